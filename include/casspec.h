@@ -1,0 +1,250 @@
+/*
+ * casspec.h -- C ABI of the CAS-Spec token-tree decode step for NVIDIA GB300 (sm_103a).
+ *
+ * CAS-Spec (arXiv 2510.26843) drafts with "virtual" draft models derived from the target model
+ * itself by dynamically switchable inference acceleration (DSIA, Sec. 4.1, Def. 4.1) and verifies
+ * token trees with tree attention (Sec. 4.2).  Every draft and verify pass is the same operation:
+ * one forward of a Llama-style decoder over n tree nodes (1 <= n <= 64) against a prefix KV cache,
+ * optionally with some layers switched off (layer-sparsity DSIA) or with W8A8 GEMMs
+ * (activation-quantisation DSIA, App. C).  After the target's pass, the longest root-to-node path
+ * that greedy decoding would have produced is accepted (lossless, Sec. 5.1) and its K/V entries are
+ * moved into the committed cache.  This library implements exactly that hot path.
+ *
+ * Conventions shared by every entry point
+ *  - Pointers marked "dev" are device pointers on the current CUDA device; "host" are host
+ *    pointers.  The library allocates no device memory: model weights, the KV cache and all
+ *    scratch live in caller-provided buffers sized by the *_bytes() queries.  It keeps only small
+ *    host handles and never retains tokens / parent_idx / output pointers after a call returns.
+ *  - Work is enqueued asynchronously on the model's stream (casspec_set_stream; default: the legacy
+ *    default stream).  Only casspec_kv_length and casspec_get_status synchronise it.
+ *  - Return value: CASSPEC_OK or a negative casspec_status.  Argument errors are reported
+ *    synchronously and enqueue nothing.  Errors detected on the device (invalid parent_idx, an
+ *    inconsistent accepted path, an expired bounded wait) are written to a device status word (the
+ *    first error wins) and read with casspec_get_status; nothing traps.
+ *  - bf16 tensors are passed as uint16_t bit patterns; matrices are row-major.  A weight W of a
+ *    linear layer is [out][in] and the layer computes y = x * W^T.
+ */
+#ifndef CASSPEC_H
+#define CASSPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Entry points are the library's only exported symbols. */
+#define CASSPEC_API __attribute__((visibility("default")))
+
+#define CASSPEC_MAX_TREE 64 /* tree slots per round; also the largest n of one call */
+
+typedef enum casspec_status {
+  CASSPEC_OK = 0,
+  CASSPEC_E_INVAL = -1,    /* NULL pointer, bad enum value, inconsistent configuration */
+  CASSPEC_E_SHAPE = -2,    /* a size outside the supported range */
+  CASSPEC_E_CAPACITY = -3, /* tree or KV capacity exceeded, or a caller buffer too small */
+  CASSPEC_E_CUDA = -4,     /* a CUDA runtime call failed (including a failed launch) */
+  CASSPEC_E_TREE = -5,     /* device: parent_idx invalid, or accepted path inconsistent */
+  CASSPEC_E_TIMEOUT = -6,  /* device: a bounded wait inside a kernel expired */
+  CASSPEC_E_STATE = -7     /* call-order rule violated (e.g. a layer's tree K/V missing) */
+} casspec_status;
+
+/* Model shape.  Requirements: d_model = n_heads * head_dim; head_dim in {64, 128};
+ * d_model % 128 == 0; ffn % 16 == 0; vocab % 8 == 0; 1 <= n_layers <= 256. */
+typedef struct casspec_model_config {
+  int32_t n_layers;
+  int32_t d_model;
+  int32_t n_heads;
+  int32_t head_dim;
+  int32_t ffn;       /* SwiGLU hidden size F */
+  int32_t vocab;
+  float rope_base;   /* rotary base (10000 for Llama-2) */
+  float rms_eps;     /* RMSNorm epsilon (1e-5 for Llama-2) */
+  int32_t with_int8; /* nonzero: reserve int8 weights + scales so quant_mode 1 can run */
+} casspec_model_config;
+
+typedef struct casspec_model casspec_model; /* opaque host handle */
+typedef struct casspec_kv casspec_kv;       /* opaque host handle */
+
+/* Weight tensors (casspec_tensor).  Shapes for d = d_model, F = ffn, V = vocab:
+ *   EMBED [V][d] bf16, LM_HEAD [V][d] bf16, FINAL_NORM [d] fp32       (layer ignored)
+ *   ATTN_NORM [d] fp32, FFN_NORM [d] fp32 (RMSNorm gains)
+ *   WQKV [3d][d] bf16 (rows: Wq, then Wk, then Wv), WO [d][d], WG [F][d], WU [F][d], WD [d][F] bf16
+ * The int8 copies (written by casspec_quantize_weights) are WQKV_Q .. WD_Q int8 with the same
+ * shapes and WQKV_S .. WD_S fp32 per-output-row scales. */
+enum casspec_tensor_id {
+  CASSPEC_T_EMBED = 0,
+  CASSPEC_T_LM_HEAD = 1,
+  CASSPEC_T_FINAL_NORM = 2,
+  CASSPEC_T_ATTN_NORM = 3,
+  CASSPEC_T_FFN_NORM = 4,
+  CASSPEC_T_WQKV = 5,
+  CASSPEC_T_WO = 6,
+  CASSPEC_T_WG = 7,
+  CASSPEC_T_WU = 8,
+  CASSPEC_T_WD = 9,
+  CASSPEC_T_WQKV_Q = 10,
+  CASSPEC_T_WO_Q = 11,
+  CASSPEC_T_WG_Q = 12,
+  CASSPEC_T_WU_Q = 13,
+  CASSPEC_T_WD_Q = 14,
+  CASSPEC_T_WQKV_S = 15,
+  CASSPEC_T_WO_S = 16,
+  CASSPEC_T_WG_S = 17,
+  CASSPEC_T_WU_S = 18,
+  CASSPEC_T_WD_S = 19
+};
+
+/* Option bits for casspec_set_options. */
+#define CASSPEC_OPT_PDL 1u    /* programmatic dependent launch between the step's kernels (default on) */
+#define CASSPEC_OPT_GRAPHS 2u /* replay a captured CUDA graph per (call shape, pointers) (default off) */
+
+/* ---------------------------------------------------------------------------------------------
+ * Model
+ * ------------------------------------------------------------------------------------------- */
+
+/* Bytes of device memory a model with `cfg` needs (weights, optional int8 copies, step scratch,
+ * tensor-map-aligned).  Returns 0 if cfg is invalid. */
+CASSPEC_API size_t casspec_model_bytes(const casspec_model_config* cfg);
+
+/* Create a model in caller memory `dev_mem` (dev, >= casspec_model_bytes(cfg), 256-byte aligned).
+ * Weights are not initialised: write them through casspec_tensor.  The caller keeps ownership of
+ * dev_mem and must keep it alive until casspec_destroy_model.  Errors: E_INVAL, E_CAPACITY, E_CUDA. */
+CASSPEC_API int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t bytes, casspec_model** out);
+
+/* Release the host handle (and any captured graphs).  Does not free dev_mem. */
+CASSPEC_API void casspec_destroy_model(casspec_model* m);
+
+/* Stream on which all of the model's work is enqueued (a cudaStream_t; NULL = legacy default). */
+CASSPEC_API int casspec_set_stream(casspec_model* m, void* cuda_stream);
+
+/* Set option bits (CASSPEC_OPT_*); returns the previous bits in *old_flags if non-NULL. */
+CASSPEC_API int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags);
+
+/* Device address and size of weight tensor `tensor` (casspec_tensor_id) of `layer` (ignored for
+ * the layer-independent tensors).  The caller writes weights there (e.g. cudaMemcpyAsync).
+ * After writing the tensor maps stay valid: they are built once from these addresses.
+ * Errors: E_INVAL (bad id / layer, int8 tensor of a model created without with_int8). */
+CASSPEC_API int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size_t* bytes);
+
+/* Per-output-channel symmetric int8 copies of WQKV, WO, WG, WU, WD for every layer (App. C
+ * activation-quantisation DSIA, W8A8 reading): for each row, a = max|w|, q = rint(w * (127/a))
+ * with ties to even (fp32, IEEE division and multiply), clamped to +-127, scale = a / 127; a = 0
+ * gives q = 0, scale 0.  Enqueued on the model stream.  Errors: E_INVAL (no int8 storage). */
+CASSPEC_API int casspec_quantize_weights(casspec_model* m);
+
+/* ---------------------------------------------------------------------------------------------
+ * KV cache: one cache shared by the target and all its self-drafts (Sec. 2 and 4.1: self-
+ * speculation keeps no separate draft cache).  Layout per layer: K then V, each
+ * [n_heads][max_ctx][head_dim] bf16.  Slots [0, P) hold the committed prefix, slots
+ * [P, P + T) hold the current token tree (T <= 64).
+ * ------------------------------------------------------------------------------------------- */
+
+/* Bytes for a cache of `max_ctx` slots (max_ctx is rounded up to a multiple of 64). */
+CASSPEC_API size_t casspec_kv_bytes(const casspec_model_config* cfg, int max_ctx);
+
+/* Create a cache for model m in caller memory `dev_mem` (dev, 256-byte aligned).  The memory is
+ * zeroed on the model stream; P = T = 0.  Errors: E_INVAL, E_CAPACITY, E_CUDA. */
+CASSPEC_API int casspec_kv_create(casspec_model* m, int max_ctx, void* dev_mem, size_t bytes, casspec_kv** out);
+CASSPEC_API void casspec_kv_destroy(casspec_kv* kv);
+
+/* K and V of `layer` (dev, [n_heads][ld_slots][head_dim] bf16) so a caller can install a prefix. */
+CASSPEC_API int casspec_kv_layer(casspec_kv* kv, int layer, void** k_dev, void** v_dev, int* ld_slots);
+
+/* Declare slots [0, P) committed in every layer and clear the tree (T = 0).  Enqueued. */
+CASSPEC_API int casspec_kv_set_prefix(casspec_kv* kv, int P);
+
+/* Discard the current tree (T = 0) without committing anything, e.g. before a verify pass that
+ * re-runs the whole draft tree.  Host-side bookkeeping only. */
+CASSPEC_API int casspec_kv_reset_tree(casspec_kv* kv);
+
+/* Synchronise the model stream and return the committed length P and the tree length T. */
+CASSPEC_API int casspec_kv_length(casspec_kv* kv, int* P_out, int* T_out);
+
+/* ---------------------------------------------------------------------------------------------
+ * The tree step (Sec. 4.2: tree attention for parallel drafting and parallel verification).
+ * ------------------------------------------------------------------------------------------- */
+
+/* One decoder forward over n new tree nodes appended at tree slots T .. T+n-1.
+ *   tokens      dev int32 [n]   token id of each node (0 <= id < vocab; clamped if not)
+ *   parent_idx  dev int32 [n]   tree slot of each node's parent, in [-1, T + i); -1 makes the node
+ *                               a child of the last committed token (depth 0, position P).  A node
+ *                               at depth t sits at position P + t and attends to the whole prefix
+ *                               plus exactly its ancestors and itself.
+ *   n           1 .. 64, T + n <= 64, P + T + n <= max_ctx
+ *   skip_mask   host uint8 [n_layers] or NULL (all layers on); 0 switches layer l off: the layer
+ *               is the identity on the residual stream and writes no K/V (layer-sparsity DSIA).
+ *               Rule: every active layer must hold K/V for all T existing tree slots (nested
+ *               masks, as in a layer-sparsity cascade); otherwise E_STATE.
+ *   quant_mode  0: bf16 weights, fp32 accumulation.  1: W8A8 GEMMs for WQKV, WO, WG/WU, WD with
+ *               per-token dynamic int8 activations (activation-quantisation DSIA); attention, K/V
+ *               and the LM head stay bf16.  Mode 1 needs casspec_quantize_weights first.
+ *   logits_out  dev fp32 [n][vocab] or NULL.
+ * The row argmax of the logits (ties to the lowest id) and the top-2 margin of every node are
+ * always computed and kept in the model (casspec_argmax).  Invalid parent_idx values are reported
+ * through the status word (E_TREE); the step still runs, treating such a node as a depth-0 node.
+ * Errors (synchronous): E_INVAL, E_SHAPE, E_CAPACITY, E_STATE, E_CUDA. */
+CASSPEC_API int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent_idx,
+                      int n, const uint8_t* skip_mask, int quant_mode, float* logits_out);
+
+/* Device pointers to the argmax (int32 [64]) and top-2 margin (fp32 [64]) of the latest tree
+ * step's nodes.  Valid until the next tree step on this model. */
+CASSPEC_API int casspec_argmax(casspec_model* m, const int32_t** argmax_dev, const float** margin_dev);
+
+/* Greedy lossless acceptance (Sec. 5.1) over a whole verified tree of n nodes.
+ *   logits        dev fp32 [n][vocab] of the target's pass, or NULL to use the model's fused
+ *                 argmax of its latest tree step (which must then have covered these n nodes).
+ *   tokens, parent_idx  dev int32 [n]; node 0 must be the only root (parent -1) and
+ *                 parent_idx[c] < c for c > 0 (else E_TREE on the status word, accepted L = 0).
+ *   accepted_out  dev int32 [n + 2]: [0] = L (>= 1), [1 .. L] = node indices of the accepted path
+ *                 root first, [L + 1] = bonus token (the target's argmax at the last accepted node).
+ * A node matches when its parent matches and its token equals the parent's argmax (node 0 always
+ * matches); the accepted node is the deepest match, the lowest index among equally deep ones. */
+CASSPEC_API int casspec_accept_greedy(casspec_model* m, const float* logits, const int32_t* tokens, const int32_t* parent_idx,
+                          int n, int32_t* accepted_out);
+
+/* Move the K/V of the accepted path (accepted_out as written by casspec_accept_greedy, dev) from
+ * tree slots to committed slots P .. P+L-1 in every layer, then P += L and T = 0.  All layers must
+ * hold the tree's K/V (the verify pass ran with every layer on), else E_STATE.  A path that is
+ * inconsistent with the current tree (L < 1, L > T, an index >= T, non-increasing indices) sets
+ * E_TREE on the status word and leaves the cache unchanged. */
+CASSPEC_API int casspec_kv_compact(casspec_kv* kv, const int32_t* accepted_out);
+
+/* Synchronise the model stream; return and clear the device status word. */
+CASSPEC_API int casspec_get_status(casspec_model* m, int* status_out);
+
+CASSPEC_API const char* casspec_status_string(int status);
+
+/* ---------------------------------------------------------------------------------------------
+ * Stateless kernels of the step, exposed for composition and for per-kernel checks.  All run on
+ * `cuda_stream`; scratch is caller-provided.
+ * ------------------------------------------------------------------------------------------- */
+
+/* Scratch bytes needed by casspec_linear_bf16 for an [N][K] weight and n tokens. */
+CASSPEC_API size_t casspec_linear_workspace_bytes(int N, int K, int n);
+
+/* Y[i][o] = sum_k X[i][k] * W[o][k] (fp32 accumulation on the tensor cores) for i < n, o < N.
+ *   W dev bf16 [N][K], X dev bf16 [n][K] (row stride K), Y dev fp32 [n][ldy], ldy >= N.
+ *   1 <= n <= 64, K % 8 == 0, N >= 1; W and X 16-byte aligned.
+ *   workspace dev, >= casspec_linear_workspace_bytes(N, K, n) bytes; its first 4 KB must be zero
+ *   before the first call and are left zero by every call that completes. */
+CASSPEC_API int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int n, float* Y, int ldy,
+                        void* workspace, size_t workspace_bytes, void* cuda_stream);
+
+/* RMSNorm of n rows (Llama pre-norm): y = x / sqrt(mean(x^2) + eps) * g, fp32 arithmetic.
+ *   x dev fp32 [n][d]; g dev fp32 [d]; y_bf16 dev bf16 [n][d] (may be NULL if q is given).
+ *   If q_out (dev int8 [n][d]) and s_out (dev fp32 [n]) are non-NULL, each bf16 output row is also
+ *   quantised with the per-row int8 rule of casspec_quantize_weights (that rule, applied per token,
+ *   is the activation quantisation of the W8A8 draft). */
+CASSPEC_API int casspec_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y_bf16, int8_t* q_out,
+                    float* s_out, void* cuda_stream);
+
+/* Per-row int8 quantisation of bf16 rows x [n][d] -> q [n][d], s [n] (same rule). */
+CASSPEC_API int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q_out, float* s_out, void* cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CASSPEC_H */

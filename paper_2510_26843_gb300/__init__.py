@@ -1,0 +1,251 @@
+"""Python binding of libcasspec (include/casspec.h): argument marshalling only.
+
+Every function mirrors the C entry point of the same name without the ``casspec_`` prefix.
+Device buffers are torch CUDA tensors (passed by data pointer); streams are torch.cuda.Stream
+objects or raw handles.  Loading fails loudly if the CUDA library has not been built: there is no
+fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libcasspec.so")
+
+OK, E_INVAL, E_SHAPE, E_CAPACITY, E_CUDA, E_TREE, E_TIMEOUT, E_STATE = 0, -1, -2, -3, -4, -5, -6, -7
+MAX_TREE = 64
+OPT_PDL, OPT_GRAPHS = 1, 2
+
+(T_EMBED, T_LM_HEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WG, T_WU, T_WD,
+ T_WQKV_Q, T_WO_Q, T_WG_Q, T_WU_Q, T_WD_Q, T_WQKV_S, T_WO_S, T_WG_S, T_WU_S, T_WD_S) = range(20)
+
+EXPORTS = [
+    "casspec_model_bytes", "casspec_create_model", "casspec_destroy_model", "casspec_set_stream",
+    "casspec_set_options", "casspec_tensor", "casspec_quantize_weights", "casspec_kv_bytes", "casspec_kv_create",
+    "casspec_kv_destroy", "casspec_kv_layer", "casspec_kv_set_prefix", "casspec_kv_reset_tree", "casspec_kv_length",
+    "casspec_tree_step", "casspec_argmax", "casspec_accept_greedy", "casspec_kv_compact", "casspec_get_status",
+    "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_rmsnorm",
+    "casspec_quantize_rows",
+]
+
+
+class ModelConfig(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("rope_base", ctypes.c_float), ("rms_eps", ctypes.c_float), ("with_int8", ctypes.c_int32)]
+
+
+class CasspecError(RuntimeError):
+    def __init__(self, fn: str, rc: int):
+        super().__init__(f"{fn} failed: {rc} ({status_string(rc)})")
+        self.rc = rc
+
+
+_lib = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_SZ = ctypes.c_size_t
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libcasspec.so (raises if it is missing: build it with __graft_entry__.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: the CUDA library must be built (python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(path)
+    sig = {
+        "casspec_model_bytes": (_SZ, [ctypes.POINTER(ModelConfig)]),
+        "casspec_create_model": (_I, [ctypes.POINTER(ModelConfig), _P, _SZ, ctypes.POINTER(_P)]),
+        "casspec_destroy_model": (None, [_P]),
+        "casspec_set_stream": (_I, [_P, _P]),
+        "casspec_set_options": (_I, [_P, ctypes.c_uint, ctypes.POINTER(ctypes.c_uint)]),
+        "casspec_tensor": (_I, [_P, _I, _I, ctypes.POINTER(_P), ctypes.POINTER(_SZ)]),
+        "casspec_quantize_weights": (_I, [_P]),
+        "casspec_kv_bytes": (_SZ, [ctypes.POINTER(ModelConfig), _I]),
+        "casspec_kv_create": (_I, [_P, _I, _P, _SZ, ctypes.POINTER(_P)]),
+        "casspec_kv_destroy": (None, [_P]),
+        "casspec_kv_layer": (_I, [_P, _I, ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.POINTER(_I)]),
+        "casspec_kv_set_prefix": (_I, [_P, _I]),
+        "casspec_kv_reset_tree": (_I, [_P]),
+        "casspec_kv_length": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+        "casspec_tree_step": (_I, [_P, _P, _P, _P, _I, _P, _I, _P]),
+        "casspec_argmax": (_I, [_P, ctypes.POINTER(_P), ctypes.POINTER(_P)]),
+        "casspec_accept_greedy": (_I, [_P, _P, _P, _P, _I, _P]),
+        "casspec_kv_compact": (_I, [_P, _P]),
+        "casspec_get_status": (_I, [_P, ctypes.POINTER(_I)]),
+        "casspec_status_string": (ctypes.c_char_p, [_I]),
+        "casspec_linear_workspace_bytes": (_SZ, [_I, _I, _I]),
+        "casspec_linear_bf16": (_I, [_P, _I, _I, _P, _I, _P, _I, _P, _SZ, _P]),
+        "casspec_rmsnorm": (_I, [_P, _P, _I, _I, ctypes.c_float, _P, _P, _P, _P]),
+        "casspec_quantize_rows": (_I, [_P, _I, _I, _P, _P, _P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _ptr(t) -> int | None:
+    """Device pointer of a torch tensor (or None / raw int)."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(s) -> int | None:
+    if s is None:
+        return None
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _check(fn: str, rc: int) -> None:
+    if rc != OK:
+        raise CasspecError(fn, rc)
+
+
+def config(n_layers, d_model, n_heads, head_dim, ffn, vocab, rope_base=10000.0, rms_eps=1e-5, with_int8=0):
+    return ModelConfig(n_layers, d_model, n_heads, head_dim, ffn, vocab, rope_base, rms_eps, int(with_int8))
+
+
+def model_bytes(cfg: ModelConfig) -> int:
+    return load_library().casspec_model_bytes(ctypes.byref(cfg))
+
+
+def create_model(cfg: ModelConfig, dev_mem) -> int:
+    h = _P()
+    _check("casspec_create_model",
+           load_library().casspec_create_model(ctypes.byref(cfg), _ptr(dev_mem), dev_mem.numel() * dev_mem.element_size(),
+                                               ctypes.byref(h)))
+    return h.value
+
+
+def destroy_model(m: int) -> None:
+    load_library().casspec_destroy_model(m)
+
+
+def set_stream(m: int, stream) -> None:
+    _check("casspec_set_stream", load_library().casspec_set_stream(m, _stream(stream)))
+
+
+def set_options(m: int, flags: int) -> int:
+    old = ctypes.c_uint()
+    _check("casspec_set_options", load_library().casspec_set_options(m, flags, ctypes.byref(old)))
+    return old.value
+
+
+def tensor(m: int, tensor_id: int, layer: int = 0) -> tuple[int, int]:
+    p, nb = _P(), _SZ()
+    _check("casspec_tensor", load_library().casspec_tensor(m, tensor_id, layer, ctypes.byref(p), ctypes.byref(nb)))
+    return p.value, nb.value
+
+
+def quantize_weights(m: int) -> None:
+    _check("casspec_quantize_weights", load_library().casspec_quantize_weights(m))
+
+
+def kv_bytes(cfg: ModelConfig, max_ctx: int) -> int:
+    return load_library().casspec_kv_bytes(ctypes.byref(cfg), max_ctx)
+
+
+def kv_create(m: int, max_ctx: int, dev_mem) -> int:
+    h = _P()
+    _check("casspec_kv_create", load_library().casspec_kv_create(m, max_ctx, _ptr(dev_mem),
+                                                                 dev_mem.numel() * dev_mem.element_size(), ctypes.byref(h)))
+    return h.value
+
+
+def kv_destroy(kv: int) -> None:
+    load_library().casspec_kv_destroy(kv)
+
+
+def kv_layer(kv: int, layer: int) -> tuple[int, int, int]:
+    k, v, ld = _P(), _P(), _I()
+    _check("casspec_kv_layer", load_library().casspec_kv_layer(kv, layer, ctypes.byref(k), ctypes.byref(v), ctypes.byref(ld)))
+    return k.value, v.value, ld.value
+
+
+def kv_set_prefix(kv: int, P: int) -> None:
+    _check("casspec_kv_set_prefix", load_library().casspec_kv_set_prefix(kv, P))
+
+
+def kv_reset_tree(kv: int) -> None:
+    _check("casspec_kv_reset_tree", load_library().casspec_kv_reset_tree(kv))
+
+
+def kv_length(kv: int) -> tuple[int, int]:
+    P, T = _I(), _I()
+    _check("casspec_kv_length", load_library().casspec_kv_length(kv, ctypes.byref(P), ctypes.byref(T)))
+    return P.value, T.value
+
+
+def tree_step(m: int, kv: int, tokens, parent_idx, n: int, skip_mask=None, quant_mode: int = 0, logits_out=None,
+              check: bool = True) -> int:
+    mask = None
+    if skip_mask is not None:
+        mask = np.ascontiguousarray(np.asarray(skip_mask, dtype=np.uint8))
+    rc = load_library().casspec_tree_step(m, kv, _ptr(tokens), _ptr(parent_idx), n,
+                                          None if mask is None else mask.ctypes.data, quant_mode, _ptr(logits_out))
+    if check:
+        _check("casspec_tree_step", rc)
+    return rc
+
+
+def argmax(m: int) -> tuple[int, int]:
+    a, g = _P(), _P()
+    _check("casspec_argmax", load_library().casspec_argmax(m, ctypes.byref(a), ctypes.byref(g)))
+    return a.value, g.value
+
+
+def accept_greedy(m: int, logits, tokens, parent_idx, n: int, accepted_out) -> None:
+    _check("casspec_accept_greedy",
+           load_library().casspec_accept_greedy(m, _ptr(logits), _ptr(tokens), _ptr(parent_idx), n, _ptr(accepted_out)))
+
+
+def kv_compact(kv: int, accepted_out, check: bool = True) -> int:
+    rc = load_library().casspec_kv_compact(kv, _ptr(accepted_out))
+    if check:
+        _check("casspec_kv_compact", rc)
+    return rc
+
+
+def get_status(m: int) -> int:
+    st = _I()
+    _check("casspec_get_status", load_library().casspec_get_status(m, ctypes.byref(st)))
+    return st.value
+
+
+def status_string(rc: int) -> str:
+    try:
+        return load_library().casspec_status_string(rc).decode()
+    except RuntimeError:
+        return str(rc)
+
+
+def linear_workspace_bytes(N: int, K: int, n: int) -> int:
+    return load_library().casspec_linear_workspace_bytes(N, K, n)
+
+
+def linear_bf16(W, N: int, K: int, X, n: int, Y, ldy: int, workspace, stream=None) -> None:
+    _check("casspec_linear_bf16",
+           load_library().casspec_linear_bf16(_ptr(W), N, K, _ptr(X), n, _ptr(Y), ldy, _ptr(workspace),
+                                              workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def rmsnorm(x, g, n: int, d: int, eps: float, y=None, q=None, s=None, stream=None) -> None:
+    _check("casspec_rmsnorm", load_library().casspec_rmsnorm(_ptr(x), _ptr(g), n, d, eps, _ptr(y), _ptr(q), _ptr(s),
+                                                             _stream(stream)))
+
+
+def quantize_rows(x, n: int, d: int, q, s, stream=None) -> None:
+    _check("casspec_quantize_rows", load_library().casspec_quantize_rows(_ptr(x), n, d, _ptr(q), _ptr(s), _stream(stream)))

@@ -1,0 +1,785 @@
+// Host runtime of the C ABI (include/casspec.h): model and KV-cache descriptors in caller memory,
+// argument validation, the launch sequence of one tree step, and optional CUDA-graph replay.
+#include <cmath>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <new>
+#include <tuple>
+#include <vector>
+
+#include "kernels.h"
+#include "../../include/casspec.h"
+
+using namespace casspec;
+
+namespace {
+
+constexpr int kSmsBound = 256;  // scratch is sized for up to this many SMs
+constexpr int kMaxTree = CASSPEC_MAX_TREE;
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+struct LayerPtrs {
+  float *attn_norm, *ffn_norm;
+  uint16_t *wqkv, *wo, *wg, *wu, *wd;
+  int8_t *qkv_q, *wo_q, *wg_q, *wu_q, *wd_q;
+  float *qkv_s, *wo_s, *wg_s, *wu_s, *wd_s;
+  CUtensorMap tm_qkv, tm_o, tm_g, tm_u, tm_d;
+};
+
+// Byte layout of a model's device memory (weights, int8 copies, step scratch).
+struct Layout {
+  size_t total = 0;
+  size_t embed, lm_head, final_norm, inv_freq;
+  std::vector<size_t> attn_norm, ffn_norm, wqkv, wo, wg, wu, wd;
+  std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
+  size_t x, xn, q, o, u, xq, xs, pos, anc, rope, am_v1, am_i1, am_v2, am, margin, am2;
+  size_t gemm_part, gemm_cnt, i8_part, i8_cnt, attn_o, attn_ml, attn_cnt, status;
+  size_t scratch_begin;
+  int max_tiles, lm_tiles;
+};
+
+bool config_ok(const casspec_model_config* c) {
+  if (c == nullptr) return false;
+  if (c->n_layers < 1 || c->n_layers > 256) return false;
+  if (c->head_dim != 64 && c->head_dim != 128) return false;
+  if (c->n_heads < 1 || c->d_model != c->n_heads * c->head_dim) return false;
+  if (c->d_model % 128 != 0) return false;
+  if (c->ffn < 16 || c->ffn % 16 != 0) return false;
+  if (c->vocab < 1 || c->vocab % 8 != 0) return false;
+  if (!(c->rope_base > 0.f) || !(c->rms_eps >= 0.f)) return false;
+  return true;
+}
+
+int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
+
+Layout make_layout(const casspec_model_config& c) {
+  Layout L;
+  const size_t d = c.d_model, F = c.ffn, V = c.vocab, NL = c.n_layers;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    off = align_up(off, 256);
+    size_t r = off;
+    off += bytes;
+    return r;
+  };
+  L.embed = take(V * d * 2);
+  L.lm_head = take(V * d * 2);
+  L.final_norm = take(d * 4);
+  L.inv_freq = take((size_t)(c.head_dim / 2) * 8);
+  for (size_t l = 0; l < NL; ++l) {
+    L.attn_norm.push_back(take(d * 4));
+    L.ffn_norm.push_back(take(d * 4));
+    L.wqkv.push_back(take(3 * d * d * 2));
+    L.wo.push_back(take(d * d * 2));
+    L.wg.push_back(take(F * d * 2));
+    L.wu.push_back(take(F * d * 2));
+    L.wd.push_back(take(d * F * 2));
+  }
+  if (c.with_int8) {
+    for (size_t l = 0; l < NL; ++l) {
+      L.qkv_q.push_back(take(3 * d * d));
+      L.wo_q.push_back(take(d * d));
+      L.wg_q.push_back(take(F * d));
+      L.wu_q.push_back(take(F * d));
+      L.wd_q.push_back(take(d * F));
+      L.qkv_s.push_back(take(3 * d * 4));
+      L.wo_s.push_back(take(d * 4));
+      L.wg_s.push_back(take(F * 4));
+      L.wu_s.push_back(take(F * 4));
+      L.wd_s.push_back(take(d * 4));
+    }
+  }
+  L.scratch_begin = align_up(off, 256);
+  const size_t T = kMaxTree;
+  L.lm_tiles = cdiv(V, 128);
+  L.max_tiles = std::max(std::max(cdiv(3 * d, 128), cdiv(F, 64)), L.lm_tiles);
+  L.x = take(T * d * 4);
+  L.xn = take(T * d * 2);
+  L.q = take(T * d * 2);
+  L.o = take(T * d * 2);
+  L.u = take(T * F * 2);
+  L.xq = take(T * std::max(d, F));
+  L.xs = take(T * 4);
+  L.pos = take(T * 4);
+  L.anc = take(T * 8);
+  L.rope = take(T * (c.head_dim / 2) * 8);
+  L.am_v1 = take((size_t)L.lm_tiles * T * 4);
+  L.am_i1 = take((size_t)L.lm_tiles * T * 4);
+  L.am_v2 = take((size_t)L.lm_tiles * T * 4);
+  L.am = take(T * 4);
+  L.margin = take(T * 4);
+  L.am2 = take(T * 4);
+  L.gemm_part = take(gemm_partials_floats(L.max_tiles, kSmsBound) * 4);
+  L.gemm_cnt = take((size_t)L.max_tiles * 4);
+  L.i8_part = take((size_t)(6 * kSmsBound + 2 * L.max_tiles) * 64 * 128 * 4);
+  L.i8_cnt = take((size_t)L.max_tiles * 4);
+  L.attn_o = take((size_t)(2 * kSmsBound + 2 * c.n_heads) * 64 * c.head_dim * 4);
+  L.attn_ml = take((size_t)(2 * kSmsBound + 2 * c.n_heads) * 64 * 2 * 4);
+  L.attn_cnt = take((size_t)c.n_heads * 4);
+  L.status = take(256);
+  L.total = align_up(off, 256);
+  return L;
+}
+
+int num_sms_of_current_device() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return sms;
+}
+
+int roundup16(int n) { return (n + 15) / 16 * 16; }
+
+}  // namespace
+
+struct GraphKey {
+  const void* kv;
+  const void* tokens;
+  const void* parent;
+  const void* logits;
+  int n, T, mode;
+  std::vector<uint8_t> mask;
+  bool operator<(const GraphKey& o) const {
+    return std::tie(kv, tokens, parent, logits, n, T, mode, mask) <
+           std::tie(o.kv, o.tokens, o.parent, o.logits, o.n, o.T, o.mode, o.mask);
+  }
+};
+
+struct casspec_model {
+  casspec_model_config cfg;
+  Layout lay;
+  uint8_t* base = nullptr;
+  cudaStream_t stream = nullptr;
+  cudaStream_t cap_stream = nullptr;
+  unsigned flags = CASSPEC_OPT_PDL;
+  int num_sms = 0;
+  uint16_t *embed, *lm_head;
+  float* final_norm;
+  double* inv_freq;
+  std::vector<LayerPtrs> layers;
+  CUtensorMap tm_lm;
+  CUtensorMap tm_xn[4], tm_oact[4], tm_uact[4];
+  float* x;
+  uint16_t *xn, *q, *o, *u;
+  int8_t* xq;
+  float* xs;
+  int* pos;
+  unsigned long long* anc;
+  float2* rope;
+  float *am_v1, *am_v2, *margin;
+  int *am_i1, *am, *am2;
+  float* gemm_part;
+  unsigned* gemm_cnt;
+  int* i8_part;
+  unsigned* i8_cnt;
+  float *attn_o, *attn_ml;
+  unsigned* attn_cnt;
+  int* status;
+  std::map<GraphKey, cudaGraphExec_t> graphs;
+  std::mutex mu;
+};
+
+struct casspec_kv {
+  casspec_model* m;
+  uint16_t* base;
+  int ctx;
+  int* dP;
+  int* tdepth;
+  unsigned long long* tanc;
+  unsigned* compact_cnt;
+  int T = 0;
+  long long P_upper = 0;
+  std::vector<int> layer_valid;  // tree slots [0, layer_valid[l]) hold K/V of layer l
+};
+
+namespace {
+
+size_t kv_region_bytes(const casspec_model_config& c, int ctx) {
+  return (size_t)c.n_layers * 2 * c.n_heads * ctx * c.head_dim * 2;
+}
+int kv_ctx(int max_ctx) { return (max_ctx + 63) / 64 * 64; }
+size_t kv_meta_bytes() { return 256 + kMaxTree * 4 + kMaxTree * 8 + 256; }
+
+uint16_t* kv_layer_k(casspec_kv* kv, int l) {
+  const auto& c = kv->m->cfg;
+  return kv->base + (size_t)l * 2 * c.n_heads * kv->ctx * c.head_dim;
+}
+uint16_t* kv_layer_v(casspec_kv* kv, int l) {
+  const auto& c = kv->m->cfg;
+  return kv_layer_k(kv, l) + (size_t)c.n_heads * kv->ctx * c.head_dim;
+}
+
+#define CK(call)                              \
+  do {                                        \
+    cudaError_t e_ = (call);                  \
+    if (e_ != cudaSuccess) return CASSPEC_E_CUDA; \
+  } while (0)
+
+// Enqueue one tree step on stream s (argument checks already done).
+int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent, int n,
+                 const std::vector<uint8_t>& on, int mode, float* logits, cudaStream_t s) {
+  const auto& c = m->cfg;
+  const int d = c.d_model, F = c.ffn, V = c.vocab, hd = c.head_dim, H = c.n_heads;
+  const bool pdl = (m->flags & CASSPEC_OPT_PDL) != 0;
+  const int BN = roundup16(n);
+  const int bi = BN / 16 - 1;
+  const int T = kv->T;
+
+  CK(launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->rope, m->inv_freq, hd / 2,
+                      m->status, s, pdl));
+  CK(launch_embed(m->embed, tokens, n, d, V, m->x, s, pdl));
+
+  EpiParams base = {};
+  base.n = n;
+  base.ctx = kv->ctx;
+  base.d = d;
+  base.hd = hd;
+  base.T = T;
+  base.dP = kv->dP;
+  base.rope = m->rope;
+
+  auto gemm = [&](const CUtensorMap& tw, const CUtensorMap& tw2, const CUtensorMap& tx, int epi, int tiles,
+                  int kblocks, const EpiParams& e) -> cudaError_t {
+    GemmArgs a = {};
+    a.tiles = tiles;
+    a.kblocks = kblocks;
+    a.partials = m->gemm_part;
+    a.counters = m->gemm_cnt;
+    a.status = m->status;
+    a.ep = e;
+    return launch_gemm_bf16(tw, tw2, tx, BN, epi, a, gemm_bf16_grid(tiles, kblocks, m->num_sms), s, pdl);
+  };
+  auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
+                   int epi, const EpiParams& e) -> cudaError_t {
+    GemmI8Args a = {};
+    a.W = W;
+    a.sw = sw;
+    a.W2 = W2;
+    a.sw2 = sw2;
+    a.X = m->xq;
+    a.sx = m->xs;
+    a.N = N;
+    a.K = K;
+    a.tiles = tiles;
+    a.ksplit = gemm_i8_ksplit(tiles, K, m->num_sms);
+    a.partials = m->i8_part;
+    a.counters = m->i8_cnt;
+    a.status = m->status;
+    a.ep = e;
+    return launch_gemm_i8(a, BN, epi, s, pdl);
+  };
+
+  const long long total_slots = kv->P_upper + T + n;
+  for (int l = 0; l < c.n_layers; ++l) {
+    if (!on[l]) continue;
+    LayerPtrs& Lp = m->layers[l];
+    // attention block
+    CK(launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
+                      pdl));
+    EpiParams e = base;
+    e.N = 3 * d;
+    e.q_out = m->q;
+    e.kc = kv_layer_k(kv, l);
+    e.vc = kv_layer_v(kv, l);
+    if (mode == 0)
+      CK(gemm(Lp.tm_qkv, Lp.tm_qkv, m->tm_xn[bi], EPI_QKV, 3 * d / 128, cdiv(d, 64), e));
+    else
+      CK(gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+    AttnArgs at = {};
+    at.q = m->q;
+    at.kc = e.kc;
+    at.vc = e.vc;
+    at.o = m->o;
+    at.anc = m->anc;
+    at.dP = kv->dP;
+    at.T = T;
+    at.n = n;
+    at.ctx = kv->ctx;
+    at.d = d;
+    at.splits = attn_splits(H, (int)std::min<long long>(total_slots, kv->ctx), m->num_sms);
+    at.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
+    at.part_o = m->attn_o;
+    at.part_ml = m->attn_ml;
+    at.counters = m->attn_cnt;
+    at.status = m->status;
+    CK(launch_tree_attention(at, hd, H, s, pdl));
+    EpiParams er = base;
+    er.N = d;
+    er.y = m->x;
+    er.ldy = d;
+    if (mode == 0) {
+      CK(gemm(Lp.tm_o, Lp.tm_o, m->tm_oact[bi], EPI_RESID, d / 128, cdiv(d, 64), er));
+    } else {
+      CK(launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
+      CK(gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, er));
+    }
+    // feed-forward block
+    CK(launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
+                      pdl));
+    EpiParams eg = base;
+    eg.N = F;
+    eg.u_out = m->u;
+    if (mode == 0)
+      CK(gemm(Lp.tm_g, Lp.tm_u, m->tm_xn[bi], EPI_GLU, cdiv(F, 64), cdiv(d, 64), eg));
+    else
+      CK(gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
+    if (mode == 0) {
+      CK(gemm(Lp.tm_d, Lp.tm_d, m->tm_uact[bi], EPI_RESID, d / 128, cdiv(F, 64), er));
+    } else {
+      CK(launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
+      CK(gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, er));
+    }
+  }
+  CK(launch_rmsnorm(m->x, m->final_norm, n, d, c.rms_eps, m->xn, nullptr, nullptr, s, pdl));
+  EpiParams el = base;
+  el.N = V;
+  el.logits = logits;
+  el.am_v1 = m->am_v1;
+  el.am_i1 = m->am_i1;
+  el.am_v2 = m->am_v2;
+  CK(gemm(m->tm_lm, m->tm_lm, m->tm_xn[bi], EPI_LMHEAD, m->lay.lm_tiles, cdiv(d, 64), el));
+  CK(launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, m->lay.lm_tiles, n, m->am, m->margin, s, pdl));
+  return CASSPEC_OK;
+}
+
+bool build_tensor_maps(casspec_model* m) {
+  const auto& c = m->cfg;
+  const uint64_t d = c.d_model, F = c.ffn, V = c.vocab;
+  bool ok = true;
+  for (int l = 0; l < c.n_layers; ++l) {
+    LayerPtrs& Lp = m->layers[l];
+    ok = ok && encode_tmap_bf16(&Lp.tm_qkv, Lp.wqkv, d, 3 * d, d * 2, 64, 128);
+    ok = ok && encode_tmap_bf16(&Lp.tm_o, Lp.wo, d, d, d * 2, 64, 128);
+    ok = ok && encode_tmap_bf16(&Lp.tm_g, Lp.wg, d, F, d * 2, 64, 64);
+    ok = ok && encode_tmap_bf16(&Lp.tm_u, Lp.wu, d, F, d * 2, 64, 64);
+    ok = ok && encode_tmap_bf16(&Lp.tm_d, Lp.wd, F, d, F * 2, 64, 128);
+  }
+  ok = ok && encode_tmap_bf16(&m->tm_lm, m->lm_head, d, V, d * 2, 64, 128);
+  for (int b = 0; b < 4; ++b) {
+    const uint32_t BN = 16 * (b + 1);
+    ok = ok && encode_tmap_bf16(&m->tm_xn[b], m->xn, d, kMaxTree, d * 2, 64, BN);
+    ok = ok && encode_tmap_bf16(&m->tm_oact[b], m->o, d, kMaxTree, d * 2, 64, BN);
+    ok = ok && encode_tmap_bf16(&m->tm_uact[b], m->u, F, kMaxTree, F * 2, 64, BN);
+  }
+  return ok;
+}
+
+}  // namespace
+
+// =============================================================================================
+// C ABI
+// =============================================================================================
+extern "C" {
+
+size_t casspec_model_bytes(const casspec_model_config* cfg) {
+  if (!config_ok(cfg)) return 0;
+  return make_layout(*cfg).total;
+}
+
+int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t bytes, casspec_model** out) {
+  if (out == nullptr || dev_mem == nullptr || !config_ok(cfg)) return CASSPEC_E_INVAL;
+  if ((reinterpret_cast<uintptr_t>(dev_mem) & 255) != 0) return CASSPEC_E_INVAL;
+  Layout L = make_layout(*cfg);
+  if (bytes < L.total) return CASSPEC_E_CAPACITY;
+  const int sms = num_sms_of_current_device();
+  if (sms <= 0 || sms > kSmsBound) return CASSPEC_E_CUDA;
+  casspec_model* m = new (std::nothrow) casspec_model();
+  if (m == nullptr) return CASSPEC_E_CAPACITY;
+  m->cfg = *cfg;
+  m->lay = L;
+  m->num_sms = sms;
+  uint8_t* b = static_cast<uint8_t*>(dev_mem);
+  m->base = b;
+  m->embed = reinterpret_cast<uint16_t*>(b + L.embed);
+  m->lm_head = reinterpret_cast<uint16_t*>(b + L.lm_head);
+  m->final_norm = reinterpret_cast<float*>(b + L.final_norm);
+  m->inv_freq = reinterpret_cast<double*>(b + L.inv_freq);
+  m->layers.resize(cfg->n_layers);
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    LayerPtrs& p = m->layers[l];
+    std::memset(&p, 0, sizeof(p));
+    p.attn_norm = reinterpret_cast<float*>(b + L.attn_norm[l]);
+    p.ffn_norm = reinterpret_cast<float*>(b + L.ffn_norm[l]);
+    p.wqkv = reinterpret_cast<uint16_t*>(b + L.wqkv[l]);
+    p.wo = reinterpret_cast<uint16_t*>(b + L.wo[l]);
+    p.wg = reinterpret_cast<uint16_t*>(b + L.wg[l]);
+    p.wu = reinterpret_cast<uint16_t*>(b + L.wu[l]);
+    p.wd = reinterpret_cast<uint16_t*>(b + L.wd[l]);
+    if (cfg->with_int8) {
+      p.qkv_q = reinterpret_cast<int8_t*>(b + L.qkv_q[l]);
+      p.wo_q = reinterpret_cast<int8_t*>(b + L.wo_q[l]);
+      p.wg_q = reinterpret_cast<int8_t*>(b + L.wg_q[l]);
+      p.wu_q = reinterpret_cast<int8_t*>(b + L.wu_q[l]);
+      p.wd_q = reinterpret_cast<int8_t*>(b + L.wd_q[l]);
+      p.qkv_s = reinterpret_cast<float*>(b + L.qkv_s[l]);
+      p.wo_s = reinterpret_cast<float*>(b + L.wo_s[l]);
+      p.wg_s = reinterpret_cast<float*>(b + L.wg_s[l]);
+      p.wu_s = reinterpret_cast<float*>(b + L.wu_s[l]);
+      p.wd_s = reinterpret_cast<float*>(b + L.wd_s[l]);
+    }
+  }
+  m->x = reinterpret_cast<float*>(b + L.x);
+  m->xn = reinterpret_cast<uint16_t*>(b + L.xn);
+  m->q = reinterpret_cast<uint16_t*>(b + L.q);
+  m->o = reinterpret_cast<uint16_t*>(b + L.o);
+  m->u = reinterpret_cast<uint16_t*>(b + L.u);
+  m->xq = reinterpret_cast<int8_t*>(b + L.xq);
+  m->xs = reinterpret_cast<float*>(b + L.xs);
+  m->pos = reinterpret_cast<int*>(b + L.pos);
+  m->anc = reinterpret_cast<unsigned long long*>(b + L.anc);
+  m->rope = reinterpret_cast<float2*>(b + L.rope);
+  m->am_v1 = reinterpret_cast<float*>(b + L.am_v1);
+  m->am_i1 = reinterpret_cast<int*>(b + L.am_i1);
+  m->am_v2 = reinterpret_cast<float*>(b + L.am_v2);
+  m->am = reinterpret_cast<int*>(b + L.am);
+  m->margin = reinterpret_cast<float*>(b + L.margin);
+  m->am2 = reinterpret_cast<int*>(b + L.am2);
+  m->gemm_part = reinterpret_cast<float*>(b + L.gemm_part);
+  m->gemm_cnt = reinterpret_cast<unsigned*>(b + L.gemm_cnt);
+  m->i8_part = reinterpret_cast<int*>(b + L.i8_part);
+  m->i8_cnt = reinterpret_cast<unsigned*>(b + L.i8_cnt);
+  m->attn_o = reinterpret_cast<float*>(b + L.attn_o);
+  m->attn_ml = reinterpret_cast<float*>(b + L.attn_ml);
+  m->attn_cnt = reinterpret_cast<unsigned*>(b + L.attn_cnt);
+  m->status = reinterpret_cast<int*>(b + L.status);
+
+  std::vector<double> invf(cfg->head_dim / 2);
+  for (int j = 0; j < cfg->head_dim / 2; ++j)
+    invf[j] = std::pow((double)cfg->rope_base, -2.0 * j / (double)cfg->head_dim);
+  if (cudaMemset(b + L.scratch_begin, 0, L.total - L.scratch_begin) != cudaSuccess ||
+      cudaMemcpy(m->inv_freq, invf.data(), invf.size() * 8, cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+    delete m;
+    return CASSPEC_E_CUDA;
+  }
+  // RMSNorm gains default to 1.0
+  std::vector<float> ones(cfg->d_model, 1.0f);
+  bool ok = cudaMemcpy(m->final_norm, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess;
+  for (int l = 0; ok && l < cfg->n_layers; ++l) {
+    ok = cudaMemcpy(m->layers[l].attn_norm, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+         cudaMemcpy(m->layers[l].ffn_norm, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess;
+  }
+  if (!ok || !build_tensor_maps(m)) {
+    cudaStreamDestroy(m->cap_stream);
+    delete m;
+    return CASSPEC_E_CUDA;
+  }
+  *out = m;
+  return CASSPEC_OK;
+}
+
+void casspec_destroy_model(casspec_model* m) {
+  if (m == nullptr) return;
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
+  delete m;
+}
+
+int casspec_set_stream(casspec_model* m, void* stream) {
+  if (m == nullptr) return CASSPEC_E_INVAL;
+  m->stream = static_cast<cudaStream_t>(stream);
+  return CASSPEC_OK;
+}
+
+int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
+  if (m == nullptr || (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS)) != 0) return CASSPEC_E_INVAL;
+  if (old_flags) *old_flags = m->flags;
+  if (flags != m->flags) {
+    for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+    m->graphs.clear();
+  }
+  m->flags = flags;
+  return CASSPEC_OK;
+}
+
+int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size_t* bytes) {
+  if (m == nullptr || dev_ptr == nullptr) return CASSPEC_E_INVAL;
+  const auto& c = m->cfg;
+  const size_t d = c.d_model, F = c.ffn, V = c.vocab;
+  const bool per_layer = tensor >= CASSPEC_T_ATTN_NORM;
+  if (per_layer && (layer < 0 || layer >= c.n_layers)) return CASSPEC_E_INVAL;
+  if (tensor >= CASSPEC_T_WQKV_Q && !c.with_int8) return CASSPEC_E_INVAL;
+  void* p = nullptr;
+  size_t nb = 0;
+  const LayerPtrs* L = per_layer ? &m->layers[layer] : nullptr;
+  switch (tensor) {
+    case CASSPEC_T_EMBED: p = m->embed; nb = V * d * 2; break;
+    case CASSPEC_T_LM_HEAD: p = m->lm_head; nb = V * d * 2; break;
+    case CASSPEC_T_FINAL_NORM: p = m->final_norm; nb = d * 4; break;
+    case CASSPEC_T_ATTN_NORM: p = L->attn_norm; nb = d * 4; break;
+    case CASSPEC_T_FFN_NORM: p = L->ffn_norm; nb = d * 4; break;
+    case CASSPEC_T_WQKV: p = L->wqkv; nb = 3 * d * d * 2; break;
+    case CASSPEC_T_WO: p = L->wo; nb = d * d * 2; break;
+    case CASSPEC_T_WG: p = L->wg; nb = F * d * 2; break;
+    case CASSPEC_T_WU: p = L->wu; nb = F * d * 2; break;
+    case CASSPEC_T_WD: p = L->wd; nb = d * F * 2; break;
+    case CASSPEC_T_WQKV_Q: p = L->qkv_q; nb = 3 * d * d; break;
+    case CASSPEC_T_WO_Q: p = L->wo_q; nb = d * d; break;
+    case CASSPEC_T_WG_Q: p = L->wg_q; nb = F * d; break;
+    case CASSPEC_T_WU_Q: p = L->wu_q; nb = F * d; break;
+    case CASSPEC_T_WD_Q: p = L->wd_q; nb = d * F; break;
+    case CASSPEC_T_WQKV_S: p = L->qkv_s; nb = 3 * d * 4; break;
+    case CASSPEC_T_WO_S: p = L->wo_s; nb = d * 4; break;
+    case CASSPEC_T_WG_S: p = L->wg_s; nb = F * 4; break;
+    case CASSPEC_T_WU_S: p = L->wu_s; nb = F * 4; break;
+    case CASSPEC_T_WD_S: p = L->wd_s; nb = d * 4; break;
+    default: return CASSPEC_E_INVAL;
+  }
+  *dev_ptr = p;
+  if (bytes) *bytes = nb;
+  return CASSPEC_OK;
+}
+
+int casspec_quantize_weights(casspec_model* m) {
+  if (m == nullptr || !m->cfg.with_int8) return CASSPEC_E_INVAL;
+  const auto& c = m->cfg;
+  const int d = c.d_model, F = c.ffn;
+  for (int l = 0; l < c.n_layers; ++l) {
+    LayerPtrs& p = m->layers[l];
+    CK(launch_quant_rows(p.wqkv, 3 * d, d, d, p.qkv_q, d, p.qkv_s, m->stream, false));
+    CK(launch_quant_rows(p.wo, d, d, d, p.wo_q, d, p.wo_s, m->stream, false));
+    CK(launch_quant_rows(p.wg, F, d, d, p.wg_q, d, p.wg_s, m->stream, false));
+    CK(launch_quant_rows(p.wu, F, d, d, p.wu_q, d, p.wu_s, m->stream, false));
+    CK(launch_quant_rows(p.wd, d, F, F, p.wd_q, F, p.wd_s, m->stream, false));
+  }
+  return CASSPEC_OK;
+}
+
+size_t casspec_kv_bytes(const casspec_model_config* cfg, int max_ctx) {
+  if (!config_ok(cfg) || max_ctx < 1) return 0;
+  return kv_region_bytes(*cfg, kv_ctx(max_ctx)) + kv_meta_bytes();
+}
+
+int casspec_kv_create(casspec_model* m, int max_ctx, void* dev_mem, size_t bytes, casspec_kv** out) {
+  if (m == nullptr || dev_mem == nullptr || out == nullptr || max_ctx < 1) return CASSPEC_E_INVAL;
+  if ((reinterpret_cast<uintptr_t>(dev_mem) & 255) != 0) return CASSPEC_E_INVAL;
+  const int ctx = kv_ctx(max_ctx);
+  const size_t region = kv_region_bytes(m->cfg, ctx);
+  if (bytes < region + kv_meta_bytes()) return CASSPEC_E_CAPACITY;
+  casspec_kv* kv = new (std::nothrow) casspec_kv();
+  if (kv == nullptr) return CASSPEC_E_CAPACITY;
+  uint8_t* b = static_cast<uint8_t*>(dev_mem);
+  kv->m = m;
+  kv->base = reinterpret_cast<uint16_t*>(b);
+  kv->ctx = ctx;
+  uint8_t* meta = b + region;
+  kv->dP = reinterpret_cast<int*>(meta);
+  kv->compact_cnt = reinterpret_cast<unsigned*>(meta + 128);
+  kv->tdepth = reinterpret_cast<int*>(meta + 256);
+  kv->tanc = reinterpret_cast<unsigned long long*>(meta + 256 + kMaxTree * 4);
+  kv->layer_valid.assign(m->cfg.n_layers, 0);
+  if (cudaMemsetAsync(b, 0, region + kv_meta_bytes(), m->stream) != cudaSuccess) {
+    delete kv;
+    return CASSPEC_E_CUDA;
+  }
+  *out = kv;
+  return CASSPEC_OK;
+}
+
+void casspec_kv_destroy(casspec_kv* kv) { delete kv; }
+
+int casspec_kv_layer(casspec_kv* kv, int layer, void** k_dev, void** v_dev, int* ld_slots) {
+  if (kv == nullptr || layer < 0 || layer >= kv->m->cfg.n_layers) return CASSPEC_E_INVAL;
+  if (k_dev) *k_dev = kv_layer_k(kv, layer);
+  if (v_dev) *v_dev = kv_layer_v(kv, layer);
+  if (ld_slots) *ld_slots = kv->ctx;
+  return CASSPEC_OK;
+}
+
+int casspec_kv_set_prefix(casspec_kv* kv, int P) {
+  if (kv == nullptr || P < 0 || P > kv->ctx) return CASSPEC_E_INVAL;
+  CK(launch_set_int(kv->dP, P, kv->m->stream));
+  kv->P_upper = P;
+  kv->T = 0;
+  std::fill(kv->layer_valid.begin(), kv->layer_valid.end(), 0);
+  return CASSPEC_OK;
+}
+
+int casspec_kv_reset_tree(casspec_kv* kv) {
+  if (kv == nullptr) return CASSPEC_E_INVAL;
+  kv->T = 0;
+  std::fill(kv->layer_valid.begin(), kv->layer_valid.end(), 0);
+  return CASSPEC_OK;
+}
+
+int casspec_kv_length(casspec_kv* kv, int* P_out, int* T_out) {
+  if (kv == nullptr) return CASSPEC_E_INVAL;
+  CK(cudaStreamSynchronize(kv->m->stream));
+  int P = 0;
+  CK(cudaMemcpy(&P, kv->dP, 4, cudaMemcpyDeviceToHost));
+  kv->P_upper = P;
+  if (P_out) *P_out = P;
+  if (T_out) *T_out = kv->T;
+  return CASSPEC_OK;
+}
+
+int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent_idx, int n,
+                      const uint8_t* skip_mask, int quant_mode, float* logits_out) {
+  if (m == nullptr || kv == nullptr || tokens == nullptr || parent_idx == nullptr || kv->m != m)
+    return CASSPEC_E_INVAL;
+  if (quant_mode != 0 && quant_mode != 1) return CASSPEC_E_INVAL;
+  if (quant_mode == 1 && !m->cfg.with_int8) return CASSPEC_E_INVAL;
+  if (n < 1 || n > kMaxTree) return CASSPEC_E_SHAPE;
+  if (kv->T + n > kMaxTree || kv->P_upper + kv->T + n > kv->ctx) return CASSPEC_E_CAPACITY;
+  const int NL = m->cfg.n_layers;
+  std::vector<uint8_t> on(NL, 1);
+  if (skip_mask)
+    for (int l = 0; l < NL; ++l) on[l] = skip_mask[l] != 0;
+  for (int l = 0; l < NL; ++l)
+    if (on[l] && kv->layer_valid[l] != kv->T) return CASSPEC_E_STATE;
+
+  std::lock_guard<std::mutex> lock(m->mu);
+  int rc = CASSPEC_OK;
+  if (m->flags & CASSPEC_OPT_GRAPHS) {
+    GraphKey key{kv, tokens, parent_idx, logits_out, n, kv->T, quant_mode, on};
+    auto it = m->graphs.find(key);
+    if (it == m->graphs.end()) {
+      if (cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+        return CASSPEC_E_CUDA;
+      rc = enqueue_step(m, kv, tokens, parent_idx, n, on, quant_mode, logits_out, m->cap_stream);
+      cudaGraph_t g = nullptr;
+      const cudaError_t ec = cudaStreamEndCapture(m->cap_stream, &g);
+      if (rc != CASSPEC_OK || ec != cudaSuccess || g == nullptr) {
+        if (g) cudaGraphDestroy(g);
+        cudaGetLastError();
+        return rc != CASSPEC_OK ? rc : CASSPEC_E_CUDA;
+      }
+      cudaGraphExec_t ex = nullptr;
+      const cudaError_t ei = cudaGraphInstantiate(&ex, g, 0);
+      cudaGraphDestroy(g);
+      if (ei != cudaSuccess) return CASSPEC_E_CUDA;
+      it = m->graphs.emplace(key, ex).first;
+    }
+    if (cudaGraphLaunch(it->second, m->stream) != cudaSuccess) return CASSPEC_E_CUDA;
+  } else {
+    rc = enqueue_step(m, kv, tokens, parent_idx, n, on, quant_mode, logits_out, m->stream);
+    if (rc != CASSPEC_OK) return rc;
+  }
+  const int Tn = kv->T + n;
+  for (int l = 0; l < NL; ++l)
+    if (on[l]) kv->layer_valid[l] = Tn;
+  kv->T = Tn;
+  return CASSPEC_OK;
+}
+
+int casspec_argmax(casspec_model* m, const int32_t** argmax_dev, const float** margin_dev) {
+  if (m == nullptr) return CASSPEC_E_INVAL;
+  if (argmax_dev) *argmax_dev = m->am;
+  if (margin_dev) *margin_dev = m->margin;
+  return CASSPEC_OK;
+}
+
+int casspec_accept_greedy(casspec_model* m, const float* logits, const int32_t* tokens, const int32_t* parent_idx,
+                          int n, int32_t* accepted_out) {
+  if (m == nullptr || tokens == nullptr || parent_idx == nullptr || accepted_out == nullptr) return CASSPEC_E_INVAL;
+  if (n < 1 || n > kMaxTree) return CASSPEC_E_SHAPE;
+  const int* am = m->am;
+  if (logits != nullptr) {
+    CK(launch_row_argmax(logits, n, m->cfg.vocab, m->am2, m->stream));
+    am = m->am2;
+  }
+  CK(launch_accept(am, tokens, parent_idx, n, accepted_out, m->status, m->stream));
+  return CASSPEC_OK;
+}
+
+int casspec_kv_compact(casspec_kv* kv, const int32_t* accepted_out) {
+  if (kv == nullptr || accepted_out == nullptr) return CASSPEC_E_INVAL;
+  if (kv->T < 1) return CASSPEC_E_STATE;
+  for (int v : kv->layer_valid)
+    if (v != kv->T) return CASSPEC_E_STATE;
+  casspec_model* m = kv->m;
+  const auto& c = m->cfg;
+  CK(launch_kv_compact(kv->base, c.n_layers, c.n_heads, kv->ctx, c.head_dim, accepted_out, kv->T, kv->dP,
+                       kv->compact_cnt, m->status, m->stream));
+  kv->P_upper += kv->T;
+  kv->T = 0;
+  std::fill(kv->layer_valid.begin(), kv->layer_valid.end(), 0);
+  return CASSPEC_OK;
+}
+
+int casspec_get_status(casspec_model* m, int* status_out) {
+  if (m == nullptr) return CASSPEC_E_INVAL;
+  CK(cudaStreamSynchronize(m->stream));
+  int st = 0;
+  CK(cudaMemcpy(&st, m->status, 4, cudaMemcpyDeviceToHost));
+  if (st != 0) {
+    // a kernel that gave up may have left fix-up counters behind: clear them all
+    CK(cudaMemset(m->status, 0, 4));
+    CK(cudaMemset(m->gemm_cnt, 0, (size_t)m->lay.max_tiles * 4));
+    CK(cudaMemset(m->i8_cnt, 0, (size_t)m->lay.max_tiles * 4));
+    CK(cudaMemset(m->attn_cnt, 0, (size_t)m->cfg.n_heads * 4));
+  }
+  if (status_out) *status_out = st;
+  return CASSPEC_OK;
+}
+
+const char* casspec_status_string(int s) {
+  switch (s) {
+    case CASSPEC_OK: return "ok";
+    case CASSPEC_E_INVAL: return "invalid argument";
+    case CASSPEC_E_SHAPE: return "unsupported size";
+    case CASSPEC_E_CAPACITY: return "capacity exceeded";
+    case CASSPEC_E_CUDA: return "CUDA error";
+    case CASSPEC_E_TREE: return "invalid tree or accepted path";
+    case CASSPEC_E_TIMEOUT: return "bounded device wait expired";
+    case CASSPEC_E_STATE: return "call-order rule violated";
+  }
+  return "unknown status";
+}
+
+size_t casspec_linear_workspace_bytes(int N, int K, int n) {
+  if (N < 1 || K < 8 || n < 1) return 0;
+  const int tiles = cdiv(N, 128);
+  return 4096 + gemm_partials_floats(tiles, kSmsBound) * 4;
+}
+
+int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int n, float* Y, int ldy, void* ws,
+                        size_t ws_bytes, void* stream) {
+  if (W == nullptr || X == nullptr || Y == nullptr || ws == nullptr) return CASSPEC_E_INVAL;
+  if (n < 1 || n > kMaxTree || N < 1 || K < 8 || K % 8 != 0 || ldy < N) return CASSPEC_E_SHAPE;
+  if (((uintptr_t)W & 15) || ((uintptr_t)X & 15) || ((uintptr_t)ws & 15)) return CASSPEC_E_INVAL;
+  const int tiles = cdiv(N, 128);
+  if (tiles > 1024) return CASSPEC_E_SHAPE;
+  if (ws_bytes < casspec_linear_workspace_bytes(N, K, n)) return CASSPEC_E_CAPACITY;
+  const int sms = num_sms_of_current_device();
+  if (sms <= 0) return CASSPEC_E_CUDA;
+  const int BN = roundup16(n);
+  CUtensorMap tw, tx;
+  if (!encode_tmap_bf16(&tw, W, K, N, (uint64_t)K * 2, 64, 128) ||
+      !encode_tmap_bf16(&tx, X, K, n, (uint64_t)K * 2, 64, BN))
+    return CASSPEC_E_CUDA;
+  const int kb = cdiv(K, 64);
+  GemmArgs a = {};
+  a.tiles = tiles;
+  a.kblocks = kb;
+  a.counters = static_cast<unsigned*>(ws);
+  a.partials = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + 4096);
+  a.status = nullptr;
+  a.ep.n = n;
+  a.ep.N = N;
+  a.ep.y = Y;
+  a.ep.ldy = ldy;
+  CK(launch_gemm_bf16(tw, tw, tx, BN, EPI_STORE, a, gemm_bf16_grid(tiles, kb, sms), static_cast<cudaStream_t>(stream),
+                      false));
+  return CASSPEC_OK;
+}
+
+int casspec_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* s,
+                    void* stream) {
+  if (x == nullptr || g == nullptr || (y == nullptr && q == nullptr) || ((q == nullptr) != (s == nullptr)))
+    return CASSPEC_E_INVAL;
+  if (n < 1 || d < 1) return CASSPEC_E_SHAPE;
+  CK(launch_rmsnorm(x, g, n, d, eps, y, q, s, static_cast<cudaStream_t>(stream), false));
+  return CASSPEC_OK;
+}
+
+int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q, float* s, void* stream) {
+  if (x == nullptr || q == nullptr || s == nullptr) return CASSPEC_E_INVAL;
+  if (n < 1 || d < 1) return CASSPEC_E_SHAPE;
+  CK(launch_quant_rows(x, n, d, d, q, d, s, static_cast<cudaStream_t>(stream), false));
+  return CASSPEC_OK;
+}
+
+}  // extern "C"

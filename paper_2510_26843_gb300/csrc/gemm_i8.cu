@@ -1,0 +1,199 @@
+// W8A8 projection for the activation-quantisation draft (App. C; W8A8 reading of QSpec-style DSIA).
+//
+// y[i][o] = (sum_k qx[i][k] * qw[o][k]) * sx[i] * sw[o], with the integer sum exact in int32
+// (|sum| <= K * 127^2 < 2^31 for K < 133,000).  tcgen05.mma has no integer kind on sm_103a, so the
+// contraction uses the warp-level mma.sync.m16n8k32 s8 x s8 -> s32 path; at draft batch sizes the
+// projection is bound by streaming the int8 weights, half the bytes of the bf16 weights.
+//   * one CTA = 8 warps = one 128-row output tile (warp w: rows 16w..16w+15) x a k-range; `ksplit`
+//     CTAs share a tile along K so every SM keeps several weight streams in flight;
+//   * weights go straight from HBM into mma fragments with 16-byte loads (no shared memory), the
+//     next 128-column block prefetched in registers.  Both operands use the same permutation of
+//     the 128 columns of a block inside the fragments, which leaves the dot product unchanged:
+//     thread (group g, lane t) loads bytes [16t, 16t+16) and [64+16t, 64+16t+16) of its rows;
+//   * the CTA that finishes a tile last (atomic counter) sums the int32 partials, dequantises
+//     once, and runs the same fused epilogue as the bf16 projection.
+#include "common.cuh"
+#include "epilogue.cuh"
+#include "kernels.h"
+
+namespace casspec {
+
+constexpr int kI8Threads = 256;
+
+__device__ __forceinline__ uint4 ldg_nc16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a) {
+  extern __shared__ float stg[];  // [128][BN + 1]
+  __shared__ int s_last;
+  const int tile = blockIdx.x, ks = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
+  pdl_trigger();
+
+  const int KB = (a.K + 127) / 128;
+  const int kb0 = (int)((long long)ks * KB / a.ksplit), kb1 = (int)((long long)(ks + 1) * KB / a.ksplit);
+  const int n = a.ep.n;
+
+  // weight rows of this thread's fragments: tile rows lr and lr + 8
+  const int8_t* wrow[2];
+  bool wok[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int lr = warp * 16 + g + 8 * h;
+    if (EPI == EPI_GLU) {
+      const int ch = tile * 64 + (lr & 63);
+      wok[h] = ch < a.N;
+      wrow[h] = (lr < 64 ? a.W : a.W2) + (size_t)(wok[h] ? ch : 0) * a.K;
+    } else {
+      const int o = tile * 128 + lr;
+      wok[h] = o < a.N;
+      wrow[h] = a.W + (size_t)(wok[h] ? o : 0) * a.K;
+    }
+  }
+  auto load_a = [&](int kb, uint4* A) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int col = kb * 128 + c * 64 + 16 * t4;
+        A[2 * h + c] = (wok[h] && col < a.K) ? ldg_nc16(wrow[h] + col) : make_uint4(0, 0, 0, 0);
+      }
+    }
+  };
+
+  int acc[BN / 8][4];
+#pragma unroll
+  for (int j = 0; j < BN / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0;
+
+  uint4 A[4], An[4];
+  if (kb0 < kb1) load_a(kb0, A);  // weights do not depend on the previous kernel
+  pdl_wait();
+  for (int kb = kb0; kb < kb1; ++kb) {
+    if (kb + 1 < kb1) load_a(kb + 1, An);
+#pragma unroll
+    for (int j = 0; j < BN / 8; ++j) {
+      const int tok = 8 * j + g;
+      uint4 B[2];
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int col = kb * 128 + c * 64 + 16 * t4;
+        B[c] = (tok < n && col < a.K) ? *reinterpret_cast<const uint4*>(a.X + (size_t)tok * a.K + col)
+                                      : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int s = 0; s < 4; ++s) {
+        const uint4 lo = A[s >> 1], hi = A[2 + (s >> 1)], b = B[s >> 1];
+        const bool odd = s & 1;
+        mma_s8_16832(acc[j], odd ? lo.z : lo.x, odd ? hi.z : hi.x, odd ? lo.w : lo.y, odd ? hi.w : hi.y,
+                     odd ? b.z : b.x, odd ? b.w : b.y);
+      }
+    }
+    if (kb + 1 < kb1) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) A[q] = An[q];
+    }
+  }
+
+  auto scale_w = [&](int row) -> float {
+    if (EPI == EPI_GLU) {
+      const int ch = tile * 64 + (row & 63);
+      if (ch >= a.N) return 0.f;
+      return row < 64 ? a.sw[ch] : a.sw2[ch];
+    }
+    const int o = tile * 128 + row;
+    return o < a.N ? a.sw[o] : 0.f;
+  };
+
+  if (a.ksplit > 1) {
+    int* part = a.partials + ((size_t)tile * a.ksplit + ks) * (64 * 128);
+#pragma unroll
+    for (int j = 0; j < BN / 8; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int tok = 8 * j + 2 * t4 + (e & 1), row = warp * 16 + g + 8 * (e >> 1);
+        if (tok < n) __stcg(part + tok * 128 + row, acc[j][e]);
+      }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) s_last = (atomicAdd(&a.counters[tile], 1u) == (unsigned)(a.ksplit - 1)) ? 1 : 0;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    for (int idx = tid; idx < n * 128; idx += kI8Threads) {
+      const int tok = idx >> 7, row = idx & 127;
+      int sum = 0;
+      for (int k = 0; k < a.ksplit; ++k)
+        sum += __ldcg(a.partials + ((size_t)tile * a.ksplit + k) * (64 * 128) + tok * 128 + row);
+      stg[row * (BN + 1) + tok] = (float)sum * a.sx[tok] * scale_w(row);
+    }
+    if (tid == 0) a.counters[tile] = 0u;
+  } else {
+#pragma unroll
+    for (int j = 0; j < BN / 8; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int tok = 8 * j + 2 * t4 + (e & 1), row = warp * 16 + g + 8 * (e >> 1);
+        if (tok < n) stg[row * (BN + 1) + tok] = (float)acc[j][e] * a.sx[tok] * scale_w(row);
+      }
+  }
+  __syncthreads();
+  float v[BN];
+  if (tid < 128) {
+#pragma unroll
+    for (int i = 0; i < BN; ++i) v[i] = stg[tid * (BN + 1) + i];
+  }
+  __syncthreads();
+  if (tid < 128) run_epilogue<BN, EPI>(a.ep, tile, tid, v, stg, [] { named_bar_sync(1, 128); });
+}
+
+int gemm_i8_ksplit(int tiles, int K, int num_sms) {
+  const int KB = (K + 127) / 128;
+  int ks = (6 * num_sms + tiles - 1) / tiles;
+  if (ks > KB / 2) ks = KB / 2;
+  if (ks < 1) ks = 1;
+  return ks;
+}
+
+template <int BN, int EPI>
+static cudaError_t launch_t(const GemmI8Args& a, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.tiles, a.ksplit);
+  cfg.blockDim = dim3(kI8Threads);
+  cfg.dynamicSmemBytes = (size_t)128 * (BN + 1) * 4;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_i8_kernel<BN, EPI>, a);
+}
+
+template <int BN>
+static cudaError_t launch_bn(const GemmI8Args& a, int epi, cudaStream_t s, bool pdl) {
+  switch (epi) {
+    case EPI_STORE: return launch_t<BN, EPI_STORE>(a, s, pdl);
+    case EPI_RESID: return launch_t<BN, EPI_RESID>(a, s, pdl);
+    case EPI_QKV: return launch_t<BN, EPI_QKV>(a, s, pdl);
+    case EPI_GLU: return launch_t<BN, EPI_GLU>(a, s, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm_i8(const GemmI8Args& a, int BN, int epi, cudaStream_t stream, bool pdl) {
+  switch (BN) {
+    case 16: return launch_bn<16>(a, epi, stream, pdl);
+    case 32: return launch_bn<32>(a, epi, stream, pdl);
+    case 48: return launch_bn<48>(a, epi, stream, pdl);
+    case 64: return launch_bn<64>(a, epi, stream, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace casspec

@@ -1,0 +1,113 @@
+// Internal interface between the host runtime (api.cu) and the kernel translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace casspec {
+
+// Epilogue applied to a finished 128-row x n tile of a projection (output rows = channels).
+enum Epi : int {
+  EPI_STORE = 0,   // y[i][o] = v                              (stateless linear)
+  EPI_RESID = 1,   // y[i][o] += v                             (Wo, Wd: residual add in fp32)
+  EPI_QKV = 2,     // rotary on q,k at tree positions; q -> q_out, k,v -> cache slots P+T+i
+  EPI_GLU = 3,     // tile = 64 gate rows + 64 up rows: u_out[i][c] = silu(g) * up
+  EPI_LMHEAD = 4,  // logits[i][o] = v (optional) + per-tile (max, argmax, 2nd max) per token
+};
+
+struct EpiParams {
+  int n;        // valid tokens (columns)
+  int N;        // output channels of the projection (for EPI_GLU: F)
+  float* y;     // EPI_STORE / EPI_RESID: [n][ldy] fp32
+  int ldy;
+  // EPI_QKV
+  uint16_t* q_out;      // [64][d] bf16
+  uint16_t* kc;         // this layer's K cache [H][ctx][hd]
+  uint16_t* vc;         // this layer's V cache
+  int ctx, d, hd, T;
+  const int* dP;        // device committed length P
+  const float2* rope;   // [n][hd/2] (cos, sin) of pos(i) * base^(-2j/hd)
+  // EPI_GLU
+  uint16_t* u_out;      // [64][F] bf16
+  // EPI_LMHEAD
+  float* logits;        // [n][V] fp32 or null
+  float* am_v1;         // [tiles][64] partial max
+  int* am_i1;           // [tiles][64] partial argmax (vocab id)
+  float* am_v2;         // [tiles][64] partial second max
+};
+
+struct GemmArgs {
+  int tiles;     // 128-row output tiles
+  int kblocks;   // ceil(K / 64)
+  float* partials;     // stream-K partial tiles, (tiles + grid) slots of 64 x 128 fp32
+  unsigned* counters;  // [tiles], zero between launches
+  int* status;
+  EpiParams ep;
+};
+
+// int8 (W8A8) projection arguments
+struct GemmI8Args {
+  const int8_t* W;   // [N][K]
+  const float* sw;   // [N]
+  const int8_t* W2;  // EPI_GLU: up weights (gate in W)
+  const float* sw2;
+  const int8_t* X;   // [64][K] quantised activations
+  const float* sx;   // [64]
+  int N, K, ksplit;  // ksplit CTAs share one 128-row tile along K
+  int tiles;
+  int* partials;     // [tiles][ksplit][64][128] int32
+  unsigned* counters;
+  int* status;
+  EpiParams ep;
+};
+
+struct AttnArgs {
+  const uint16_t* q;    // [64][d] bf16 (rotated)
+  const uint16_t* kc;   // [H][ctx][hd]
+  const uint16_t* vc;
+  uint16_t* o;          // [64][d] bf16
+  const unsigned long long* anc;  // [n] ancestor masks over tree slots
+  const int* dP;
+  int T, n, ctx, d, splits;
+  float scale_log2;     // log2(e) / sqrt(hd)
+  float* part_o;        // [H][splits][64][hd]
+  float* part_ml;       // [H][splits][64][2]
+  unsigned* counters;   // [H]
+  int* status;
+};
+
+// ---- launchers (return cudaSuccess or the launch error) ----
+bool encode_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows, uint64_t row_stride_bytes,
+                      uint32_t box_inner, uint32_t box_rows);
+int gemm_bf16_grid(int tiles, int kblocks, int num_sms);
+size_t gemm_partials_floats(int tiles, int grid);
+cudaError_t launch_gemm_bf16(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int BN, int epi,
+                             const GemmArgs& args, int grid, cudaStream_t stream, bool pdl);
+
+int gemm_i8_ksplit(int tiles, int K, int num_sms);
+cudaError_t launch_gemm_i8(const GemmI8Args& args, int BN, int epi, cudaStream_t stream, bool pdl);
+
+int attn_splits(int n_heads, int total_slots, int num_sms);
+cudaError_t launch_tree_attention(const AttnArgs& a, int hd, int n_heads, cudaStream_t stream, bool pdl);
+
+cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
+                             int* pos, unsigned long long* anc_new, float2* rope, const double* inv_freq, int half,
+                             int* status, cudaStream_t s, bool pdl);
+cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, cudaStream_t s,
+                         bool pdl);
+cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
+                           cudaStream_t s, bool pdl);
+cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
+                              bool pdl);
+cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,
+                                 float* margin, cudaStream_t s, bool pdl);
+cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s);
+cudaError_t launch_accept(const int* am, const int* tokens, const int* parent, int n, int* acc, int* status,
+                          cudaStream_t s);
+cudaError_t launch_kv_compact(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* acc, int T,
+                              int* dP, unsigned* counter, int* status, cudaStream_t s);
+cudaError_t launch_set_int(int* p, int v, cudaStream_t s);
+
+}  // namespace casspec

@@ -1,0 +1,406 @@
+// The small kernels of the tree step: tree preparation, embedding gather, RMSNorm (+ per-token
+// int8 quantisation), LM-head argmax reduction, greedy acceptance and KV compaction.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace casspec {
+
+static cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl,
+                                   cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cfg;
+}
+
+// ---------------------------------------------------------------------------------------------
+// Tree preparation (Alg. 1 tree T_r; Sec. 4.2 tree attention).  New node i occupies tree slot
+// T + i; its depth is 0 for parent -1 (child of the last committed token) else depth(parent) + 1;
+// its position is P + depth; its ancestor mask is anc(parent) | bit(T + i).  Also fills the
+// rotary table (cos, sin)(pos(i) * inv_freq[j]) in fp64 -> fp32 for the QKV epilogue.
+// ---------------------------------------------------------------------------------------------
+__global__ void tree_prep_kernel(const int* __restrict__ parent, int n, int T, const int* dP, int* tdepth,
+                                 unsigned long long* tanc, int* pos, unsigned long long* anc_new, float2* rope,
+                                 const double* inv_freq, int half, int* status) {
+  __shared__ int s_depth[kMaxTree];
+  __shared__ unsigned long long s_anc[kMaxTree];
+  __shared__ int s_pos[kMaxTree];
+  pdl_trigger();
+  pdl_wait();
+  const int P = *dP;
+  if (threadIdx.x < T) {
+    s_depth[threadIdx.x] = tdepth[threadIdx.x];
+    s_anc[threadIdx.x] = tanc[threadIdx.x];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    bool bad = false;
+    for (int i = 0; i < n; ++i) {
+      const int j = T + i;
+      const int p = parent[i];
+      int dep;
+      unsigned long long an;
+      if (p == -1) {
+        dep = 0;
+        an = 1ull << j;
+      } else if (p >= 0 && p < j) {
+        dep = s_depth[p] + 1;
+        an = s_anc[p] | (1ull << j);
+      } else {
+        bad = true;  // reported; the node is treated as a depth-0 node so the step stays well defined
+        dep = 0;
+        an = 1ull << j;
+      }
+      s_depth[j] = dep;
+      s_anc[j] = an;
+      s_pos[i] = P + dep;
+    }
+    if (bad) set_status(status, CASSPEC_E_TREE);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+    tdepth[T + i] = s_depth[T + i];
+    tanc[T + i] = s_anc[T + i];
+    pos[i] = s_pos[i];
+    anc_new[i] = s_anc[T + i];
+  }
+  for (int idx = threadIdx.x; idx < n * half; idx += blockDim.x) {
+    const int i = idx / half, j = idx % half;
+    double sn, cs;
+    sincos((double)s_pos[i] * inv_freq[j], &sn, &cs);
+    rope[idx] = make_float2((float)cs, (float)sn);
+  }
+}
+
+cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
+                             int* pos, unsigned long long* anc_new, float2* rope, const double* inv_freq, int half,
+                             int* status, cudaStream_t s, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(256), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, tree_prep_kernel, parent, n, T, dP, tdepth, tanc, pos, anc_new, rope, inv_freq,
+                            half, status);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Embedding gather: x[i][:] = E[tokens[i]][:] widened to the fp32 residual stream.
+// ---------------------------------------------------------------------------------------------
+__global__ void embed_kernel(const uint16_t* __restrict__ E, const int* __restrict__ tokens, int d, int vocab,
+                             float* __restrict__ x) {
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x;
+  int tok = tokens[i];
+  tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);
+  const uint16_t* row = E + (size_t)tok * d;
+  for (int c = threadIdx.x * 2; c < d; c += blockDim.x * 2) {
+    const uint32_t two = *reinterpret_cast<const uint32_t*>(row + c);
+    *reinterpret_cast<float2*>(x + (size_t)i * d + c) = make_float2(bf2f(two & 0xFFFF), bf2f(two >> 16));
+  }
+}
+
+cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, cudaStream_t s,
+                         bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, embed_kernel, E, tokens, d, vocab, x);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Block reductions (256 threads)
+// ---------------------------------------------------------------------------------------------
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int k = 0; k < (int)(blockDim.x >> 5); ++k) t += red[k];  // fixed order: deterministic
+  return t;
+}
+__device__ __forceinline__ float block_max(float v, float* red) {
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = red[0];
+  for (int k = 1; k < (int)(blockDim.x >> 5); ++k) t = fmaxf(t, red[k]);
+  return t;
+}
+
+// Per-row symmetric int8 quantisation rule (App. C activation-quantisation DSIA, W8A8 reading):
+// inv = 127 / amax (IEEE division), q = rint(x * inv) (IEEE multiply, ties to even), clamp +-127,
+// scale = amax / 127; amax = 0 gives q = 0, scale 0.
+__device__ __forceinline__ int8_t quant_one(float x, float inv) {
+  int q = __float2int_rn(__fmul_rn(x, inv));
+  q = q > 127 ? 127 : (q < -127 ? -127 : q);
+  return (int8_t)q;
+}
+
+// ---------------------------------------------------------------------------------------------
+// RMSNorm (pre-norm): y = bf16(x * rsqrt(mean(x^2) + eps) * g), fp32 arithmetic; optionally the
+// per-token int8 quantisation of the bf16 row.
+// ---------------------------------------------------------------------------------------------
+__global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g, int d, float eps,
+                               uint16_t* __restrict__ y, int8_t* __restrict__ q, float* __restrict__ sq) {
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x;
+  const float* xr = x + (size_t)i * d;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += xr[c] * xr[c];
+  ss = block_sum(ss, red);
+  const float r = rsqrtf(ss / (float)d + eps);
+  float amax = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const uint16_t b = f2bf(xr[c] * r * g[c]);
+    if (y) y[(size_t)i * d + c] = b;
+    amax = fmaxf(amax, fabsf(bf2f(b)));
+  }
+  if (q == nullptr) return;
+  amax = block_max(amax, red);
+  const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const float v = bf2f(f2bf(xr[c] * r * g[c]));
+    q[(size_t)i * d + c] = amax > 0.f ? quant_one(v, inv) : (int8_t)0;
+  }
+  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
+}
+
+cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
+                           cudaStream_t s, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, x, g, d, eps, y, q, sq);
+}
+
+__global__ void quant_rows_kernel(const uint16_t* __restrict__ x, int d, int ldx, int8_t* __restrict__ q, int ldq,
+                                  float* __restrict__ sq) {
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x;
+  const uint16_t* xr = x + (size_t)i * ldx;
+  float amax = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) amax = fmaxf(amax, fabsf(bf2f(xr[c])));
+  amax = block_max(amax, red);
+  const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x)
+    q[(size_t)i * ldq + c] = amax > 0.f ? quant_one(bf2f(xr[c]), inv) : (int8_t)0;
+  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
+}
+
+cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
+                              bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Argmax over the vocabulary: (max, lowest index of the max, second max) partials per LM-head
+// tile are merged; the merge is a total order (ties -> lower id), so lane order does not matter.
+// ---------------------------------------------------------------------------------------------
+struct Top2 {
+  float v1;
+  int i1;
+  float v2;
+};
+__device__ __forceinline__ Top2 merge_top2(Top2 a, Top2 b) {
+  Top2 r;
+  const bool b_wins = (b.v1 > a.v1) || (b.v1 == a.v1 && b.i1 < a.i1);
+  r.v1 = b_wins ? b.v1 : a.v1;
+  r.i1 = b_wins ? b.i1 : a.i1;
+  r.v2 = fmaxf(fmaxf(a.v2, b.v2), fminf(a.v1, b.v1));
+  return r;
+}
+
+__global__ void argmax_reduce_kernel(const float* __restrict__ v1, const int* __restrict__ i1,
+                                     const float* __restrict__ v2, int tiles, int* am, float* margin) {
+  pdl_trigger();
+  pdl_wait();
+  const int row = blockIdx.x, lane = threadIdx.x;
+  Top2 acc = {-INFINITY, 0x7fffffff, -INFINITY};
+  for (int t = lane; t < tiles; t += 32) acc = merge_top2(acc, Top2{v1[t * 64 + row], i1[t * 64 + row], v2[t * 64 + row]});
+  for (int o = 16; o > 0; o >>= 1) {
+    Top2 other{__shfl_xor_sync(0xffffffffu, acc.v1, o), __shfl_xor_sync(0xffffffffu, acc.i1, o),
+               __shfl_xor_sync(0xffffffffu, acc.v2, o)};
+    acc = merge_top2(acc, other);
+  }
+  if (lane == 0) {
+    am[row] = acc.i1;
+    margin[row] = acc.v1 - acc.v2;
+  }
+}
+
+cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,
+                                 float* margin, cudaStream_t s, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(32), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, argmax_reduce_kernel, v1, i1, v2, tiles, am, margin);
+}
+
+__global__ void row_argmax_kernel(const float* __restrict__ logits, int V, int* am) {
+  __shared__ float sv[8];
+  __shared__ int si[8];
+  const int row = blockIdx.x;
+  const float* lr = logits + (size_t)row * V;
+  float best = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int c = threadIdx.x; c < V; c += blockDim.x) {
+    const float x = lr[c];
+    if (x > best || (x == best && c < bi)) {
+      best = x;
+      bi = c;
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ov > best || (ov == best && oi < bi)) {
+      best = ov;
+      bi = oi;
+    }
+  }
+  if ((threadIdx.x & 31) == 0) {
+    sv[threadIdx.x >> 5] = best;
+    si[threadIdx.x >> 5] = bi;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
+      if (sv[w] > best || (sv[w] == best && si[w] < bi)) {
+        best = sv[w];
+        bi = si[w];
+      }
+    am[row] = bi;
+  }
+}
+
+cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s) {
+  row_argmax_kernel<<<n, 256, 0, s>>>(logits, V, am);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------------------------
+// Greedy acceptance (Sec. 5.1 lossless verification): a node matches when its parent matches and
+// its token equals the parent's argmax; the deepest match (lowest index among equals) is accepted
+// with its root path; the bonus token is the argmax there.
+// ---------------------------------------------------------------------------------------------
+__global__ void accept_kernel(const int* __restrict__ am, const int* __restrict__ tokens,
+                              const int* __restrict__ parent, int n, int* acc, int* status) {
+  __shared__ int s_par[kMaxTree], s_tok[kMaxTree], s_am[kMaxTree], s_depth[kMaxTree], s_match[kMaxTree];
+  const int tid = threadIdx.x;
+  if (tid < n) {
+    s_par[tid] = parent[tid];
+    s_tok[tid] = tokens[tid];
+    s_am[tid] = am[tid];
+  }
+  __syncthreads();
+  if (tid != 0) return;
+  bool ok = s_par[0] == -1;
+  for (int c = 1; c < n && ok; ++c) ok = s_par[c] >= 0 && s_par[c] < c;
+  if (!ok) {
+    set_status(status, CASSPEC_E_TREE);
+    acc[0] = 0;
+    return;
+  }
+  s_depth[0] = 0;
+  s_match[0] = 1;
+  int best = 0;
+  for (int c = 1; c < n; ++c) {
+    const int p = s_par[c];
+    s_depth[c] = s_depth[p] + 1;
+    s_match[c] = s_match[p] && (s_tok[c] == s_am[p]);
+    if (s_match[c] && s_depth[c] > s_depth[best]) best = c;
+  }
+  const int L = s_depth[best] + 1;
+  int node = best;
+  for (int k = L; k >= 1; --k) {
+    acc[k] = node;
+    node = s_par[node];
+  }
+  acc[0] = L;
+  acc[L + 1] = s_am[best];
+}
+
+cudaError_t launch_accept(const int* am, const int* tokens, const int* parent, int n, int* acc, int* status,
+                          cudaStream_t s) {
+  accept_kernel<<<1, 64, 0, s>>>(am, tokens, parent, n, acc, status);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------------------------
+// KV compaction: K/V of accepted tree slot path[k] -> committed slot P + k in every layer.  One
+// thread owns one 16-byte chunk of one (layer, K|V, head) row and walks k upwards; since
+// path[k] >= k, a source slot is never overwritten before it is read.  The CTA that finishes last
+// advances P (all CTAs read P before any of them can finish).
+// ---------------------------------------------------------------------------------------------
+__global__ void kv_compact_kernel(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* __restrict__ acc,
+                                  int T, int* dP, unsigned* counter, int* status) {
+  __shared__ int s_path[kMaxTree];
+  __shared__ int s_ok, s_last;
+  const int P = *dP;
+  if (threadIdx.x == 0) {
+    const int L = acc[0];
+    bool ok = L >= 1 && L <= T;
+    for (int k = 0; ok && k < L; ++k) {
+      const int j = acc[1 + k];
+      ok = j >= 0 && j < T && (k == 0 ? j == 0 : j > s_path[k - 1]);
+      s_path[k] = j;
+    }
+    s_ok = ok ? L : 0;
+    if (!ok && blockIdx.x == 0) set_status(status, CASSPEC_E_TREE);
+  }
+  __syncthreads();
+  const int L = s_ok;
+  const int chunks = hd / 8;
+  const long long items = (long long)n_layers * 2 * n_heads * chunks;
+  for (long long it = (long long)blockIdx.x * blockDim.x + threadIdx.x; L > 0 && it < items;
+       it += (long long)gridDim.x * blockDim.x) {
+    const int c = (int)(it % chunks);
+    const long long row = it / chunks;  // (layer, kv, head) rows of [ctx][hd]
+    uint16_t* base = kv + (size_t)row * ctx * hd + c * 8;
+    for (int k = 0; k < L; ++k) {
+      const int src = P + s_path[k], dst = P + k;
+      if (src != dst)
+        *reinterpret_cast<uint4*>(base + (size_t)dst * hd) = *reinterpret_cast<const uint4*>(base + (size_t)src * hd);
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned old = atomicAdd(counter, 1u);
+    s_last = (old == gridDim.x - 1) ? 1 : 0;
+  }
+  __syncthreads();
+  if (s_last && threadIdx.x == 0) {
+    if (L > 0) *dP = P + L;
+    *counter = 0u;
+  }
+}
+
+cudaError_t launch_kv_compact(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* acc, int T, int* dP,
+                              unsigned* counter, int* status, cudaStream_t s) {
+  const long long items = (long long)n_layers * 2 * n_heads * (hd / 8);
+  long long blocks = (items + 255) / 256;
+  if (blocks > 1024) blocks = 1024;
+  kv_compact_kernel<<<(int)blocks, 256, 0, s>>>(kv, n_layers, n_heads, ctx, hd, acc, T, dP, counter, status);
+  return cudaGetLastError();
+}
+
+__global__ void set_int_kernel(int* p, int v) { *p = v; }
+cudaError_t launch_set_int(int* p, int v, cudaStream_t s) {
+  set_int_kernel<<<1, 1, 0, s>>>(p, v);
+  return cudaGetLastError();
+}
+
+}  // namespace casspec
