@@ -1,0 +1,434 @@
+"""Benchmark of the CAS-Spec tree-verify step on GB300.
+
+Workload (one "step"): the 32-layer Llama-7B-shaped model (d=4096, 32 heads x 128, SwiGLU 11008,
+vocab 32000, bf16 weights N(0, 0.02) from the seeded generator), prefix of 2048 committed slots
+(N(0, 1) bf16 stand-in K/V), a 64-node seeded token tree (depth <= 8): tree verify pass (all layers,
+LM head, fused argmax) -> greedy acceptance -> KV compaction -> rollback of the prefix to 2048 so
+every step sees the same workload.  Weights (13.2 GB) and KV (1.1 GB) exceed the 129 MB L2 many
+times over, so no L2 flush is needed between steps.
+
+Output: one JSON line (rank 0).  value = device-timed step latency in microseconds (lower is
+better); e2e = the same through the C ABI with host-resident inputs copied in and the accepted
+path copied out every step; roofline = the dominant kernel (gate/up projection) from a separate
+kernel-timing pass with CUDA events around each launch; cpu_baseline = the fp64 oracle on a
+bounded sample (embedding + 1 of 32 layers + LM head, scaled to 32 layers) on the host cores.
+
+`--impl reference` times the CPU oracle alone (the reference arm) on the same metric.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "7B tree-verify step latency (µs, n=64) and % of 8 TB/s HBM roofline"
+SEED = 20251026
+FALLBACK_HBM_GBS = 6800.0
+
+# name -> (layers kept of the 7B shape, prefix P, tree nodes n, max depth, max branching, fraction of
+#          layers skipped, quant mode, verify (accept + compact) or draft (tree reset))
+WORKLOADS = {
+    "verify7b": (32, 2048, 64, 8, None, 0.0, 0, True),
+    "layer7b": (1, 1024, 32, 6, 4, 0.0, 0, True),
+}
+for _n in (1, 2, 4, 8):
+    WORKLOADS[f"draft7b-skip50-n{_n}"] = (32, 2048, _n, 8, None, 0.5, 0, False)
+    WORKLOADS[f"draft7b-int8-n{_n}"] = (32, 2048, _n, 8, None, 0.0, 1, False)
+    WORKLOADS[f"draft7b-skip50-int8-n{_n}"] = (32, 2048, _n, 8, None, 0.5, 1, False)
+
+
+def _shape(layers: int = 32):
+    import synth
+
+    s = synth.LLAMA7B
+    return synth.ModelShape(layers, s.d_model, s.n_heads, s.head_dim, s.ffn, s.vocab)
+
+
+def algorithmic_bytes(shape, n: int, P: int, layers_on: int | None = None, quant: int = 0) -> dict:
+    """Bytes the step must move: every active weight once (int8 + fp32 row scales in W8A8 mode), the
+    prefix K/V of active layers, the tree K/V written once, fp32 logits written once (activations
+    are < 0.1% and left out)."""
+    L = shape.n_layers if layers_on is None else layers_on
+    d, F, V = shape.d_model, shape.ffn, shape.vocab
+    w = L * (4 * d * d + 3 * d * F) * (1 if quant else 2) + (L * (5 * d + 2 * F) * 4 if quant else 0)
+    lm = V * d * 2
+    kv_read = L * 2 * P * d * 2
+    kv_write = L * 2 * n * d * 2
+    logits = n * V * 4
+    return {"weights": w, "lm_head": lm, "kv_read": kv_read, "kv_write": kv_write, "logits": logits,
+            "total": w + lm + kv_read + kv_write + logits}
+
+
+def gateup_bytes(shape, n: int, quant: int = 0) -> int:
+    """Wg, Wu read (+ row scales) + activations read + U written (bf16)."""
+    d, F = shape.d_model, shape.ffn
+    if quant:
+        return 2 * F * d + 2 * F * 4 + n * d + n * F * 2
+    return 2 * F * d * 2 + n * d * 2 + n * F * 2
+
+
+def measured_peaks() -> tuple[float, str]:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def recorded_traffic() -> float | None:
+    """DRAM bytes per launch of the gate/up projection from the committed ncu summary, if it was taken
+    on the current kernel source (the summary records the source hash)."""
+    path = os.path.join(ROOT, "profiles", "gemm_bf16_gateup_7b_n64.md")
+    src = os.path.join(ROOT, "paper_2510_26843_gb300", "csrc", "gemm_tc.cu")
+    try:
+        text = open(path).read()
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        m_hash = re.search(r"source_sha256_16:\s*([0-9a-f]+)", text)
+        m_tr = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+        if m_hash and m_tr and m_hash.group(1) == h:
+            return float(m_tr.group(1))
+    except OSError:
+        pass
+    return None
+
+
+# ------------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ------------------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(prefix="clocks_", suffix=".csv")
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
+                 "-i", str(gpu_index)], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        self.t0 = self.t1 = None
+
+    def mark(self, start: bool) -> None:
+        if start:
+            self.t0 = time.time()
+        else:
+            self.t1 = time.time()
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.12)
+        self.proc.terminate()
+        self.proc.wait()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[3], parts[4:]))
+            except (ValueError, IndexError):
+                continue
+        os.unlink(self.path)
+        inside = [r for r in rows if self.t0 - 0.06 <= r[0] <= self.t1 + 0.06]
+        if not inside and rows:
+            mid = 0.5 * (self.t0 + self.t1)
+            inside = sorted(rows, key=lambda r: abs(r[0] - mid))[:3]
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[4][1:5]) if v.lower().startswith("active")})
+        return {"sm_mhz": float(np.median([r[1] for r in inside])), "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": reasons, "samples": len(inside)}
+
+
+# ------------------------------------------------------------------------------------------------
+# CPU oracle sample (the reference arm and the cpu_baseline)
+# ------------------------------------------------------------------------------------------------
+class OracleSampler:
+    """fp64 oracle on the 7B shape truncated to its first layer; one sample runs the verify step with
+    that layer on (t1) and the step with no layer (t0: embedding, final norm, LM head); the full
+    step is estimated as t0 + 32 * (t1 - t0)."""
+
+    def __init__(self, parent, toks, P: int, n_layers: int, mode: int = 0):
+        import oracle
+        import synth
+
+        sh = _shape()
+        self.sh1 = synth.ModelShape(1, sh.d_model, sh.n_heads, sh.head_dim, sh.ffn, sh.vocab)
+        self.w = oracle.Weights.from_seed(SEED, self.sh1, keep_layers=1)
+        for name in ("wqkv", "wo", "wg", "wu", "wd"):
+            self.w.f64(name, 0)
+        self.w.f64("embed")
+        self.w.f64("lm_head")
+        self.kv = oracle.KVCache(1, sh.n_heads, sh.head_dim, P + len(toks))
+        k = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, sh, 0, "k", P)).astype(np.float64)
+        v = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, sh, 0, "v", P)).astype(np.float64)
+        self.kv.load_prefix(0, k, v)
+        self.parent, self.toks = parent, toks
+        self.n_layers = n_layers
+        self.mode = mode
+        if mode:
+            for name in ("wqkv", "wo", "wg", "wu", "wd"):
+                self.w.int8(name, 0)
+        self.t0 = None
+
+    def _run(self, on: int) -> float:
+        import oracle
+
+        self.kv.reset_tree()
+        t = time.perf_counter()
+        oracle.tree_step(self.w, self.kv, self.toks, self.parent, skip_mask=np.array([on], np.uint8),
+                         quant_mode=self.mode)
+        return time.perf_counter() - t
+
+    def sample_us(self) -> float:
+        if self.t0 is None:
+            self.t0 = self._run(0)
+        t1 = self._run(1)
+        return (self.t0 + self.n_layers * max(t1 - self.t0, 0.0)) * 1e6
+
+
+def workload_tree(wl):
+    import synth
+
+    layers, P, n, depth, branch, skip, mode, verify = wl
+    parent = synth.tree(SEED, n, depth, branch)
+    toks = synth.tokens(SEED, n, _shape().vocab)
+    return parent, toks
+
+
+def describe(name: str, wl) -> str:
+    layers, P, n, depth, branch, skip, mode, verify = wl
+    kind = "tree verify + accept + compact" if verify else "draft step (tree reset after)"
+    extra = (f", {int(skip * 100)}% layers skipped" if skip else "") + (", W8A8" if mode else ", bf16")
+    br = f", branching<={branch}" if branch else ""
+    return (f"{name}: llama7b-shape {layers} layer(s), d4096, n={n} nodes (depth<={depth}{br}), prefix {P}{extra}; "
+            f"{kind}")
+
+
+def config_block(args, name, wl, graphs: bool) -> dict:
+    layers, P, n, depth, branch, skip, mode, verify = wl
+    return {"workload": describe(name, wl), "n_tree": n, "prefix_len": P, "tree_depth_max": depth, "seed": SEED,
+            "l2": "no flush: the weights + KV streamed per step exceed the 129 MB L2 many times",
+            "cuda_graphs": graphs, "pdl": True, "parallelism": f"replicas{args.gpus}"}
+
+
+def run_reference(args) -> None:
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = WORKLOADS[args.workload]
+    parent, toks = workload_tree(wl)
+    s = OracleSampler(parent, toks, wl[1], wl[0] if not wl[5] else int(round(wl[0] * (1 - wl[5]))), wl[6])
+    for _ in range(args.warmup):
+        s.sample_us()
+    vals = [s.sample_us() for _ in range(args.steps)]
+    v = float(np.mean(vals))
+    cores = os.cpu_count()
+    out = {"impl": "reference", "metric": METRIC, "value": round(v, 1), "unit": "us", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(v / 1e3, 3), "higher_is_better": False,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": config_block(args, args.workload, wl, False),
+           "cpu_baseline": {"value": round(v, 1), "unit": "us", "cores": cores, "kind": "oracle",
+                            "sample": f"fp64 oracle, embedding + 1 of {wl[0]} layers + LM head per step, "
+                                      f"scaled to {wl[0]} layers"},
+           "e2e": {"value": round(v, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+# ------------------------------------------------------------------------------------------------
+# the GPU arm
+# ------------------------------------------------------------------------------------------------
+def run_gpu(args) -> None:
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    import synth
+    import paper_2510_26843_gb300 as cs
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    cs.load_library()
+    wl = WORKLOADS[args.workload]
+    layers, P, n, depth, branch, skip, mode, verify = wl
+    sh = _shape(layers)
+    dm = DeviceModel(sh, SEED, with_int8=bool(mode))
+    kv = DeviceKV(dm, P + 2 * n + 64)
+    kv.load_random_prefix(SEED, P)
+    parent, toks = workload_tree(wl)
+    mask = synth.skip_masks(SEED, layers, [skip])[0] if skip else None
+    layers_on = layers if mask is None else int(mask.sum())
+    stream = torch.cuda.current_stream()
+    cs.set_stream(dm.h, stream)
+    tok_d = torch.tensor(toks, dtype=torch.int32, device="cuda")
+    par_d = torch.tensor(parent, dtype=torch.int32, device="cuda")
+    logits = torch.empty(n, sh.vocab, dtype=torch.float32, device="cuda")
+    acc = torch.zeros(n + 2, dtype=torch.int32, device="cuda")
+    graphs = not args.no_graphs
+    cs.set_options(dm.h, cs.OPT_PDL | (cs.OPT_GRAPHS if graphs else 0))
+
+    def step():
+        cs.tree_step(dm.h, kv.h, tok_d, par_d, n, mask, mode, logits)
+        if verify:
+            cs.accept_greedy(dm.h, None, tok_d, par_d, n, acc)
+            cs.kv_compact(kv.h, acc)
+            cs.kv_set_prefix(kv.h, P)
+        else:
+            cs.kv_reset_tree(kv.h)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    barrier()
+    st = cs.get_status(dm.h)
+    if st != 0:
+        raise RuntimeError(f"device status after warm-up: {st} ({cs.status_string(st)})")
+
+    # ---- device-timed region ----
+    clocks = ClockSampler(local)
+    time.sleep(0.2)
+    n0 = cs.launch_count(dm.h)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    clocks.mark(True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    barrier()
+    clocks.mark(False)
+    launches = cs.launch_count(dm.h) - n0
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    us = ms * 1e3
+
+    # ---- end to end through the C ABI with host buffers ----
+    tok_h = torch.from_numpy(np.asarray(toks, dtype=np.int32)).pin_memory()
+    par_h = torch.from_numpy(np.asarray(parent, dtype=np.int32)).pin_memory()
+    out_d = acc if verify else logits[:, :1]
+    out_h = torch.zeros(out_d.shape, dtype=out_d.dtype).pin_memory()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        tok_d.copy_(tok_h, non_blocking=True)
+        par_d.copy_(par_h, non_blocking=True)
+        step()
+        out_h.copy_(out_d, non_blocking=True)
+        stream.synchronize()
+    e2e_us = (time.perf_counter() - t0) / args.steps * 1e6
+    if verify:
+        assert 1 <= int(out_h[0]) <= n
+
+    # ---- kernel-timing pass: eager launches bracketed by CUDA events on the launch stream ----
+    cs.set_options(dm.h, cs.OPT_PDL)
+    cs.profile(dm.h, True)
+    for _ in range(args.steps):
+        step()
+    per_kind = {}
+    names = ["qkv", "attention", "wo", "gateup", "down", "lm_head", "other"]
+    for k, name in enumerate(names):
+        tot, cnt = cs.profile_read(dm.h, k)
+        per_kind[name] = {"ms_per_step": round(tot / args.steps, 4), "launches_per_step": cnt // max(args.steps, 1),
+                          "avg_us": round(tot / max(cnt, 1) * 1e3, 2)}
+    cs.profile(dm.h, False)
+    st = cs.get_status(dm.h)
+    if st != 0:
+        raise RuntimeError(f"device status after timing: {st} ({cs.status_string(st)})")
+
+    peak, peak_kind = measured_peaks()
+    gu_bytes = gateup_bytes(sh, n, mode)
+    gu_avg_s = per_kind["gateup"]["avg_us"] * 1e-6
+    achieved = gu_bytes / gu_avg_s / 1e9
+    ab = algorithmic_bytes(sh, n, P, layers_on, mode)
+    kern = "gemm_i8_kernel (W8A8 gate/up + SwiGLU)" if mode else "gemm_bf16_tc_kernel (gate/up + SwiGLU)"
+
+    out = {
+        "metric": METRIC, "value": round(us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int8" if mode else "bf16",
+        "data": "synthetic (seeded N(0,0.02) weights, N(0,1) prefix KV)",
+        "config": config_block(args, args.workload, wl, graphs),
+        "step_roofline": {"algorithmic_bytes": ab["total"],
+                          "pct_of_8TBps": round(100 * ab["total"] / (us * 1e-6) / 8e12, 2),
+                          "frac_of_hbm_peak": round(ab["total"] / (us * 1e-6) / 1e9 / peak, 4),
+                          "tokens_per_s": round(n / (us * 1e-6) * world, 1)},
+        "roofline": {"kernel": f"{kern}, {args.workload}", "bound": "hbm", "achieved": round(achieved, 1),
+                     "peak": peak, "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+                     else "fallback", "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": recorded_traffic() if (args.workload == "verify7b") else None,
+                     "algorithmic_bytes_per_launch": gu_bytes},
+        "kernels": per_kind,
+        "e2e": {"value": round(e2e_us, 1), "unit": "us", "h2d_bytes_per_step": 2 * n * 4,
+                "d2h_bytes_per_step": int(out_d.numel() * out_d.element_size())},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        s = OracleSampler(parent, toks, P, layers_on, mode)
+        t_start = time.perf_counter()
+        vals = []
+        while not vals or (time.perf_counter() - t_start < args.cpu_seconds and len(vals) < 20):
+            vals.append(s.sample_us())
+        out["cpu_baseline"] = {"value": round(float(np.mean(vals)), 1), "unit": "us", "cores": os.cpu_count(),
+                               "kind": "oracle",
+                               "sample": f"fp64 oracle, {len(vals)} x (embedding + 1 of {layers_on} layers + LM head), "
+                                         f"scaled to {layers_on} layers"}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    kv.close()
+    dm.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main() -> None:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-graphs", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--workload", default="verify7b", choices=sorted(WORKLOADS))
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

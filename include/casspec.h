@@ -211,6 +211,32 @@ CASSPEC_API int casspec_accept_greedy(casspec_model* m, const float* logits, con
  * E_TREE on the status word and leaves the cache unchanged. */
 CASSPEC_API int casspec_kv_compact(casspec_kv* kv, const int32_t* accepted_out);
 
+/* ---------------------------------------------------------------------------------------------
+ * Tracing: per-kernel device time measured with CUDA events on the launch stream.
+ * ------------------------------------------------------------------------------------------- */
+enum casspec_kernel_kind {
+  CASSPEC_K_QKV = 0,    /* QKV projection + rotary + K/V write */
+  CASSPEC_K_ATTN = 1,   /* tree attention */
+  CASSPEC_K_WO = 2,     /* output projection + residual */
+  CASSPEC_K_GATEUP = 3, /* gate/up projection + SwiGLU */
+  CASSPEC_K_DOWN = 4,   /* down projection + residual */
+  CASSPEC_K_LMHEAD = 5, /* LM head + argmax partials */
+  CASSPEC_K_OTHER = 6,  /* tree prep, embedding, RMSNorm, quantisation, argmax merge */
+  CASSPEC_K_COUNT = 7
+};
+
+/* enable != 0: clear the records and bracket every kernel the model launches eagerly from now on
+ * with a CUDA event pair (graph replays are not instrumented); enable == 0: stop recording. */
+CASSPEC_API int casspec_profile(casspec_model* m, int enable);
+
+/* Synchronise the model stream; total device time in ms and number of recorded launches of
+ * kernel kind `kind` (casspec_kernel_kind) since profiling was enabled. */
+CASSPEC_API int casspec_profile_read(casspec_model* m, int kind, double* total_ms, int* launches);
+
+/* Number of kernels the model has enqueued so far: eager launches plus the kernels contained in
+ * every replayed CUDA graph. */
+CASSPEC_API int casspec_launch_count(casspec_model* m, uint64_t* count);
+
 /* Synchronise the model stream; return and clear the device status word. */
 CASSPEC_API int casspec_get_status(casspec_model* m, int* status_out);
 

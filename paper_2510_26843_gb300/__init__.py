@@ -28,8 +28,9 @@ EXPORTS = [
     "casspec_kv_destroy", "casspec_kv_layer", "casspec_kv_set_prefix", "casspec_kv_reset_tree", "casspec_kv_length",
     "casspec_tree_step", "casspec_argmax", "casspec_accept_greedy", "casspec_kv_compact", "casspec_get_status",
     "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_rmsnorm",
-    "casspec_quantize_rows",
+    "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
 ]
+K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
 
 class ModelConfig(ctypes.Structure):
@@ -83,6 +84,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_linear_bf16": (_I, [_P, _I, _I, _P, _I, _P, _I, _P, _SZ, _P]),
         "casspec_rmsnorm": (_I, [_P, _P, _I, _I, ctypes.c_float, _P, _P, _P, _P]),
         "casspec_quantize_rows": (_I, [_P, _I, _I, _P, _P, _P]),
+        "casspec_profile": (_I, [_P, _I]),
+        "casspec_profile_read": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(_I)]),
+        "casspec_launch_count": (_I, [_P, ctypes.POINTER(ctypes.c_uint64)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -249,3 +253,20 @@ def rmsnorm(x, g, n: int, d: int, eps: float, y=None, q=None, s=None, stream=Non
 
 def quantize_rows(x, n: int, d: int, q, s, stream=None) -> None:
     _check("casspec_quantize_rows", load_library().casspec_quantize_rows(_ptr(x), n, d, _ptr(q), _ptr(s), _stream(stream)))
+
+
+def profile(m: int, enable: bool) -> None:
+    _check("casspec_profile", load_library().casspec_profile(m, int(enable)))
+
+
+def profile_read(m: int, kind: int) -> tuple[float, int]:
+    """(total device ms, launches) of kernel kind `kind` since profiling was enabled."""
+    t, c = ctypes.c_double(), _I()
+    _check("casspec_profile_read", load_library().casspec_profile_read(m, kind, ctypes.byref(t), ctypes.byref(c)))
+    return t.value, c.value
+
+
+def launch_count(m: int) -> int:
+    c = ctypes.c_uint64()
+    _check("casspec_launch_count", load_library().casspec_launch_count(m, ctypes.byref(c)))
+    return c.value

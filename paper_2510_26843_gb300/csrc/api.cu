@@ -177,8 +177,12 @@ struct casspec_model {
   float *attn_o, *attn_ml;
   unsigned* attn_cnt;
   int* status;
-  std::map<GraphKey, cudaGraphExec_t> graphs;
+  std::map<GraphKey, std::pair<cudaGraphExec_t, int>> graphs;  // exec + kernels it contains
   std::mutex mu;
+  bool prof_on = false;
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> prof_ev[CASSPEC_K_COUNT];
+  int prof_used[CASSPEC_K_COUNT] = {};
+  uint64_t launches = 0;
 };
 
 struct casspec_kv {
@@ -217,9 +221,41 @@ uint16_t* kv_layer_v(casspec_kv* kv, int l) {
     if (e_ != cudaSuccess) return CASSPEC_E_CUDA; \
   } while (0)
 
-// Enqueue one tree step on stream s (argument checks already done).
+// Event pair bracketing one launch of `kind` while profiling (eager launches only).
+cudaEvent_t prof_begin(casspec_model* m, int kind, cudaStream_t s) {
+  auto& v = m->prof_ev[kind];
+  int& used = m->prof_used[kind];
+  if (used == (int)v.size()) {
+    cudaEvent_t a, b;
+    if (cudaEventCreate(&a) != cudaSuccess) return nullptr;
+    if (cudaEventCreate(&b) != cudaSuccess) {
+      cudaEventDestroy(a);
+      return nullptr;
+    }
+    v.emplace_back(a, b);
+  }
+  cudaEventRecord(v[used].first, s);
+  return v[used].second;
+}
+
+// Launch `call` (a cudaError_t expression) as one kernel of kind `kind`: count it, and bracket it
+// with events when profiling an eager step.
+#define LAUNCH(kind, call)                                                   \
+  do {                                                                       \
+    cudaEvent_t stop_ = prof ? prof_begin(m, (kind), s) : nullptr;            \
+    const cudaError_t e_ = (call);                                           \
+    if (e_ != cudaSuccess) return CASSPEC_E_CUDA;                            \
+    if (stop_ != nullptr) {                                                  \
+      cudaEventRecord(stop_, s);                                             \
+      m->prof_used[(kind)]++;                                                \
+    }                                                                        \
+    ++count;                                                                 \
+  } while (0)
+
+// Enqueue one tree step on stream s (argument checks already done).  `count` receives the number
+// of kernels enqueued; profiling events are recorded only when `prof` is set.
 int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent, int n,
-                 const std::vector<uint8_t>& on, int mode, float* logits, cudaStream_t s) {
+                 const std::vector<uint8_t>& on, int mode, float* logits, cudaStream_t s, bool prof, int& count) {
   const auto& c = m->cfg;
   const int d = c.d_model, F = c.ffn, V = c.vocab, hd = c.head_dim, H = c.n_heads;
   const bool pdl = (m->flags & CASSPEC_OPT_PDL) != 0;
@@ -227,9 +263,9 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   const int bi = BN / 16 - 1;
   const int T = kv->T;
 
-  CK(launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->rope, m->inv_freq, hd / 2,
+  LAUNCH(CASSPEC_K_OTHER, launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->rope, m->inv_freq, hd / 2,
                       m->status, s, pdl));
-  CK(launch_embed(m->embed, tokens, n, d, V, m->x, s, pdl));
+  LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, m->x, s, pdl));
 
   EpiParams base = {};
   base.n = n;
@@ -276,7 +312,7 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     if (!on[l]) continue;
     LayerPtrs& Lp = m->layers[l];
     // attention block
-    CK(launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
+    LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
                       pdl));
     EpiParams e = base;
     e.N = 3 * d;
@@ -284,9 +320,9 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     e.kc = kv_layer_k(kv, l);
     e.vc = kv_layer_v(kv, l);
     if (mode == 0)
-      CK(gemm(Lp.tm_qkv, Lp.tm_qkv, m->tm_xn[bi], EPI_QKV, 3 * d / 128, cdiv(d, 64), e));
+      LAUNCH(CASSPEC_K_QKV, gemm(Lp.tm_qkv, Lp.tm_qkv, m->tm_xn[bi], EPI_QKV, 3 * d / 128, cdiv(d, 64), e));
     else
-      CK(gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+      LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
     AttnArgs at = {};
     at.q = m->q;
     at.kc = e.kc;
@@ -304,43 +340,43 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     at.part_ml = m->attn_ml;
     at.counters = m->attn_cnt;
     at.status = m->status;
-    CK(launch_tree_attention(at, hd, H, s, pdl));
+    LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(at, hd, H, s, pdl));
     EpiParams er = base;
     er.N = d;
     er.y = m->x;
     er.ldy = d;
     if (mode == 0) {
-      CK(gemm(Lp.tm_o, Lp.tm_o, m->tm_oact[bi], EPI_RESID, d / 128, cdiv(d, 64), er));
+      LAUNCH(CASSPEC_K_WO, gemm(Lp.tm_o, Lp.tm_o, m->tm_oact[bi], EPI_RESID, d / 128, cdiv(d, 64), er));
     } else {
-      CK(launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
-      CK(gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, er));
+      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
+      LAUNCH(CASSPEC_K_WO, gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, er));
     }
     // feed-forward block
-    CK(launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
+    LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
                       pdl));
     EpiParams eg = base;
     eg.N = F;
     eg.u_out = m->u;
     if (mode == 0)
-      CK(gemm(Lp.tm_g, Lp.tm_u, m->tm_xn[bi], EPI_GLU, cdiv(F, 64), cdiv(d, 64), eg));
+      LAUNCH(CASSPEC_K_GATEUP, gemm(Lp.tm_g, Lp.tm_u, m->tm_xn[bi], EPI_GLU, cdiv(F, 64), cdiv(d, 64), eg));
     else
-      CK(gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
+      LAUNCH(CASSPEC_K_GATEUP, gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
     if (mode == 0) {
-      CK(gemm(Lp.tm_d, Lp.tm_d, m->tm_uact[bi], EPI_RESID, d / 128, cdiv(F, 64), er));
+      LAUNCH(CASSPEC_K_DOWN, gemm(Lp.tm_d, Lp.tm_d, m->tm_uact[bi], EPI_RESID, d / 128, cdiv(F, 64), er));
     } else {
-      CK(launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
-      CK(gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, er));
+      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
+      LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, er));
     }
   }
-  CK(launch_rmsnorm(m->x, m->final_norm, n, d, c.rms_eps, m->xn, nullptr, nullptr, s, pdl));
+  LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, m->final_norm, n, d, c.rms_eps, m->xn, nullptr, nullptr, s, pdl));
   EpiParams el = base;
   el.N = V;
   el.logits = logits;
   el.am_v1 = m->am_v1;
   el.am_i1 = m->am_i1;
   el.am_v2 = m->am_v2;
-  CK(gemm(m->tm_lm, m->tm_lm, m->tm_xn[bi], EPI_LMHEAD, m->lay.lm_tiles, cdiv(d, 64), el));
-  CK(launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, m->lay.lm_tiles, n, m->am, m->margin, s, pdl));
+  LAUNCH(CASSPEC_K_LMHEAD, gemm(m->tm_lm, m->tm_lm, m->tm_xn[bi], EPI_LMHEAD, m->lay.lm_tiles, cdiv(d, 64), el));
+  LAUNCH(CASSPEC_K_OTHER, launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, m->lay.lm_tiles, n, m->am, m->margin, s, pdl));
   return CASSPEC_OK;
 }
 
@@ -472,7 +508,12 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
 
 void casspec_destroy_model(casspec_model* m) {
   if (m == nullptr) return;
-  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second.first);
+  for (auto& v : m->prof_ev)
+    for (auto& e : v) {
+      cudaEventDestroy(e.first);
+      cudaEventDestroy(e.second);
+    }
   if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
   delete m;
 }
@@ -487,7 +528,7 @@ int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
   if (m == nullptr || (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS)) != 0) return CASSPEC_E_INVAL;
   if (old_flags) *old_flags = m->flags;
   if (flags != m->flags) {
-    for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+    for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second.first);
     m->graphs.clear();
   }
   m->flags = flags;
@@ -591,6 +632,7 @@ int casspec_kv_layer(casspec_kv* kv, int layer, void** k_dev, void** v_dev, int*
 int casspec_kv_set_prefix(casspec_kv* kv, int P) {
   if (kv == nullptr || P < 0 || P > kv->ctx) return CASSPEC_E_INVAL;
   CK(launch_set_int(kv->dP, P, kv->m->stream));
+  kv->m->launches++;
   kv->P_upper = P;
   kv->T = 0;
   std::fill(kv->layer_valid.begin(), kv->layer_valid.end(), 0);
@@ -638,7 +680,8 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
     if (it == m->graphs.end()) {
       if (cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
         return CASSPEC_E_CUDA;
-      rc = enqueue_step(m, kv, tokens, parent_idx, n, on, quant_mode, logits_out, m->cap_stream);
+      int count = 0;
+      rc = enqueue_step(m, kv, tokens, parent_idx, n, on, quant_mode, logits_out, m->cap_stream, false, count);
       cudaGraph_t g = nullptr;
       const cudaError_t ec = cudaStreamEndCapture(m->cap_stream, &g);
       if (rc != CASSPEC_OK || ec != cudaSuccess || g == nullptr) {
@@ -650,11 +693,14 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
       const cudaError_t ei = cudaGraphInstantiate(&ex, g, 0);
       cudaGraphDestroy(g);
       if (ei != cudaSuccess) return CASSPEC_E_CUDA;
-      it = m->graphs.emplace(key, ex).first;
+      it = m->graphs.emplace(key, std::make_pair(ex, count)).first;
     }
-    if (cudaGraphLaunch(it->second, m->stream) != cudaSuccess) return CASSPEC_E_CUDA;
+    if (cudaGraphLaunch(it->second.first, m->stream) != cudaSuccess) return CASSPEC_E_CUDA;
+    m->launches += (uint64_t)it->second.second;
   } else {
-    rc = enqueue_step(m, kv, tokens, parent_idx, n, on, quant_mode, logits_out, m->stream);
+    int count = 0;
+    rc = enqueue_step(m, kv, tokens, parent_idx, n, on, quant_mode, logits_out, m->stream, m->prof_on, count);
+    m->launches += (uint64_t)count;
     if (rc != CASSPEC_OK) return rc;
   }
   const int Tn = kv->T + n;
@@ -679,8 +725,10 @@ int casspec_accept_greedy(casspec_model* m, const float* logits, const int32_t* 
   if (logits != nullptr) {
     CK(launch_row_argmax(logits, n, m->cfg.vocab, m->am2, m->stream));
     am = m->am2;
+    m->launches++;
   }
   CK(launch_accept(am, tokens, parent_idx, n, accepted_out, m->status, m->stream));
+  m->launches++;
   return CASSPEC_OK;
 }
 
@@ -693,9 +741,38 @@ int casspec_kv_compact(casspec_kv* kv, const int32_t* accepted_out) {
   const auto& c = m->cfg;
   CK(launch_kv_compact(kv->base, c.n_layers, c.n_heads, kv->ctx, c.head_dim, accepted_out, kv->T, kv->dP,
                        kv->compact_cnt, m->status, m->stream));
+  m->launches++;
   kv->P_upper += kv->T;
   kv->T = 0;
   std::fill(kv->layer_valid.begin(), kv->layer_valid.end(), 0);
+  return CASSPEC_OK;
+}
+
+int casspec_profile(casspec_model* m, int enable) {
+  if (m == nullptr) return CASSPEC_E_INVAL;
+  m->prof_on = enable != 0;
+  if (m->prof_on)
+    for (int k = 0; k < CASSPEC_K_COUNT; ++k) m->prof_used[k] = 0;
+  return CASSPEC_OK;
+}
+
+int casspec_profile_read(casspec_model* m, int kind, double* total_ms, int* launches) {
+  if (m == nullptr || kind < 0 || kind >= CASSPEC_K_COUNT) return CASSPEC_E_INVAL;
+  CK(cudaStreamSynchronize(m->stream));
+  double t = 0.0;
+  for (int i = 0; i < m->prof_used[kind]; ++i) {
+    float ms = 0.f;
+    CK(cudaEventElapsedTime(&ms, m->prof_ev[kind][i].first, m->prof_ev[kind][i].second));
+    t += ms;
+  }
+  if (total_ms) *total_ms = t;
+  if (launches) *launches = m->prof_used[kind];
+  return CASSPEC_OK;
+}
+
+int casspec_launch_count(casspec_model* m, uint64_t* count) {
+  if (m == nullptr || count == nullptr) return CASSPEC_E_INVAL;
+  *count = m->launches;
   return CASSPEC_OK;
 }
 
