@@ -31,10 +31,10 @@ struct LayerPtrs {
 // Byte layout of a model's device memory (weights, int8 copies, step scratch).
 struct Layout {
   size_t total = 0;
-  size_t embed, lm_head, final_norm, inv_freq;
+  size_t embed, lm_head, final_norm;
   std::vector<size_t> attn_norm, ffn_norm, wqkv, wo, wg, wu, wd;
   std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
-  size_t x, xn, q, o, u, xq, xs, pos, anc, rope, am_v1, am_i1, am_v2, am, margin, am2;
+  size_t x, xn, q, o, u, xq, xs, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
   size_t gemm_part, gemm_cnt, i8_part, i8_cnt, attn_o, attn_ml, attn_cnt, status;
   size_t scratch_begin;
   int max_tiles, lm_tiles;
@@ -67,7 +67,6 @@ Layout make_layout(const casspec_model_config& c) {
   L.embed = take(V * d * 2);
   L.lm_head = take(V * d * 2);
   L.final_norm = take(d * 4);
-  L.inv_freq = take((size_t)(c.head_dim / 2) * 8);
   for (size_t l = 0; l < NL; ++l) {
     L.attn_norm.push_back(take(d * 4));
     L.ffn_norm.push_back(take(d * 4));
@@ -104,7 +103,6 @@ Layout make_layout(const casspec_model_config& c) {
   L.xs = take(T * 4);
   L.pos = take(T * 4);
   L.anc = take(T * 8);
-  L.rope = take(T * (c.head_dim / 2) * 8);
   L.am_v1 = take((size_t)L.lm_tiles * T * 4);
   L.am_i1 = take((size_t)L.lm_tiles * T * 4);
   L.am_v2 = take((size_t)L.lm_tiles * T * 4);
@@ -157,7 +155,6 @@ struct casspec_model {
   int num_sms = 0;
   uint16_t *embed, *lm_head;
   float* final_norm;
-  double* inv_freq;
   std::vector<LayerPtrs> layers;
   CUtensorMap tm_lm;
   CUtensorMap tm_xn[4], tm_oact[4], tm_uact[4];
@@ -167,7 +164,6 @@ struct casspec_model {
   float* xs;
   int* pos;
   unsigned long long* anc;
-  float2* rope;
   float *am_v1, *am_v2, *margin;
   int *am_i1, *am, *am2;
   float* gemm_part;
@@ -193,6 +189,7 @@ struct casspec_kv {
   int* tdepth;
   unsigned long long* tanc;
   unsigned* compact_cnt;
+  float2* rope;  // [ctx][hd/2] rotary (cos, sin) per position
   int T = 0;
   long long P_upper = 0;
   std::vector<int> layer_valid;  // tree slots [0, layer_valid[l]) hold K/V of layer l
@@ -204,7 +201,9 @@ size_t kv_region_bytes(const casspec_model_config& c, int ctx) {
   return (size_t)c.n_layers * 2 * c.n_heads * ctx * c.head_dim * 2;
 }
 int kv_ctx(int max_ctx) { return (max_ctx + 63) / 64 * 64; }
-size_t kv_meta_bytes() { return 256 + kMaxTree * 4 + kMaxTree * 8 + 256; }
+size_t kv_meta_bytes(const casspec_model_config& c, int ctx) {
+  return 1024 + (size_t)ctx * (c.head_dim / 2) * 8;
+}
 
 uint16_t* kv_layer_k(casspec_kv* kv, int l) {
   const auto& c = kv->m->cfg;
@@ -263,8 +262,8 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   const int bi = BN / 16 - 1;
   const int T = kv->T;
 
-  LAUNCH(CASSPEC_K_OTHER, launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->rope, m->inv_freq, hd / 2,
-                      m->status, s, pdl));
+  LAUNCH(CASSPEC_K_OTHER, launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->status, s,
+                                           pdl));
   LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, m->x, s, pdl));
 
   EpiParams base = {};
@@ -274,7 +273,8 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   base.hd = hd;
   base.T = T;
   base.dP = kv->dP;
-  base.rope = m->rope;
+  base.pos = m->pos;
+  base.rope = kv->rope;
 
   auto gemm = [&](const CUtensorMap& tw, const CUtensorMap& tw2, const CUtensorMap& tx, int epi, int tiles,
                   int kblocks, const EpiParams& e) -> cudaError_t {
@@ -431,7 +431,6 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   m->embed = reinterpret_cast<uint16_t*>(b + L.embed);
   m->lm_head = reinterpret_cast<uint16_t*>(b + L.lm_head);
   m->final_norm = reinterpret_cast<float*>(b + L.final_norm);
-  m->inv_freq = reinterpret_cast<double*>(b + L.inv_freq);
   m->layers.resize(cfg->n_layers);
   for (int l = 0; l < cfg->n_layers; ++l) {
     LayerPtrs& p = m->layers[l];
@@ -465,7 +464,6 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   m->xs = reinterpret_cast<float*>(b + L.xs);
   m->pos = reinterpret_cast<int*>(b + L.pos);
   m->anc = reinterpret_cast<unsigned long long*>(b + L.anc);
-  m->rope = reinterpret_cast<float2*>(b + L.rope);
   m->am_v1 = reinterpret_cast<float*>(b + L.am_v1);
   m->am_i1 = reinterpret_cast<int*>(b + L.am_i1);
   m->am_v2 = reinterpret_cast<float*>(b + L.am_v2);
@@ -481,11 +479,7 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   m->attn_cnt = reinterpret_cast<unsigned*>(b + L.attn_cnt);
   m->status = reinterpret_cast<int*>(b + L.status);
 
-  std::vector<double> invf(cfg->head_dim / 2);
-  for (int j = 0; j < cfg->head_dim / 2; ++j)
-    invf[j] = std::pow((double)cfg->rope_base, -2.0 * j / (double)cfg->head_dim);
   if (cudaMemset(b + L.scratch_begin, 0, L.total - L.scratch_begin) != cudaSuccess ||
-      cudaMemcpy(m->inv_freq, invf.data(), invf.size() * 8, cudaMemcpyHostToDevice) != cudaSuccess ||
       cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
     delete m;
     return CASSPEC_E_CUDA;
@@ -590,7 +584,7 @@ int casspec_quantize_weights(casspec_model* m) {
 
 size_t casspec_kv_bytes(const casspec_model_config* cfg, int max_ctx) {
   if (!config_ok(cfg) || max_ctx < 1) return 0;
-  return kv_region_bytes(*cfg, kv_ctx(max_ctx)) + kv_meta_bytes();
+  return kv_region_bytes(*cfg, kv_ctx(max_ctx)) + kv_meta_bytes(*cfg, kv_ctx(max_ctx));
 }
 
 int casspec_kv_create(casspec_model* m, int max_ctx, void* dev_mem, size_t bytes, casspec_kv** out) {
@@ -598,7 +592,8 @@ int casspec_kv_create(casspec_model* m, int max_ctx, void* dev_mem, size_t bytes
   if ((reinterpret_cast<uintptr_t>(dev_mem) & 255) != 0) return CASSPEC_E_INVAL;
   const int ctx = kv_ctx(max_ctx);
   const size_t region = kv_region_bytes(m->cfg, ctx);
-  if (bytes < region + kv_meta_bytes()) return CASSPEC_E_CAPACITY;
+  const size_t meta_bytes = kv_meta_bytes(m->cfg, ctx);
+  if (bytes < region + meta_bytes) return CASSPEC_E_CAPACITY;
   casspec_kv* kv = new (std::nothrow) casspec_kv();
   if (kv == nullptr) return CASSPEC_E_CAPACITY;
   uint8_t* b = static_cast<uint8_t*>(dev_mem);
@@ -610,8 +605,20 @@ int casspec_kv_create(casspec_model* m, int max_ctx, void* dev_mem, size_t bytes
   kv->compact_cnt = reinterpret_cast<unsigned*>(meta + 128);
   kv->tdepth = reinterpret_cast<int*>(meta + 256);
   kv->tanc = reinterpret_cast<unsigned long long*>(meta + 256 + kMaxTree * 4);
+  kv->rope = reinterpret_cast<float2*>(meta + 1024);
   kv->layer_valid.assign(m->cfg.n_layers, 0);
-  if (cudaMemsetAsync(b, 0, region + kv_meta_bytes(), m->stream) != cudaSuccess) {
+  // rotary table for every position of the cache, evaluated in fp64 on the host
+  const int half = m->cfg.head_dim / 2;
+  std::vector<float2> table((size_t)ctx * half);
+  for (int p = 0; p < ctx; ++p)
+    for (int j = 0; j < half; ++j) {
+      const double ang = (double)p * std::pow((double)m->cfg.rope_base, -2.0 * j / (double)m->cfg.head_dim);
+      table[(size_t)p * half + j] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+    }
+  if (cudaMemsetAsync(b, 0, region + 1024, m->stream) != cudaSuccess ||
+      cudaMemcpyAsync(kv->rope, table.data(), table.size() * sizeof(float2), cudaMemcpyHostToDevice, m->stream) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(m->stream) != cudaSuccess) {
     delete kv;
     return CASSPEC_E_CUDA;
   }

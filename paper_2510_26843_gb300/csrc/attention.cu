@@ -234,25 +234,41 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attn_kernel(const AttnArgs 
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  for (int idx = tid; idx < a.n * (HD / 2); idx += kAttnThreads) {
-    const int row = idx / (HD / 2), c2 = (idx % (HD / 2)) * 2;
+  // merge: per-(row, split) weights 2^(m_s - M) / L staged in shared memory first (one pass of
+  // independent loads), then every output is a weighted sum over splits with independent loads.
+  float* w_s = reinterpret_cast<float*>(Ks);  // [64][splits] (K/V staging is free now)
+  const int S = a.splits;
+  for (int row = tid; row < a.n; row += kAttnThreads) {
     float M = -INFINITY;
-    for (int sp = 0; sp < a.splits; ++sp) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.part_ml + (((size_t)head * a.splits + sp) * 64 + row) * 2));
-      M = fmaxf(M, ml.x);
-    }
-    float L = 0.f, o0 = 0.f, o1 = 0.f;
-    for (int sp = 0; sp < a.splits; ++sp) {
-      const size_t pb = ((size_t)head * a.splits + sp) * 64 + row;
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.part_ml + pb * 2));
-      if (ml.x == -INFINITY) continue;
-      const float w = exp2f(ml.x - M);
-      const float2 ov = __ldcg(reinterpret_cast<const float2*>(a.part_o + pb * HD + c2));
+    for (int sp = 0; sp < S; ++sp)
+      M = fmaxf(M, __ldcg(a.part_ml + (((size_t)head * S + sp) * 64 + row) * 2));
+    float L = 0.f;
+    for (int sp = 0; sp < S; ++sp) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.part_ml + (((size_t)head * S + sp) * 64 + row) * 2));
+      const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
+      w_s[row * S + sp] = w;
       L += ml.y * w;
-      o0 += ov.x * w;
-      o1 += ov.y * w;
     }
-    *reinterpret_cast<uint32_t*>(a.o + (size_t)row * a.d + head * HD + c2) = pack_bf16x2(o0 / L, o1 / L);
+    const float invL = 1.f / L;
+    for (int sp = 0; sp < S; ++sp) w_s[row * S + sp] *= invL;
+  }
+  __syncthreads();
+  for (int idx = tid; idx < a.n * (HD / 4); idx += kAttnThreads) {
+    const int row = idx / (HD / 4), c4 = (idx % (HD / 4)) * 4;
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int sp = 0; sp < S; ++sp) {
+      const float w = w_s[row * S + sp];
+      if (w == 0.f) continue;
+      const float4 ov = __ldcg(reinterpret_cast<const float4*>(a.part_o + (((size_t)head * S + sp) * 64 + row) * HD + c4));
+      o.x += ov.x * w;
+      o.y += ov.y * w;
+      o.z += ov.z * w;
+      o.w += ov.w * w;
+    }
+    uint2 pk;
+    pk.x = pack_bf16x2(o.x, o.y);
+    pk.y = pack_bf16x2(o.z, o.w);
+    *reinterpret_cast<uint2*>(a.o + (size_t)row * a.d + head * HD + c4) = pk;
   }
   if (tid == 0) a.counters[head] = 0u;
 }
@@ -261,6 +277,7 @@ int attn_splits(int n_heads, int total_slots, int num_sms) {
   const int nblk = (total_slots + kAttnBlk - 1) / kAttnBlk;
   int s = (2 * num_sms + n_heads - 1) / n_heads;  // about two CTAs per SM
   if (s > nblk) s = nblk;
+  if (s > 64) s = 64;  // the merge stages 64 x splits weights in the K staging area
   if (s < 1) s = 1;
   return s;
 }

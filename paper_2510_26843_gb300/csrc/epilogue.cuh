@@ -29,7 +29,7 @@ __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, con
 #pragma unroll
     for (int i = 0; i < BN; ++i) {
       if (i < e.n) {
-        const float2 cs = e.rope[i * half + jj];
+        const float2 cs = e.rope[(size_t)e.pos[i] * half + jj];
         const float out = v[i] * cs.x + sgn * stg[rp * (BN + 1) + i] * cs.y;
         if (part == 0)
           e.q_out[(size_t)i * e.d + within] = f2bf(out);

@@ -31,10 +31,17 @@ constexpr uint32_t kATileBytes = 128 * 128;  // 128 rows x 64 bf16
 
 __host__ __device__ constexpr uint32_t gemm_stage_bytes(int BN) { return kATileBytes + (uint32_t)BN * 128u; }
 __host__ __device__ constexpr uint32_t gemm_staging_bytes(int BN) { return 128u * (uint32_t)(BN + 1) * 4u; }
+#ifndef CASSPEC_GEMM_SMEM_BUDGET
+#define CASSPEC_GEMM_SMEM_BUDGET (200u * 1024u)
+#endif
+#ifndef CASSPEC_GEMM_MAX_STAGES
+#define CASSPEC_GEMM_MAX_STAGES 8
+#endif
 __host__ __device__ constexpr int gemm_stages(int BN) {
-  return (int)((200u * 1024u - gemm_staging_bytes(BN) - 1024u) / gemm_stage_bytes(BN)) > 8
-             ? 8
-             : (int)((200u * 1024u - gemm_staging_bytes(BN) - 1024u) / gemm_stage_bytes(BN));
+  return (int)((CASSPEC_GEMM_SMEM_BUDGET - gemm_staging_bytes(BN) - 1024u) / gemm_stage_bytes(BN)) >
+                 CASSPEC_GEMM_MAX_STAGES
+             ? CASSPEC_GEMM_MAX_STAGES
+             : (int)((CASSPEC_GEMM_SMEM_BUDGET - gemm_staging_bytes(BN) - 1024u) / gemm_stage_bytes(BN));
 }
 __host__ __device__ constexpr size_t gemm_smem_bytes(int BN) {
   return 1024 + (size_t)gemm_stages(BN) * gemm_stage_bytes(BN) + gemm_staging_bytes(BN) + 256;
@@ -110,10 +117,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int t = (int)(u / kb), k = (int)(u % kb);
         uint8_t* sa = smem + stage * STAGE;
         if (EPI == EPI_GLU) {
-          tma_load_2d(sa, &tmW, &full[stage], k * 64, t * 64, pol_w);                 // gate rows
-          tma_load_2d(sa + kATileBytes / 2, &tmW2, &full[stage], k * 64, t * 64, pol_w);  // up rows
+          const int x = a.w_blocked ? 0 : k * 64, y = a.w_blocked ? (int)u * 64 : t * 64;
+          tma_load_2d(sa, &tmW, &full[stage], x, y, pol_w);                    // gate rows
+          tma_load_2d(sa + kATileBytes / 2, &tmW2, &full[stage], x, y, pol_w);  // up rows
         } else {
-          tma_load_2d(sa, &tmW, &full[stage], k * 64, t * 128, pol_w);
+          const int x = a.w_blocked ? 0 : k * 64, y = a.w_blocked ? (int)u * 128 : t * 128;
+          tma_load_2d(sa, &tmW, &full[stage], x, y, pol_w);
         }
       };
       auto load_x = [&](int stage, long long u) {

@@ -28,7 +28,8 @@ struct EpiParams {
   uint16_t* vc;         // this layer's V cache
   int ctx, d, hd, T;
   const int* dP;        // device committed length P
-  const float2* rope;   // [n][hd/2] (cos, sin) of pos(i) * base^(-2j/hd)
+  const int* pos;       // [n] position of each new node (P + depth)
+  const float2* rope;   // [ctx][hd/2] (cos, sin) of p * base^(-2j/hd) for every position p
   // EPI_GLU
   uint16_t* u_out;      // [64][F] bf16
   // EPI_LMHEAD
@@ -41,6 +42,7 @@ struct EpiParams {
 struct GemmArgs {
   int tiles;     // 128-row output tiles
   int kblocks;   // ceil(K / 64)
+  int w_blocked; // weights stored tile-blocked: box (t, k) is rows [(t * kblocks + k) * R, +R) of a 64-wide map
   float* partials;     // stream-K partial tiles, (tiles + grid) slots of 64 x 128 fp32
   unsigned* counters;  // [tiles], zero between launches
   int* status;
@@ -93,8 +95,7 @@ int attn_splits(int n_heads, int total_slots, int num_sms);
 cudaError_t launch_tree_attention(const AttnArgs& a, int hd, int n_heads, cudaStream_t stream, bool pdl);
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
-                             int* pos, unsigned long long* anc_new, float2* rope, const double* inv_freq, int half,
-                             int* status, cudaStream_t s, bool pdl);
+                             int* pos, unsigned long long* anc_new, int* status, cudaStream_t s, bool pdl);
 cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, cudaStream_t s,
                          bool pdl);
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,

@@ -22,15 +22,13 @@ static cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, size_t smem, cudaStrea
 // ---------------------------------------------------------------------------------------------
 // Tree preparation (Alg. 1 tree T_r; Sec. 4.2 tree attention).  New node i occupies tree slot
 // T + i; its depth is 0 for parent -1 (child of the last committed token) else depth(parent) + 1;
-// its position is P + depth; its ancestor mask is anc(parent) | bit(T + i).  Also fills the
-// rotary table (cos, sin)(pos(i) * inv_freq[j]) in fp64 -> fp32 for the QKV epilogue.
+// its position is P + depth; its ancestor mask is anc(parent) | bit(T + i).
 // ---------------------------------------------------------------------------------------------
 __global__ void tree_prep_kernel(const int* __restrict__ parent, int n, int T, const int* dP, int* tdepth,
-                                 unsigned long long* tanc, int* pos, unsigned long long* anc_new, float2* rope,
-                                 const double* inv_freq, int half, int* status) {
+                                 unsigned long long* tanc, int* pos, unsigned long long* anc_new, int* status) {
   __shared__ int s_depth[kMaxTree];
   __shared__ unsigned long long s_anc[kMaxTree];
-  __shared__ int s_pos[kMaxTree];
+  __shared__ int s_par[kMaxTree];
   pdl_trigger();
   pdl_wait();
   const int P = *dP;
@@ -38,12 +36,13 @@ __global__ void tree_prep_kernel(const int* __restrict__ parent, int n, int T, c
     s_depth[threadIdx.x] = tdepth[threadIdx.x];
     s_anc[threadIdx.x] = tanc[threadIdx.x];
   }
+  if (threadIdx.x < n) s_par[threadIdx.x] = parent[threadIdx.x];
   __syncthreads();
   if (threadIdx.x == 0) {
     bool bad = false;
     for (int i = 0; i < n; ++i) {
       const int j = T + i;
-      const int p = parent[i];
+      const int p = s_par[i];
       int dep;
       unsigned long long an;
       if (p == -1) {
@@ -59,32 +58,24 @@ __global__ void tree_prep_kernel(const int* __restrict__ parent, int n, int T, c
       }
       s_depth[j] = dep;
       s_anc[j] = an;
-      s_pos[i] = P + dep;
     }
     if (bad) set_status(status, CASSPEC_E_TREE);
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    tdepth[T + i] = s_depth[T + i];
-    tanc[T + i] = s_anc[T + i];
-    pos[i] = s_pos[i];
-    anc_new[i] = s_anc[T + i];
-  }
-  for (int idx = threadIdx.x; idx < n * half; idx += blockDim.x) {
-    const int i = idx / half, j = idx % half;
-    double sn, cs;
-    sincos((double)s_pos[i] * inv_freq[j], &sn, &cs);
-    rope[idx] = make_float2((float)cs, (float)sn);
+  if (threadIdx.x < n) {
+    const int j = T + threadIdx.x;
+    tdepth[j] = s_depth[j];
+    tanc[j] = s_anc[j];
+    pos[threadIdx.x] = P + s_depth[j];
+    anc_new[threadIdx.x] = s_anc[j];
   }
 }
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
-                             int* pos, unsigned long long* anc_new, float2* rope, const double* inv_freq, int half,
-                             int* status, cudaStream_t s, bool pdl) {
+                             int* pos, unsigned long long* anc_new, int* status, cudaStream_t s, bool pdl) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(256), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, tree_prep_kernel, parent, n, T, dP, tdepth, tanc, pos, anc_new, rope, inv_freq,
-                            half, status);
+  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(64), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, tree_prep_kernel, parent, n, T, dP, tdepth, tanc, pos, anc_new, status);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -146,62 +137,133 @@ __device__ __forceinline__ int8_t quant_one(float x, float inv) {
 
 // ---------------------------------------------------------------------------------------------
 // RMSNorm (pre-norm): y = bf16(x * rsqrt(mean(x^2) + eps) * g), fp32 arithmetic; optionally the
-// per-token int8 quantisation of the bf16 row.
+// per-token int8 quantisation of the bf16 row.  One CTA per row; the row stays in registers
+// (16-byte loads, all issued before the first reduction), so the kernel is one memory round trip.
 // ---------------------------------------------------------------------------------------------
-__global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g, int d, float eps,
-                               uint16_t* __restrict__ y, int8_t* __restrict__ q, float* __restrict__ sq) {
+constexpr int kRowThreads = 512;
+constexpr int kRowVec = 8;  // float4 per thread: rows up to 16384 fp32 values
+
+__global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g,
+                                                              int d, float eps, uint16_t* __restrict__ y,
+                                                              int8_t* __restrict__ q, float* __restrict__ sq) {
   __shared__ float red[32];
   pdl_trigger();
-  pdl_wait();
   const int i = blockIdx.x;
-  const float* xr = x + (size_t)i * d;
+  const int nv = d / 4;
+  float4 gv[kRowVec];
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    gv[k] = c < nv ? reinterpret_cast<const float4*>(g)[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  pdl_wait();
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)i * d);
+  float4 xv[kRowVec];
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    xv[k] = c < nv ? xr[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += xr[c] * xr[c];
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) ss += xv[k].x * xv[k].x + xv[k].y * xv[k].y + xv[k].z * xv[k].z + xv[k].w * xv[k].w;
   ss = block_sum(ss, red);
   const float r = rsqrtf(ss / (float)d + eps);
+  uint16_t b[kRowVec][4];
   float amax = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const uint16_t b = f2bf(xr[c] * r * g[c]);
-    if (y) y[(size_t)i * d + c] = b;
-    amax = fmaxf(amax, fabsf(bf2f(b)));
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    b[k][0] = f2bf(xv[k].x * r * gv[k].x);
+    b[k][1] = f2bf(xv[k].y * r * gv[k].y);
+    b[k][2] = f2bf(xv[k].z * r * gv[k].z);
+    b[k][3] = f2bf(xv[k].w * r * gv[k].w);
+    const int c = threadIdx.x + k * kRowThreads;
+    if (c < nv) {
+      if (y) {
+        uint2 pk;
+        pk.x = (uint32_t)b[k][0] | ((uint32_t)b[k][1] << 16);
+        pk.y = (uint32_t)b[k][2] | ((uint32_t)b[k][3] << 16);
+        reinterpret_cast<uint2*>(y + (size_t)i * d)[c] = pk;
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) amax = fmaxf(amax, fabsf(bf2f(b[k][e])));
+    }
   }
   if (q == nullptr) return;
   amax = block_max(amax, red);
   const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const float v = bf2f(f2bf(xr[c] * r * g[c]));
-    q[(size_t)i * d + c] = amax > 0.f ? quant_one(v, inv) : (int8_t)0;
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    if (c < nv) {
+      char4 o;
+      o.x = amax > 0.f ? quant_one(bf2f(b[k][0]), inv) : 0;
+      o.y = amax > 0.f ? quant_one(bf2f(b[k][1]), inv) : 0;
+      o.z = amax > 0.f ? quant_one(bf2f(b[k][2]), inv) : 0;
+      o.w = amax > 0.f ? quant_one(bf2f(b[k][3]), inv) : 0;
+      reinterpret_cast<char4*>(q + (size_t)i * d)[c] = o;
+    }
   }
   if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
 }
 
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
                            cudaStream_t s, bool pdl) {
+  if (d % 4 != 0 || d > 4 * kRowVec * kRowThreads) return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
   return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, x, g, d, eps, y, q, sq);
 }
 
-__global__ void quant_rows_kernel(const uint16_t* __restrict__ x, int d, int ldx, int8_t* __restrict__ q, int ldq,
-                                  float* __restrict__ sq) {
+// Per-row int8 quantisation of bf16 rows (16-byte loads kept in registers; rows up to 16384).
+constexpr int kQVec = 4;  // uint4 (8 bf16) per thread
+__global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t* __restrict__ x, int d, int ldx,
+                                                                 int8_t* __restrict__ q, int ldq,
+                                                                 float* __restrict__ sq) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
   const int i = blockIdx.x;
+  const int nv = d / 8;
   const uint16_t* xr = x + (size_t)i * ldx;
+  uint4 xv[kQVec];
+#pragma unroll
+  for (int k = 0; k < kQVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    xv[k] = c < nv ? reinterpret_cast<const uint4*>(xr)[c] : make_uint4(0, 0, 0, 0);
+  }
   float amax = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) amax = fmaxf(amax, fabsf(bf2f(xr[c])));
+#pragma unroll
+  for (int k = 0; k < kQVec; ++k) {
+    const uint32_t w[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) amax = fmaxf(amax, fmaxf(fabsf(bf2f(w[e] & 0xFFFF)), fabsf(bf2f(w[e] >> 16))));
+  }
   amax = block_max(amax, red);
   const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x)
-    q[(size_t)i * ldq + c] = amax > 0.f ? quant_one(bf2f(xr[c]), inv) : (int8_t)0;
+#pragma unroll
+  for (int k = 0; k < kQVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    if (c < nv) {
+      const uint32_t w[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+      uint32_t o[2] = {0u, 0u};
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float v = bf2f(e & 1 ? (w[e >> 1] >> 16) : (w[e >> 1] & 0xFFFF));
+        const int8_t qq = amax > 0.f ? quant_one(v, inv) : (int8_t)0;
+        o[e >> 2] |= ((uint32_t)(uint8_t)qq) << (8 * (e & 3));
+      }
+      reinterpret_cast<uint2*>(q + (size_t)i * ldq)[c] = make_uint2(o[0], o[1]);
+    }
+  }
   if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
 }
 
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
                               bool pdl) {
+  if (d % 8 != 0 || ldx % 8 != 0 || ldq % 8 != 0 || d > 8 * kQVec * kRowThreads) return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
   return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq);
 }
 

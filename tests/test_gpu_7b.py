@@ -1,0 +1,185 @@
+"""GPU parity at the Llama-7B shapes (d=4096, 32 heads x 128, F=11008, V=32000) against the CPU oracle,
+in the launch configuration the benchmark times (CUDA graphs + programmatic dependent launch):
+
+  * one 7B-shaped layer with LM head: prefix of 1024 stand-in K/V slots, 32-node tree (depth <= 6,
+    branching <= 4): logits, the tree K/V the step writes, and acceptance of a planted path;
+  * the full 32-layer verify: prefix 2048, 64-node tree (depth <= 8): all 64 x 32000 logits,
+    acceptance, and compaction (moved K/V bit-identical to the tree slots they came from);
+  * draft steps on the same model: 50% of layers skipped, W8A8, and both, at n = 8.
+
+Tolerances as in test_gpu_step.py (2e-2 / 5e-2 of the oracle's logit range; bit-exact indices
+unless the oracle's top-2 margin is below 1e-3).
+"""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+SEED = 777
+SH7 = synth.LLAMA7B
+TOL_BF16, TOL_INT8, MARGIN = 2e-2, 5e-2, 1e-3
+
+
+@pytest.fixture(scope="module")
+def cs():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import paper_2510_26843_gb300 as m
+
+    m.load_library()
+    return m
+
+
+def _i32(a):
+    return torch.tensor(np.asarray(a, dtype=np.int32), device="cuda")
+
+
+def rel_err(got, ref):
+    return np.max(np.abs(got - ref) / np.ptp(ref, axis=1, keepdims=True), axis=1)
+
+
+def oracle_cache(shape, P, extra):
+    okv = oracle.KVCache(shape.n_layers, shape.n_heads, shape.head_dim, P + extra)
+    for l in range(shape.n_layers):
+        k = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, shape, l, "k", P)).astype(np.float64)
+        v = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, shape, l, "v", P)).astype(np.float64)
+        okv.load_prefix(l, k, v)
+    return okv
+
+
+def gpu_step(cs, dm, kv, toks, parent, vocab, mask=None, mode=0):
+    n = len(toks)
+    t, p = _i32(toks), _i32(parent)
+    logits = torch.full((n, vocab), float("nan"), device="cuda")
+    cs.tree_step(dm.h, kv.h, t, p, n, mask, mode, logits)
+    torch.cuda.synchronize()
+    return logits.cpu().numpy().astype(np.float64), t, p
+
+
+# ------------------------------------------------------------------------------------------------
+# single 7B-shaped layer
+# ------------------------------------------------------------------------------------------------
+def test_single_layer_7b(cs):
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel, bf16_bits_to_float
+
+    sh = synth.ModelShape(1, SH7.d_model, SH7.n_heads, SH7.head_dim, SH7.ffn, SH7.vocab)
+    P, n = 1024, 32
+    dm = DeviceModel(sh, SEED)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS)
+    kv = DeviceKV(dm, P + 64)
+    kv.load_random_prefix(SEED, P)
+    ow = oracle.Weights.from_seed(SEED, sh, keep_layers=1)
+    parent = synth.tree(SEED, n, 6, 4)
+    toks = synth.tokens(SEED, n, sh.vocab)
+    # plant the oracle's greedy tokens along the root path of the deepest node
+    deepest = max(range(n), key=lambda i: (len(_path(parent, i)), -i))
+    branch = _path(parent, deepest)
+    for a, b in zip(branch, branch[1:]):
+        okv = oracle_cache(sh, P, n)
+        toks[b] = oracle.argmax_lowest(oracle.tree_step(ow, okv, toks, parent))[a]
+    okv = oracle_cache(sh, P, n)
+    trace = {}
+    ref = oracle.tree_step(ow, okv, toks, parent, trace=trace)
+    got, t, p = gpu_step(cs, dm, kv, toks, parent, sh.vocab)
+    assert np.all(rel_err(got, ref) < TOL_BF16), rel_err(got, ref).max()
+    # K/V the step wrote into the tree slots
+    K, V = kv.layer(0)
+    for dev, refkv in ((K, okv.K[0]), (V, okv.V[0])):
+        g = bf16_bits_to_float(dev[:, P:P + n])
+        r = refkv[:, P:P + n]
+        assert np.max(np.abs(g - r)) <= 1e-2 * np.max(np.abs(r))
+    acc = torch.zeros(n + 2, dtype=torch.int32, device="cuda")
+    cs.accept_greedy(dm.h, None, t, p, n, acc)
+    torch.cuda.synchronize()
+    path, bonus = oracle.accept_greedy(oracle.argmax_lowest(ref), toks, parent)
+    assert path == branch
+    if np.all(oracle.top2_margin(ref)[path] >= MARGIN):
+        L = int(acc[0])
+        assert acc[1:1 + L].cpu().tolist() == path and int(acc[L + 1]) == bonus
+    assert cs.get_status(dm.h) == 0
+    kv.close()
+    dm.close()
+
+
+def _path(parent, i):
+    out = []
+    while i != -1:
+        out.append(int(i))
+        i = parent[i]
+    return out[::-1]
+
+
+# ------------------------------------------------------------------------------------------------
+# full 32-layer model: verify and drafts
+# ------------------------------------------------------------------------------------------------
+@pytest.fixture(scope="module")
+def dm7(cs):
+    from paper_2510_26843_gb300.workload import DeviceModel
+
+    dm = DeviceModel(SH7, SEED, with_int8=True)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS)
+    yield dm
+    dm.close()
+
+
+@pytest.fixture(scope="module")
+def ow7():
+    return oracle.Weights.from_seed(SEED, SH7, keep_layers=1)
+
+
+def test_full_7b_verify_accept_compact(cs, dm7, ow7):
+    from paper_2510_26843_gb300.workload import DeviceKV
+
+    P, n = 2048, 64
+    kv = DeviceKV(dm7, P + 2 * n)
+    kv.load_random_prefix(SEED, P)
+    parent = synth.tree(SEED, n, 8)
+    toks = synth.tokens(SEED, n, SH7.vocab)
+    got, t, p = gpu_step(cs, dm7, kv, toks, parent, SH7.vocab)
+    # tree K/V of the last layer before compaction
+    K_last, V_last = (x[:, P:P + n].clone() for x in kv.layer(SH7.n_layers - 1))
+    acc = torch.zeros(n + 2, dtype=torch.int32, device="cuda")
+    cs.accept_greedy(dm7.h, None, t, p, n, acc)
+    cs.kv_compact(kv.h, acc)
+    torch.cuda.synchronize()
+    L = int(acc[0])
+    gpu_path = acc[1:1 + L].cpu().tolist()
+    assert cs.kv_length(kv.h) == (P + L, 0)
+    K_new, V_new = kv.layer(SH7.n_layers - 1)
+    for k, j in enumerate(gpu_path):  # compaction moves bytes exactly
+        assert torch.equal(K_new[:, P + k], K_last[:, j]) and torch.equal(V_new[:, P + k], V_last[:, j])
+    assert cs.get_status(dm7.h) == 0
+
+    okv = oracle_cache(SH7, P, n)
+    ref = oracle.tree_step(ow7, okv, toks, parent)
+    err = rel_err(got, ref)
+    assert np.all(err < TOL_BF16), err.max()
+    path, bonus = oracle.accept_greedy(oracle.argmax_lowest(ref), toks, parent)
+    if np.all(oracle.top2_margin(ref)[path] >= MARGIN):
+        assert gpu_path == path and int(acc[L + 1]) == bonus
+    kv.close()
+
+
+@pytest.mark.parametrize("skip,mode", [(0.5, 0), (0.0, 1), (0.5, 1)])
+def test_7b_draft_steps(cs, dm7, ow7, skip, mode):
+    from paper_2510_26843_gb300.workload import DeviceKV
+
+    P, n = 2048, 8
+    kv = DeviceKV(dm7, P + 64)
+    kv.load_random_prefix(SEED, P)
+    parent = synth.tree(SEED + 1, n, 8)
+    toks = synth.tokens(SEED + 1, n, SH7.vocab)
+    mask = synth.skip_masks(SEED, SH7.n_layers, [skip])[0] if skip else None
+    got, _, _ = gpu_step(cs, dm7, kv, toks, parent, SH7.vocab, mask=mask, mode=mode)
+    assert cs.get_status(dm7.h) == 0
+    okv = oracle_cache(SH7, P, n)
+    ref = oracle.tree_step(ow7, okv, toks, parent, skip_mask=mask, quant_mode=mode)
+    err = rel_err(got, ref)
+    assert np.all(err < (TOL_INT8 if mode else TOL_BF16)), err.max()
+    kv.close()
