@@ -38,7 +38,7 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attn_kernel(const AttnArgs 
   pdl_trigger();
   pdl_wait();
 
-  const int P = *a.dP;
+  const int P = __ldcg(a.dP);
   const int total = P + a.T + a.n;
   const int nblk = (total + kAttnBlk - 1) / kAttnBlk;
   const int b0 = (int)((long long)split * nblk / a.splits);
@@ -49,7 +49,7 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attn_kernel(const AttnArgs 
   for (int idx = tid; idx < 64 * C8; idx += kAttnThreads) {
     const int row = idx / C8, c8 = idx % C8;
     uint4 val = make_uint4(0, 0, 0, 0);
-    if (row < a.n) val = *reinterpret_cast<const uint4*>(a.q + (size_t)row * a.d + head * HD + c8 * 8);
+    if (row < a.n) val = __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)row * a.d + head * HD + c8 * 8));
     *reinterpret_cast<uint4*>(Qs + row * PITCH + c8 * 8) = val;
   }
   auto load_block = [&](int b, int buf) {
@@ -76,8 +76,8 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attn_kernel(const AttnArgs 
   const bool active = row0 < a.n;
   const int g = lane >> 2, t4 = lane & 3;
   const int rA = row0 + g, rB = rA + 8;
-  const unsigned long long ancA = rA < a.n ? a.anc[rA] : 0ull;
-  const unsigned long long ancB = rB < a.n ? a.anc[rB] : 0ull;
+  const unsigned long long ancA = rA < a.n ? __ldcg(a.anc + rA) : 0ull;
+  const unsigned long long ancB = rB < a.n ? __ldcg(a.anc + rB) : 0ull;
 
   uint32_t qf[HD / 16][4];
   if (active) {
@@ -275,7 +275,7 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attn_kernel(const AttnArgs 
 
 int attn_splits(int n_heads, int total_slots, int num_sms) {
   const int nblk = (total_slots + kAttnBlk - 1) / kAttnBlk;
-  int s = (2 * num_sms + n_heads - 1) / n_heads;  // about two CTAs per SM
+  int s = (2 * num_sms) / n_heads;  // two CTAs per SM: the whole grid runs in one wave
   if (s > nblk) s = nblk;
   if (s > 64) s = 64;  // the merge stages 64 x splits weights in the K staging area
   if (s < 1) s = 1;

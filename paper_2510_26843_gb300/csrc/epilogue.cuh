@@ -22,14 +22,14 @@ __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, con
   for (int i = 0; i < BN; ++i) stg[r * (BN + 1) + i] = v[i];
   bar();
   const int rp = r ^ half;  // heads are aligned to tiles (d % 128 == 0, hd | 128)
-  const int P = *e.dP;
+  const int P = __ldcg(e.dP);
   const int jj = j & (half - 1);
   if (part < 2) {
     const float sgn = (j < half) ? -1.f : 1.f;
 #pragma unroll
     for (int i = 0; i < BN; ++i) {
       if (i < e.n) {
-        const float2 cs = e.rope[(size_t)e.pos[i] * half + jj];
+        const float2 cs = e.rope[(size_t)__ldcg(e.pos + i) * half + jj];
         const float out = v[i] * cs.x + sgn * stg[rp * (BN + 1) + i] * cs.y;
         if (part == 0)
           e.q_out[(size_t)i * e.d + within] = f2bf(out);
@@ -106,7 +106,7 @@ __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, c
     for (int i = 0; i < BN; ++i) {
       if (i < e.n) {
         float* p = e.y + (size_t)i * e.ldy + o;
-        *p = store ? v[i] : (*p + v[i]);
+        *p = store ? v[i] : (__ldcg(p) + v[i]);
       }
     }
   }

@@ -83,7 +83,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         const int col = kb * 128 + c * 64 + 16 * t4;
-        B[c] = (tok < n && col < a.K) ? *reinterpret_cast<const uint4*>(a.X + (size_t)tok * a.K + col)
+        B[c] = (tok < n && col < a.K) ? __ldcg(reinterpret_cast<const uint4*>(a.X + (size_t)tok * a.K + col))
                                       : make_uint4(0, 0, 0, 0);
       }
 #pragma unroll
@@ -130,7 +130,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
       int sum = 0;
       for (int k = 0; k < a.ksplit; ++k)
         sum += __ldcg(a.partials + ((size_t)tile * a.ksplit + k) * (64 * 128) + tok * 128 + row);
-      stg[row * (BN + 1) + tok] = (float)sum * a.sx[tok] * scale_w(row);
+      stg[row * (BN + 1) + tok] = (float)sum * __ldcg(a.sx + tok) * scale_w(row);
     }
     if (tid == 0) a.counters[tile] = 0u;
   } else {
@@ -139,7 +139,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int tok = 8 * j + 2 * t4 + (e & 1), row = warp * 16 + g + 8 * (e >> 1);
-        if (tok < n) stg[row * (BN + 1) + tok] = (float)acc[j][e] * a.sx[tok] * scale_w(row);
+        if (tok < n) stg[row * (BN + 1) + tok] = (float)acc[j][e] * __ldcg(a.sx + tok) * scale_w(row);
       }
   }
   __syncthreads();

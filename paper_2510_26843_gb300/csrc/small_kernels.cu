@@ -19,6 +19,11 @@ static cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, size_t smem, cudaStrea
   return cfg;
 }
 
+// Note on loads: a kernel launched with programmatic dependent launch may start before its
+// predecessor finishes; everything a predecessor kernel wrote is therefore read with L1-bypassing
+// loads (__ldcg / ld.global.cg), never through L1 or the read-only path, which could hold lines
+// cached before griddepcontrol.wait returned.
+
 // ---------------------------------------------------------------------------------------------
 // Tree preparation (Alg. 1 tree T_r; Sec. 4.2 tree attention).  New node i occupies tree slot
 // T + i; its depth is 0 for parent -1 (child of the last committed token) else depth(parent) + 1;
@@ -31,12 +36,12 @@ __global__ void tree_prep_kernel(const int* __restrict__ parent, int n, int T, c
   __shared__ int s_par[kMaxTree];
   pdl_trigger();
   pdl_wait();
-  const int P = *dP;
+  const int P = __ldcg(dP);
   if (threadIdx.x < T) {
-    s_depth[threadIdx.x] = tdepth[threadIdx.x];
-    s_anc[threadIdx.x] = tanc[threadIdx.x];
+    s_depth[threadIdx.x] = __ldcg(tdepth + threadIdx.x);
+    s_anc[threadIdx.x] = __ldcg(tanc + threadIdx.x);
   }
-  if (threadIdx.x < n) s_par[threadIdx.x] = parent[threadIdx.x];
+  if (threadIdx.x < n) s_par[threadIdx.x] = __ldcg(parent + threadIdx.x);
   __syncthreads();
   if (threadIdx.x == 0) {
     bool bad = false;
@@ -86,7 +91,7 @@ __global__ void embed_kernel(const uint16_t* __restrict__ E, const int* __restri
   pdl_trigger();
   pdl_wait();
   const int i = blockIdx.x;
-  int tok = tokens[i];
+  int tok = __ldcg(tokens + i);
   tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);
   const uint16_t* row = E + (size_t)tok * d;
   for (int c = threadIdx.x * 2; c < d; c += blockDim.x * 2) {
@@ -148,6 +153,7 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __res
                                                               int8_t* __restrict__ q, float* __restrict__ sq) {
   __shared__ float red[32];
   pdl_trigger();
+  pdl_wait();
   const int i = blockIdx.x;
   const int nv = d / 4;
   float4 gv[kRowVec];
@@ -156,13 +162,12 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __res
     const int c = threadIdx.x + k * kRowThreads;
     gv[k] = c < nv ? reinterpret_cast<const float4*>(g)[c] : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  pdl_wait();
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)i * d);
   float4 xv[kRowVec];
 #pragma unroll
   for (int k = 0; k < kRowVec; ++k) {
     const int c = threadIdx.x + k * kRowThreads;
-    xv[k] = c < nv ? xr[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+    xv[k] = c < nv ? __ldcg(xr + c) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   float ss = 0.f;
 #pragma unroll
@@ -230,7 +235,7 @@ __global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t*
 #pragma unroll
   for (int k = 0; k < kQVec; ++k) {
     const int c = threadIdx.x + k * kRowThreads;
-    xv[k] = c < nv ? reinterpret_cast<const uint4*>(xr)[c] : make_uint4(0, 0, 0, 0);
+    xv[k] = c < nv ? __ldcg(reinterpret_cast<const uint4*>(xr) + c) : make_uint4(0, 0, 0, 0);
   }
   float amax = 0.f;
 #pragma unroll
@@ -291,7 +296,8 @@ __global__ void argmax_reduce_kernel(const float* __restrict__ v1, const int* __
   pdl_wait();
   const int row = blockIdx.x, lane = threadIdx.x;
   Top2 acc = {-INFINITY, 0x7fffffff, -INFINITY};
-  for (int t = lane; t < tiles; t += 32) acc = merge_top2(acc, Top2{v1[t * 64 + row], i1[t * 64 + row], v2[t * 64 + row]});
+  for (int t = lane; t < tiles; t += 32)
+    acc = merge_top2(acc, Top2{__ldcg(v1 + t * 64 + row), __ldcg(i1 + t * 64 + row), __ldcg(v2 + t * 64 + row)});
   for (int o = 16; o > 0; o >>= 1) {
     Top2 other{__shfl_xor_sync(0xffffffffu, acc.v1, o), __shfl_xor_sync(0xffffffffu, acc.i1, o),
                __shfl_xor_sync(0xffffffffu, acc.v2, o)};
@@ -318,7 +324,7 @@ __global__ void row_argmax_kernel(const float* __restrict__ logits, int V, int* 
   float best = -INFINITY;
   int bi = 0x7fffffff;
   for (int c = threadIdx.x; c < V; c += blockDim.x) {
-    const float x = lr[c];
+    const float x = __ldcg(lr + c);
     if (x > best || (x == best && c < bi)) {
       best = x;
       bi = c;
@@ -362,9 +368,9 @@ __global__ void accept_kernel(const int* __restrict__ am, const int* __restrict_
   __shared__ int s_par[kMaxTree], s_tok[kMaxTree], s_am[kMaxTree], s_depth[kMaxTree], s_match[kMaxTree];
   const int tid = threadIdx.x;
   if (tid < n) {
-    s_par[tid] = parent[tid];
-    s_tok[tid] = tokens[tid];
-    s_am[tid] = am[tid];
+    s_par[tid] = __ldcg(parent + tid);
+    s_tok[tid] = __ldcg(tokens + tid);
+    s_am[tid] = __ldcg(am + tid);
   }
   __syncthreads();
   if (tid != 0) return;
@@ -410,12 +416,12 @@ __global__ void kv_compact_kernel(uint16_t* kv, int n_layers, int n_heads, int c
                                   int T, int* dP, unsigned* counter, int* status) {
   __shared__ int s_path[kMaxTree];
   __shared__ int s_ok, s_last;
-  const int P = *dP;
+  const int P = __ldcg(dP);
   if (threadIdx.x == 0) {
-    const int L = acc[0];
+    const int L = __ldcg(acc);
     bool ok = L >= 1 && L <= T;
     for (int k = 0; ok && k < L; ++k) {
-      const int j = acc[1 + k];
+      const int j = __ldcg(acc + 1 + k);
       ok = j >= 0 && j < T && (k == 0 ? j == 0 : j > s_path[k - 1]);
       s_path[k] = j;
     }
