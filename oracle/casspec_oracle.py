@@ -30,7 +30,8 @@ Readings where the paper is silent (each also listed in the design notes):
   * quantisation: q = rint(x * (127 / amax)) with ties to even, clamped to [-127, 127], scale
     amax / 127; amax = 0 gives q = 0 and scale 0.  Weights are quantised with this rule evaluated
     in fp32 (IEEE round-to-nearest division and multiply, no fused multiply-add) from the bf16
-    weights; activations in the end-to-end oracle use the same rule in fp64.
+    weights; activations are quantised with the same fp32 rule from their bf16 rounding (the
+    precision in which the draft stores them), so both sides take the integer decisions alike.
 
 Everything here is fp64 unless stated; bf16 inputs are widened exactly.
 """
@@ -243,9 +244,18 @@ def tree_topology(parent: np.ndarray, T: int, depth_prev: list, anc_prev: list) 
 # ----------------------------------------------------------------------------------------------
 
 
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest bf16 value (ties to even) via fp32; returned as fp32."""
+    u = np.ascontiguousarray(np.asarray(x, dtype=np.float64).astype(np.float32)).view(np.uint32)
+    u = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) & np.uint32(0xFFFF0000)
+    return u.view(np.float32)
+
+
 def _linear(x: np.ndarray, w: Weights, name: str, layer: int, quant: bool) -> np.ndarray:
     if quant:
-        qx, sx = quantize_rows_f64(x)
+        # The quantiser's integer decisions are taken on the activation as the draft stores it
+        # (bf16) with the fp32 rule, i.e. in the kernel's precision.
+        qx, sx = quantize_rows_f32(round_bf16(x))
         qw, sw = w.int8(name, layer)
         return linear_w8a8(qx, sx, qw, sw)
     return x @ w.f64(name, layer).T
