@@ -190,6 +190,7 @@ struct casspec_kv {
   unsigned long long* tanc;
   unsigned* compact_cnt;
   float2* rope;  // [ctx][hd/2] rotary (cos, sin) per position
+  CUtensorMap tm_kv;  // the whole cache as [layers * 2 * heads * ctx][hd] bf16, 64 x 64 boxes
   int T = 0;
   long long P_upper = 0;
   std::vector<int> layer_valid;  // tree slots [0, layer_valid[l]) hold K/V of layer l
@@ -325,8 +326,6 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
     AttnArgs at = {};
     at.q = m->q;
-    at.kc = e.kc;
-    at.vc = e.vc;
     at.o = m->o;
     at.anc = m->anc;
     at.dP = kv->dP;
@@ -334,13 +333,15 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     at.n = n;
     at.ctx = kv->ctx;
     at.d = d;
-    at.splits = attn_splits(H, (int)std::min<long long>(total_slots, kv->ctx), m->num_sms);
+    at.n_heads = H;
+    at.layer = l;
     at.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
     at.part_o = m->attn_o;
     at.part_ml = m->attn_ml;
     at.counters = m->attn_cnt;
     at.status = m->status;
-    LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(at, hd, H, s, pdl));
+    const int agrid = attn_grid(H, (int)std::min<long long>(total_slots, kv->ctx), m->num_sms);
+    LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(kv->tm_kv, at, hd, agrid, s, pdl));
     EpiParams er = base;
     er.N = d;
     er.y = m->x;
@@ -607,6 +608,11 @@ int casspec_kv_create(casspec_model* m, int max_ctx, void* dev_mem, size_t bytes
   kv->tanc = reinterpret_cast<unsigned long long*>(meta + 256 + kMaxTree * 4);
   kv->rope = reinterpret_cast<float2*>(meta + 1024);
   kv->layer_valid.assign(m->cfg.n_layers, 0);
+  if (!encode_tmap_bf16(&kv->tm_kv, kv->base, (uint64_t)m->cfg.head_dim,
+                        (uint64_t)m->cfg.n_layers * 2 * m->cfg.n_heads * ctx, (uint64_t)m->cfg.head_dim * 2, 64, 64)) {
+    delete kv;
+    return CASSPEC_E_CUDA;
+  }
   // rotary table for every position of the cache, evaluated in fp64 on the host
   const int half = m->cfg.head_dim / 2;
   std::vector<float2> table((size_t)ctx * half);

@@ -67,15 +67,14 @@ struct GemmI8Args {
 
 struct AttnArgs {
   const uint16_t* q;    // [64][d] bf16 (rotated)
-  const uint16_t* kc;   // [H][ctx][hd]
-  const uint16_t* vc;
   uint16_t* o;          // [64][d] bf16
   const unsigned long long* anc;  // [n] ancestor masks over tree slots
   const int* dP;
-  int T, n, ctx, d, splits;
+  int T, n, ctx, d, n_heads;
+  int layer;            // K/V rows of this layer in the cache tensor map: ((layer * 2 + kv) * H + h) * ctx + slot
   float scale_log2;     // log2(e) / sqrt(hd)
-  float* part_o;        // [H][splits][64][hd]
-  float* part_ml;       // [H][splits][64][2]
+  float* part_o;        // [n_heads + grid][64][hd]
+  float* part_ml;       // [n_heads + grid][64][2]
   unsigned* counters;   // [H]
   int* status;
 };
@@ -91,8 +90,9 @@ cudaError_t launch_gemm_bf16(const CUtensorMap& tmW, const CUtensorMap& tmW2, co
 int gemm_i8_ksplit(int tiles, int K, int num_sms);
 cudaError_t launch_gemm_i8(const GemmI8Args& args, int BN, int epi, cudaStream_t stream, bool pdl);
 
-int attn_splits(int n_heads, int total_slots, int num_sms);
-cudaError_t launch_tree_attention(const AttnArgs& a, int hd, int n_heads, cudaStream_t stream, bool pdl);
+int attn_grid(int n_heads, int total_slots, int num_sms);
+cudaError_t launch_tree_attention(const CUtensorMap& tmKV, const AttnArgs& a, int hd, int grid, cudaStream_t stream,
+                                  bool pdl);
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
                              int* pos, unsigned long long* anc_new, int* status, cudaStream_t s, bool pdl);
