@@ -35,7 +35,7 @@ struct Layout {
   std::vector<size_t> attn_norm, ffn_norm, wqkv, wo, wg, wu, wd;
   std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
   size_t x, xn, q, o, u, xq, xs, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
-  size_t gemm_part, gemm_cnt, i8_part, i8_cnt, attn_o, attn_ml, attn_cnt, status;
+  size_t gemm_part, gemm_cnt, i8_part, i8_cnt, status;
   size_t scratch_begin;
   int max_tiles, lm_tiles;
 };
@@ -113,9 +113,6 @@ Layout make_layout(const casspec_model_config& c) {
   L.gemm_cnt = take((size_t)L.max_tiles * 4);
   L.i8_part = take((size_t)(6 * kSmsBound + 2 * L.max_tiles) * 64 * 128 * 4);
   L.i8_cnt = take((size_t)L.max_tiles * 4);
-  L.attn_o = take((size_t)(2 * kSmsBound + 2 * c.n_heads) * 64 * c.head_dim * 4);
-  L.attn_ml = take((size_t)(2 * kSmsBound + 2 * c.n_heads) * 64 * 2 * 4);
-  L.attn_cnt = take((size_t)c.n_heads * 4);
   L.status = take(256);
   L.total = align_up(off, 256);
   return L;
@@ -170,8 +167,6 @@ struct casspec_model {
   unsigned* gemm_cnt;
   int* i8_part;
   unsigned* i8_cnt;
-  float *attn_o, *attn_ml;
-  unsigned* attn_cnt;
   int* status;
   std::map<GraphKey, std::pair<cudaGraphExec_t, int>> graphs;  // exec + kernels it contains
   std::mutex mu;
@@ -308,7 +303,6 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     return launch_gemm_i8(a, BN, epi, s, pdl);
   };
 
-  const long long total_slots = kv->P_upper + T + n;
   for (int l = 0; l < c.n_layers; ++l) {
     if (!on[l]) continue;
     LayerPtrs& Lp = m->layers[l];
@@ -335,13 +329,10 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     at.d = d;
     at.n_heads = H;
     at.layer = l;
+    at.cluster = attn_cluster(H, m->num_sms);
     at.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
-    at.part_o = m->attn_o;
-    at.part_ml = m->attn_ml;
-    at.counters = m->attn_cnt;
     at.status = m->status;
-    const int agrid = attn_grid(H, (int)std::min<long long>(total_slots, kv->ctx), m->num_sms);
-    LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(kv->tm_kv, at, hd, agrid, s, pdl));
+    LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(kv->tm_kv, at, hd, s, pdl));
     EpiParams er = base;
     er.N = d;
     er.y = m->x;
@@ -475,9 +466,6 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   m->gemm_cnt = reinterpret_cast<unsigned*>(b + L.gemm_cnt);
   m->i8_part = reinterpret_cast<int*>(b + L.i8_part);
   m->i8_cnt = reinterpret_cast<unsigned*>(b + L.i8_cnt);
-  m->attn_o = reinterpret_cast<float*>(b + L.attn_o);
-  m->attn_ml = reinterpret_cast<float*>(b + L.attn_ml);
-  m->attn_cnt = reinterpret_cast<unsigned*>(b + L.attn_cnt);
   m->status = reinterpret_cast<int*>(b + L.status);
 
   if (cudaMemset(b + L.scratch_begin, 0, L.total - L.scratch_begin) != cudaSuccess ||
@@ -799,7 +787,6 @@ int casspec_get_status(casspec_model* m, int* status_out) {
     CK(cudaMemset(m->status, 0, 4));
     CK(cudaMemset(m->gemm_cnt, 0, (size_t)m->lay.max_tiles * 4));
     CK(cudaMemset(m->i8_cnt, 0, (size_t)m->lay.max_tiles * 4));
-    CK(cudaMemset(m->attn_cnt, 0, (size_t)m->cfg.n_heads * 4));
   }
   if (status_out) *status_out = st;
   return CASSPEC_OK;

@@ -72,10 +72,8 @@ struct AttnArgs {
   const int* dP;
   int T, n, ctx, d, n_heads;
   int layer;            // K/V rows of this layer in the cache tensor map: ((layer * 2 + kv) * H + h) * ctx + slot
+  int cluster;          // CTAs per head (thread-block cluster size, <= 8)
   float scale_log2;     // log2(e) / sqrt(hd)
-  float* part_o;        // [n_heads + grid][64][hd]
-  float* part_ml;       // [n_heads + grid][64][2]
-  unsigned* counters;   // [H]
   int* status;
 };
 
@@ -90,9 +88,8 @@ cudaError_t launch_gemm_bf16(const CUtensorMap& tmW, const CUtensorMap& tmW2, co
 int gemm_i8_ksplit(int tiles, int K, int num_sms);
 cudaError_t launch_gemm_i8(const GemmI8Args& args, int BN, int epi, cudaStream_t stream, bool pdl);
 
-int attn_grid(int n_heads, int total_slots, int num_sms);
-cudaError_t launch_tree_attention(const CUtensorMap& tmKV, const AttnArgs& a, int hd, int grid, cudaStream_t stream,
-                                  bool pdl);
+int attn_cluster(int n_heads, int num_sms);
+cudaError_t launch_tree_attention(const CUtensorMap& tmKV, const AttnArgs& a, int hd, cudaStream_t stream, bool pdl);
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
                              int* pos, unsigned long long* anc_new, int* status, cudaStream_t s, bool pdl);
