@@ -51,7 +51,9 @@ typedef enum casspec_status {
 } casspec_status;
 
 /* Model shape.  Requirements: d_model = n_heads * head_dim; head_dim in {64, 128};
- * d_model % 128 == 0; ffn % 16 == 0; vocab % 8 == 0; 1 <= n_layers <= 256. */
+ * d_model % 128 == 0, d_model <= 16384; ffn % 16 == 0, ffn <= 65536; vocab % 8 == 0,
+ * vocab <= 131072; 1 <= n_layers <= 256.  The upper bounds keep every projection at most 1024
+ * output tiles (one stream-K counter page per phase). */
 typedef struct casspec_model_config {
   int32_t n_layers;
   int32_t d_model;

@@ -34,8 +34,8 @@ struct Layout {
   size_t embed, lm_head, final_norm;
   std::vector<size_t> attn_norm, ffn_norm, wqkv, wo, wg, wu, wd;
   std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
-  size_t x, xn, q, o, u, xq, xs, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
-  size_t gemm_part, gemm_cnt, i8_part, i8_cnt, status;
+  size_t x, q, o, u, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
+  size_t gemm_part, gemm_cnt, chain_cnt, chain_bar, i8_part, i8_cnt, status;
   size_t scratch_begin;
   int max_tiles, lm_tiles;
 };
@@ -45,9 +45,9 @@ bool config_ok(const casspec_model_config* c) {
   if (c->n_layers < 1 || c->n_layers > 256) return false;
   if (c->head_dim != 64 && c->head_dim != 128) return false;
   if (c->n_heads < 1 || c->d_model != c->n_heads * c->head_dim) return false;
-  if (c->d_model % 128 != 0) return false;
-  if (c->ffn < 16 || c->ffn % 16 != 0) return false;
-  if (c->vocab < 1 || c->vocab % 8 != 0) return false;
+  if (c->d_model % 128 != 0 || c->d_model > 16384) return false;
+  if (c->ffn < 16 || c->ffn % 16 != 0 || c->ffn > 65536) return false;
+  if (c->vocab < 1 || c->vocab % 8 != 0 || c->vocab > 131072) return false;
   if (!(c->rope_base > 0.f) || !(c->rms_eps >= 0.f)) return false;
   return true;
 }
@@ -95,12 +95,12 @@ Layout make_layout(const casspec_model_config& c) {
   L.lm_tiles = cdiv(V, 128);
   L.max_tiles = std::max(std::max(cdiv(3 * d, 128), cdiv(F, 64)), L.lm_tiles);
   L.x = take(T * d * 4);
-  L.xn = take(T * d * 2);
   L.q = take(T * d * 2);
-  L.o = take(T * d * 2);
-  L.u = take(T * F * 2);
+  L.o = take(T * d * 4);
+  L.u = take(T * F * 4);
   L.xq = take(T * std::max(d, F));
   L.xs = take(T * 4);
+  L.ssp = take((size_t)std::max<size_t>(d / 128, 1) * T * 4);
   L.pos = take(T * 4);
   L.anc = take(T * 8);
   L.am_v1 = take((size_t)L.lm_tiles * T * 4);
@@ -111,6 +111,8 @@ Layout make_layout(const casspec_model_config& c) {
   L.am2 = take(T * 4);
   L.gemm_part = take(gemm_partials_floats(L.max_tiles, kSmsBound) * 4);
   L.gemm_cnt = take((size_t)L.max_tiles * 4);
+  L.chain_cnt = take((size_t)kMaxPhases * 1024 * 4);
+  L.chain_bar = take(256);
   L.i8_part = take((size_t)(6 * kSmsBound + 2 * L.max_tiles) * 64 * 128 * 4);
   L.i8_cnt = take((size_t)L.max_tiles * 4);
   L.status = take(256);
@@ -154,11 +156,11 @@ struct casspec_model {
   float* final_norm;
   std::vector<LayerPtrs> layers;
   CUtensorMap tm_lm;
-  CUtensorMap tm_xn[4], tm_oact[4], tm_uact[4];
-  float* x;
-  uint16_t *xn, *q, *o, *u;
+  float *x, *o, *u, *ssp;
+  uint16_t* q;
   int8_t* xq;
   float* xs;
+  unsigned *chain_cnt, *chain_bar;
   int* pos;
   unsigned long long* anc;
   float *am_v1, *am_v2, *margin;
@@ -249,18 +251,24 @@ cudaEvent_t prof_begin(casspec_model* m, int kind, cudaStream_t s) {
 
 // Enqueue one tree step on stream s (argument checks already done).  `count` receives the number
 // of kernels enqueued; profiling events are recorded only when `prof` is set.
+//   bf16 mode: tree prep -> embedding (+ row sums of squares) -> chain[QKV of the first active
+//   layer] -> for each active layer: attention, chain[Wo, Wgate/Wup, Wdown, next layer's QKV or the
+//   LM head] -> argmax merge.  RMSNorm is folded into the chain phases that consume it.
+//   int8 mode: per-projection W8A8 kernels with RMSNorm / quantisation kernels, then chain[LM head].
 int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent, int n,
                  const std::vector<uint8_t>& on, int mode, float* logits, cudaStream_t s, bool prof, int& count) {
   const auto& c = m->cfg;
   const int d = c.d_model, F = c.ffn, V = c.vocab, hd = c.head_dim, H = c.n_heads;
   const bool pdl = (m->flags & CASSPEC_OPT_PDL) != 0;
   const int BN = roundup16(n);
-  const int bi = BN / 16 - 1;
   const int T = kv->T;
+  std::vector<int> act;
+  for (int l = 0; l < c.n_layers; ++l)
+    if (on[l]) act.push_back(l);
 
   LAUNCH(CASSPEC_K_OTHER, launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->status, s,
                                            pdl));
-  LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, m->x, s, pdl));
+  LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, m->x, m->ssp, s, pdl));
 
   EpiParams base = {};
   base.n = n;
@@ -272,52 +280,86 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   base.pos = m->pos;
   base.rope = kv->rope;
 
-  auto gemm = [&](const CUtensorMap& tw, const CUtensorMap& tw2, const CUtensorMap& tx, int epi, int tiles,
-                  int kblocks, const EpiParams& e) -> cudaError_t {
-    GemmArgs a = {};
-    a.tiles = tiles;
-    a.kblocks = kblocks;
-    a.partials = m->gemm_part;
-    a.counters = m->gemm_cnt;
-    a.status = m->status;
-    a.ep = e;
-    return launch_gemm_bf16(tw, tw2, tx, BN, epi, a, gemm_bf16_grid(tiles, kblocks, m->num_sms), s, pdl);
+  // ---- phase descriptors of the projection chain ----
+  auto ph_qkv = [&](int l, int ss_tiles, PhaseDesc& p, CUtensorMap& w) {
+    p = PhaseDesc{};
+    p.epi = EPI_QKV;
+    p.tiles = 3 * d / 128;
+    p.kblocks = cdiv(d, 64);
+    p.K = d;
+    p.in = m->x;
+    p.ld_in = d;
+    p.ss = m->ssp;
+    p.ss_tiles = ss_tiles;
+    p.g = m->layers[l].attn_norm;
+    p.eps = c.rms_eps;
+    p.ep = base;
+    p.ep.N = 3 * d;
+    p.ep.q_out = m->q;
+    p.ep.kc = kv_layer_k(kv, l);
+    p.ep.vc = kv_layer_v(kv, l);
+    w = m->layers[l].tm_qkv;
   };
-  auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
-                   int epi, const EpiParams& e) -> cudaError_t {
-    GemmI8Args a = {};
-    a.W = W;
-    a.sw = sw;
-    a.W2 = W2;
-    a.sw2 = sw2;
-    a.X = m->xq;
-    a.sx = m->xs;
-    a.N = N;
-    a.K = K;
-    a.tiles = tiles;
-    a.ksplit = gemm_i8_ksplit(tiles, K, m->num_sms);
-    a.partials = m->i8_part;
-    a.counters = m->i8_cnt;
-    a.status = m->status;
-    a.ep = e;
-    return launch_gemm_i8(a, BN, epi, s, pdl);
+  auto ph_resid = [&](const float* in, int K, PhaseDesc& p) {
+    p = PhaseDesc{};
+    p.epi = EPI_RESID;
+    p.tiles = d / 128;
+    p.kblocks = cdiv(K, 64);
+    p.K = K;
+    p.in = in;
+    p.ld_in = K;
+    p.ep = base;
+    p.ep.N = d;
+    p.ep.y = m->x;
+    p.ep.ldy = d;
+    p.ep.ss_out = m->ssp;
   };
-
-  for (int l = 0; l < c.n_layers; ++l) {
-    if (!on[l]) continue;
-    LayerPtrs& Lp = m->layers[l];
-    // attention block
-    LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
-                      pdl));
-    EpiParams e = base;
-    e.N = 3 * d;
-    e.q_out = m->q;
-    e.kc = kv_layer_k(kv, l);
-    e.vc = kv_layer_v(kv, l);
-    if (mode == 0)
-      LAUNCH(CASSPEC_K_QKV, gemm(Lp.tm_qkv, Lp.tm_qkv, m->tm_xn[bi], EPI_QKV, 3 * d / 128, cdiv(d, 64), e));
-    else
-      LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+  auto ph_gu = [&](int l, PhaseDesc& p) {
+    p = PhaseDesc{};
+    p.epi = EPI_GLU;
+    p.tiles = cdiv(F, 64);
+    p.kblocks = cdiv(d, 64);
+    p.K = d;
+    p.in = m->x;
+    p.ld_in = d;
+    p.ss = m->ssp;
+    p.ss_tiles = d / 128;
+    p.g = m->layers[l].ffn_norm;
+    p.eps = c.rms_eps;
+    p.ep = base;
+    p.ep.N = F;
+    p.ep.u_out = m->u;
+  };
+  auto ph_lm = [&](int ss_tiles, PhaseDesc& p, CUtensorMap& w) {
+    p = PhaseDesc{};
+    p.epi = EPI_LMHEAD;
+    p.tiles = m->lay.lm_tiles;
+    p.kblocks = cdiv(d, 64);
+    p.K = d;
+    p.in = m->x;
+    p.ld_in = d;
+    p.ss = m->ssp;
+    p.ss_tiles = ss_tiles;
+    p.g = m->final_norm;
+    p.eps = c.rms_eps;
+    p.ep = base;
+    p.ep.N = V;
+    p.ep.logits = logits;
+    p.ep.am_v1 = m->am_v1;
+    p.ep.am_i1 = m->am_i1;
+    p.ep.am_v2 = m->am_v2;
+    w = m->tm_lm;
+  };
+  const int cgrid = chain_grid(m->num_sms);
+  auto chain = [&](ChainArgs& ca, ChainMaps& cm, int kind) -> int {
+    ca.partials = m->gemm_part;
+    ca.counters = m->chain_cnt;
+    ca.bar = m->chain_bar;
+    ca.status = m->status;
+    LAUNCH(kind, launch_chain(cm, ca, BN, cgrid, s, pdl));
+    return CASSPEC_OK;
+  };
+  auto attention = [&](int l) -> int {
     AttnArgs at = {};
     at.q = m->q;
     at.o = m->o;
@@ -333,41 +375,96 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     at.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
     at.status = m->status;
     LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(kv->tm_kv, at, hd, s, pdl));
-    EpiParams er = base;
-    er.N = d;
-    er.y = m->x;
-    er.ldy = d;
-    if (mode == 0) {
-      LAUNCH(CASSPEC_K_WO, gemm(Lp.tm_o, Lp.tm_o, m->tm_oact[bi], EPI_RESID, d / 128, cdiv(d, 64), er));
+    return CASSPEC_OK;
+  };
+
+  if (mode == 0) {
+    ChainArgs ca = {};
+    ChainMaps cm = {};
+    int rc;
+    if (act.empty()) {
+      ca.nphases = 1;
+      ph_lm(1, ca.ph[0], cm.w[0]);
+      if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
     } else {
-      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
+      ca.nphases = 1;
+      ph_qkv(act[0], 1, ca.ph[0], cm.w[0]);
+      if ((rc = chain(ca, cm, CASSPEC_K_QKV)) != CASSPEC_OK) return rc;
+      for (size_t i = 0; i < act.size(); ++i) {
+        const int l = act[i];
+        if ((rc = attention(l)) != CASSPEC_OK) return rc;
+        ChainArgs cb = {};
+        ChainMaps cn = {};
+        cb.nphases = 4;
+        ph_resid(m->o, d, cb.ph[0]);
+        cn.w[0] = m->layers[l].tm_o;
+        ph_gu(l, cb.ph[1]);
+        cn.w[1] = m->layers[l].tm_g;
+        cn.w2[1] = m->layers[l].tm_u;
+        ph_resid(m->u, F, cb.ph[2]);
+        cn.w[2] = m->layers[l].tm_d;
+        if (i + 1 < act.size())
+          ph_qkv(act[i + 1], d / 128, cb.ph[3], cn.w[3]);
+        else
+          ph_lm(d / 128, cb.ph[3], cn.w[3]);
+        if ((rc = chain(cb, cn, CASSPEC_K_GATEUP)) != CASSPEC_OK) return rc;
+      }
+    }
+  } else {
+    auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
+                     int epi, const EpiParams& e) -> cudaError_t {
+      GemmI8Args g8 = {};
+      g8.W = W;
+      g8.sw = sw;
+      g8.W2 = W2;
+      g8.sw2 = sw2;
+      g8.X = m->xq;
+      g8.sx = m->xs;
+      g8.N = N;
+      g8.K = K;
+      g8.tiles = tiles;
+      g8.ksplit = gemm_i8_ksplit(tiles, K, m->num_sms);
+      g8.partials = m->i8_part;
+      g8.counters = m->i8_cnt;
+      g8.status = m->status;
+      g8.ep = e;
+      return launch_gemm_i8(g8, BN, epi, s, pdl);
+    };
+    for (size_t i = 0; i < act.size(); ++i) {
+      const int l = act[i];
+      LayerPtrs& Lp = m->layers[l];
+      LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
+      EpiParams e = base;
+      e.N = 3 * d;
+      e.q_out = m->q;
+      e.kc = kv_layer_k(kv, l);
+      e.vc = kv_layer_v(kv, l);
+      LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+      int rc;
+      if ((rc = attention(l)) != CASSPEC_OK) return rc;
+      EpiParams er = base;
+      er.N = d;
+      er.y = m->x;
+      er.ldy = d;
+      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows_f32(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
       LAUNCH(CASSPEC_K_WO, gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, er));
-    }
-    // feed-forward block
-    LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, mode ? nullptr : m->xn, mode ? m->xq : nullptr, m->xs, s,
-                      pdl));
-    EpiParams eg = base;
-    eg.N = F;
-    eg.u_out = m->u;
-    if (mode == 0)
-      LAUNCH(CASSPEC_K_GATEUP, gemm(Lp.tm_g, Lp.tm_u, m->tm_xn[bi], EPI_GLU, cdiv(F, 64), cdiv(d, 64), eg));
-    else
+      LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
+      EpiParams eg = base;
+      eg.N = F;
+      eg.u_out = m->u;
       LAUNCH(CASSPEC_K_GATEUP, gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
-    if (mode == 0) {
-      LAUNCH(CASSPEC_K_DOWN, gemm(Lp.tm_d, Lp.tm_d, m->tm_uact[bi], EPI_RESID, d / 128, cdiv(F, 64), er));
-    } else {
-      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
-      LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, er));
+      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows_f32(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
+      EpiParams ed = er;
+      ed.ss_out = m->ssp;  // the LM head's RMSNorm scale
+      LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
     }
+    ChainArgs ca = {};
+    ChainMaps cm = {};
+    ca.nphases = 1;
+    ph_lm(act.empty() ? 1 : d / 128, ca.ph[0], cm.w[0]);
+    int rc;
+    if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
   }
-  LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, m->final_norm, n, d, c.rms_eps, m->xn, nullptr, nullptr, s, pdl));
-  EpiParams el = base;
-  el.N = V;
-  el.logits = logits;
-  el.am_v1 = m->am_v1;
-  el.am_i1 = m->am_i1;
-  el.am_v2 = m->am_v2;
-  LAUNCH(CASSPEC_K_LMHEAD, gemm(m->tm_lm, m->tm_lm, m->tm_xn[bi], EPI_LMHEAD, m->lay.lm_tiles, cdiv(d, 64), el));
   LAUNCH(CASSPEC_K_OTHER, launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, m->lay.lm_tiles, n, m->am, m->margin, s, pdl));
   return CASSPEC_OK;
 }
@@ -385,12 +482,6 @@ bool build_tensor_maps(casspec_model* m) {
     ok = ok && encode_tmap_bf16(&Lp.tm_d, Lp.wd, F, d, F * 2, 64, 128);
   }
   ok = ok && encode_tmap_bf16(&m->tm_lm, m->lm_head, d, V, d * 2, 64, 128);
-  for (int b = 0; b < 4; ++b) {
-    const uint32_t BN = 16 * (b + 1);
-    ok = ok && encode_tmap_bf16(&m->tm_xn[b], m->xn, d, kMaxTree, d * 2, 64, BN);
-    ok = ok && encode_tmap_bf16(&m->tm_oact[b], m->o, d, kMaxTree, d * 2, 64, BN);
-    ok = ok && encode_tmap_bf16(&m->tm_uact[b], m->u, F, kMaxTree, F * 2, 64, BN);
-  }
   return ok;
 }
 
@@ -448,10 +539,12 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
     }
   }
   m->x = reinterpret_cast<float*>(b + L.x);
-  m->xn = reinterpret_cast<uint16_t*>(b + L.xn);
   m->q = reinterpret_cast<uint16_t*>(b + L.q);
-  m->o = reinterpret_cast<uint16_t*>(b + L.o);
-  m->u = reinterpret_cast<uint16_t*>(b + L.u);
+  m->o = reinterpret_cast<float*>(b + L.o);
+  m->u = reinterpret_cast<float*>(b + L.u);
+  m->ssp = reinterpret_cast<float*>(b + L.ssp);
+  m->chain_cnt = reinterpret_cast<unsigned*>(b + L.chain_cnt);
+  m->chain_bar = reinterpret_cast<unsigned*>(b + L.chain_bar);
   m->xq = reinterpret_cast<int8_t*>(b + L.xq);
   m->xs = reinterpret_cast<float*>(b + L.xs);
   m->pos = reinterpret_cast<int*>(b + L.pos);
@@ -787,6 +880,8 @@ int casspec_get_status(casspec_model* m, int* status_out) {
     CK(cudaMemset(m->status, 0, 4));
     CK(cudaMemset(m->gemm_cnt, 0, (size_t)m->lay.max_tiles * 4));
     CK(cudaMemset(m->i8_cnt, 0, (size_t)m->lay.max_tiles * 4));
+    CK(cudaMemset(m->chain_cnt, 0, (size_t)kMaxPhases * 1024 * 4));
+    CK(cudaMemset(m->chain_bar, 0, 256));
   }
   if (status_out) *status_out = st;
   return CASSPEC_OK;

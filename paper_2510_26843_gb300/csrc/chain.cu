@@ -1,0 +1,480 @@
+// Persistent projection chain on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+//
+// One launch runs a list of dependent projections of a tree step -- e.g. Wo (+residual), Wgate/Wup
+// (+SwiGLU), Wdown (+residual), and the next layer's Wqkv (+rotary, K/V write) -- with a grid-wide
+// barrier between phases.  Only the activations depend on the previous phase; the weights do not,
+// so the weight stream runs on across phase boundaries and the HBM pipeline never drains between
+// projections.  Per CTA (one per SM):
+//   * warp 0 -- TMA producer: streams the CTA's weight tiles (128 x 64 bf16, 128-byte swizzle,
+//     L2 evict-first) of every phase through a deep mbarrier ring, never waiting on activations;
+//   * warps 6-9 -- activation transform: after the phase barrier, build the B operand tile of each
+//     k-block from fp32 rows (the residual stream scaled by its RMSNorm factor and gains, the
+//     attention output, or the SwiGLU output), split into hi + lo bf16 parts (16 significant bits)
+//     and stored in the MMA's swizzled K-major layout;
+//   * warp 1 -- TMEM owner and single-thread MMA issuer: D += W * hi^T + W * lo^T (tcgen05.mma
+//     kind::f16, M = 128 channels, N = BN tokens), double-buffered accumulators in TMEM;
+//   * warps 2-5 -- epilogue: TMEM -> registers, stream-K fix-up (last CTA of a tile sums the partials
+//     in CTA order), fused epilogue; then the CTA's arrival at the phase barrier.
+// Work of each phase is split stream-K over (tile, k-block) units so all SMs stream equal bytes.
+// Every wait is bounded (2 s) and reports CASSPEC_E_TIMEOUT instead of hanging.
+#include "common.cuh"
+#include "epilogue.cuh"
+#include "kernels.h"
+
+namespace casspec {
+
+constexpr int kChainThreads = 320;
+constexpr uint32_t kWTile = 128 * 128;  // 128 rows x 64 bf16
+constexpr int kXStages = 3;
+constexpr uint32_t kChainSmemBudget = 232448u;  // 227 KB per CTA
+
+__host__ __device__ constexpr uint32_t chain_x_stage(int BN) { return 2u * (uint32_t)BN * 128u; }
+__host__ __device__ constexpr uint32_t chain_staging(int BN) { return 128u * (uint32_t)(BN + 1) * 4u; }
+__host__ __device__ constexpr uint32_t chain_fixed(int BN) {
+  return 1024u + kXStages * chain_x_stage(BN) + chain_staging(BN) + 64u * 4u + 512u;
+}
+__host__ __device__ constexpr int chain_w_stages(int BN) {
+  return (int)((kChainSmemBudget - chain_fixed(BN)) / kWTile) > 12 ? 12
+                                                                   : (int)((kChainSmemBudget - chain_fixed(BN)) / kWTile);
+}
+__host__ __device__ constexpr size_t chain_smem(int BN) { return chain_fixed(BN) + (size_t)chain_w_stages(BN) * kWTile; }
+__host__ __device__ constexpr uint32_t chain_tmem_cols(int BN) { return 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : 128); }
+
+__device__ __forceinline__ int chain_cta_of(long long x, long long U, int G) {
+  return (int)(((x + 1) * (long long)G - 1) / U);
+}
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
+template <int BN, typename Bar>
+__device__ __forceinline__ void chain_epilogue(int epi, const EpiParams& e, int tile, int r, const float* v, float* stg,
+                                               Bar bar) {
+  switch (epi) {
+    case EPI_RESID: run_epilogue<BN, EPI_RESID>(e, tile, r, v, stg, bar); break;
+    case EPI_QKV: run_epilogue<BN, EPI_QKV>(e, tile, r, v, stg, bar); break;
+    case EPI_GLU: run_epilogue<BN, EPI_GLU>(e, tile, r, v, stg, bar); break;
+    case EPI_LMHEAD: run_epilogue<BN, EPI_LMHEAD>(e, tile, r, v, stg, bar); break;
+    default: run_epilogue<BN, EPI_STORE>(e, tile, r, v, stg, bar); break;
+  }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kChainThreads, 1)
+    chain_kernel(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs a) {
+  constexpr int SW = chain_w_stages(BN);
+  constexpr int SX = kXStages;
+  constexpr uint32_t XT = (uint32_t)BN * 128u;  // one hi or lo tile
+  constexpr uint32_t XS = 2 * XT;
+  constexpr uint32_t TMEM_COLS = chain_tmem_cols(BN);
+  constexpr uint32_t IDESC = idesc_bf16_f32(128, BN);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* wring = smem;
+  uint8_t* xring = smem + SW * kWTile;
+  float* stg = reinterpret_cast<float*>(xring + SX * XS);
+  float* rs = stg + 128 * (BN + 1);
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(rs + 64);
+  uint64_t* wempty = wfull + SW;
+  uint64_t* xfull = wempty + SW;
+  uint64_t* xempty = xfull + SX;
+  uint64_t* tfull = xempty + SX;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  // [0] abort, [1] last-arriver, [2..9] per-warp accumulator-ready votes (two segments), [10] go
+  volatile int* flags = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = gridDim.x, cta = blockIdx.x;
+  const int np = a.nphases;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < SW; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], 1);
+    }
+    for (int s = 0; s < SX; ++s) {
+      mbar_init(&xfull[s], 4);
+      mbar_init(&xempty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
+    mbar_init(drain, 1);
+    flags[0] = 0;
+    flags[1] = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    for (int p = 0; p < np; ++p) {
+      tma_prefetch_desc(&maps.w[p]);
+      if (a.ph[p].epi == EPI_GLU) tma_prefetch_desc(&maps.w2[p]);
+    }
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- weight producer (never waits on activations) ----------------
+      const uint64_t pol = policy_evict_first();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, armed_parity = 0;
+      for (int p = 0; p < np && !flags[0]; ++p) {
+        const PhaseDesc& ph = a.ph[p];
+        const int kb = ph.kblocks;
+        const long long U = (long long)ph.tiles * kb;
+        const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
+        for (long long u = u0; u < u1; ++u) {
+          if (!mbar_wait_bounded(&wempty[stage], phase ^ 1, flags)) {
+            flags[0] = 1;
+            set_status(a.status, CASSPEC_E_TIMEOUT);
+            break;
+          }
+          const int t = (int)(u / kb), k = (int)(u % kb);
+          mbar_expect_tx(&wfull[stage], kWTile);
+          armed |= 1u << stage;
+          armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
+          uint8_t* sa = wring + stage * kWTile;
+          if (ph.epi == EPI_GLU) {
+            tma_load_2d(sa, &maps.w[p], &wfull[stage], k * 64, t * 64, pol);
+            tma_load_2d(sa + kWTile / 2, &maps.w2[p], &wfull[stage], k * 64, t * 64, pol);
+          } else {
+            tma_load_2d(sa, &maps.w[p], &wfull[stage], k * 64, t * 128, pol);
+          }
+          if (++stage == SW) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (flags[0]) {  // abort: let the copies already issued land before the CTA exits
+        for (int s = 0; s < SW; ++s)
+          if (armed & (1u << s)) mbar_wait_bounded(&wfull[s], (armed_parity >> s) & 1, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      int ws = 0, xs = 0;
+      uint32_t wph = 0, xph = 0;
+      uint32_t used[2] = {0, 0};
+      int buf = 0;
+      bool ok = true;
+      for (int p = 0; p < np && ok; ++p) {
+        const PhaseDesc& ph = a.ph[p];
+        const int kb = ph.kblocks;
+        const long long U = (long long)ph.tiles * kb;
+        const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
+        long long u = u0;
+        while (u < u1 && ok) {
+          const int t = (int)(u / kb);
+          const long long seg_end = ((long long)(t + 1) * kb < u1) ? (long long)(t + 1) * kb : u1;
+          if (!mbar_wait_bounded(&tempty[buf], (used[buf] & 1) ^ 1, flags)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+          for (long long uu = u; uu < seg_end; ++uu) {
+            if (!mbar_wait_bounded(&wfull[ws], wph, flags) || !mbar_wait_bounded(&xfull[xs], xph, flags)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(wring + ws * kWTile);
+            const uint32_t sh = smem_u32(xring + xs * XS), sl = sh + XT;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint64_t ad = sw128_kmajor_desc(sa + kk * 32);
+              tc_mma_bf16(d_tmem, ad, sw128_kmajor_desc(sh + kk * 32), IDESC, (uu > u || kk > 0) ? 1u : 0u);
+              tc_mma_bf16(d_tmem, ad, sw128_kmajor_desc(sl + kk * 32), IDESC, 1u);
+            }
+            tc_commit(&wempty[ws]);
+            tc_commit(&xempty[xs]);
+            if (++ws == SW) {
+              ws = 0;
+              wph ^= 1;
+            }
+            if (++xs == SX) {
+              xs = 0;
+              xph ^= 1;
+            }
+          }
+          if (!ok) break;
+          tc_commit(&tfull[buf]);
+          used[buf]++;
+          buf ^= 1;
+          u = seg_end;
+        }
+      }
+      if (!ok) {
+        flags[0] = 1;
+        set_status(a.status, CASSPEC_E_TIMEOUT);
+      }
+      tc_commit(drain);  // all MMAs complete before TMEM is released
+      mbar_wait_bounded(drain, 0, nullptr);
+    }
+  } else if (warp < 6) {
+    // ---------------- epilogue warps 2..5 ----------------
+    // Control flow is identical in the four warps (every decision that follows a bounded wait is
+    // voted through shared memory), so their named barriers always match, even after a timeout.
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    auto bar = [] { named_bar_sync(1, 128); };
+    uint32_t used[2] = {0, 0};
+    int buf = 0, seg = 0;
+    for (int p = 0; p < np; ++p) {
+      const PhaseDesc& ph = a.ph[p];
+      const int kb = ph.kblocks;
+      const long long U = (long long)ph.tiles * kb;
+      const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
+      unsigned* counters = a.counters + p * 1024;
+      long long u = u0;
+      while (u < u1) {
+        const int t = (int)(u / kb);
+        const long long seg_end = ((long long)(t + 1) * kb < u1) ? (long long)(t + 1) * kb : u1;
+        const bool got = mbar_wait_bounded(&tfull[buf], used[buf] & 1, flags);
+        if (lane == 0) flags[2 + (seg & 1) * 4 + q] = got ? 1 : 0;
+        bar();
+        const int vote = (seg & 1) * 4;
+        const bool ready = flags[2 + vote] && flags[3 + vote] && flags[4 + vote] && flags[5 + vote];
+        ++seg;
+        used[buf]++;
+        if (!ready) {  // the accumulator never arrived: give up on the rest (uniformly)
+          flags[0] = 1;
+          set_status(a.status, CASSPEC_E_TIMEOUT);
+          u = seg_end;
+          buf ^= 1;
+          continue;
+        }
+        tc_fence_after();
+        float v[BN];
+        const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
+#pragma unroll
+        for (int c = 0; c < BN; c += 16) tmem_ld_x16(taddr + c, &v[c]);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[buf]);
+        buf ^= 1;
+
+        const int c_first = chain_cta_of((long long)t * kb, U, G);
+        const int c_last = chain_cta_of((long long)(t + 1) * kb - 1, U, G);
+        bool finish = true;
+        if (c_first != c_last) {
+          float* mine = a.partials + (size_t)(t + cta) * (64 * 128);
+#pragma unroll
+          for (int i = 0; i < BN; ++i)
+            if (i < ph.ep.n) __stcg(mine + i * 128 + r, v[i]);
+          __threadfence();
+          bar();
+          if (threadIdx.x == 64) {
+            const unsigned old = atomicAdd(&counters[t], 1u);
+            flags[1] = (old == (unsigned)(c_last - c_first)) ? 1 : 0;
+          }
+          bar();
+          finish = flags[1] != 0;
+          if (finish) {
+            __threadfence();
+            float acc[BN];
+#pragma unroll
+            for (int i = 0; i < BN; ++i) acc[i] = 0.f;
+            for (int cc = c_first; cc <= c_last; ++cc) {
+              if (cc == cta) {
+#pragma unroll
+                for (int i = 0; i < BN; ++i) acc[i] += v[i];
+              } else {
+                const float* pp = a.partials + (size_t)(t + cc) * (64 * 128);
+#pragma unroll
+                for (int i = 0; i < BN; ++i)
+                  if (i < ph.ep.n) acc[i] += __ldcg(pp + i * 128 + r);
+              }
+            }
+#pragma unroll
+            for (int i = 0; i < BN; ++i) v[i] = acc[i];
+            if (threadIdx.x == 64) counters[t] = 0u;  // ready for the next launch
+          }
+        }
+        if (finish) chain_epilogue<BN>(ph.epi, ph.ep, t, r, v, stg, bar);
+        u = seg_end;
+      }
+      if (p + 1 < np) {  // this CTA's writes of phase p are done: arrive at the phase barrier
+        __threadfence();
+        bar();
+        if (threadIdx.x == 64) {
+          __threadfence();
+          atomicAdd(&a.bar[0], 1u);
+        }
+      }
+    }
+  } else {
+    // ---------------- activation transform warps 6..9 ----------------
+    // Thread tt == 0 alone polls the phase barrier and publishes the outcome before the named
+    // barrier; after an abort every wait below returns at once, so the loops run out uniformly.
+    const int tt = threadIdx.x - 192;  // 0..127
+    auto tbar = [] { named_bar_sync(2, 128); };
+    int xs = 0;
+    uint32_t xph = 0;
+    for (int p = 0; p < np; ++p) {
+      const PhaseDesc& ph = a.ph[p];
+      // the inputs of phase p were written by the previous kernel (p = 0) or by phase p - 1
+      if (p == 0) {
+        pdl_wait();
+      } else if (tt == 0) {
+        const unsigned target = (unsigned)p * (unsigned)G;
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_acquire_u32(a.bar) < target) {
+          if (flags[0]) break;
+          if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            flags[0] = 1;
+            set_status(a.status, CASSPEC_E_TIMEOUT);
+            break;
+          }
+        }
+      }
+      tbar();
+      const int n = ph.ep.n;
+      if (ph.ss != nullptr) {
+        if (tt < 64) {
+          float ssum = 0.f;
+          for (int t = 0; t < ph.ss_tiles; ++t) ssum += __ldcg(ph.ss + t * 64 + tt);
+          rs[tt] = tt < n ? rsqrtf(ssum / (float)ph.K + ph.eps) : 0.f;
+        }
+        tbar();
+      }
+      const int kb = ph.kblocks;
+      const long long U = (long long)ph.tiles * kb;
+      const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
+      for (long long u = u0; u < u1; ++u) {
+        const bool free_slot = mbar_wait_bounded(&xempty[xs], xph ^ 1, flags);
+        if (free_slot && !flags[0]) {
+          const int k = (int)(u % kb);
+          const uint32_t th = smem_u32(xring + xs * XS), tl = th + XT;
+          for (int item = tt; item < BN * 8; item += 128) {
+            const int row = item >> 3, c = item & 7;
+            const int col = k * 64 + c * 8;
+            float vv[8];
+            if (row < n && col < ph.K) {
+              const float4 f0 = __ldcg(reinterpret_cast<const float4*>(ph.in + (size_t)row * ph.ld_in + col));
+              const float4 f1 = __ldcg(reinterpret_cast<const float4*>(ph.in + (size_t)row * ph.ld_in + col + 4));
+              vv[0] = f0.x, vv[1] = f0.y, vv[2] = f0.z, vv[3] = f0.w, vv[4] = f1.x, vv[5] = f1.y, vv[6] = f1.z,
+              vv[7] = f1.w;
+              if (ph.ss != nullptr) {
+                const float sc = rs[row];
+                const float4 g0 = __ldg(reinterpret_cast<const float4*>(ph.g + col));
+                const float4 g1 = __ldg(reinterpret_cast<const float4*>(ph.g + col + 4));
+                vv[0] = vv[0] * sc * g0.x, vv[1] = vv[1] * sc * g0.y, vv[2] = vv[2] * sc * g0.z,
+                vv[3] = vv[3] * sc * g0.w;
+                vv[4] = vv[4] * sc * g1.x, vv[5] = vv[5] * sc * g1.y, vv[6] = vv[6] * sc * g1.z,
+                vv[7] = vv[7] * sc * g1.w;
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 8; ++j) vv[j] = 0.f;
+            }
+            uint32_t hi[4], lo[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const uint16_t h0 = f2bf(vv[2 * j]), h1 = f2bf(vv[2 * j + 1]);
+              hi[j] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+              lo[j] = pack_bf16x2(vv[2 * j] - bf2f(h0), vv[2 * j + 1] - bf2f(h1));
+            }
+            const uint32_t off = (uint32_t)row * 128u + ((uint32_t)(c ^ (row & 7)) << 4);
+            st_shared_v4(th + off, hi[0], hi[1], hi[2], hi[3]);
+            st_shared_v4(tl + off, lo[0], lo[1], lo[2], lo[3]);
+          }
+          fence_proxy_async_smem();  // generic-proxy smem writes -> visible to the tensor cores
+        } else if (!free_slot && !flags[0]) {
+          flags[0] = 1;
+          set_status(a.status, CASSPEC_E_TIMEOUT);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&xfull[xs]);
+        if (++xs == SX) {
+          xs = 0;
+          xph ^= 1;
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && np > 1) {  // the last CTA out resets the phase-barrier counters
+    __threadfence();
+    if (atomicAdd(&a.bar[1], 1u) == (unsigned)(G - 1)) {
+      a.bar[0] = 0u;
+      a.bar[1] = 0u;
+    }
+  }
+}
+
+int chain_grid(int num_sms) { return num_sms; }
+
+size_t chain_smem_bytes(int BN) {
+  switch (BN) {
+    case 16: return chain_smem(16);
+    case 32: return chain_smem(32);
+    case 48: return chain_smem(48);
+    default: return chain_smem(64);
+  }
+}
+
+template <int BN>
+static cudaError_t launch_bn(const ChainMaps& maps, const ChainArgs& args, int grid, cudaStream_t stream, bool pdl) {
+  auto kern = chain_kernel<BN>;
+  constexpr size_t smem = chain_smem(BN);
+  static int configured = -1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (configured != dev) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    configured = dev;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kChainThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, maps, args);
+}
+
+cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int BN, int grid, cudaStream_t stream, bool pdl) {
+  if (args.nphases < 1 || args.nphases > kMaxPhases) return cudaErrorInvalidValue;
+  switch (BN) {
+    case 16: return launch_bn<16>(maps, args, grid, stream, pdl);
+    case 32: return launch_bn<32>(maps, args, grid, stream, pdl);
+    case 48: return launch_bn<48>(maps, args, grid, stream, pdl);
+    case 64: return launch_bn<64>(maps, args, grid, stream, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace casspec

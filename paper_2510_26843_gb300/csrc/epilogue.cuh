@@ -59,7 +59,7 @@ __device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, con
       if (i < e.n) {
         const float g = v[i];
         const float up = stg[(r + 64) * (BN + 1) + i];
-        e.u_out[(size_t)i * e.N + ch] = f2bf(g / (1.f + expf(-g)) * up);
+        e.u_out[(size_t)i * e.N + ch] = g / (1.f + expf(-g)) * up;
       }
     }
   }
@@ -99,23 +99,45 @@ __device__ __forceinline__ void epi_lmhead(const EpiParams& e, int tile, int r, 
 }
 
 template <int BN>
-__device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, const float* v, bool store) {
+__device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, const float* v) {
   const int o = tile * 128 + r;
   if (o < e.N) {
 #pragma unroll
-    for (int i = 0; i < BN; ++i) {
-      if (i < e.n) {
-        float* p = e.y + (size_t)i * e.ldy + o;
-        *p = store ? v[i] : (__ldcg(p) + v[i]);
-      }
-    }
+    for (int i = 0; i < BN; ++i)
+      if (i < e.n) e.y[(size_t)i * e.ldy + o] = v[i];
   }
+}
+
+// y += v (fp32 residual stream); optionally the tile's per-token sum of squares of the updated rows,
+// the partial sums from which the next RMSNorm takes its scale (fixed order: deterministic).
+template <int BN, typename Bar>
+__device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+  const int o = tile * 128 + r;
+  const bool valid = o < e.N;
+#pragma unroll
+  for (int i = 0; i < BN; ++i) {
+    float nv = 0.f;
+    if (i < e.n && valid) {
+      float* p = e.y + (size_t)i * e.ldy + o;
+      nv = __ldcg(p) + v[i];
+      *p = nv;
+    }
+    if (e.ss_out != nullptr) stg[r * (BN + 1) + i] = nv * nv;
+  }
+  if (e.ss_out == nullptr) return;
+  bar();
+  if (r < e.n) {
+    float s = 0.f;
+    for (int row = 0; row < 128; ++row) s += stg[row * (BN + 1) + r];
+    e.ss_out[tile * 64 + r] = s;
+  }
+  bar();
 }
 
 template <int BN, int EPI, typename Bar>
 __device__ __forceinline__ void run_epilogue(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  if constexpr (EPI == EPI_STORE) epi_resid<BN>(e, tile, r, v, true);
-  if constexpr (EPI == EPI_RESID) epi_resid<BN>(e, tile, r, v, false);
+  if constexpr (EPI == EPI_STORE) epi_store<BN>(e, tile, r, v);
+  if constexpr (EPI == EPI_RESID) epi_resid<BN>(e, tile, r, v, stg, bar);
   if constexpr (EPI == EPI_QKV) epi_qkv<BN>(e, tile, r, v, stg, bar);
   if constexpr (EPI == EPI_GLU) epi_glu<BN>(e, tile, r, v, stg, bar);
   if constexpr (EPI == EPI_LMHEAD) epi_lmhead<BN>(e, tile, r, v, stg, bar);

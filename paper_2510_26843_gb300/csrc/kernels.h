@@ -30,8 +30,9 @@ struct EpiParams {
   const int* dP;        // device committed length P
   const int* pos;       // [n] position of each new node (P + depth)
   const float2* rope;   // [ctx][hd/2] (cos, sin) of p * base^(-2j/hd) for every position p
+  float* ss_out;        // EPI_RESID (optional): [tiles][64] sum over the tile's columns of updated y^2
   // EPI_GLU
-  uint16_t* u_out;      // [64][F] bf16
+  float* u_out;         // [64][F] fp32
   // EPI_LMHEAD
   float* logits;        // [n][V] fp32 or null
   float* am_v1;         // [tiles][64] partial max
@@ -67,7 +68,7 @@ struct GemmI8Args {
 
 struct AttnArgs {
   const uint16_t* q;    // [64][d] bf16 (rotated)
-  uint16_t* o;          // [64][d] bf16
+  float* o;             // [64][d] fp32
   const unsigned long long* anc;  // [n] ancestor masks over tree slots
   const int* dP;
   int T, n, ctx, d, n_heads;
@@ -75,6 +76,35 @@ struct AttnArgs {
   int cluster;          // CTAs per head (thread-block cluster size, <= 8)
   float scale_log2;     // log2(e) / sqrt(hd)
   int* status;
+};
+
+// One phase of the persistent projection chain: Y = A(X) W^T with A(X) built on the fly from fp32
+// rows (optionally RMS-normalised) and split into hi + lo bf16 parts.
+constexpr int kMaxPhases = 4;
+struct PhaseDesc {
+  int epi;           // EPI_QKV, EPI_RESID, EPI_GLU or EPI_LMHEAD
+  int tiles;         // 128-row output tiles (EPI_GLU: 64 gate + 64 up rows per tile)
+  int kblocks;       // ceil(K / 64)
+  int K;             // input width
+  const float* in;   // fp32 input rows [64][ld_in]
+  int ld_in;
+  const float* ss;   // normalise rows: per-tile partial sums of squares [ss_tiles][64] (null: no norm)
+  int ss_tiles;
+  const float* g;    // RMSNorm gains [K]
+  float eps;
+  EpiParams ep;
+};
+struct ChainArgs {
+  int nphases;
+  PhaseDesc ph[kMaxPhases];
+  float* partials;     // stream-K partial tiles (shared by the phases)
+  unsigned* counters;  // [kMaxPhases][1024] fix-up counters, zero between launches
+  unsigned* bar;       // [2] grid-barrier counters, zero between launches
+  int* status;
+};
+struct ChainMaps {
+  CUtensorMap w[kMaxPhases];   // weights (EPI_GLU: gate)
+  CUtensorMap w2[kMaxPhases];  // EPI_GLU: up
 };
 
 // ---- launchers (return cudaSuccess or the launch error) ----
@@ -93,12 +123,17 @@ cudaError_t launch_tree_attention(const CUtensorMap& tmKV, const AttnArgs& a, in
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
                              int* pos, unsigned long long* anc_new, int* status, cudaStream_t s, bool pdl);
-cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, cudaStream_t s,
-                         bool pdl);
+cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, float* ss,
+                         cudaStream_t s, bool pdl);
+int chain_grid(int num_sms);
+size_t chain_smem_bytes(int BN);
+cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int BN, int grid, cudaStream_t stream, bool pdl);
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
                            cudaStream_t s, bool pdl);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
                               bool pdl);
+cudaError_t launch_quant_rows_f32(const float* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
+                                  bool pdl);
 cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,
                                  float* margin, cudaStream_t s, bool pdl);
 cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s);

@@ -84,30 +84,6 @@ cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int
 }
 
 // ---------------------------------------------------------------------------------------------
-// Embedding gather: x[i][:] = E[tokens[i]][:] widened to the fp32 residual stream.
-// ---------------------------------------------------------------------------------------------
-__global__ void embed_kernel(const uint16_t* __restrict__ E, const int* __restrict__ tokens, int d, int vocab,
-                             float* __restrict__ x) {
-  pdl_trigger();
-  pdl_wait();
-  const int i = blockIdx.x;
-  int tok = __ldcg(tokens + i);
-  tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);
-  const uint16_t* row = E + (size_t)tok * d;
-  for (int c = threadIdx.x * 2; c < d; c += blockDim.x * 2) {
-    const uint32_t two = *reinterpret_cast<const uint32_t*>(row + c);
-    *reinterpret_cast<float2*>(x + (size_t)i * d + c) = make_float2(bf2f(two & 0xFFFF), bf2f(two >> 16));
-  }
-}
-
-cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, cudaStream_t s,
-                         bool pdl) {
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, embed_kernel, E, tokens, d, vocab, x);
-}
-
-// ---------------------------------------------------------------------------------------------
 // Block reductions (256 threads)
 // ---------------------------------------------------------------------------------------------
 __device__ __forceinline__ float block_sum(float v, float* red) {
@@ -138,6 +114,37 @@ __device__ __forceinline__ int8_t quant_one(float x, float inv) {
   int q = __float2int_rn(__fmul_rn(x, inv));
   q = q > 127 ? 127 : (q < -127 ? -127 : q);
   return (int8_t)q;
+}
+
+// ---------------------------------------------------------------------------------------------
+// Embedding gather: x[i][:] = E[tokens[i]][:] widened to the fp32 residual stream, plus the row's
+// sum of squares (the first RMSNorm's scale), ss[i].
+// ---------------------------------------------------------------------------------------------
+__global__ void embed_kernel(const uint16_t* __restrict__ E, const int* tokens, int d, int vocab,
+                             float* __restrict__ x, float* __restrict__ ss) {
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x;
+  int tok = __ldcg(tokens + i);
+  tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);
+  const uint16_t* row = E + (size_t)tok * d;
+  float acc = 0.f;
+  for (int c = threadIdx.x * 2; c < d; c += blockDim.x * 2) {
+    const uint32_t two = *reinterpret_cast<const uint32_t*>(row + c);
+    const float f0 = bf2f(two & 0xFFFF), f1 = bf2f(two >> 16);
+    *reinterpret_cast<float2*>(x + (size_t)i * d + c) = make_float2(f0, f1);
+    acc += f0 * f0 + f1 * f1;
+  }
+  acc = block_sum(acc, red);
+  if (threadIdx.x == 0) ss[i] = acc;
+}
+
+cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, float* ss,
+                         cudaStream_t s, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, embed_kernel, E, tokens, d, vocab, x, ss);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -270,6 +277,54 @@ cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* 
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
   return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq);
+}
+
+// Per-row int8 quantisation of fp32 rows as stored in bf16 (each value is rounded to bf16 first,
+// the precision in which the W8A8 draft keeps its activations).
+__global__ void __launch_bounds__(kRowThreads) quant_rows_f32_kernel(const float* __restrict__ x, int d, int ldx,
+                                                                     int8_t* __restrict__ q, int ldq,
+                                                                     float* __restrict__ sq) {
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x;
+  const int nv = d / 4;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)i * ldx);
+  float4 xv[kRowVec];
+  float amax = 0.f;
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    xv[k] = c < nv ? __ldcg(xr + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    xv[k].x = bf2f(f2bf(xv[k].x));
+    xv[k].y = bf2f(f2bf(xv[k].y));
+    xv[k].z = bf2f(f2bf(xv[k].z));
+    xv[k].w = bf2f(f2bf(xv[k].w));
+    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(xv[k].x), fabsf(xv[k].y)), fmaxf(fabsf(xv[k].z), fabsf(xv[k].w))));
+  }
+  amax = block_max(amax, red);
+  const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int c = threadIdx.x + k * kRowThreads;
+    if (c < nv) {
+      char4 o;
+      o.x = amax > 0.f ? quant_one(xv[k].x, inv) : 0;
+      o.y = amax > 0.f ? quant_one(xv[k].y, inv) : 0;
+      o.z = amax > 0.f ? quant_one(xv[k].z, inv) : 0;
+      o.w = amax > 0.f ? quant_one(xv[k].w, inv) : 0;
+      reinterpret_cast<char4*>(q + (size_t)i * ldq)[c] = o;
+    }
+  }
+  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
+}
+
+cudaError_t launch_quant_rows_f32(const float* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
+                                  bool pdl) {
+  if (d % 4 != 0 || ldx % 4 != 0 || ldq % 4 != 0 || d > 4 * kRowVec * kRowThreads) return cudaErrorInvalidValue;
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, quant_rows_f32_kernel, x, d, ldx, q, ldq, sq);
 }
 
 // ---------------------------------------------------------------------------------------------
