@@ -9,7 +9,8 @@ times over, so no L2 flush is needed between steps.
 
 Output: one JSON line (rank 0).  value = device-timed step latency in microseconds (lower is
 better); e2e = the same through the C ABI with host-resident inputs copied in and the accepted
-path copied out every step; roofline = the dominant kernel (gate/up projection) from a separate
+path copied out every step; roofline = the dominant kernel (bf16: the per-layer projection chain
+Wo -> gate/up -> down -> next QKV or LM head; int8: the W8A8 gate/up projection) from a separate
 kernel-timing pass with CUDA events around each launch; cpu_baseline = the fp64 oracle on a
 bounded sample (embedding + 1 of 32 layers + LM head, scaled to 32 layers) on the host cores.
 
@@ -70,6 +71,17 @@ def algorithmic_bytes(shape, n: int, P: int, layers_on: int | None = None, quant
             "total": w + lm + kv_read + kv_write + logits}
 
 
+def chain_bytes(shape, n: int, layers_on: int) -> int:
+    """Mean algorithmic bytes of one per-layer chain launch (bf16 mode): Wo, Wg, Wu, Wd and the next
+    active layer's Wqkv (the LM head after the last layer) read once; the attention output read
+    (bf16), the residual stream read and written twice (fp32), the SwiGLU output written and read
+    (bf16), q written and the new K/V written (bf16), the logits written once (fp32)."""
+    d, F, V, L = shape.d_model, shape.ffn, shape.vocab, layers_on
+    w = L * (d * d + 3 * F * d) * 2 + (L - 1) * 3 * d * d * 2 + V * d * 2
+    act = L * (n * d * 2 + 4 * n * d * 4 + 2 * n * F * 2) + (L - 1) * 3 * n * d * 2 + n * V * 4
+    return (w + act) // L
+
+
 def gateup_bytes(shape, n: int, quant: int = 0) -> int:
     """Wg, Wu read (+ row scales) + activations read + U written (bf16)."""
     d, F = shape.d_model, shape.ffn
@@ -88,10 +100,10 @@ def measured_peaks() -> tuple[float, str]:
 
 
 def recorded_traffic() -> float | None:
-    """DRAM bytes per launch of the gate/up projection from the committed ncu summary, if it was taken
-    on the current kernel source (the summary records the source hash)."""
-    path = os.path.join(ROOT, "profiles", "gemm_bf16_gateup_7b_n64.md")
-    src = os.path.join(ROOT, "paper_2510_26843_gb300", "csrc", "gemm_tc.cu")
+    """DRAM bytes per launch of the per-layer chain kernel from the committed ncu summary, if it was
+    taken on the current kernel source (the summary records the source hash)."""
+    path = os.path.join(ROOT, "profiles", "chain_7b_verify_n64.md")
+    src = os.path.join(ROOT, "paper_2510_26843_gb300", "csrc", "chain.cu")
     try:
         text = open(path).read()
         h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
@@ -357,6 +369,7 @@ def run_gpu(args) -> None:
     for _ in range(args.steps):
         step()
     per_kind = {}
+    # bf16 mode: "qkv" is the first layer's QKV chain launch, "gateup" the per-layer chains
     names = ["qkv", "attention", "wo", "gateup", "down", "lm_head", "other"]
     for k, name in enumerate(names):
         tot, cnt = cs.profile_read(dm.h, k)
@@ -368,11 +381,12 @@ def run_gpu(args) -> None:
         raise RuntimeError(f"device status after timing: {st} ({cs.status_string(st)})")
 
     peak, peak_kind = measured_peaks()
-    gu_bytes = gateup_bytes(sh, n, mode)
+    gu_bytes = gateup_bytes(sh, n, mode) if mode else chain_bytes(sh, n, layers_on)
     gu_avg_s = per_kind["gateup"]["avg_us"] * 1e-6
     achieved = gu_bytes / gu_avg_s / 1e9
     ab = algorithmic_bytes(sh, n, P, layers_on, mode)
-    kern = "gemm_i8_kernel (W8A8 gate/up + SwiGLU)" if mode else "gemm_bf16_tc_kernel (gate/up + SwiGLU)"
+    kern = ("gemm_i8_kernel (W8A8 gate/up + SwiGLU)" if mode else
+            "chain_kernel (Wo + residual, gate/up + SwiGLU, down + residual, next QKV or LM head)")
 
     out = {
         "metric": METRIC, "value": round(us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,

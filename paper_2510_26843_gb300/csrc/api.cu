@@ -34,7 +34,7 @@ struct Layout {
   size_t embed, lm_head, final_norm;
   std::vector<size_t> attn_norm, ffn_norm, wqkv, wo, wg, wu, wd;
   std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
-  size_t x, q, o, u, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
+  size_t x, q, o, u, xa, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
   size_t gemm_part, gemm_cnt, chain_cnt, chain_bar, i8_part, i8_cnt, status;
   size_t scratch_begin;
   int max_tiles, lm_tiles;
@@ -96,8 +96,9 @@ Layout make_layout(const casspec_model_config& c) {
   L.max_tiles = std::max(std::max(cdiv(3 * d, 128), cdiv(F, 64)), L.lm_tiles);
   L.x = take(T * d * 4);
   L.q = take(T * d * 2);
-  L.o = take(T * d * 4);
-  L.u = take(T * F * 4);
+  L.o = take(2 * T * d * 2);  // split activations: hi plane rows 0..63, lo plane rows 64..127
+  L.u = take(2 * T * F * 2);
+  L.xa = take(2 * T * d * 2);
   L.xq = take(T * std::max(d, F));
   L.xs = take(T * 4);
   L.ssp = take((size_t)std::max<size_t>(d / 128, 1) * T * 4);
@@ -156,8 +157,9 @@ struct casspec_model {
   float* final_norm;
   std::vector<LayerPtrs> layers;
   CUtensorMap tm_lm;
-  float *x, *o, *u, *ssp;
-  uint16_t* q;
+  float *x, *ssp;
+  uint16_t *q, *o, *u, *xa;       // o, u, xa: split activations [128][K] bf16 (hi, lo planes)
+  CUtensorMap tm_o[4], tm_u[4], tm_xa[4];  // their 64 x BN boxes, BN = 16, 32, 48, 64
   int8_t* xq;
   float* xs;
   unsigned *chain_cnt, *chain_bar;
@@ -268,7 +270,10 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
 
   LAUNCH(CASSPEC_K_OTHER, launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->status, s,
                                            pdl));
-  LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, m->x, m->ssp, s, pdl));
+  // the first projection that reads x normalises it with these gains (null: an int8 layer does)
+  const float* g_first = act.empty() ? m->final_norm : (mode == 0 ? m->layers[act[0]].attn_norm : nullptr);
+  LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, g_first, m->x, m->ssp, m->xa, s, pdl));
+  const int bi = BN / 16 - 1;  // tensor maps of the split activations for this BN
 
   EpiParams base = {};
   base.n = n;
@@ -281,17 +286,14 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   base.rope = kv->rope;
 
   // ---- phase descriptors of the projection chain ----
-  auto ph_qkv = [&](int l, int ss_tiles, PhaseDesc& p, CUtensorMap& w) {
+  auto ph_qkv = [&](int l, int ss_tiles, PhaseDesc& p, CUtensorMap& w, CUtensorMap& x) {
     p = PhaseDesc{};
     p.epi = EPI_QKV;
     p.tiles = 3 * d / 128;
     p.kblocks = cdiv(d, 64);
     p.K = d;
-    p.in = m->x;
-    p.ld_in = d;
     p.ss = m->ssp;
     p.ss_tiles = ss_tiles;
-    p.g = m->layers[l].attn_norm;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = 3 * d;
@@ -299,48 +301,44 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.kc = kv_layer_k(kv, l);
     p.ep.vc = kv_layer_v(kv, l);
     w = m->layers[l].tm_qkv;
+    x = m->tm_xa[bi];
   };
-  auto ph_resid = [&](const float* in, int K, PhaseDesc& p) {
+  // residual projection; g_next: gains of the RMSNorm that the next projection applies to x
+  auto ph_resid = [&](int K, const float* g_next, PhaseDesc& p) {
     p = PhaseDesc{};
     p.epi = EPI_RESID;
     p.tiles = d / 128;
     p.kblocks = cdiv(K, 64);
     p.K = K;
-    p.in = in;
-    p.ld_in = K;
     p.ep = base;
     p.ep.N = d;
     p.ep.y = m->x;
     p.ep.ldy = d;
     p.ep.ss_out = m->ssp;
+    p.ep.xa_out = m->xa;
+    p.ep.g_next = g_next;
   };
-  auto ph_gu = [&](int l, PhaseDesc& p) {
+  auto ph_gu = [&](PhaseDesc& p) {
     p = PhaseDesc{};
     p.epi = EPI_GLU;
     p.tiles = cdiv(F, 64);
     p.kblocks = cdiv(d, 64);
     p.K = d;
-    p.in = m->x;
-    p.ld_in = d;
     p.ss = m->ssp;
     p.ss_tiles = d / 128;
-    p.g = m->layers[l].ffn_norm;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = F;
     p.ep.u_out = m->u;
   };
-  auto ph_lm = [&](int ss_tiles, PhaseDesc& p, CUtensorMap& w) {
+  auto ph_lm = [&](int ss_tiles, PhaseDesc& p, CUtensorMap& w, CUtensorMap& x) {
     p = PhaseDesc{};
     p.epi = EPI_LMHEAD;
     p.tiles = m->lay.lm_tiles;
     p.kblocks = cdiv(d, 64);
     p.K = d;
-    p.in = m->x;
-    p.ld_in = d;
     p.ss = m->ssp;
     p.ss_tiles = ss_tiles;
-    p.g = m->final_norm;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = V;
@@ -349,6 +347,7 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.am_i1 = m->am_i1;
     p.ep.am_v2 = m->am_v2;
     w = m->tm_lm;
+    x = m->tm_xa[bi];
   };
   const int cgrid = chain_grid(m->num_sms);
   auto chain = [&](ChainArgs& ca, ChainMaps& cm, int kind) -> int {
@@ -382,31 +381,34 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     ChainArgs ca = {};
     ChainMaps cm = {};
     int rc;
+    ca.nphases = 1;
     if (act.empty()) {
-      ca.nphases = 1;
-      ph_lm(1, ca.ph[0], cm.w[0]);
+      ph_lm(1, ca.ph[0], cm.w[0], cm.x[0]);
       if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
     } else {
-      ca.nphases = 1;
-      ph_qkv(act[0], 1, ca.ph[0], cm.w[0]);
+      ph_qkv(act[0], 1, ca.ph[0], cm.w[0], cm.x[0]);
       if ((rc = chain(ca, cm, CASSPEC_K_QKV)) != CASSPEC_OK) return rc;
       for (size_t i = 0; i < act.size(); ++i) {
         const int l = act[i];
+        const bool last = i + 1 == act.size();
         if ((rc = attention(l)) != CASSPEC_OK) return rc;
         ChainArgs cb = {};
         ChainMaps cn = {};
         cb.nphases = 4;
-        ph_resid(m->o, d, cb.ph[0]);
+        ph_resid(d, m->layers[l].ffn_norm, cb.ph[0]);
         cn.w[0] = m->layers[l].tm_o;
-        ph_gu(l, cb.ph[1]);
+        cn.x[0] = m->tm_o[bi];
+        ph_gu(cb.ph[1]);
         cn.w[1] = m->layers[l].tm_g;
         cn.w2[1] = m->layers[l].tm_u;
-        ph_resid(m->u, F, cb.ph[2]);
+        cn.x[1] = m->tm_xa[bi];
+        ph_resid(F, last ? m->final_norm : m->layers[act[i + 1]].attn_norm, cb.ph[2]);
         cn.w[2] = m->layers[l].tm_d;
-        if (i + 1 < act.size())
-          ph_qkv(act[i + 1], d / 128, cb.ph[3], cn.w[3]);
+        cn.x[2] = m->tm_u[bi];
+        if (!last)
+          ph_qkv(act[i + 1], d / 128, cb.ph[3], cn.w[3], cn.x[3]);
         else
-          ph_lm(d / 128, cb.ph[3], cn.w[3]);
+          ph_lm(d / 128, cb.ph[3], cn.w[3], cn.x[3]);
         if ((rc = chain(cb, cn, CASSPEC_K_GATEUP)) != CASSPEC_OK) return rc;
       }
     }
@@ -446,22 +448,27 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       er.N = d;
       er.y = m->x;
       er.ldy = d;
-      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows_f32(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
+      // W8A8 activations are the bf16 values: the hi plane of the split output
+      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
       LAUNCH(CASSPEC_K_WO, gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, er));
       LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
       EpiParams eg = base;
       eg.N = F;
       eg.u_out = m->u;
       LAUNCH(CASSPEC_K_GATEUP, gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
-      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows_f32(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
+      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
       EpiParams ed = er;
-      ed.ss_out = m->ssp;  // the LM head's RMSNorm scale
+      if (i + 1 == act.size()) {  // the LM head's RMSNorm scale and operand
+        ed.ss_out = m->ssp;
+        ed.xa_out = m->xa;
+        ed.g_next = m->final_norm;
+      }
       LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
     }
     ChainArgs ca = {};
     ChainMaps cm = {};
     ca.nphases = 1;
-    ph_lm(act.empty() ? 1 : d / 128, ca.ph[0], cm.w[0]);
+    ph_lm(act.empty() ? 1 : d / 128, ca.ph[0], cm.w[0], cm.x[0]);
     int rc;
     if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
   }
@@ -482,6 +489,12 @@ bool build_tensor_maps(casspec_model* m) {
     ok = ok && encode_tmap_bf16(&Lp.tm_d, Lp.wd, F, d, F * 2, 64, 128);
   }
   ok = ok && encode_tmap_bf16(&m->tm_lm, m->lm_head, d, V, d * 2, 64, 128);
+  for (int b = 0; b < 4; ++b) {
+    const uint32_t BN = 16u * (uint32_t)(b + 1);
+    ok = ok && encode_tmap_bf16(&m->tm_o[b], m->o, d, 2 * kMaxTree, d * 2, 64, BN);
+    ok = ok && encode_tmap_bf16(&m->tm_u[b], m->u, F, 2 * kMaxTree, F * 2, 64, BN);
+    ok = ok && encode_tmap_bf16(&m->tm_xa[b], m->xa, d, 2 * kMaxTree, d * 2, 64, BN);
+  }
   return ok;
 }
 
@@ -540,8 +553,9 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   }
   m->x = reinterpret_cast<float*>(b + L.x);
   m->q = reinterpret_cast<uint16_t*>(b + L.q);
-  m->o = reinterpret_cast<float*>(b + L.o);
-  m->u = reinterpret_cast<float*>(b + L.u);
+  m->o = reinterpret_cast<uint16_t*>(b + L.o);
+  m->u = reinterpret_cast<uint16_t*>(b + L.u);
+  m->xa = reinterpret_cast<uint16_t*>(b + L.xa);
   m->ssp = reinterpret_cast<float*>(b + L.ssp);
   m->chain_cnt = reinterpret_cast<unsigned*>(b + L.chain_cnt);
   m->chain_bar = reinterpret_cast<unsigned*>(b + L.chain_bar);

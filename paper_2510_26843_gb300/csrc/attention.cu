@@ -298,10 +298,15 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
       }
     }
     const float inv = 1.f / L;
-    uint2 pk;
-    pk.x = pack_bf16x2(o.x * inv, o.y * inv);
-    pk.y = pack_bf16x2(o.z * inv, o.w * inv);
-    *reinterpret_cast<uint2*>(a.o + (size_t)row * a.d + head * HD + c4) = pk;
+    const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
+    const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
+    uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
+    hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
+    hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
+    lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
+    lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
+    *reinterpret_cast<uint2*>(a.o + (size_t)row * a.d + head * HD + c4) = hi;
+    *reinterpret_cast<uint2*>(a.o + (size_t)(64 + row) * a.d + head * HD + c4) = lo;
   }
   cluster_sync();  // no rank leaves while another still reads its shared memory
 }

@@ -5,16 +5,15 @@
 // barrier between phases.  Only the activations depend on the previous phase; the weights do not,
 // so the weight stream runs on across phase boundaries and the HBM pipeline never drains between
 // projections.  Per CTA (one per SM):
-//   * warp 0 -- TMA producer: streams the CTA's weight tiles (128 x 64 bf16, 128-byte swizzle,
+//   * warp 0 -- weight producer: streams the CTA's weight tiles (128 x 64 bf16, 128-byte swizzle,
 //     L2 evict-first) of every phase through a deep mbarrier ring, never waiting on activations;
-//   * warps 6-9 -- activation transform: after the phase barrier, build the B operand tile of each
-//     k-block from fp32 rows (the residual stream scaled by its RMSNorm factor and gains, the
-//     attention output, or the SwiGLU output), split into hi + lo bf16 parts (16 significant bits)
-//     and stored in the MMA's swizzled K-major layout;
-//   * warp 1 -- TMEM owner and single-thread MMA issuer: D += W * hi^T + W * lo^T (tcgen05.mma
+//   * warp 6 -- activation producer: after the phase barrier, streams the B operand tiles (BN x 64
+//     of the hi plane and of the lo plane of the split activation, 128-byte swizzle) by TMA;
+//   * warp 1 -- TMEM owner and single-thread MMA issuer: D += W hi^T + W lo^T (tcgen05.mma
 //     kind::f16, M = 128 channels, N = BN tokens), double-buffered accumulators in TMEM;
 //   * warps 2-5 -- epilogue: TMEM -> registers, stream-K fix-up (last CTA of a tile sums the partials
-//     in CTA order), fused epilogue; then the CTA's arrival at the phase barrier.
+//     in CTA order), the per-token RMSNorm factor, fused epilogue; then the CTA's arrival at the
+//     phase barrier.
 // Work of each phase is split stream-K over (tile, k-block) units so all SMs stream equal bytes.
 // Every wait is bounded (2 s) and reports CASSPEC_E_TIMEOUT instead of hanging.
 #include "common.cuh"
@@ -23,9 +22,9 @@
 
 namespace casspec {
 
-constexpr int kChainThreads = 320;
+constexpr int kChainThreads = 224;
 constexpr uint32_t kWTile = 128 * 128;  // 128 rows x 64 bf16
-constexpr int kXStages = 3;
+constexpr int kXStages = 4;
 constexpr uint32_t kChainSmemBudget = 232448u;  // 227 KB per CTA
 
 __host__ __device__ constexpr uint32_t chain_x_stage(int BN) { return 2u * (uint32_t)BN * 128u; }
@@ -40,6 +39,8 @@ __host__ __device__ constexpr int chain_w_stages(int BN) {
 __host__ __device__ constexpr size_t chain_smem(int BN) { return chain_fixed(BN) + (size_t)chain_w_stages(BN) * kWTile; }
 __host__ __device__ constexpr uint32_t chain_tmem_cols(int BN) { return 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : 128); }
 
+__device__ __forceinline__ long long chain_u0(int c, long long U, int G) { return (long long)c * U / G; }
+// CTA that owns unit x when U units are split into G contiguous ranges [c U / G, (c + 1) U / G)
 __device__ __forceinline__ int chain_cta_of(long long x, long long U, int G) {
   return (int)(((x + 1) * (long long)G - 1) / U);
 }
@@ -48,9 +49,8 @@ __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
+// generic-proxy global writes <-> async-proxy (TMA) reads of the split activations
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
 template <int BN, typename Bar>
 __device__ __forceinline__ void chain_epilogue(int epi, const EpiParams& e, int tile, int r, const float* v, float* stg,
@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
-  // [0] abort, [1] last-arriver, [2..9] per-warp accumulator-ready votes (two segments), [10] go
+  // [0] abort, [1] last-arriver, [2..9] per-warp accumulator-ready votes (two segments)
   volatile int* flags = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       mbar_init(&wempty[s], 1);
     }
     for (int s = 0; s < SX; ++s) {
-      mbar_init(&xfull[s], 4);
+      mbar_init(&xfull[s], 1);
       mbar_init(&xempty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -109,14 +109,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       mbar_init(&tempty[b], 4);
     }
     mbar_init(drain, 1);
-    flags[0] = 0;
-    flags[1] = 0;
+    for (int f = 0; f < 10; ++f) flags[f] = 0;
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
     for (int p = 0; p < np; ++p) {
       tma_prefetch_desc(&maps.w[p]);
       if (a.ph[p].epi == EPI_GLU) tma_prefetch_desc(&maps.w2[p]);
+      tma_prefetch_desc(&maps.x[p]);
     }
   }
   if (warp == 1) {
@@ -140,8 +140,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         const PhaseDesc& ph = a.ph[p];
         const int kb = ph.kblocks;
         const long long U = (long long)ph.tiles * kb;
-        const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
-        for (long long u = u0; u < u1; ++u) {
+        const long long u1 = chain_u0(cta + 1, U, G);
+        for (long long u = chain_u0(cta, U, G); u < u1; ++u) {
           if (!mbar_wait_bounded(&wempty[stage], phase ^ 1, flags)) {
             flags[0] = 1;
             set_status(a.status, CASSPEC_E_TIMEOUT);
@@ -169,6 +169,58 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           if (armed & (1u << s)) mbar_wait_bounded(&wfull[s], (armed_parity >> s) & 1, nullptr);
       }
     }
+  } else if (warp == 6) {
+    if (lane == 0) {
+      // ---------------- activation producer (waits for the phase barrier) ----------------
+      const uint64_t pol = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, armed_parity = 0;
+      for (int p = 0; p < np && !flags[0]; ++p) {
+        const PhaseDesc& ph = a.ph[p];
+        if (p == 0) {
+          pdl_wait();  // inputs of the first phase come from the previous kernel
+        } else {       // ... of the others from phase p - 1 of every CTA (one counter per phase:
+                       // a CTA with no work may run ahead and arrive at later phases early)
+          const uint64_t t0 = globaltimer_ns();
+          while (ld_acquire_u32(a.bar + (p - 1)) < (unsigned)G) {
+            if (flags[0]) break;
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+              flags[0] = 1;
+              set_status(a.status, CASSPEC_E_TIMEOUT);
+              break;
+            }
+          }
+          if (flags[0]) break;
+        }
+        fence_proxy_async_global();
+        const int kb = ph.kblocks;
+        const long long U = (long long)ph.tiles * kb;
+        const long long u1 = chain_u0(cta + 1, U, G);
+        for (long long u = chain_u0(cta, U, G); u < u1; ++u) {
+          if (!mbar_wait_bounded(&xempty[stage], phase ^ 1, flags)) {
+            flags[0] = 1;
+            set_status(a.status, CASSPEC_E_TIMEOUT);
+            break;
+          }
+          const int k = (int)(u % kb);
+          mbar_expect_tx(&xfull[stage], XS);
+          armed |= 1u << stage;
+          armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
+          uint8_t* sx = xring + stage * XS;
+          tma_load_2d(sx, &maps.x[p], &xfull[stage], k * 64, 0, pol);        // hi plane, tokens 0..BN-1
+          tma_load_2d(sx + XT, &maps.x[p], &xfull[stage], k * 64, 64, pol);  // lo plane
+          if (++stage == SX) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (flags[0]) {
+        for (int s = 0; s < SX; ++s)
+          if (armed & (1u << s)) mbar_wait_bounded(&xfull[s], (armed_parity >> s) & 1, nullptr);
+      }
+    }
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
@@ -181,8 +233,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         const PhaseDesc& ph = a.ph[p];
         const int kb = ph.kblocks;
         const long long U = (long long)ph.tiles * kb;
-        const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
-        long long u = u0;
+        const long long u1 = chain_u0(cta + 1, U, G);
+        long long u = chain_u0(cta, U, G);
         while (u < u1 && ok) {
           const int t = (int)(u / kb);
           const long long seg_end = ((long long)(t + 1) * kb < u1) ? (long long)(t + 1) * kb : u1;
@@ -231,22 +283,26 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       tc_commit(drain);  // all MMAs complete before TMEM is released
       mbar_wait_bounded(drain, 0, nullptr);
     }
-  } else if (warp < 6) {
+  } else {
     // ---------------- epilogue warps 2..5 ----------------
     // Control flow is identical in the four warps (every decision that follows a bounded wait is
     // voted through shared memory), so their named barriers always match, even after a timeout.
     const int q = warp & 3;
     const int r = q * 32 + lane;
     auto bar = [] { named_bar_sync(1, 128); };
+    // The phase-barrier counters belong to the previous launch until it has completed (its last
+    // CTA resets them); a CTA without units could otherwise arrive before that reset.
+    pdl_wait();
     uint32_t used[2] = {0, 0};
     int buf = 0, seg = 0;
     for (int p = 0; p < np; ++p) {
       const PhaseDesc& ph = a.ph[p];
       const int kb = ph.kblocks;
       const long long U = (long long)ph.tiles * kb;
-      const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
+      const long long u1 = chain_u0(cta + 1, U, G);
       unsigned* counters = a.counters + p * 1024;
-      long long u = u0;
+      bool have_rs = false;
+      long long u = chain_u0(cta, U, G);
       while (u < u1) {
         const int t = (int)(u / kb);
         const long long seg_end = ((long long)(t + 1) * kb < u1) ? (long long)(t + 1) * kb : u1;
@@ -264,6 +320,16 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           buf ^= 1;
           continue;
         }
+        if (ph.ss != nullptr && !have_rs) {
+          // the phase's inputs are visible here: this accumulator was computed from them
+          if (r < 64) {
+            float ssum = 0.f;
+            for (int j = 0; j < ph.ss_tiles; ++j) ssum += __ldcg(ph.ss + j * 64 + r);
+            rs[r] = rsqrtf(ssum / (float)ph.K + ph.eps);
+          }
+          bar();
+          have_rs = true;
+        }
         tc_fence_after();
         float v[BN];
         const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
@@ -275,10 +341,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         if (lane == 0) mbar_arrive(&tempty[buf]);
         buf ^= 1;
 
+        // stream-K fix-up over the CTAs that own units of tile t (CTAs with no unit at all, which
+        // exist when the phase has fewer units than CTAs, are skipped)
         const int c_first = chain_cta_of((long long)t * kb, U, G);
         const int c_last = chain_cta_of((long long)(t + 1) * kb - 1, U, G);
         bool finish = true;
         if (c_first != c_last) {
+          int owners = 0;
+          for (int cc = c_first; cc <= c_last; ++cc) owners += chain_u0(cc + 1, U, G) > chain_u0(cc, U, G);
           float* mine = a.partials + (size_t)(t + cta) * (64 * 128);
 #pragma unroll
           for (int i = 0; i < BN; ++i)
@@ -287,7 +357,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           bar();
           if (threadIdx.x == 64) {
             const unsigned old = atomicAdd(&counters[t], 1u);
-            flags[1] = (old == (unsigned)(c_last - c_first)) ? 1 : 0;
+            flags[1] = (old == (unsigned)(owners - 1)) ? 1 : 0;
           }
           bar();
           finish = flags[1] != 0;
@@ -300,7 +370,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
               if (cc == cta) {
 #pragma unroll
                 for (int i = 0; i < BN; ++i) acc[i] += v[i];
-              } else {
+              } else if (chain_u0(cc + 1, U, G) > chain_u0(cc, U, G)) {
                 const float* pp = a.partials + (size_t)(t + cc) * (64 * 128);
 #pragma unroll
                 for (int i = 0; i < BN; ++i)
@@ -312,104 +382,23 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             if (threadIdx.x == 64) counters[t] = 0u;  // ready for the next launch
           }
         }
-        if (finish) chain_epilogue<BN>(ph.epi, ph.ep, t, r, v, stg, bar);
+        if (finish) {
+          if (ph.ss != nullptr) {
+#pragma unroll
+            for (int i = 0; i < BN; ++i) v[i] *= rs[i < 64 ? i : 63];
+          }
+          chain_epilogue<BN>(ph.epi, ph.ep, t, r, v, stg, bar);
+        }
         u = seg_end;
       }
+      if (have_rs) bar();  // rs is rewritten by the next phase only after every thread used it
       if (p + 1 < np) {  // this CTA's writes of phase p are done: arrive at the phase barrier
+        fence_proxy_async_global();
         __threadfence();
         bar();
         if (threadIdx.x == 64) {
           __threadfence();
-          atomicAdd(&a.bar[0], 1u);
-        }
-      }
-    }
-  } else {
-    // ---------------- activation transform warps 6..9 ----------------
-    // Thread tt == 0 alone polls the phase barrier and publishes the outcome before the named
-    // barrier; after an abort every wait below returns at once, so the loops run out uniformly.
-    const int tt = threadIdx.x - 192;  // 0..127
-    auto tbar = [] { named_bar_sync(2, 128); };
-    int xs = 0;
-    uint32_t xph = 0;
-    for (int p = 0; p < np; ++p) {
-      const PhaseDesc& ph = a.ph[p];
-      // the inputs of phase p were written by the previous kernel (p = 0) or by phase p - 1
-      if (p == 0) {
-        pdl_wait();
-      } else if (tt == 0) {
-        const unsigned target = (unsigned)p * (unsigned)G;
-        const uint64_t t0 = globaltimer_ns();
-        while (ld_acquire_u32(a.bar) < target) {
-          if (flags[0]) break;
-          if (globaltimer_ns() - t0 > kWaitLimitNs) {
-            flags[0] = 1;
-            set_status(a.status, CASSPEC_E_TIMEOUT);
-            break;
-          }
-        }
-      }
-      tbar();
-      const int n = ph.ep.n;
-      if (ph.ss != nullptr) {
-        if (tt < 64) {
-          float ssum = 0.f;
-          for (int t = 0; t < ph.ss_tiles; ++t) ssum += __ldcg(ph.ss + t * 64 + tt);
-          rs[tt] = tt < n ? rsqrtf(ssum / (float)ph.K + ph.eps) : 0.f;
-        }
-        tbar();
-      }
-      const int kb = ph.kblocks;
-      const long long U = (long long)ph.tiles * kb;
-      const long long u0 = (long long)cta * U / G, u1 = (long long)(cta + 1) * U / G;
-      for (long long u = u0; u < u1; ++u) {
-        const bool free_slot = mbar_wait_bounded(&xempty[xs], xph ^ 1, flags);
-        if (free_slot && !flags[0]) {
-          const int k = (int)(u % kb);
-          const uint32_t th = smem_u32(xring + xs * XS), tl = th + XT;
-          for (int item = tt; item < BN * 8; item += 128) {
-            const int row = item >> 3, c = item & 7;
-            const int col = k * 64 + c * 8;
-            float vv[8];
-            if (row < n && col < ph.K) {
-              const float4 f0 = __ldcg(reinterpret_cast<const float4*>(ph.in + (size_t)row * ph.ld_in + col));
-              const float4 f1 = __ldcg(reinterpret_cast<const float4*>(ph.in + (size_t)row * ph.ld_in + col + 4));
-              vv[0] = f0.x, vv[1] = f0.y, vv[2] = f0.z, vv[3] = f0.w, vv[4] = f1.x, vv[5] = f1.y, vv[6] = f1.z,
-              vv[7] = f1.w;
-              if (ph.ss != nullptr) {
-                const float sc = rs[row];
-                const float4 g0 = __ldg(reinterpret_cast<const float4*>(ph.g + col));
-                const float4 g1 = __ldg(reinterpret_cast<const float4*>(ph.g + col + 4));
-                vv[0] = vv[0] * sc * g0.x, vv[1] = vv[1] * sc * g0.y, vv[2] = vv[2] * sc * g0.z,
-                vv[3] = vv[3] * sc * g0.w;
-                vv[4] = vv[4] * sc * g1.x, vv[5] = vv[5] * sc * g1.y, vv[6] = vv[6] * sc * g1.z,
-                vv[7] = vv[7] * sc * g1.w;
-              }
-            } else {
-#pragma unroll
-              for (int j = 0; j < 8; ++j) vv[j] = 0.f;
-            }
-            uint32_t hi[4], lo[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const uint16_t h0 = f2bf(vv[2 * j]), h1 = f2bf(vv[2 * j + 1]);
-              hi[j] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-              lo[j] = pack_bf16x2(vv[2 * j] - bf2f(h0), vv[2 * j + 1] - bf2f(h1));
-            }
-            const uint32_t off = (uint32_t)row * 128u + ((uint32_t)(c ^ (row & 7)) << 4);
-            st_shared_v4(th + off, hi[0], hi[1], hi[2], hi[3]);
-            st_shared_v4(tl + off, lo[0], lo[1], lo[2], lo[3]);
-          }
-          fence_proxy_async_smem();  // generic-proxy smem writes -> visible to the tensor cores
-        } else if (!free_slot && !flags[0]) {
-          flags[0] = 1;
-          set_status(a.status, CASSPEC_E_TIMEOUT);
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&xfull[xs]);
-        if (++xs == SX) {
-          xs = 0;
-          xph ^= 1;
+          atomicAdd(&a.bar[p], 1u);
         }
       }
     }
@@ -422,10 +411,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     tmem_dealloc(tmem_base, TMEM_COLS);
   }
   if (threadIdx.x == 0 && np > 1) {  // the last CTA out resets the phase-barrier counters
+    pdl_wait();  // (the exit counter, too, is the previous launch's until it completes)
     __threadfence();
-    if (atomicAdd(&a.bar[1], 1u) == (unsigned)(G - 1)) {
-      a.bar[0] = 0u;
-      a.bar[1] = 0u;
+    if (atomicAdd(&a.bar[kMaxPhases], 1u) == (unsigned)(G - 1)) {
+      for (int p = 0; p <= kMaxPhases; ++p) a.bar[p] = 0u;
     }
   }
 }

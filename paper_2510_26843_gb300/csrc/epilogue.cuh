@@ -59,7 +59,10 @@ __device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, con
       if (i < e.n) {
         const float g = v[i];
         const float up = stg[(r + 64) * (BN + 1) + i];
-        e.u_out[(size_t)i * e.N + ch] = g / (1.f + expf(-g)) * up;
+        const float u = g / (1.f + expf(-g)) * up;
+        const uint16_t hi = f2bf(u);
+        e.u_out[(size_t)i * e.N + ch] = hi;
+        e.u_out[(size_t)(64 + i) * e.N + ch] = f2bf(u - bf2f(hi));
       }
     }
   }
@@ -109,11 +112,13 @@ __device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, c
 }
 
 // y += v (fp32 residual stream); optionally the tile's per-token sum of squares of the updated rows,
-// the partial sums from which the next RMSNorm takes its scale (fixed order: deterministic).
+// the partial sums from which the next RMSNorm takes its scale (fixed order: deterministic), and
+// split(y * g_next), the operand of the next projection.
 template <int BN, typename Bar>
 __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
   const int o = tile * 128 + r;
   const bool valid = o < e.N;
+  const float gn = (e.xa_out != nullptr && valid) ? e.g_next[o] : 0.f;
 #pragma unroll
   for (int i = 0; i < BN; ++i) {
     float nv = 0.f;
@@ -121,6 +126,12 @@ __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, c
       float* p = e.y + (size_t)i * e.ldy + o;
       nv = __ldcg(p) + v[i];
       *p = nv;
+      if (e.xa_out != nullptr) {
+        const float a = nv * gn;
+        const uint16_t hi = f2bf(a);
+        e.xa_out[(size_t)i * e.ldy + o] = hi;
+        e.xa_out[(size_t)(64 + i) * e.ldy + o] = f2bf(a - bf2f(hi));
+      }
     }
     if (e.ss_out != nullptr) stg[r * (BN + 1) + i] = nv * nv;
   }

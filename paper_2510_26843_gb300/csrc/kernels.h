@@ -13,7 +13,7 @@ enum Epi : int {
   EPI_STORE = 0,   // y[i][o] = v                              (stateless linear)
   EPI_RESID = 1,   // y[i][o] += v                             (Wo, Wd: residual add in fp32)
   EPI_QKV = 2,     // rotary on q,k at tree positions; q -> q_out, k,v -> cache slots P+T+i
-  EPI_GLU = 3,     // tile = 64 gate rows + 64 up rows: u_out[i][c] = silu(g) * up
+  EPI_GLU = 3,     // tile = 64 gate rows + 64 up rows: u_out = split(silu(g) * up)
   EPI_LMHEAD = 4,  // logits[i][o] = v (optional) + per-tile (max, argmax, 2nd max) per token
 };
 
@@ -31,8 +31,13 @@ struct EpiParams {
   const int* pos;       // [n] position of each new node (P + depth)
   const float2* rope;   // [ctx][hd/2] (cos, sin) of p * base^(-2j/hd) for every position p
   float* ss_out;        // EPI_RESID (optional): [tiles][64] sum over the tile's columns of updated y^2
+  uint16_t* xa_out;     // EPI_RESID (optional): split(y * g_next) as [128][ldy] bf16 (see below)
+  const float* g_next;  // RMSNorm gains of the projection that reads xa_out
   // EPI_GLU
-  float* u_out;         // [64][F] fp32
+  uint16_t* u_out;      // split(silu(g) * up) as [128][N] bf16
+  // A "split" activation matrix holds fp32 values v as two bf16 planes, hi = bf16(v) in rows
+  // 0..63 and lo = bf16(v - hi) in rows 64..127 (16 significant bits in all): the B operand of the
+  // chained tensor-core projections, which multiply both planes with the same weights.
   // EPI_LMHEAD
   float* logits;        // [n][V] fp32 or null
   float* am_v1;         // [tiles][64] partial max
@@ -68,7 +73,7 @@ struct GemmI8Args {
 
 struct AttnArgs {
   const uint16_t* q;    // [64][d] bf16 (rotated)
-  float* o;             // [64][d] fp32
+  uint16_t* o;          // split attention output [128][d] bf16
   const unsigned long long* anc;  // [n] ancestor masks over tree slots
   const int* dP;
   int T, n, ctx, d, n_heads;
@@ -78,19 +83,18 @@ struct AttnArgs {
   int* status;
 };
 
-// One phase of the persistent projection chain: Y = A(X) W^T with A(X) built on the fly from fp32
-// rows (optionally RMS-normalised) and split into hi + lo bf16 parts.
+// One phase of the persistent projection chain: Y = W (hi + lo)^T over a split activation matrix
+// (tensor map ChainMaps::x), optionally scaled per token by an RMSNorm factor: when `ss` is set the
+// activation is x * g (gains already applied by its producer) and the token's result is multiplied
+// by rsqrt(sum(ss) / K + eps), which equals projecting RMSNorm(x) * g.
 constexpr int kMaxPhases = 4;
 struct PhaseDesc {
   int epi;           // EPI_QKV, EPI_RESID, EPI_GLU or EPI_LMHEAD
   int tiles;         // 128-row output tiles (EPI_GLU: 64 gate + 64 up rows per tile)
   int kblocks;       // ceil(K / 64)
   int K;             // input width
-  const float* in;   // fp32 input rows [64][ld_in]
-  int ld_in;
-  const float* ss;   // normalise rows: per-tile partial sums of squares [ss_tiles][64] (null: no norm)
+  const float* ss;   // per-tile partial sums of squares [ss_tiles][64] of x (null: no norm)
   int ss_tiles;
-  const float* g;    // RMSNorm gains [K]
   float eps;
   EpiParams ep;
 };
@@ -99,12 +103,13 @@ struct ChainArgs {
   PhaseDesc ph[kMaxPhases];
   float* partials;     // stream-K partial tiles (shared by the phases)
   unsigned* counters;  // [kMaxPhases][1024] fix-up counters, zero between launches
-  unsigned* bar;       // [2] grid-barrier counters, zero between launches
+  unsigned* bar;       // [kMaxPhases + 1] phase-barrier arrival counters + exit counter, zero between launches
   int* status;
 };
 struct ChainMaps {
-  CUtensorMap w[kMaxPhases];   // weights (EPI_GLU: gate)
+  CUtensorMap w[kMaxPhases];   // weights (EPI_GLU: gate), 64 x 128 boxes (EPI_GLU: 64 x 64)
   CUtensorMap w2[kMaxPhases];  // EPI_GLU: up
+  CUtensorMap x[kMaxPhases];   // split activations [128][K] bf16, 64 x BN boxes
 };
 
 // ---- launchers (return cudaSuccess or the launch error) ----
@@ -123,8 +128,8 @@ cudaError_t launch_tree_attention(const CUtensorMap& tmKV, const AttnArgs& a, in
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
                              int* pos, unsigned long long* anc_new, int* status, cudaStream_t s, bool pdl);
-cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, float* ss,
-                         cudaStream_t s, bool pdl);
+cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, const float* g, float* x,
+                         float* ss, uint16_t* xa, cudaStream_t s, bool pdl);
 int chain_grid(int num_sms);
 size_t chain_smem_bytes(int BN);
 cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int BN, int grid, cudaStream_t stream, bool pdl);
@@ -132,8 +137,6 @@ cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float e
                            cudaStream_t s, bool pdl);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
                               bool pdl);
-cudaError_t launch_quant_rows_f32(const float* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
-                                  bool pdl);
 cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,
                                  float* margin, cudaStream_t s, bool pdl);
 cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s);

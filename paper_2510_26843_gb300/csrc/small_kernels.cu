@@ -121,7 +121,8 @@ __device__ __forceinline__ int8_t quant_one(float x, float inv) {
 // sum of squares (the first RMSNorm's scale), ss[i].
 // ---------------------------------------------------------------------------------------------
 __global__ void embed_kernel(const uint16_t* __restrict__ E, const int* tokens, int d, int vocab,
-                             float* __restrict__ x, float* __restrict__ ss) {
+                             const float* __restrict__ g, float* __restrict__ x, float* __restrict__ ss,
+                             uint16_t* __restrict__ xa) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
@@ -135,16 +136,22 @@ __global__ void embed_kernel(const uint16_t* __restrict__ E, const int* tokens, 
     const float f0 = bf2f(two & 0xFFFF), f1 = bf2f(two >> 16);
     *reinterpret_cast<float2*>(x + (size_t)i * d + c) = make_float2(f0, f1);
     acc += f0 * f0 + f1 * f1;
+    if (xa != nullptr) {  // split(x * g) for the first projection that normalises x
+      const float a0 = f0 * g[c], a1 = f1 * g[c + 1];
+      const uint16_t h0 = f2bf(a0), h1 = f2bf(a1);
+      *reinterpret_cast<uint32_t*>(xa + (size_t)i * d + c) = (uint32_t)h0 | ((uint32_t)h1 << 16);
+      *reinterpret_cast<uint32_t*>(xa + (size_t)(64 + i) * d + c) = pack_bf16x2(a0 - bf2f(h0), a1 - bf2f(h1));
+    }
   }
   acc = block_sum(acc, red);
   if (threadIdx.x == 0) ss[i] = acc;
 }
 
-cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, float* x, float* ss,
-                         cudaStream_t s, bool pdl) {
+cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, const float* g, float* x,
+                         float* ss, uint16_t* xa, cudaStream_t s, bool pdl) {
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(256), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, embed_kernel, E, tokens, d, vocab, x, ss);
+  return cudaLaunchKernelEx(&cfg, embed_kernel, E, tokens, d, vocab, g, x, ss, g != nullptr ? xa : nullptr);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -277,54 +284,6 @@ cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* 
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
   return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq);
-}
-
-// Per-row int8 quantisation of fp32 rows as stored in bf16 (each value is rounded to bf16 first,
-// the precision in which the W8A8 draft keeps its activations).
-__global__ void __launch_bounds__(kRowThreads) quant_rows_f32_kernel(const float* __restrict__ x, int d, int ldx,
-                                                                     int8_t* __restrict__ q, int ldq,
-                                                                     float* __restrict__ sq) {
-  __shared__ float red[32];
-  pdl_trigger();
-  pdl_wait();
-  const int i = blockIdx.x;
-  const int nv = d / 4;
-  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)i * ldx);
-  float4 xv[kRowVec];
-  float amax = 0.f;
-#pragma unroll
-  for (int k = 0; k < kRowVec; ++k) {
-    const int c = threadIdx.x + k * kRowThreads;
-    xv[k] = c < nv ? __ldcg(xr + c) : make_float4(0.f, 0.f, 0.f, 0.f);
-    xv[k].x = bf2f(f2bf(xv[k].x));
-    xv[k].y = bf2f(f2bf(xv[k].y));
-    xv[k].z = bf2f(f2bf(xv[k].z));
-    xv[k].w = bf2f(f2bf(xv[k].w));
-    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(xv[k].x), fabsf(xv[k].y)), fmaxf(fabsf(xv[k].z), fabsf(xv[k].w))));
-  }
-  amax = block_max(amax, red);
-  const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
-#pragma unroll
-  for (int k = 0; k < kRowVec; ++k) {
-    const int c = threadIdx.x + k * kRowThreads;
-    if (c < nv) {
-      char4 o;
-      o.x = amax > 0.f ? quant_one(xv[k].x, inv) : 0;
-      o.y = amax > 0.f ? quant_one(xv[k].y, inv) : 0;
-      o.z = amax > 0.f ? quant_one(xv[k].z, inv) : 0;
-      o.w = amax > 0.f ? quant_one(xv[k].w, inv) : 0;
-      reinterpret_cast<char4*>(q + (size_t)i * ldq)[c] = o;
-    }
-  }
-  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
-}
-
-cudaError_t launch_quant_rows_f32(const float* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
-                                  bool pdl) {
-  if (d % 4 != 0 || ldx % 4 != 0 || ldq % 4 != 0 || d > 4 * kRowVec * kRowThreads) return cudaErrorInvalidValue;
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, quant_rows_f32_kernel, x, d, ldx, q, ldq, sq);
 }
 
 // ---------------------------------------------------------------------------------------------
