@@ -28,7 +28,7 @@ constexpr int kXStages = 4;
 constexpr uint32_t kChainSmemBudget = 232448u;  // 227 KB per CTA
 
 __host__ __device__ constexpr uint32_t chain_x_stage(int BN) { return 2u * (uint32_t)BN * 128u; }
-__host__ __device__ constexpr uint32_t chain_staging(int BN) { return 128u * (uint32_t)(BN + 1) * 4u; }
+__host__ __device__ constexpr uint32_t chain_staging(int BN) { return (uint32_t)epi_staging_floats(BN) * 4u; }
 __host__ __device__ constexpr uint32_t chain_fixed(int BN) {
   return 1024u + kXStages * chain_x_stage(BN) + chain_staging(BN) + 64u * 4u + 512u;
 }
@@ -79,7 +79,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint8_t* wring = smem;
   uint8_t* xring = smem + SW * kWTile;
   float* stg = reinterpret_cast<float*>(xring + SX * XS);
-  float* rs = stg + 128 * (BN + 1);
+  float* rs = stg + epi_staging_floats(BN);
   uint64_t* wfull = reinterpret_cast<uint64_t*>(rs + 64);
   uint64_t* wempty = wfull + SW;
   uint64_t* xfull = wempty + SW;
@@ -137,9 +137,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       uint32_t phase = 0;
       uint32_t armed = 0, armed_parity = 0;
       for (int p = 0; p < np && !flags[0]; ++p) {
-        const PhaseDesc& ph = a.ph[p];
-        const int kb = ph.kblocks;
-        const long long U = (long long)ph.tiles * kb;
+        const int kb = a.ph[p].kblocks;
+        const bool glu = a.ph[p].epi == EPI_GLU;
+        const long long U = (long long)a.ph[p].tiles * kb;
         const long long u1 = chain_u0(cta + 1, U, G);
         for (long long u = chain_u0(cta, U, G); u < u1; ++u) {
           if (!mbar_wait_bounded(&wempty[stage], phase ^ 1, flags)) {
@@ -152,7 +152,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           armed |= 1u << stage;
           armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
           uint8_t* sa = wring + stage * kWTile;
-          if (ph.epi == EPI_GLU) {
+          if (glu) {
             tma_load_2d(sa, &maps.w[p], &wfull[stage], k * 64, t * 64, pol);
             tma_load_2d(sa + kWTile / 2, &maps.w2[p], &wfull[stage], k * 64, t * 64, pol);
           } else {
@@ -177,7 +177,6 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       uint32_t phase = 0;
       uint32_t armed = 0, armed_parity = 0;
       for (int p = 0; p < np && !flags[0]; ++p) {
-        const PhaseDesc& ph = a.ph[p];
         if (p == 0) {
           pdl_wait();  // inputs of the first phase come from the previous kernel
         } else {       // ... of the others from phase p - 1 of every CTA (one counter per phase:
@@ -194,8 +193,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           if (flags[0]) break;
         }
         fence_proxy_async_global();
-        const int kb = ph.kblocks;
-        const long long U = (long long)ph.tiles * kb;
+        const int kb = a.ph[p].kblocks;
+        const long long U = (long long)a.ph[p].tiles * kb;
         const long long u1 = chain_u0(cta + 1, U, G);
         for (long long u = chain_u0(cta, U, G); u < u1; ++u) {
           if (!mbar_wait_bounded(&xempty[stage], phase ^ 1, flags)) {
@@ -230,9 +229,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       int buf = 0;
       bool ok = true;
       for (int p = 0; p < np && ok; ++p) {
-        const PhaseDesc& ph = a.ph[p];
-        const int kb = ph.kblocks;
-        const long long U = (long long)ph.tiles * kb;
+        const int kb = a.ph[p].kblocks;
+        const long long U = (long long)a.ph[p].tiles * kb;
         const long long u1 = chain_u0(cta + 1, U, G);
         long long u = chain_u0(cta, U, G);
         while (u < u1 && ok) {
@@ -296,9 +294,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     uint32_t used[2] = {0, 0};
     int buf = 0, seg = 0;
     for (int p = 0; p < np; ++p) {
-      const PhaseDesc& ph = a.ph[p];
-      const int kb = ph.kblocks;
-      const long long U = (long long)ph.tiles * kb;
+      // The phase descriptor sits in parameter space behind a runtime index: copy what the loops
+      // use into registers once, so no load of it is ordered behind the epilogue's stores.
+      const EpiParams ep = a.ph[p].ep;
+      const int epi = a.ph[p].epi, kb = a.ph[p].kblocks, Kp = a.ph[p].K, n = ep.n;
+      const float* ss = a.ph[p].ss;
+      const int ss_tiles = a.ph[p].ss_tiles;
+      const float eps = a.ph[p].eps;
+      const long long U = (long long)a.ph[p].tiles * kb;
       const long long u1 = chain_u0(cta + 1, U, G);
       unsigned* counters = a.counters + p * 1024;
       bool have_rs = false;
@@ -320,12 +323,18 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           buf ^= 1;
           continue;
         }
-        if (ph.ss != nullptr && !have_rs) {
+        if (ss != nullptr && !have_rs) {
           // the phase's inputs are visible here: this accumulator was computed from them
           if (r < 64) {
-            float ssum = 0.f;
-            for (int j = 0; j < ph.ss_tiles; ++j) ssum += __ldcg(ph.ss + j * 64 + r);
-            rs[r] = rsqrtf(ssum / (float)ph.K + ph.eps);
+            float ssum = 0.f;  // fixed summation order; loads issued 8 at a time
+            for (int j0 = 0; j0 < ss_tiles; j0 += 8) {
+              float t8[8];
+#pragma unroll
+              for (int k = 0; k < 8; ++k) t8[k] = j0 + k < ss_tiles ? __ldcg(ss + (j0 + k) * 64 + r) : 0.f;
+#pragma unroll
+              for (int k = 0; k < 8; ++k) ssum += t8[k];
+            }
+            rs[r] = rsqrtf(ssum / (float)Kp + eps);
           }
           bar();
           have_rs = true;
@@ -352,42 +361,67 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           float* mine = a.partials + (size_t)(t + cta) * (64 * 128);
 #pragma unroll
           for (int i = 0; i < BN; ++i)
-            if (i < ph.ep.n) __stcg(mine + i * 128 + r, v[i]);
-          __threadfence();
-          bar();
+            if (i < n) __stcg(mine + i * 128 + r, v[i]);
+          bar();  // then one gpu-scope fence (cumulative over the CTA's stores) before the arrival
           if (threadIdx.x == 64) {
+            __threadfence();
             const unsigned old = atomicAdd(&counters[t], 1u);
             flags[1] = (old == (unsigned)(owners - 1)) ? 1 : 0;
           }
           bar();
           finish = flags[1] != 0;
           if (finish) {
-            __threadfence();
-            float acc[BN];
+            // The last owner sums every owner's partial in CTA order.  Partials are [token][row]
+            // slots; own values go through shared memory in the same layout so that each thread
+            // accumulates whole float4s with coalesced 16-byte loads, all loads of one owner in
+            // flight together.
 #pragma unroll
-            for (int i = 0; i < BN; ++i) acc[i] = 0.f;
+            for (int i = 0; i < BN; ++i) stg[i * 128 + r] = v[i];
+            bar();
+            __threadfence();
+            float4 acc[BN / 4];
+#pragma unroll
+            for (int j = 0; j < BN / 4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+            const int nf4 = n * 32;  // float4s of the valid tokens
+            const float4* own4 = reinterpret_cast<const float4*>(stg);
             for (int cc = c_first; cc <= c_last; ++cc) {
+              float4 t4[BN / 4];
               if (cc == cta) {
 #pragma unroll
-                for (int i = 0; i < BN; ++i) acc[i] += v[i];
+                for (int j = 0; j < BN / 4; ++j) t4[j] = r + 128 * j < nf4 ? own4[r + 128 * j] : make_float4(0.f, 0.f, 0.f, 0.f);
               } else if (chain_u0(cc + 1, U, G) > chain_u0(cc, U, G)) {
-                const float* pp = a.partials + (size_t)(t + cc) * (64 * 128);
+                const float4* pp = reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128));
 #pragma unroll
-                for (int i = 0; i < BN; ++i)
-                  if (i < ph.ep.n) acc[i] += __ldcg(pp + i * 128 + r);
+                for (int j = 0; j < BN / 4; ++j) t4[j] = r + 128 * j < nf4 ? __ldcg(pp + r + 128 * j) : make_float4(0.f, 0.f, 0.f, 0.f);
+              } else {
+                continue;
+              }
+#pragma unroll
+              for (int j = 0; j < BN / 4; ++j) {
+                acc[j].x += t4[j].x;
+                acc[j].y += t4[j].y;
+                acc[j].z += t4[j].z;
+                acc[j].w += t4[j].w;
               }
             }
+            bar();
+            float4* st4 = reinterpret_cast<float4*>(stg);
 #pragma unroll
-            for (int i = 0; i < BN; ++i) v[i] = acc[i];
+            for (int j = 0; j < BN / 4; ++j)
+              if (r + 128 * j < nf4) st4[r + 128 * j] = acc[j];
+            bar();
+#pragma unroll
+            for (int i = 0; i < BN; ++i) v[i] = stg[i * 128 + r];
+            bar();  // the epilogue reuses the staging area
             if (threadIdx.x == 64) counters[t] = 0u;  // ready for the next launch
           }
         }
         if (finish) {
-          if (ph.ss != nullptr) {
+          if (ss != nullptr) {
 #pragma unroll
-            for (int i = 0; i < BN; ++i) v[i] *= rs[i < 64 ? i : 63];
+            for (int i = 0; i < BN; ++i) v[i] *= rs[i];
           }
-          chain_epilogue<BN>(ph.epi, ph.ep, t, r, v, stg, bar);
+          chain_epilogue<BN>(epi, ep, t, r, v, stg, bar);
         }
         u = seg_end;
       }

@@ -1,7 +1,9 @@
-// Epilogues of the projections.  A finished 128-row tile is held one row (output channel) per
-// thread by 128 cooperating threads; thread r owns row r and the values v[0..BN) of tokens
-// 0..BN-1 (only i < n are meaningful).  `stg` is a [128][BN+1] fp32 staging area in shared memory
-// used where a row needs another row's values (rotary partner, gate/up pair, argmax over rows);
+// Epilogues of the projections.  A finished 128-row tile arrives one row (output channel) per
+// thread from 128 cooperating threads: thread r owns row r and the values v[0..BN) of tokens
+// 0..BN-1 (only i < n are meaningful).  The tile is first staged token-major in shared memory
+// (`stg`, epi_staging_floats(BN) floats); then each warp takes whole tokens and each lane four
+// consecutive channels, so every global access is a 16- or 8-byte vector and the per-token
+// reductions (sum of squares, argmax) are warp shuffles in a fixed order (deterministic).
 // `bar` synchronises the 128 threads (a named barrier).
 #pragma once
 
@@ -10,144 +12,247 @@
 
 namespace casspec {
 
+constexpr int kEpiStride = 132;  // staging row of one token: 128 channels + 4 pad floats
+
+__host__ __device__ constexpr int epi_staging_floats(int BN) {
+  return 128 * (BN + 1) > BN * kEpiStride ? 128 * (BN + 1) : BN * kEpiStride;
+}
+
+template <int BN, typename Bar>
+__device__ __forceinline__ void epi_stage(int r, const float* v, float* stg, Bar bar) {
+  bar();  // the previous user of the staging area is done
+#pragma unroll
+  for (int i = 0; i < BN; ++i) stg[i * kEpiStride + r] = v[i];
+  bar();
+}
+
+__device__ __forceinline__ float4 stg4(const float* stg, int i, int c) {
+  return *reinterpret_cast<const float4*>(stg + i * kEpiStride + c);
+}
+
+__device__ __forceinline__ uint2 pack4_bf16(float a, float b, float c, float d) {
+  return make_uint2(pack_bf16x2(a, b), pack_bf16x2(c, d));
+}
+
+// hi = bf16(x), lo = bf16(x - hi) of four values
+__device__ __forceinline__ void split4(float4 x, uint2& hi, uint2& lo) {
+  const uint16_t h0 = f2bf(x.x), h1 = f2bf(x.y), h2 = f2bf(x.z), h3 = f2bf(x.w);
+  hi = make_uint2((uint32_t)h0 | ((uint32_t)h1 << 16), (uint32_t)h2 | ((uint32_t)h3 << 16));
+  lo = pack4_bf16(x.x - bf2f(h0), x.y - bf2f(h1), x.z - bf2f(h2), x.w - bf2f(h3));
+}
+
+__device__ __forceinline__ float warp_sum(float s) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  return s;
+}
+
+// Q/K/V: rotary on q and k at the node's tree position; q -> q_out, k, v -> cache slot P + T + i.
 template <int BN, typename Bar>
 __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  const int o = tile * 128 + r;  // row of [Wq; Wk; Wv]
-  const int part = o / e.d;      // 0: q, 1: k, 2: v
+  epi_stage<BN>(r, v, stg, bar);
+  const int w = r >> 5, l = r & 31;
+  const int row = 4 * l;
+  const int o = tile * 128 + row;  // first of this lane's 4 rows of [Wq; Wk; Wv]
+  const int part = o / e.d;        // 0: q, 1: k, 2: v (a tile never straddles parts: d % 128 == 0)
   const int within = o - part * e.d;
   const int head = within / e.hd;
   const int j = within - head * e.hd;
   const int half = e.hd >> 1;
-#pragma unroll
-  for (int i = 0; i < BN; ++i) stg[r * (BN + 1) + i] = v[i];
-  bar();
-  const int rp = r ^ half;  // heads are aligned to tiles (d % 128 == 0, hd | 128)
-  const int P = __ldcg(e.dP);
+  const int prow = row ^ half;  // rotary partner rows (half is a multiple of 4)
   const int jj = j & (half - 1);
+  const float sgn = (j < half) ? -1.f : 1.f;
+  const int P = __ldcg(e.dP);
+  constexpr int M = (BN + 3) / 4;  // tokens per warp: i = w + 4 m
   if (part < 2) {
-    const float sgn = (j < half) ? -1.f : 1.f;
+    int pos[M];
 #pragma unroll
-    for (int i = 0; i < BN; ++i) {
-      if (i < e.n) {
-        const float2 cs = e.rope[(size_t)__ldcg(e.pos + i) * half + jj];
-        const float out = v[i] * cs.x + sgn * stg[rp * (BN + 1) + i] * cs.y;
-        if (part == 0)
-          e.q_out[(size_t)i * e.d + within] = f2bf(out);
-        else
-          e.kc[((size_t)head * e.ctx + (P + e.T + i)) * e.hd + j] = f2bf(out);
+    for (int m = 0; m < M; ++m) pos[m] = (w + 4 * m < e.n) ? __ldcg(e.pos + w + 4 * m) : 0;
+#pragma unroll
+    for (int m0 = 0; m0 < M; m0 += 8) {  // rotary tables of 8 tokens in flight at a time
+      float4 c01[8], c23[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (m0 + k < M) {
+          const float4* cs = reinterpret_cast<const float4*>(e.rope + (size_t)pos[m0 + k] * half + jj);
+          c01[k] = cs[0];
+          c23[k] = cs[1];
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int i = w + 4 * (m0 + k);
+        if (m0 + k < M && i < e.n) {
+          const float4 x = stg4(stg, i, row), y = stg4(stg, i, prow);
+          const uint2 out = pack4_bf16(x.x * c01[k].x + sgn * y.x * c01[k].y, x.y * c01[k].z + sgn * y.y * c01[k].w,
+                                       x.z * c23[k].x + sgn * y.z * c23[k].y, x.w * c23[k].z + sgn * y.w * c23[k].w);
+          if (part == 0)
+            *reinterpret_cast<uint2*>(e.q_out + (size_t)i * e.d + within) = out;
+          else
+            *reinterpret_cast<uint2*>(e.kc + ((size_t)head * e.ctx + (P + e.T + i)) * e.hd + j) = out;
+        }
       }
     }
   } else {
 #pragma unroll
-    for (int i = 0; i < BN; ++i)
-      if (i < e.n) e.vc[((size_t)head * e.ctx + (P + e.T + i)) * e.hd + j] = f2bf(v[i]);
+    for (int m = 0; m < M; ++m) {
+      const int i = w + 4 * m;
+      if (i < e.n) {
+        const float4 x = stg4(stg, i, row);
+        *reinterpret_cast<uint2*>(e.vc + ((size_t)head * e.ctx + (P + e.T + i)) * e.hd + j) =
+            pack4_bf16(x.x, x.y, x.z, x.w);
+      }
+    }
   }
   bar();
 }
 
+// gate/up tile (rows 0..63 gate, 64..127 up of channels tile*64..): u = silu(gate) * up, split.
 template <int BN, typename Bar>
 __device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  if (r >= 64) {
+  epi_stage<BN>(r, v, stg, bar);
+  const int w = r >> 5, l = r & 31;
+  const int c4 = (l & 15) * 4;  // 16 lanes per token, 4 channels each
+  const int ch = tile * 64 + c4;
+  if (ch < e.N) {  // N % 16 == 0: a 4-channel group is entirely valid or not
+    constexpr int M = (BN + 7) / 8;  // token pairs per warp: i = 2 (w + 4 m) + (l >> 4)
 #pragma unroll
-    for (int i = 0; i < BN; ++i) stg[r * (BN + 1) + i] = v[i];
-  }
-  bar();
-  const int ch = tile * 64 + r;
-  if (r < 64 && ch < e.N) {
-#pragma unroll
-    for (int i = 0; i < BN; ++i) {
+    for (int m = 0; m < M; ++m) {
+      const int i = 2 * (w + 4 * m) + (l >> 4);
       if (i < e.n) {
-        const float g = v[i];
-        const float up = stg[(r + 64) * (BN + 1) + i];
-        const float u = g / (1.f + expf(-g)) * up;
-        const uint16_t hi = f2bf(u);
-        e.u_out[(size_t)i * e.N + ch] = hi;
-        e.u_out[(size_t)(64 + i) * e.N + ch] = f2bf(u - bf2f(hi));
+        const float4 g = stg4(stg, i, c4), up = stg4(stg, i, 64 + c4);
+        float4 u;
+        u.x = g.x / (1.f + expf(-g.x)) * up.x;
+        u.y = g.y / (1.f + expf(-g.y)) * up.y;
+        u.z = g.z / (1.f + expf(-g.z)) * up.z;
+        u.w = g.w / (1.f + expf(-g.w)) * up.w;
+        uint2 hi, lo;
+        split4(u, hi, lo);
+        *reinterpret_cast<uint2*>(e.u_out + (size_t)i * e.N + ch) = hi;
+        *reinterpret_cast<uint2*>(e.u_out + (size_t)(64 + i) * e.N + ch) = lo;
       }
     }
   }
   bar();
 }
 
+// LM head: logits (optional) and, per token, the tile's (max, argmax, second max) over its rows;
+// ties go to the lowest vocabulary id.
 template <int BN, typename Bar>
 __device__ __forceinline__ void epi_lmhead(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  const int o = tile * 128 + r;
-  const bool valid = o < e.N;
-  if (e.logits != nullptr && valid) {
+  epi_stage<BN>(r, v, stg, bar);
+  const int w = r >> 5, l = r & 31;
+  const int o = tile * 128 + 4 * l;
+  const bool valid = o < e.N;  // N % 8 == 0: a 4-row group is entirely valid or not
+  constexpr int M = (BN + 3) / 4;
 #pragma unroll
-    for (int i = 0; i < BN; ++i)
-      if (i < e.n) e.logits[(size_t)i * e.N + o] = v[i];
-  }
-#pragma unroll
-  for (int i = 0; i < BN; ++i) stg[r * (BN + 1) + i] = valid ? v[i] : -INFINITY;
-  bar();
-  if (r < e.n) {
+  for (int m = 0; m < M; ++m) {
+    const int i = w + 4 * m;
+    if (i >= e.n) continue;  // warp-uniform
+    const float4 x = stg4(stg, i, 4 * l);
+    if (e.logits != nullptr && valid) *reinterpret_cast<float4*>(e.logits + (size_t)i * e.N + o) = x;
     float m1 = -INFINITY, m2 = -INFINITY;
-    int i1 = 0;
-    for (int row = 0; row < 128; ++row) {
-      const float x = stg[row * (BN + 1) + r];
-      if (x > m1) {
-        m2 = m1;
-        m1 = x;
-        i1 = row;
-      } else if (x > m2) {
-        m2 = x;
+    int i1 = 0x7fffffff;
+    if (valid) {
+      const float xs[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        if (xs[k] > m1) {
+          m2 = m1;
+          m1 = xs[k];
+          i1 = 4 * l + k;
+        } else if (xs[k] > m2) {
+          m2 = xs[k];
+        }
       }
     }
-    e.am_v1[tile * 64 + r] = m1;
-    e.am_i1[tile * 64 + r] = tile * 128 + i1;
-    e.am_v2[tile * 64 + r] = m2;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float om1 = __shfl_xor_sync(0xffffffffu, m1, off);
+      const float om2 = __shfl_xor_sync(0xffffffffu, m2, off);
+      const int oi1 = __shfl_xor_sync(0xffffffffu, i1, off);
+      if (om1 > m1 || (om1 == m1 && oi1 < i1)) {
+        m2 = fmaxf(m1, om2);
+        m1 = om1;
+        i1 = oi1;
+      } else {
+        m2 = fmaxf(m2, om1);
+      }
+    }
+    if (l == 0) {
+      e.am_v1[tile * 64 + i] = m1;
+      e.am_i1[tile * 64 + i] = tile * 128 + (i1 == 0x7fffffff ? 0 : i1);
+      e.am_v2[tile * 64 + i] = m2;
+    }
   }
   bar();
 }
 
-template <int BN>
-__device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, const float* v) {
-  const int o = tile * 128 + r;
-  if (o < e.N) {
+// y = v (stateless projection); any N and ldy.
+template <int BN, typename Bar>
+__device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+  epi_stage<BN>(r, v, stg, bar);
+  const int w = r >> 5, l = r & 31;
+  constexpr int M = (BN + 3) / 4;
 #pragma unroll
-    for (int i = 0; i < BN; ++i)
-      if (i < e.n) e.y[(size_t)i * e.ldy + o] = v[i];
+  for (int m = 0; m < M; ++m) {
+    const int i = w + 4 * m;
+    if (i >= e.n) continue;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {  // lane l: channels l, l + 32, l + 64, l + 96 (coalesced rows)
+      const int c = l + 32 * k, o = tile * 128 + c;
+      if (o < e.N) e.y[(size_t)i * e.ldy + o] = stg[i * kEpiStride + c];
+    }
   }
+  bar();
 }
 
-// y += v (fp32 residual stream); optionally the tile's per-token sum of squares of the updated rows,
-// the partial sums from which the next RMSNorm takes its scale (fixed order: deterministic), and
-// split(y * g_next), the operand of the next projection.
+// y += v (fp32 residual stream); optionally the tile's per-token sum of squares of the updated rows
+// (the partial sums from which the next RMSNorm takes its scale) and split(y * g_next), the operand
+// of the next projection.  N = d (a multiple of 128).
 template <int BN, typename Bar>
 __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  const int o = tile * 128 + r;
-  const bool valid = o < e.N;
-  const float gn = (e.xa_out != nullptr && valid) ? e.g_next[o] : 0.f;
+  epi_stage<BN>(r, v, stg, bar);
+  const int w = r >> 5, l = r & 31;
+  const int o = tile * 128 + 4 * l;
+  constexpr int M = (BN + 3) / 4;
+  float4 old[M];  // every load first: one memory round trip
 #pragma unroll
-  for (int i = 0; i < BN; ++i) {
-    float nv = 0.f;
-    if (i < e.n && valid) {
-      float* p = e.y + (size_t)i * e.ldy + o;
-      nv = __ldcg(p) + v[i];
-      *p = nv;
-      if (e.xa_out != nullptr) {
-        const float a = nv * gn;
-        const uint16_t hi = f2bf(a);
-        e.xa_out[(size_t)i * e.ldy + o] = hi;
-        e.xa_out[(size_t)(64 + i) * e.ldy + o] = f2bf(a - bf2f(hi));
-      }
-    }
-    if (e.ss_out != nullptr) stg[r * (BN + 1) + i] = nv * nv;
+  for (int m = 0; m < M; ++m) {
+    const int i = w + 4 * m;
+    old[m] = i < e.n ? __ldcg(reinterpret_cast<const float4*>(e.y + (size_t)i * e.ldy + o))
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  if (e.ss_out == nullptr) return;
-  bar();
-  if (r < e.n) {
-    float s = 0.f;
-    for (int row = 0; row < 128; ++row) s += stg[row * (BN + 1) + r];
-    e.ss_out[tile * 64 + r] = s;
+  const float4 gn =
+      e.xa_out != nullptr ? *reinterpret_cast<const float4*>(e.g_next + o) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int m = 0; m < M; ++m) {
+    const int i = w + 4 * m;
+    if (i >= e.n) continue;  // warp-uniform
+    const float4 x = stg4(stg, i, 4 * l);
+    float4 nv;
+    nv.x = old[m].x + x.x;
+    nv.y = old[m].y + x.y;
+    nv.z = old[m].z + x.z;
+    nv.w = old[m].w + x.w;
+    *reinterpret_cast<float4*>(e.y + (size_t)i * e.ldy + o) = nv;
+    if (e.xa_out != nullptr) {
+      uint2 hi, lo;
+      split4(make_float4(nv.x * gn.x, nv.y * gn.y, nv.z * gn.z, nv.w * gn.w), hi, lo);
+      *reinterpret_cast<uint2*>(e.xa_out + (size_t)i * e.ldy + o) = hi;
+      *reinterpret_cast<uint2*>(e.xa_out + (size_t)(64 + i) * e.ldy + o) = lo;
+    }
+    if (e.ss_out != nullptr) {
+      const float s = warp_sum(nv.x * nv.x + nv.y * nv.y + nv.z * nv.z + nv.w * nv.w);
+      if (l == 0) e.ss_out[tile * 64 + i] = s;
+    }
   }
   bar();
 }
 
 template <int BN, int EPI, typename Bar>
 __device__ __forceinline__ void run_epilogue(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  if constexpr (EPI == EPI_STORE) epi_store<BN>(e, tile, r, v);
+  if constexpr (EPI == EPI_STORE) epi_store<BN>(e, tile, r, v, stg, bar);
   if constexpr (EPI == EPI_RESID) epi_resid<BN>(e, tile, r, v, stg, bar);
   if constexpr (EPI == EPI_QKV) epi_qkv<BN>(e, tile, r, v, stg, bar);
   if constexpr (EPI == EPI_GLU) epi_glu<BN>(e, tile, r, v, stg, bar);

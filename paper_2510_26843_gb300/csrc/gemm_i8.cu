@@ -30,7 +30,7 @@ __device__ __forceinline__ uint4 ldg_nc16(const void* p) {
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a) {
-  extern __shared__ float stg[];  // [128][BN + 1]
+  extern __shared__ float stg[];  // [128][BN + 1] dequantised tile, then the epilogue's staging
   __shared__ int s_last;
   const int tile = blockIdx.x, ks = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
@@ -165,7 +165,7 @@ static cudaError_t launch_t(const GemmI8Args& a, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.tiles, a.ksplit);
   cfg.blockDim = dim3(kI8Threads);
-  cfg.dynamicSmemBytes = (size_t)128 * (BN + 1) * 4;
+  cfg.dynamicSmemBytes = (size_t)epi_staging_floats(BN) * 4;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -30,7 +30,7 @@ constexpr int kGemmThreads = 192;
 constexpr uint32_t kATileBytes = 128 * 128;  // 128 rows x 64 bf16
 
 __host__ __device__ constexpr uint32_t gemm_stage_bytes(int BN) { return kATileBytes + (uint32_t)BN * 128u; }
-__host__ __device__ constexpr uint32_t gemm_staging_bytes(int BN) { return 128u * (uint32_t)(BN + 1) * 4u; }
+__host__ __device__ constexpr uint32_t gemm_staging_bytes(int BN) { return (uint32_t)epi_staging_floats(BN) * 4u; }
 #ifndef CASSPEC_GEMM_SMEM_BUDGET
 #define CASSPEC_GEMM_SMEM_BUDGET (200u * 1024u)
 #endif
