@@ -54,13 +54,13 @@ __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence
 
 template <int BN, typename Bar>
 __device__ __forceinline__ void chain_epilogue(int epi, const EpiParams& e, int tile, int r, const float* v, float* stg,
-                                               Bar bar) {
+                                               Bar bar, int i0, int i1) {
   switch (epi) {
-    case EPI_RESID: run_epilogue<BN, EPI_RESID>(e, tile, r, v, stg, bar); break;
-    case EPI_QKV: run_epilogue<BN, EPI_QKV>(e, tile, r, v, stg, bar); break;
-    case EPI_GLU: run_epilogue<BN, EPI_GLU>(e, tile, r, v, stg, bar); break;
-    case EPI_LMHEAD: run_epilogue<BN, EPI_LMHEAD>(e, tile, r, v, stg, bar); break;
-    default: run_epilogue<BN, EPI_STORE>(e, tile, r, v, stg, bar); break;
+    case EPI_RESID: run_epilogue<BN, EPI_RESID>(e, tile, r, v, stg, bar, i0, i1); break;
+    case EPI_QKV: run_epilogue<BN, EPI_QKV>(e, tile, r, v, stg, bar, i0, i1); break;
+    case EPI_GLU: run_epilogue<BN, EPI_GLU>(e, tile, r, v, stg, bar, i0, i1); break;
+    case EPI_LMHEAD: run_epilogue<BN, EPI_LMHEAD>(e, tile, r, v, stg, bar, i0, i1); break;
+    default: run_epilogue<BN, EPI_STORE>(e, tile, r, v, stg, bar, i0, i1); break;
   }
 }
 
@@ -88,7 +88,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
-  // [0] abort, [1] last-arriver, [2..9] per-warp accumulator-ready votes (two segments)
+  // [0] abort, [1] fix-up wait result, [2..9] per-warp accumulator-ready votes (two segments),
+  // [2] after the main loops: this CTA is the last out
   volatile int* flags = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -350,49 +351,82 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         if (lane == 0) mbar_arrive(&tempty[buf]);
         buf ^= 1;
 
-        // stream-K fix-up over the CTAs that own units of tile t (CTAs with no unit at all, which
-        // exist when the phase has fewer units than CTAs, are skipped)
+        // Stream-K fix-up.  Every owner of a shared tile deposits its partial ([token][row] slot
+        // t + cta) and counts itself in.  The owners for which the tile is their last segment of
+        // the phase (all but possibly the one that holds the tile's tail at the start of its range)
+        // reach it together at the end of the phase: each waits for every deposit, sums one slice
+        // of the tokens over the owners in CTA order (deterministic) and runs the epilogue on it.
+        // CTAs with no unit at all (phases with fewer units than CTAs) are not owners.
         const int c_first = chain_cta_of((long long)t * kb, U, G);
         const int c_last = chain_cta_of((long long)(t + 1) * kb - 1, U, G);
+        int i0 = 0, i1 = n;
         bool finish = true;
         if (c_first != c_last) {
-          int owners = 0;
-          for (int cc = c_first; cc <= c_last; ++cc) owners += chain_u0(cc + 1, U, G) > chain_u0(cc, U, G);
+          const long long tile_end = (long long)(t + 1) * kb;
+          int owners = 0, parts = 0, rank = 0;
+          for (int cc = c_first; cc <= c_last; ++cc) {
+            const long long b0 = chain_u0(cc, U, G), b1 = chain_u0(cc + 1, U, G);
+            if (b1 <= b0) continue;
+            ++owners;
+            if (b1 <= tile_end) {
+              if (cc == cta) rank = parts;
+              ++parts;
+            }
+          }
           float* mine = a.partials + (size_t)(t + cta) * (64 * 128);
 #pragma unroll
           for (int i = 0; i < BN; ++i)
             if (i < n) __stcg(mine + i * 128 + r, v[i]);
-          bar();  // then one gpu-scope fence (cumulative over the CTA's stores) before the arrival
+          bar();  // then one gpu-scope fence (cumulative over the CTA's stores) before counting in
           if (threadIdx.x == 64) {
             __threadfence();
-            const unsigned old = atomicAdd(&counters[t], 1u);
-            flags[1] = (old == (unsigned)(owners - 1)) ? 1 : 0;
+            atomicAdd(&counters[t], 1u);
           }
-          bar();
-          finish = flags[1] != 0;
+          finish = seg_end == u1;  // a participant: this is the CTA's last segment of the phase
           if (finish) {
-            // The last owner sums every owner's partial in CTA order.  Partials are [token][row]
-            // slots; own values go through shared memory in the same layout so that each thread
-            // accumulates whole float4s with coalesced 16-byte loads, all loads of one owner in
-            // flight together.
-#pragma unroll
-            for (int i = 0; i < BN; ++i) stg[i * 128 + r] = v[i];
+            if (threadIdx.x == 64) {
+              const uint64_t t0 = globaltimer_ns();
+              int ok = 1;
+              while (ld_acquire_u32(counters + t) < (unsigned)owners) {
+                if (flags[0] || globaltimer_ns() - t0 > kWaitLimitNs) {
+                  ok = 0;
+                  flags[0] = 1;
+                  set_status(a.status, CASSPEC_E_TIMEOUT);
+                  break;
+                }
+              }
+              flags[1] = ok;
+            }
             bar();
+            finish = flags[1] != 0;
+            i0 = rank * n / parts;
+            i1 = (rank + 1) * n / parts;
+          }
+          if (finish && i1 > i0) {
             __threadfence();
+#pragma unroll
+            for (int i = 0; i < BN; ++i) stg[i * 128 + r] = v[i];  // own partial, same layout
+            bar();
+            const int f0 = i0 * 32, f1 = i1 * 32;  // float4s of the slice
             float4 acc[BN / 4];
 #pragma unroll
             for (int j = 0; j < BN / 4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-            const int nf4 = n * 32;  // float4s of the valid tokens
             const float4* own4 = reinterpret_cast<const float4*>(stg);
             for (int cc = c_first; cc <= c_last; ++cc) {
               float4 t4[BN / 4];
               if (cc == cta) {
 #pragma unroll
-                for (int j = 0; j < BN / 4; ++j) t4[j] = r + 128 * j < nf4 ? own4[r + 128 * j] : make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int j = 0; j < BN / 4; ++j) {
+                  const int f = f0 + r + 128 * j;
+                  t4[j] = f < f1 ? own4[f] : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
               } else if (chain_u0(cc + 1, U, G) > chain_u0(cc, U, G)) {
                 const float4* pp = reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128));
 #pragma unroll
-                for (int j = 0; j < BN / 4; ++j) t4[j] = r + 128 * j < nf4 ? __ldcg(pp + r + 128 * j) : make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int j = 0; j < BN / 4; ++j) {
+                  const int f = f0 + r + 128 * j;
+                  t4[j] = f < f1 ? __ldcg(pp + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
               } else {
                 continue;
               }
@@ -407,21 +441,21 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             bar();
             float4* st4 = reinterpret_cast<float4*>(stg);
 #pragma unroll
-            for (int j = 0; j < BN / 4; ++j)
-              if (r + 128 * j < nf4) st4[r + 128 * j] = acc[j];
+            for (int j = 0; j < BN / 4; ++j) {
+              const int f = f0 + r + 128 * j;
+              if (f < f1) st4[f] = acc[j];
+            }
             bar();
 #pragma unroll
             for (int i = 0; i < BN; ++i) v[i] = stg[i * 128 + r];
-            bar();  // the epilogue reuses the staging area
-            if (threadIdx.x == 64) counters[t] = 0u;  // ready for the next launch
           }
         }
-        if (finish) {
+        if (finish && i1 > i0) {
           if (ss != nullptr) {
 #pragma unroll
             for (int i = 0; i < BN; ++i) v[i] *= rs[i];
           }
-          chain_epilogue<BN>(epi, ep, t, r, v, stg, bar);
+          chain_epilogue<BN>(epi, ep, t, r, v, stg, bar, i0, i1);
         }
         u = seg_end;
       }
@@ -444,12 +478,19 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem_base, TMEM_COLS);
   }
-  if (threadIdx.x == 0 && np > 1) {  // the last CTA out resets the phase-barrier counters
-    pdl_wait();  // (the exit counter, too, is the previous launch's until it completes)
+  // The last CTA out returns the phase-barrier, exit and fix-up counters to zero for the next
+  // launch (they belong to the previous launch until it completes, hence the dependency wait).
+  if (threadIdx.x == 0) {
+    pdl_wait();
     __threadfence();
-    if (atomicAdd(&a.bar[kMaxPhases], 1u) == (unsigned)(G - 1)) {
-      for (int p = 0; p <= kMaxPhases; ++p) a.bar[p] = 0u;
-    }
+    flags[2] = atomicAdd(&a.bar[kMaxPhases], 1u) == (unsigned)(G - 1) ? 1 : 0;
+  }
+  __syncthreads();
+  if (flags[2]) {
+    __threadfence();
+    for (int p = threadIdx.x; p <= kMaxPhases; p += blockDim.x) a.bar[p] = 0u;
+    for (int p = 0; p < np; ++p)
+      for (int t = threadIdx.x; t < a.ph[p].tiles; t += blockDim.x) a.counters[p * 1024 + t] = 0u;
   }
 }
 

@@ -4,7 +4,8 @@
 // (`stg`, epi_staging_floats(BN) floats); then each warp takes whole tokens and each lane four
 // consecutive channels, so every global access is a 16- or 8-byte vector and the per-token
 // reductions (sum of squares, argmax) are warp shuffles in a fixed order (deterministic).
-// `bar` synchronises the 128 threads (a named barrier).
+// `bar` synchronises the 128 threads (a named barrier).  Only tokens [i0, i1) (i1 <= n) are
+// written: a tile may be finished in token slices by several CTAs.
 #pragma once
 
 #include "common.cuh"
@@ -49,7 +50,8 @@ __device__ __forceinline__ float warp_sum(float s) {
 
 // Q/K/V: rotary on q and k at the node's tree position; q -> q_out, k, v -> cache slot P + T + i.
 template <int BN, typename Bar>
-__device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+__device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar,
+                                         int i0, int i1) {
   epi_stage<BN>(r, v, stg, bar);
   const int w = r >> 5, l = r & 31;
   const int row = 4 * l;
@@ -67,7 +69,7 @@ __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, con
   if (part < 2) {
     int pos[M];
 #pragma unroll
-    for (int m = 0; m < M; ++m) pos[m] = (w + 4 * m < e.n) ? __ldcg(e.pos + w + 4 * m) : 0;
+    for (int m = 0; m < M; ++m) pos[m] = (w + 4 * m >= i0 && w + 4 * m < i1) ? __ldcg(e.pos + w + 4 * m) : 0;
 #pragma unroll
     for (int m0 = 0; m0 < M; m0 += 8) {  // rotary tables of 8 tokens in flight at a time
       float4 c01[8], c23[8];
@@ -82,7 +84,7 @@ __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, con
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         const int i = w + 4 * (m0 + k);
-        if (m0 + k < M && i < e.n) {
+        if (m0 + k < M && i >= i0 && i < i1) {
           const float4 x = stg4(stg, i, row), y = stg4(stg, i, prow);
           const uint2 out = pack4_bf16(x.x * c01[k].x + sgn * y.x * c01[k].y, x.y * c01[k].z + sgn * y.y * c01[k].w,
                                        x.z * c23[k].x + sgn * y.z * c23[k].y, x.w * c23[k].z + sgn * y.w * c23[k].w);
@@ -97,7 +99,7 @@ __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, con
 #pragma unroll
     for (int m = 0; m < M; ++m) {
       const int i = w + 4 * m;
-      if (i < e.n) {
+      if (i >= i0 && i < i1) {
         const float4 x = stg4(stg, i, row);
         *reinterpret_cast<uint2*>(e.vc + ((size_t)head * e.ctx + (P + e.T + i)) * e.hd + j) =
             pack4_bf16(x.x, x.y, x.z, x.w);
@@ -109,7 +111,8 @@ __device__ __forceinline__ void epi_qkv(const EpiParams& e, int tile, int r, con
 
 // gate/up tile (rows 0..63 gate, 64..127 up of channels tile*64..): u = silu(gate) * up, split.
 template <int BN, typename Bar>
-__device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+__device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar,
+                                         int i0, int i1) {
   epi_stage<BN>(r, v, stg, bar);
   const int w = r >> 5, l = r & 31;
   const int c4 = (l & 15) * 4;  // 16 lanes per token, 4 channels each
@@ -119,13 +122,14 @@ __device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, con
 #pragma unroll
     for (int m = 0; m < M; ++m) {
       const int i = 2 * (w + 4 * m) + (l >> 4);
-      if (i < e.n) {
+      if (i >= i0 && i < i1) {
         const float4 g = stg4(stg, i, c4), up = stg4(stg, i, 64 + c4);
         float4 u;
-        u.x = g.x / (1.f + expf(-g.x)) * up.x;
-        u.y = g.y / (1.f + expf(-g.y)) * up.y;
-        u.z = g.z / (1.f + expf(-g.z)) * up.z;
-        u.w = g.w / (1.f + expf(-g.w)) * up.w;
+        // fast exponential and division: ~1e-6 relative error, below the 16-bit split
+        u.x = __fdividef(g.x, 1.f + __expf(-g.x)) * up.x;
+        u.y = __fdividef(g.y, 1.f + __expf(-g.y)) * up.y;
+        u.z = __fdividef(g.z, 1.f + __expf(-g.z)) * up.z;
+        u.w = __fdividef(g.w, 1.f + __expf(-g.w)) * up.w;
         uint2 hi, lo;
         split4(u, hi, lo);
         *reinterpret_cast<uint2*>(e.u_out + (size_t)i * e.N + ch) = hi;
@@ -139,7 +143,8 @@ __device__ __forceinline__ void epi_glu(const EpiParams& e, int tile, int r, con
 // LM head: logits (optional) and, per token, the tile's (max, argmax, second max) over its rows;
 // ties go to the lowest vocabulary id.
 template <int BN, typename Bar>
-__device__ __forceinline__ void epi_lmhead(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+__device__ __forceinline__ void epi_lmhead(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar,
+                                         int i0, int i1) {
   epi_stage<BN>(r, v, stg, bar);
   const int w = r >> 5, l = r & 31;
   const int o = tile * 128 + 4 * l;
@@ -148,7 +153,7 @@ __device__ __forceinline__ void epi_lmhead(const EpiParams& e, int tile, int r, 
 #pragma unroll
   for (int m = 0; m < M; ++m) {
     const int i = w + 4 * m;
-    if (i >= e.n) continue;  // warp-uniform
+    if (i < i0 || i >= i1) continue;  // warp-uniform
     const float4 x = stg4(stg, i, 4 * l);
     if (e.logits != nullptr && valid) *reinterpret_cast<float4*>(e.logits + (size_t)i * e.N + o) = x;
     float m1 = -INFINITY, m2 = -INFINITY;
@@ -190,14 +195,15 @@ __device__ __forceinline__ void epi_lmhead(const EpiParams& e, int tile, int r, 
 
 // y = v (stateless projection); any N and ldy.
 template <int BN, typename Bar>
-__device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+__device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar,
+                                         int i0, int i1) {
   epi_stage<BN>(r, v, stg, bar);
   const int w = r >> 5, l = r & 31;
   constexpr int M = (BN + 3) / 4;
 #pragma unroll
   for (int m = 0; m < M; ++m) {
     const int i = w + 4 * m;
-    if (i >= e.n) continue;
+    if (i < i0 || i >= i1) continue;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {  // lane l: channels l, l + 32, l + 64, l + 96 (coalesced rows)
       const int c = l + 32 * k, o = tile * 128 + c;
@@ -211,7 +217,8 @@ __device__ __forceinline__ void epi_store(const EpiParams& e, int tile, int r, c
 // (the partial sums from which the next RMSNorm takes its scale) and split(y * g_next), the operand
 // of the next projection.  N = d (a multiple of 128).
 template <int BN, typename Bar>
-__device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
+__device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar,
+                                         int i0, int i1) {
   epi_stage<BN>(r, v, stg, bar);
   const int w = r >> 5, l = r & 31;
   const int o = tile * 128 + 4 * l;
@@ -220,7 +227,7 @@ __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, c
 #pragma unroll
   for (int m = 0; m < M; ++m) {
     const int i = w + 4 * m;
-    old[m] = i < e.n ? __ldcg(reinterpret_cast<const float4*>(e.y + (size_t)i * e.ldy + o))
+    old[m] = (i >= i0 && i < i1) ? __ldcg(reinterpret_cast<const float4*>(e.y + (size_t)i * e.ldy + o))
                      : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   const float4 gn =
@@ -228,7 +235,7 @@ __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, c
 #pragma unroll
   for (int m = 0; m < M; ++m) {
     const int i = w + 4 * m;
-    if (i >= e.n) continue;  // warp-uniform
+    if (i < i0 || i >= i1) continue;  // warp-uniform
     const float4 x = stg4(stg, i, 4 * l);
     float4 nv;
     nv.x = old[m].x + x.x;
@@ -251,12 +258,13 @@ __device__ __forceinline__ void epi_resid(const EpiParams& e, int tile, int r, c
 }
 
 template <int BN, int EPI, typename Bar>
-__device__ __forceinline__ void run_epilogue(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar) {
-  if constexpr (EPI == EPI_STORE) epi_store<BN>(e, tile, r, v, stg, bar);
-  if constexpr (EPI == EPI_RESID) epi_resid<BN>(e, tile, r, v, stg, bar);
-  if constexpr (EPI == EPI_QKV) epi_qkv<BN>(e, tile, r, v, stg, bar);
-  if constexpr (EPI == EPI_GLU) epi_glu<BN>(e, tile, r, v, stg, bar);
-  if constexpr (EPI == EPI_LMHEAD) epi_lmhead<BN>(e, tile, r, v, stg, bar);
+__device__ __forceinline__ void run_epilogue(const EpiParams& e, int tile, int r, const float* v, float* stg, Bar bar,
+                                             int i0, int i1) {
+  if constexpr (EPI == EPI_STORE) epi_store<BN>(e, tile, r, v, stg, bar, i0, i1);
+  if constexpr (EPI == EPI_RESID) epi_resid<BN>(e, tile, r, v, stg, bar, i0, i1);
+  if constexpr (EPI == EPI_QKV) epi_qkv<BN>(e, tile, r, v, stg, bar, i0, i1);
+  if constexpr (EPI == EPI_GLU) epi_glu<BN>(e, tile, r, v, stg, bar, i0, i1);
+  if constexpr (EPI == EPI_LMHEAD) epi_lmhead<BN>(e, tile, r, v, stg, bar, i0, i1);
 }
 
 }  // namespace casspec

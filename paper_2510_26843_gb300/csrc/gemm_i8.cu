@@ -149,7 +149,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
     for (int i = 0; i < BN; ++i) v[i] = stg[tid * (BN + 1) + i];
   }
   __syncthreads();
-  if (tid < 128) run_epilogue<BN, EPI>(a.ep, tile, tid, v, stg, [] { named_bar_sync(1, 128); });
+  if (tid < 128) run_epilogue<BN, EPI>(a.ep, tile, tid, v, stg, [] { named_bar_sync(1, 128); }, 0, a.ep.n);
 }
 
 int gemm_i8_ksplit(int tiles, int K, int num_sms) {

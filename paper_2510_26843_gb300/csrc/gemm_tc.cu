@@ -279,7 +279,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           if (threadIdx.x == 64) a.counters[t] = 0u;  // ready for the next launch
         }
       }
-      if (finish) run_epilogue<BN, EPI>(a.ep, t, r, v, stg, bar);
+      if (finish) run_epilogue<BN, EPI>(a.ep, t, r, v, stg, bar, 0, a.ep.n);
       u = seg_end;
     }
   }
