@@ -130,12 +130,19 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
     const uint32_t qbase = smem_u32(qs);
     const unsigned long long ancA = rA < a.n ? __ldcg(a.anc + rA) : 0ull;
     const unsigned long long ancB = rB < a.n ? __ldcg(a.anc + rB) : 0ull;
-    for (int idx = tid; idx < 64 * NCH; idx += kAttnCompute) {
-      const int row = idx / NCH, c = idx % NCH;
-      uint4 val = make_uint4(0, 0, 0, 0);
-      if (row < a.n) val = __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)row * a.d + head * HD + c * 8));
-      asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(swz(qbase, row, c)), "r"(val.x), "r"(val.y),
-                   "r"(val.z), "r"(val.w)
+    constexpr int QPT = 64 * NCH / kAttnCompute;  // 16-byte chunks of Q per thread
+    uint4 qv[QPT];  // every load in flight before the first shared-memory store
+#pragma unroll
+    for (int k = 0; k < QPT; ++k) {
+      const int idx = tid + k * kAttnCompute, row = idx / NCH, c = idx % NCH;
+      qv[k] = row < a.n ? __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)row * a.d + head * HD + c * 8))
+                        : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int k = 0; k < QPT; ++k) {
+      const int idx = tid + k * kAttnCompute, row = idx / NCH, c = idx % NCH;
+      asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(swz(qbase, row, c)), "r"(qv[k].x), "r"(qv[k].y),
+                   "r"(qv[k].z), "r"(qv[k].w)
                    : "memory");
     }
     cbar();
@@ -174,25 +181,38 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
         }
         const int sbase = b * kAttnBlk;
         float mxA = -INFINITY, mxB = -INFINITY;
+        if (sbase + kAttnBlk <= P) {  // a block of the committed prefix: visible to every node
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
+          for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int slot = sbase + nt * 8 + 2 * t4 + e;
-            bool visA, visB;
-            if (slot < P) {
-              visA = visB = true;
-            } else if (slot < total) {
-              const int j = slot - P;
-              visA = (ancA >> j) & 1ull;
-              visB = (ancB >> j) & 1ull;
-            } else {
-              visA = visB = false;
+            for (int e = 0; e < 2; ++e) {
+              s[nt][e] *= a.scale_log2;
+              s[nt][2 + e] *= a.scale_log2;
+              mxA = fmaxf(mxA, s[nt][e]);
+              mxB = fmaxf(mxB, s[nt][2 + e]);
             }
-            s[nt][e] = visA ? s[nt][e] * a.scale_log2 : -INFINITY;
-            s[nt][2 + e] = visB ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
-            mxA = fmaxf(mxA, s[nt][e]);
-            mxB = fmaxf(mxB, s[nt][2 + e]);
+          }
+        } else {
+#pragma unroll
+          for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int slot = sbase + nt * 8 + 2 * t4 + e;
+              bool visA, visB;
+              if (slot < P) {
+                visA = visB = true;
+              } else if (slot < total) {
+                const int j = slot - P;
+                visA = (ancA >> j) & 1ull;
+                visB = (ancB >> j) & 1ull;
+              } else {
+                visA = visB = false;
+              }
+              s[nt][e] = visA ? s[nt][e] * a.scale_log2 : -INFINITY;
+              s[nt][2 + e] = visB ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
+              mxA = fmaxf(mxA, s[nt][e]);
+              mxB = fmaxf(mxB, s[nt][2 + e]);
+            }
           }
         }
         mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 1));
