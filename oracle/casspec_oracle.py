@@ -292,12 +292,15 @@ def tree_attention(q: np.ndarray, kv: KVCache, layer: int, slots: list, anc: lis
 
 def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
               skip_mask: np.ndarray | None = None, quant_mode: int = 0,
-              trace: dict | None = None) -> np.ndarray:
+              trace: dict | None = None, attn_bf16: bool = False) -> np.ndarray:
     """One draft/verify pass over n new tree nodes; returns logits [n, V] (fp64).
 
     The nodes occupy tree slots T .. T+n-1 (cache slots P+T .. P+T+n-1); each active layer writes
     their K/V there.  skip_mask[l] == 0 switches layer l off (Sec. 4.1 layer sparsity).
     quant_mode 1 runs the W8A8 draft (App. C).  `trace`, if given, receives per-layer intermediates.
+    attn_bf16 rounds q and the K/V written to the cache to bf16 (a bf16 cache and bf16 attention
+    operands).  It is a perturbation of the size of bf16 storage, used by tests to measure how far
+    the method's own output moves under it; the reference result keeps it off.
     """
     sh = w.shape
     tokens = np.asarray(tokens, dtype=np.int64)
@@ -322,6 +325,8 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
         q = rope(qkv[:, :d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
         k = rope(qkv[:, d:2 * d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
         v = qkv[:, 2 * d:].reshape(n, H, h)
+        if attn_bf16:
+            q, k, v = round_bf16(q), round_bf16(k), round_bf16(v)
         for i, s in enumerate(slots):
             kv.K[l][:, s] = k[i]
             kv.V[l][:, s] = v[i]

@@ -329,6 +329,28 @@ def test_int8_mode_close_to_bf16_mode(tiny):
     assert 1e-5 < err < 0.1, err
 
 
+def test_attn_bf16_rounds_only_the_attention_operands(tiny):
+    """attn_bf16 stores bf16 K/V and uses bf16 q: the cache entries it writes are bf16 values,
+    everything else is the fp64 model, and the logits move by about the bf16 rounding."""
+    w, ref, prefix = tiny
+    toks, parent = synth.tokens(5, 8, SH.vocab), synth.tree(5, 8, 4)
+    kv1, _ = _prefilled(w, prefix)
+    kv2, _ = _prefilled(w, prefix)
+    tr1, tr2 = {}, {}
+    a = oracle.tree_step(w, kv1, toks, parent, trace=tr1)
+    b = oracle.tree_step(w, kv2, toks, parent, trace=tr2, attn_bf16=True)
+    P = len(prefix)
+    for l in range(SH.n_layers):
+        new_k = kv2.K[l][:, P:P + 8]
+        assert np.array_equal(new_k, oracle.round_bf16(new_k))
+        assert np.array_equal(tr2[l]["q"], oracle.round_bf16(tr2[l]["q"]))
+        assert not np.array_equal(kv1.K[l][:, P:P + 8], oracle.round_bf16(kv1.K[l][:, P:P + 8]))
+    # layer 0's normalised input does not depend on attention: identical
+    assert np.array_equal(tr1[0]["xn"], tr2[0]["xn"])
+    err = np.max(np.abs(a - b) / np.ptp(a, axis=1, keepdims=True))
+    assert 1e-6 < err < 1e-2, err
+
+
 # ------------------------------------------------------------------------------------------------
 # acceptance vs brute force; losslessness; compaction
 # ------------------------------------------------------------------------------------------------
