@@ -260,6 +260,20 @@ CASSPEC_API size_t casspec_linear_workspace_bytes(int N, int K, int n);
 CASSPEC_API int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int n, float* Y, int ldy,
                         void* workspace, size_t workspace_bytes, void* cuda_stream);
 
+/* casspec_linear_bf16 without a caller workspace: the same projection (Y = X W^T, fp32 accumulation
+ * on the tensor cores, same arguments and layout as casspec_linear_bf16), with its stream-K scratch
+ * in a static device array of the library (8 MB + 4 KB per device).  The paper has no counterpart:
+ * this is plumbing for callers that cannot allocate device memory at the call site.
+ *   Allocates nothing.  The first call on a device looks up the scratch address (with that device
+ *   current); make that first call before capturing any stream.  Every call clears the scratch's
+ *   counter block on `cuda_stream` before its kernel, so nothing needs to be zeroed by the caller.
+ *   The scratch is shared by all calls on a device: calls that overlap in time (other streams or
+ *   threads) race on it and must be serialised by the caller.
+ *   Returns CASSPEC_E_CAPACITY when ceil(N / 128) + min(ceil(N/128) * ceil(K/64), SM count) > 256
+ *   (N up to 13,312 on a 152-SM GB300); other errors as casspec_linear_bf16. */
+CASSPEC_API int casspec_linear_bf16_static(const uint16_t* W, int N, int K, const uint16_t* X, int n, float* Y, int ldy,
+                               void* cuda_stream);
+
 /* RMSNorm of n rows (Llama pre-norm): y = x / sqrt(mean(x^2) + eps) * g, fp32 arithmetic.
  *   x dev fp32 [n][d]; g dev fp32 [d]; y_bf16 dev bf16 [n][d] (may be NULL if q is given).
  *   If q_out (dev int8 [n][d]) and s_out (dev fp32 [n]) are non-NULL, each bf16 output row is also

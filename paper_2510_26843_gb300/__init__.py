@@ -27,7 +27,8 @@ EXPORTS = [
     "casspec_set_options", "casspec_tensor", "casspec_quantize_weights", "casspec_kv_bytes", "casspec_kv_create",
     "casspec_kv_destroy", "casspec_kv_layer", "casspec_kv_set_prefix", "casspec_kv_reset_tree", "casspec_kv_length",
     "casspec_tree_step", "casspec_argmax", "casspec_accept_greedy", "casspec_kv_compact", "casspec_get_status",
-    "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_rmsnorm",
+    "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_linear_bf16_static",
+    "casspec_rmsnorm",
     "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
@@ -82,6 +83,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_status_string": (ctypes.c_char_p, [_I]),
         "casspec_linear_workspace_bytes": (_SZ, [_I, _I, _I]),
         "casspec_linear_bf16": (_I, [_P, _I, _I, _P, _I, _P, _I, _P, _SZ, _P]),
+        "casspec_linear_bf16_static": (_I, [_P, _I, _I, _P, _I, _P, _I, _P]),
         "casspec_rmsnorm": (_I, [_P, _P, _I, _I, ctypes.c_float, _P, _P, _P, _P]),
         "casspec_quantize_rows": (_I, [_P, _I, _I, _P, _P, _P]),
         "casspec_profile": (_I, [_P, _I]),
@@ -244,6 +246,11 @@ def linear_bf16(W, N: int, K: int, X, n: int, Y, ldy: int, workspace, stream=Non
     _check("casspec_linear_bf16",
            load_library().casspec_linear_bf16(_ptr(W), N, K, _ptr(X), n, _ptr(Y), ldy, _ptr(workspace),
                                               workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def linear_bf16_static(W, N: int, K: int, X, n: int, Y, ldy: int, stream=None) -> None:
+    _check("casspec_linear_bf16_static",
+           load_library().casspec_linear_bf16_static(_ptr(W), N, K, _ptr(X), n, _ptr(Y), ldy, _stream(stream)))
 
 
 def rmsnorm(x, g, n: int, d: int, eps: float, y=None, q=None, s=None, stream=None) -> None:
