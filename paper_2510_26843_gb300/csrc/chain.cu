@@ -37,7 +37,12 @@ __host__ __device__ constexpr int chain_w_stages(int BN) {
                                                                    : (int)((kChainSmemBudget - chain_fixed(BN)) / kWTile);
 }
 __host__ __device__ constexpr size_t chain_smem(int BN) { return chain_fixed(BN) + (size_t)chain_w_stages(BN) * kWTile; }
-__host__ __device__ constexpr uint32_t chain_tmem_cols(int BN) { return 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : 128); }
+// TMEM per accumulator buffer: two accumulators (alternate k-steps) of 2*BN columns (the hi and
+// lo planes stacked as one N = 2*BN operand); two buffers.
+__host__ __device__ constexpr uint32_t chain_buf_cols(int BN) { return 4u * (uint32_t)BN; }
+__host__ __device__ constexpr uint32_t chain_tmem_cols(int BN) {
+  return 2 * chain_buf_cols(BN) <= 128 ? 128 : (2 * chain_buf_cols(BN) <= 256 ? 256 : 512);
+}
 
 __device__ __forceinline__ long long chain_u0(int c, long long U, int G) { return (long long)c * U / G; }
 // CTA that owns unit x when U units are split into G contiguous ranges [c U / G, (c + 1) U / G)
@@ -72,7 +77,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   constexpr uint32_t XT = (uint32_t)BN * 128u;  // one hi or lo tile
   constexpr uint32_t XS = 2 * XT;
   constexpr uint32_t TMEM_COLS = chain_tmem_cols(BN);
-  constexpr uint32_t IDESC = idesc_bf16_f32(128, BN);
+  constexpr uint32_t IDESC = idesc_bf16_f32(128, 2 * BN);  // B = [hi; lo], N = 2 * BN
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -242,7 +247,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+          const uint32_t d_tmem = tmem_base + (uint32_t)buf * chain_buf_cols(BN);
           for (long long uu = u; uu < seg_end; ++uu) {
             if (!mbar_wait_bounded(&wfull[ws], wph, flags) || !mbar_wait_bounded(&xfull[xs], xph, flags)) {
               ok = false;
@@ -250,13 +255,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             }
             tc_fence_after();
             const uint32_t sa = smem_u32(wring + ws * kWTile);
-            const uint32_t sh = smem_u32(xring + xs * XS), sl = sh + XT;
+            const uint32_t sh = smem_u32(xring + xs * XS);
+            // One MMA per 16-column k-step with the hi and lo planes stacked (N = 2 * BN, the X stage
+            // holds them back to back); even and odd k-steps go to two accumulators so that
+            // consecutive MMAs do not depend on each other.
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t ad = sw128_kmajor_desc(sa + kk * 32);
-              tc_mma_bf16(d_tmem, ad, sw128_kmajor_desc(sh + kk * 32), IDESC, (uu > u || kk > 0) ? 1u : 0u);
-              tc_mma_bf16(d_tmem, ad, sw128_kmajor_desc(sl + kk * 32), IDESC, 1u);
-            }
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_bf16(d_tmem + (uint32_t)(kk & 1) * (2u * BN), sw128_kmajor_desc(sa + kk * 32),
+                          sw128_kmajor_desc(sh + kk * 32), IDESC, (uu > u || kk >= 2) ? 1u : 0u);
             tc_commit(&wempty[ws]);
             tc_commit(&xempty[xs]);
             if (++ws == SW) {
@@ -342,10 +348,18 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         }
         tc_fence_after();
         float v[BN];
-        const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
+        const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)buf * chain_buf_cols(BN);
 #pragma unroll
-        for (int c = 0; c < BN; c += 16) tmem_ld_x16(taddr + c, &v[c]);
-        tmem_ld_wait();
+        for (int c = 0; c < BN; c += 16) {  // (acc0 hi + acc0 lo) + (acc1 hi + acc1 lo), fixed order
+          float t1[16], t2[16], t3[16];
+          tmem_ld_x16(taddr + c, &v[c]);
+          tmem_ld_x16(taddr + BN + c, t1);
+          tmem_ld_x16(taddr + 2 * BN + c, t2);
+          tmem_ld_x16(taddr + 3 * BN + c, t3);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) v[c + j] = (v[c + j] + t1[j]) + (t2[j] + t3[j]);
+        }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
@@ -364,19 +378,32 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         if (c_first != c_last) {
           const long long tile_end = (long long)(t + 1) * kb;
           int owners = 0, parts = 0, rank = 0;
+          int own_list[6];  // the first 6 owners in CTA order
           for (int cc = c_first; cc <= c_last; ++cc) {
             const long long b0 = chain_u0(cc, U, G), b1 = chain_u0(cc + 1, U, G);
             if (b1 <= b0) continue;
+#pragma unroll
+            for (int o = 0; o < 6; ++o)
+              if (o == owners) own_list[o] = cc;
             ++owners;
             if (b1 <= tile_end) {
               if (cc == cta) rank = parts;
               ++parts;
             }
           }
-          float* mine = a.partials + (size_t)(t + cta) * (64 * 128);
+          // own partial token-major in shared memory ([token][row], the slot layout), then coalesced
+          // 16-byte stores of the valid tokens into slot t + cta
 #pragma unroll
-          for (int i = 0; i < BN; ++i)
-            if (i < n) __stcg(mine + i * 128 + r, v[i]);
+          for (int i = 0; i < BN; ++i) stg[i * 128 + r] = v[i];
+          bar();
+          const int nf4 = n * 32;
+          const float4* own4 = reinterpret_cast<const float4*>(stg);
+          {
+            float4* mine4 = reinterpret_cast<float4*>(a.partials + (size_t)(t + cta) * (64 * 128));
+#pragma unroll
+            for (int j = 0; j < BN / 4; ++j)
+              if (r + 128 * j < nf4) __stcg(mine4 + r + 128 * j, own4[r + 128 * j]);
+          }
           bar();  // then one gpu-scope fence (cumulative over the CTA's stores) before counting in
           if (threadIdx.x == 64) {
             __threadfence();
@@ -404,38 +431,53 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           }
           if (finish && i1 > i0) {
             __threadfence();
-#pragma unroll
-            for (int i = 0; i < BN; ++i) stg[i * 128 + r] = v[i];  // own partial, same layout
-            bar();
             const int f0 = i0 * 32, f1 = i1 * 32;  // float4s of the slice
             float4 acc[BN / 4];
 #pragma unroll
             for (int j = 0; j < BN / 4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-            const float4* own4 = reinterpret_cast<const float4*>(stg);
-            for (int cc = c_first; cc <= c_last; ++cc) {
-              float4 t4[BN / 4];
-              if (cc == cta) {
+            auto add4 = [](float4& x, const float4& y) {
+              x.x += y.x;
+              x.y += y.y;
+              x.z += y.z;
+              x.w += y.w;
+            };
+            if (owners <= 6 && f1 - f0 <= 4 * 128) {
+              // a small slice (at most 4 float4s per thread) from at most 6 owners: every load in
+              // flight together; sums in CTA order
+              float4 t4[6][4];
 #pragma unroll
-                for (int j = 0; j < BN / 4; ++j) {
-                  const int f = f0 + r + 128 * j;
-                  t4[j] = f < f1 ? own4[f] : make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-              } else if (chain_u0(cc + 1, U, G) > chain_u0(cc, U, G)) {
-                const float4* pp = reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128));
+              for (int o = 0; o < 6; ++o) {
 #pragma unroll
-                for (int j = 0; j < BN / 4; ++j) {
+                for (int j = 0; j < 4; ++j) {
                   const int f = f0 + r + 128 * j;
-                  t4[j] = f < f1 ? __ldcg(pp + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+                  float4 val = make_float4(0.f, 0.f, 0.f, 0.f);
+                  if (o < owners && f < f1) {
+                    const int cc = own_list[o];
+                    val = cc == cta ? own4[f]
+                                    : __ldcg(reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128)) + f);
+                  }
+                  t4[o][j] = val;
                 }
-              } else {
-                continue;
               }
 #pragma unroll
-              for (int j = 0; j < BN / 4; ++j) {
-                acc[j].x += t4[j].x;
-                acc[j].y += t4[j].y;
-                acc[j].z += t4[j].z;
-                acc[j].w += t4[j].w;
+              for (int o = 0; o < 6; ++o) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                  if (j < BN / 4) add4(acc[j], t4[o][j]);
+              }
+            } else {  // larger slices or many owners: one owner at a time, all its loads in flight
+              for (int cc = c_first; cc <= c_last; ++cc) {
+                if (cc != cta && chain_u0(cc + 1, U, G) <= chain_u0(cc, U, G)) continue;
+                const float4* src = cc == cta ? own4
+                                              : reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128));
+                float4 t4[BN / 4];
+#pragma unroll
+                for (int j = 0; j < BN / 4; ++j) {
+                  const int f = f0 + r + 128 * j;
+                  t4[j] = f < f1 ? (cc == cta ? src[f] : __ldcg(src + f)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int j = 0; j < BN / 4; ++j) add4(acc[j], t4[j]);
               }
             }
             bar();
