@@ -42,18 +42,25 @@ FALLBACK_HBM_GBS = 6800.0
 WORKLOADS = {
     "verify7b": (32, 2048, 64, 8, None, 0.0, 0, True),
     "layer7b": (1, 1024, 32, 6, 4, 0.0, 0, True),
+    "verify13b": (40, 4096, 64, 8, None, 0.0, 0, True),
+    # one cascade round: the 60%-skip W8A8 draft appends the tree level by level, the 40%-skip bf16
+    # draft re-checks all 64 nodes, then the full verify, acceptance and compaction
+    "cascade13b": (40, 4096, 64, 8, None, 0.0, 0, True),
 }
 for _n in (1, 2, 4, 8):
     WORKLOADS[f"draft7b-skip50-n{_n}"] = (32, 2048, _n, 8, None, 0.5, 0, False)
     WORKLOADS[f"draft7b-int8-n{_n}"] = (32, 2048, _n, 8, None, 0.0, 1, False)
     WORKLOADS[f"draft7b-skip50-int8-n{_n}"] = (32, 2048, _n, 8, None, 0.5, 1, False)
+FAMILY = {"verify13b": "13b", "cascade13b": "13b"}  # others: 7B shape
+CASCADE_SKIP = (0.4, 0.6)  # d1 (bf16) and d2 (W8A8) layer-skip fractions of the 13B cascade
 
 
-def _shape(layers: int = 32):
+def _shape(layers: int | None = None, family: str = "7b"):
     import synth
 
-    s = synth.LLAMA7B
-    return synth.ModelShape(layers, s.d_model, s.n_heads, s.head_dim, s.ffn, s.vocab)
+    s = synth.LLAMA13B if family == "13b" else synth.LLAMA7B
+    return synth.ModelShape(s.n_layers if layers is None else layers, s.d_model, s.n_heads, s.head_dim, s.ffn,
+                            s.vocab)
 
 
 def algorithmic_bytes(shape, n: int, P: int, layers_on: int | None = None, quant: int = 0) -> dict:
@@ -179,11 +186,11 @@ class OracleSampler:
     that layer on (t1) and the step with no layer (t0: embedding, final norm, LM head); the full
     step is estimated as t0 + 32 * (t1 - t0)."""
 
-    def __init__(self, parent, toks, P: int, n_layers: int, mode: int = 0):
+    def __init__(self, parent, toks, P: int, n_layers: int, mode: int = 0, family: str = "7b"):
         import oracle
         import synth
 
-        sh = _shape()
+        sh = _shape(None, family)
         self.sh1 = synth.ModelShape(1, sh.d_model, sh.n_heads, sh.head_dim, sh.ffn, sh.vocab)
         self.w = oracle.Weights.from_seed(SEED, self.sh1, keep_layers=1)
         for name in ("wqkv", "wo", "wg", "wu", "wd"):
@@ -227,12 +234,36 @@ def workload_tree(wl):
     return parent, toks
 
 
+def bfs_levels(parent, toks):
+    """The tree reordered by depth (parents first) and the [start, end) node range of each level."""
+    n = len(parent)
+    depth = [0] * n
+    for i in range(1, n):
+        depth[i] = depth[parent[i]] + 1
+    order = sorted(range(n), key=lambda i: (depth[i], i))
+    pos = {old: new for new, old in enumerate(order)}
+    par = np.array([-1 if parent[o] < 0 else pos[int(parent[o])] for o in order], dtype=np.int32)
+    tk = np.array([toks[o] for o in order], dtype=np.int32)
+    levels, start = [], 0
+    for d in range(max(depth) + 1):
+        cnt = sum(1 for x in depth if x == d)
+        levels.append((start, start + cnt))
+        start += cnt
+    return par, tk, levels
+
+
 def describe(name: str, wl) -> str:
     layers, P, n, depth, branch, skip, mode, verify = wl
+    fam = FAMILY.get(name, "7b")
+    d = _shape(None, fam).d_model
+    if name.startswith("cascade"):
+        return (f"{name}: llama{fam}-shape {layers} layers, d{d}, prefix {P}; one cascade round on a {n}-node tree "
+                f"(depth<={depth}): {int(CASCADE_SKIP[1] * 100)}%-skip W8A8 draft level by level, "
+                f"{int(CASCADE_SKIP[0] * 100)}%-skip bf16 re-check of all nodes, full verify + accept + compact")
     kind = "tree verify + accept + compact" if verify else "draft step (tree reset after)"
     extra = (f", {int(skip * 100)}% layers skipped" if skip else "") + (", W8A8" if mode else ", bf16")
     br = f", branching<={branch}" if branch else ""
-    return (f"{name}: llama7b-shape {layers} layer(s), d4096, n={n} nodes (depth<={depth}{br}), prefix {P}{extra}; "
+    return (f"{name}: llama{fam}-shape {layers} layer(s), d{d}, n={n} nodes (depth<={depth}{br}), prefix {P}{extra}; "
             f"{kind}")
 
 
@@ -243,25 +274,54 @@ def config_block(args, name, wl, graphs: bool) -> dict:
             "cuda_graphs": graphs, "pdl": True, "parallelism": f"replicas{args.gpus}"}
 
 
+def oracle_estimate(name, wl, parent, toks, seconds: float, steps: int | None = None) -> tuple[float, str]:
+    """The oracle's time for one step (or one cascade round) of workload `name`, from bounded samples:
+    embedding + 1 layer + LM head, scaled to the active layers of each tree step involved."""
+    layers, P, n, depth, branch, skip, mode, verify = wl
+    family = FAMILY.get(name, "7b")
+    if name.startswith("cascade"):
+        import synth
+
+        par, tk, levels = bfs_levels(parent, toks)
+        m1, m2 = synth.skip_masks(SEED, layers, list(CASCADE_SKIP))
+        parts = [(tk[a:b], np.where(par[a:b] < a, -1, par[a:b] - a), int(m2.sum()), 1) for (a, b) in levels]
+        parts += [(tk, par, int(m1.sum()), 0), (tk, par, layers, 0)]
+        total, desc = 0.0, []
+        for tks, prt, on, md in parts:
+            s = OracleSampler(prt, tks, P, on, md, family)
+            total += float(np.mean([s.sample_us() for _ in range(2)]))
+        return total, (f"fp64 oracle, each of the round's {len(parts)} tree steps sampled as embedding + 1 layer + "
+                       f"LM head and scaled to its active layers (draft levels rooted at the level's first node)")
+    layers_on = layers if not skip else int(round(layers * (1 - skip)))
+    s = OracleSampler(parent, toks, P, layers_on, mode, family)
+    t_start = time.perf_counter()
+    vals = []
+    limit = steps if steps is not None else 20
+    while not vals or (time.perf_counter() - t_start < seconds and len(vals) < limit):
+        vals.append(s.sample_us())
+    return float(np.mean(vals)), (f"fp64 oracle, {len(vals)} x (embedding + 1 of {layers_on} layers + LM head), "
+                                  f"scaled to {layers_on} layers")
+
+
 def run_reference(args) -> None:
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     wl = WORKLOADS[args.workload]
     parent, toks = workload_tree(wl)
-    s = OracleSampler(parent, toks, wl[1], wl[0] if not wl[5] else int(round(wl[0] * (1 - wl[5]))), wl[6])
-    for _ in range(args.warmup):
-        s.sample_us()
-    vals = [s.sample_us() for _ in range(args.steps)]
-    v = float(np.mean(vals))
+    vals = []
+    sample = ""
+    for _ in range(args.warmup + args.steps):
+        v1, sample = oracle_estimate(args.workload, wl, parent, toks, 0.0, 1)
+        vals.append(v1)
+    v = float(np.mean(vals[args.warmup:]))
     cores = os.cpu_count()
     out = {"impl": "reference", "metric": METRIC, "value": round(v, 1), "unit": "us", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(v / 1e3, 3), "higher_is_better": False,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": config_block(args, args.workload, wl, False),
            "cpu_baseline": {"value": round(v, 1), "unit": "us", "cores": cores, "kind": "oracle",
-                            "sample": f"fp64 oracle, embedding + 1 of {wl[0]} layers + LM head per step, "
-                                      f"scaled to {wl[0]} layers"},
+                            "sample": sample},
            "e2e": {"value": round(v, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
 
@@ -287,13 +347,18 @@ def run_gpu(args) -> None:
     cs.load_library()
     wl = WORKLOADS[args.workload]
     layers, P, n, depth, branch, skip, mode, verify = wl
-    sh = _shape(layers)
-    dm = DeviceModel(sh, SEED, with_int8=bool(mode))
+    family = FAMILY.get(args.workload, "7b")
+    cascade = args.workload.startswith("cascade")
+    sh = _shape(layers, family)
+    dm = DeviceModel(sh, SEED, with_int8=bool(mode) or cascade)
     kv = DeviceKV(dm, P + 2 * n + 64)
     kv.load_random_prefix(SEED, P)
     parent, toks = workload_tree(wl)
     mask = synth.skip_masks(SEED, layers, [skip])[0] if skip else None
     layers_on = layers if mask is None else int(mask.sum())
+    if cascade:  # the tree in level order; nested draft masks d1 (bf16) and d2 (W8A8)
+        parent, toks, levels = bfs_levels(parent, toks)
+        m1, m2 = synth.skip_masks(SEED, layers, list(CASCADE_SKIP))
     stream = torch.cuda.current_stream()
     cs.set_stream(dm.h, stream)
     tok_d = torch.tensor(toks, dtype=torch.int32, device="cuda")
@@ -304,6 +369,12 @@ def run_gpu(args) -> None:
     cs.set_options(dm.h, cs.OPT_PDL | (cs.OPT_GRAPHS if graphs else 0))
 
     def step():
+        if cascade:
+            for (a, b) in levels:  # d2 drafts one level at a time, appended to the tree
+                cs.tree_step(dm.h, kv.h, tok_d[a:], par_d[a:], b - a, m2, 1, None)
+            cs.kv_reset_tree(kv.h)
+            cs.tree_step(dm.h, kv.h, tok_d, par_d, n, m1, 0, None)  # d1 re-checks every node
+            cs.kv_reset_tree(kv.h)
         cs.tree_step(dm.h, kv.h, tok_d, par_d, n, mask, mode, logits)
         if verify:
             cs.accept_greedy(dm.h, None, tok_d, par_d, n, acc)
@@ -367,7 +438,13 @@ def run_gpu(args) -> None:
     cs.set_options(dm.h, cs.OPT_PDL)
     cs.profile(dm.h, True)
     for _ in range(args.steps):
-        step()
+        if cascade:  # per-kernel figures of the round's verify step (the drafts mix kernel kinds)
+            cs.tree_step(dm.h, kv.h, tok_d, par_d, n, mask, mode, logits)
+            cs.accept_greedy(dm.h, None, tok_d, par_d, n, acc)
+            cs.kv_compact(kv.h, acc)
+            cs.kv_set_prefix(kv.h, P)
+        else:
+            step()
     per_kind = {}
     # bf16 mode: "qkv" is the first layer's QKV chain launch, "gateup" the per-layer chains
     names = ["qkv", "attention", "wo", "gateup", "down", "lm_head", "other"]
@@ -385,6 +462,16 @@ def run_gpu(args) -> None:
     gu_avg_s = per_kind["gateup"]["avg_us"] * 1e-6
     achieved = gu_bytes / gu_avg_s / 1e9
     ab = algorithmic_bytes(sh, n, P, layers_on, mode)
+    if cascade:  # the round's bytes: every draft level, the re-check and the verify
+        ab = dict(ab)
+        on1, on2 = int(m1.sum()), int(m2.sum())
+        total = ab["total"]
+        T = 0
+        for (a, b) in levels:
+            total += algorithmic_bytes(sh, b - a, P + T, on2, 1)["total"]
+            T += b - a
+        total += algorithmic_bytes(sh, n, P, on1, 0)["total"]
+        ab["total"] = total
     kern = ("gemm_i8_kernel (W8A8 gate/up + SwiGLU)" if mode else
             "chain_kernel (Wo + residual, gate/up + SwiGLU, down + residual, next QKV or LM head)")
 
@@ -410,15 +497,9 @@ def run_gpu(args) -> None:
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        s = OracleSampler(parent, toks, P, layers_on, mode)
-        t_start = time.perf_counter()
-        vals = []
-        while not vals or (time.perf_counter() - t_start < args.cpu_seconds and len(vals) < 20):
-            vals.append(s.sample_us())
-        out["cpu_baseline"] = {"value": round(float(np.mean(vals)), 1), "unit": "us", "cores": os.cpu_count(),
-                               "kind": "oracle",
-                               "sample": f"fp64 oracle, {len(vals)} x (embedding + 1 of {layers_on} layers + LM head), "
-                                         f"scaled to {layers_on} layers"}
+        v, sample = oracle_estimate(args.workload, wl, parent, toks, args.cpu_seconds)
+        out["cpu_baseline"] = {"value": round(v, 1), "unit": "us", "cores": os.cpu_count(), "kind": "oracle",
+                               "sample": sample}
     if rank == 0:
         print(json.dumps(out), flush=True)
     kv.close()
