@@ -114,7 +114,12 @@ Layout make_layout(const casspec_model_config& c) {
   L.gemm_cnt = take((size_t)L.max_tiles * 4);
   L.chain_cnt = take((size_t)kMaxPhases * 1024 * 4);
   L.chain_bar = take(256);
-  L.i8_part = take((size_t)(6 * kSmsBound + 2 * L.max_tiles) * 64 * 128 * 4);
+  {  // int32 partial tiles of the W8A8 projections: tiles x ksplit slots of 64 x 128
+    const size_t kq = (size_t)(cdiv(d, 128) + 3) / 4, kf = (size_t)(cdiv(F, 128) + 3) / 4;
+    const size_t slots = std::max(std::max((size_t)cdiv(3 * d, 128) * kq, (size_t)cdiv(F, 64) * kq),
+                                  (size_t)cdiv(d, 128) * kf);
+    L.i8_part = take(slots * 64 * 128 * 4);
+  }
   L.i8_cnt = take((size_t)L.max_tiles * 4);
   L.status = take(256);
   L.total = align_up(off, 256);

@@ -4,12 +4,13 @@
 // (|sum| <= K * 127^2 < 2^31 for K < 133,000).  tcgen05.mma has no integer kind on sm_103a, so the
 // contraction uses the warp-level mma.sync.m16n8k32 s8 x s8 -> s32 path; at draft batch sizes the
 // projection is bound by streaming the int8 weights, half the bytes of the bf16 weights.
-//   * one CTA = 8 warps = one 128-row output tile (warp w: rows 16w..16w+15) x a k-range; `ksplit`
-//     CTAs share a tile along K so every SM keeps several weight streams in flight;
-//   * weights go straight from HBM into mma fragments with 16-byte loads (no shared memory), the
-//     next 128-column block prefetched in registers.  Both operands use the same permutation of
-//     the 128 columns of a block inside the fragments, which leaves the dot product unchanged:
-//     thread (group g, lane t) loads bytes [16t, 16t+16) and [64+16t, 64+16t+16) of its rows;
+//   * one CTA = 8 warps = one 128-row output tile (warp w: rows 16w..16w+15) x at most 4 blocks of
+//     128 columns; `ksplit` CTAs share a tile along K;
+//   * weights go straight from HBM into mma fragments with 16-byte loads (no shared memory), all
+//     of the CTA's loads issued before the first MMA, so each CTA pays one memory latency.  The
+//     activation slice of the k-range is staged once in shared memory.  Both operands use the same
+//     permutation of the 128 columns of a block inside the fragments, which leaves the dot product
+//     unchanged: thread (group g, lane t) takes bytes [16t, 16t+16) and [64+16t, 64+16t+16);
 //   * the CTA that finishes a tile last (atomic counter) sums the int32 partials, dequantises
 //     once, and runs the same fused epilogue as the bf16 projection.
 #include "common.cuh"
@@ -28,9 +29,11 @@ __device__ __forceinline__ uint4 ldg_nc16(const void* p) {
   return v;
 }
 
+constexpr int kI8MaxKb = 4;  // k-blocks of 128 per CTA (all of its weight loads in flight at once)
+
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a) {
-  extern __shared__ float stg[];  // [128][BN + 1] dequantised tile, then the epilogue's staging
+  extern __shared__ float stg[];  // the CTA's X slice, then the dequantised tile, then the epilogue staging
   __shared__ int s_last;
   const int tile = blockIdx.x, ks = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
@@ -38,6 +41,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
 
   const int KB = (a.K + 127) / 128;
   const int kb0 = (int)((long long)ks * KB / a.ksplit), kb1 = (int)((long long)(ks + 1) * KB / a.ksplit);
+  const int nkb = kb1 - kb0;  // <= kI8MaxKb: ksplit >= ceil(KB / kI8MaxKb)
   const int n = a.ep.n;
 
   // weight rows of this thread's fragments: tile rows lr and lr + 8
@@ -56,49 +60,69 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
       wrow[h] = a.W + (size_t)(wok[h] ? o : 0) * a.K;
     }
   }
-  auto load_a = [&](int kb, uint4* A) {
+  // every weight load of the CTA's k-range first (the weights do not depend on the previous kernel)
+  uint4 A[kI8MaxKb][4];
+#pragma unroll
+  for (int j = 0; j < kI8MaxKb; ++j) {
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
-        const int col = kb * 128 + c * 64 + 16 * t4;
-        A[2 * h + c] = (wok[h] && col < a.K) ? ldg_nc16(wrow[h] + col) : make_uint4(0, 0, 0, 0);
+        const int col = (kb0 + j) * 128 + c * 64 + 16 * t4;
+        A[j][2 * h + c] = (j < nkb && wok[h] && col < a.K) ? ldg_nc16(wrow[h] + col) : make_uint4(0, 0, 0, 0);
       }
     }
-  };
+  }
+  pdl_wait();
+  // the activations of the k-range, [BN][nkb * 128] int8 in shared memory (zero beyond n and K)
+  int8_t* xs = reinterpret_cast<int8_t*>(stg);
+  const int xrow = nkb * 128;
+  {
+    constexpr int kPieces = (BN * kI8MaxKb * 8 + kI8Threads - 1) / kI8Threads;  // 16-byte pieces per thread
+    const int per_tok = nkb * 8;
+    const int pieces = BN * per_tok;
+    uint4 xv[kPieces];
+#pragma unroll
+    for (int k = 0; k < kPieces; ++k) {
+      const int idx = tid + k * kI8Threads;
+      const int tok = idx / per_tok, c = (idx % per_tok) * 16;
+      const int col = kb0 * 128 + c;
+      xv[k] = (idx < pieces && tok < n && col < a.K)
+                  ? __ldcg(reinterpret_cast<const uint4*>(a.X + (size_t)tok * a.K + col))
+                  : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int k = 0; k < kPieces; ++k) {
+      const int idx = tid + k * kI8Threads;
+      if (idx < pieces) *reinterpret_cast<uint4*>(xs + (idx / per_tok) * xrow + (idx % per_tok) * 16) = xv[k];
+    }
+  }
+  __syncthreads();
 
   int acc[BN / 8][4];
 #pragma unroll
   for (int j = 0; j < BN / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0;
-
-  uint4 A[4], An[4];
-  if (kb0 < kb1) load_a(kb0, A);  // weights do not depend on the previous kernel
-  pdl_wait();
-  for (int kb = kb0; kb < kb1; ++kb) {
-    if (kb + 1 < kb1) load_a(kb + 1, An);
 #pragma unroll
-    for (int j = 0; j < BN / 8; ++j) {
-      const int tok = 8 * j + g;
-      uint4 B[2];
+  for (int kbl = 0; kbl < kI8MaxKb; ++kbl) {
+    if (kbl < nkb) {
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        const int col = kb * 128 + c * 64 + 16 * t4;
-        B[c] = (tok < n && col < a.K) ? __ldcg(reinterpret_cast<const uint4*>(a.X + (size_t)tok * a.K + col))
-                                      : make_uint4(0, 0, 0, 0);
+      for (int j = 0; j < BN / 8; ++j) {
+        const int tok = 8 * j + g;
+        uint4 B[2];
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+          B[c] = *reinterpret_cast<const uint4*>(xs + tok * xrow + kbl * 128 + c * 64 + 16 * t4);
+#pragma unroll
+        for (int s2 = 0; s2 < 4; ++s2) {
+          const uint4 lo = A[kbl][s2 >> 1], hi = A[kbl][2 + (s2 >> 1)], b = B[s2 >> 1];
+          const bool odd = s2 & 1;
+          mma_s8_16832(acc[j], odd ? lo.z : lo.x, odd ? hi.z : hi.x, odd ? lo.w : lo.y, odd ? hi.w : hi.y,
+                       odd ? b.z : b.x, odd ? b.w : b.y);
+        }
       }
-#pragma unroll
-      for (int s = 0; s < 4; ++s) {
-        const uint4 lo = A[s >> 1], hi = A[2 + (s >> 1)], b = B[s >> 1];
-        const bool odd = s & 1;
-        mma_s8_16832(acc[j], odd ? lo.z : lo.x, odd ? hi.z : hi.x, odd ? lo.w : lo.y, odd ? hi.w : hi.y,
-                     odd ? b.z : b.x, odd ? b.w : b.y);
-      }
-    }
-    if (kb + 1 < kb1) {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) A[q] = An[q];
     }
   }
+  __syncthreads();  // the X slice is dead: the shared memory now takes the dequantised tile
 
   auto scale_w = [&](int row) -> float {
     if (EPI == EPI_GLU) {
@@ -119,9 +143,11 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
         const int tok = 8 * j + 2 * t4 + (e & 1), row = warp * 16 + g + 8 * (e >> 1);
         if (tok < n) __stcg(part + tok * 128 + row, acc[j][e]);
       }
-    __threadfence();
     __syncthreads();
-    if (tid == 0) s_last = (atomicAdd(&a.counters[tile], 1u) == (unsigned)(a.ksplit - 1)) ? 1 : 0;
+    if (tid == 0) {
+      __threadfence();
+      s_last = (atomicAdd(&a.counters[tile], 1u) == (unsigned)(a.ksplit - 1)) ? 1 : 0;
+    }
     __syncthreads();
     if (!s_last) return;
     __threadfence();
@@ -153,11 +179,9 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
 }
 
 int gemm_i8_ksplit(int tiles, int K, int num_sms) {
-  const int KB = (K + 127) / 128;
-  int ks = (6 * num_sms + tiles - 1) / tiles;
-  if (ks > KB / 2) ks = KB / 2;
-  if (ks < 1) ks = 1;
-  return ks;
+  (void)tiles;
+  (void)num_sms;
+  return ((K + 127) / 128 + kI8MaxKb - 1) / kI8MaxKb;
 }
 
 template <int BN, int EPI>
@@ -165,7 +189,7 @@ static cudaError_t launch_t(const GemmI8Args& a, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.tiles, a.ksplit);
   cfg.blockDim = dim3(kI8Threads);
-  cfg.dynamicSmemBytes = (size_t)epi_staging_floats(BN) * 4;
+  cfg.dynamicSmemBytes = (size_t)epi_staging_floats(BN) * 4;  // >= BN * 4 * 128 bytes of X slice
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
