@@ -2,17 +2,17 @@
 //
 // Node i of the tree attends to every committed prefix slot [0, P) and to the tree slots of its
 // ancestors and itself (bit j of anc[i] <=> tree slot j, cache slot P + j).
-//   * one thread-block cluster of C CTAs per head; CTA rank r handles the r-th contiguous share of
-//     the head's 64-slot KV blocks (split-KV), so every SM streams about the same K/V bytes;
+//   * S CTAs per head (split-KV, S * heads <= 2 per SM, so the whole grid is resident at once);
+//     split s handles the s-th contiguous share of the head's 64-slot KV blocks;
 //   * K/V blocks arrive by TMA (2-D tensor map over the whole cache, 128-byte swizzle, 64 slots x 64
 //     dims per box) in an S-stage mbarrier ring fed by a dedicated producer warp;
 //   * four compute warps, 16 query rows each, run QK^T and PV on tensor cores (mma.sync m16n8k16
 //     bf16 -> fp32) with ldmatrix addresses XOR-swizzled to match the TMA layout, the ancestor mask
 //     applied to the scores, and an online softmax whose row reductions are quad shuffles;
-//   * the split-KV partials (running max, sum, unnormalised output) stay in each CTA's shared memory
-//     and are merged across the cluster through distributed shared memory: rank r merges rows
-//     r, r + C, ... reading all C partials, between two hardware cluster barriers.  No global
-//     scratch, no atomics, and a fixed merge order, so results do not depend on timing.
+//   * each split writes its partial (running max, sum, unnormalised output) to global scratch and
+//     counts itself in; once all S splits of the head have arrived, split s merges rows
+//     s, s + S, ... over the S partials in split order (fixed, so results do not depend on timing)
+//     and the last split out returns the head's counters to zero.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -22,7 +22,6 @@ constexpr int kAttnCompute = 128;                // 4 compute warps
 constexpr int kAttnThreads = kAttnCompute + 32;  // + producer warp
 constexpr int kAttnBlk = 64;
 constexpr int kAttnStages = 3;
-constexpr int kAttnMaxCluster = 8;
 
 template <int HD>
 __host__ __device__ constexpr uint32_t attn_tile_bytes() {
@@ -46,26 +45,24 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
   constexpr uint32_t STAGE = 2 * TILE;
   constexpr int S = kAttnStages;
   constexpr int NCH = HD / 8;  // 16-byte chunks per row
-  static_assert(64 * HD * 4 + 64 * 8 <= S * STAGE, "partials must fit in the K/V ring");
   extern __shared__ __align__(1024) uint8_t sm[];
   uint8_t* ring = sm;
   uint8_t* qs = sm + S * STAGE;
   uint64_t* full = reinterpret_cast<uint64_t*>(qs + 64 * HD * 2);
   uint64_t* empty = full + S;
-  volatile int* flags = reinterpret_cast<volatile int*>(empty + S);  // [0] abort
-  float* part_o = reinterpret_cast<float*>(ring);                    // [64][HD], after the main loop
-  float2* part_ml = reinterpret_cast<float2*>(ring + 64 * HD * 4);   // [64] (max, sum)
+  volatile int* flags = reinterpret_cast<volatile int*>(empty + S);  // [0] abort, [1] merge go-ahead
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int C = a.cluster;
+  const int C = a.splits;
   const int head = blockIdx.x / C;
-  const int rank = (int)cluster_ctarank();
+  const int rank = blockIdx.x % C;
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 4);
     }
     flags[0] = 0;
+    flags[1] = 0;
     fence_mbar_init();
   }
   if (tid == kAttnCompute) tma_prefetch_desc(&tmKV);
@@ -268,72 +265,95 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
     }
   }
 
-  // ---- partials into this CTA's shared memory (the K/V ring is drained) ----
-  __syncthreads();
+  // ---- this split's partial to global scratch, then count in ----
+  const int n = a.n;
+  const size_t pslot = (size_t)head * C + rank;
   if (warp < 4) {
     lA += __shfl_xor_sync(0xffffffffu, lA, 1);
     lA += __shfl_xor_sync(0xffffffffu, lA, 2);
     lB += __shfl_xor_sync(0xffffffffu, lB, 1);
     lB += __shfl_xor_sync(0xffffffffu, lB, 2);
+    float* po = a.part_o + pslot * 64 * HD;
 #pragma unroll
     for (int dt = 0; dt < HD / 8; ++dt) {
       const int col = dt * 8 + 2 * t4;
-      *reinterpret_cast<float2*>(part_o + rA * HD + col) = make_float2(oacc[dt][0], oacc[dt][1]);
-      *reinterpret_cast<float2*>(part_o + rB * HD + col) = make_float2(oacc[dt][2], oacc[dt][3]);
+      if (rA < n) __stcg(reinterpret_cast<float2*>(po + rA * HD + col), make_float2(oacc[dt][0], oacc[dt][1]));
+      if (rB < n) __stcg(reinterpret_cast<float2*>(po + rB * HD + col), make_float2(oacc[dt][2], oacc[dt][3]));
     }
     if (t4 == 0) {
-      part_ml[rA] = make_float2(mA, lA);
-      part_ml[rB] = make_float2(mB, lB);
+      if (rA < n) __stcg(a.part_ml + pslot * 64 + rA, make_float2(mA, lA));
+      if (rB < n) __stcg(a.part_ml + pslot * 64 + rB, make_float2(mB, lB));
     }
   }
-  cluster_sync();  // every rank's partials are visible cluster-wide
+  __syncthreads();
+  if (tid == 0) {
+    // every split of this head is resident (the grid fits the GPU at two CTAs per SM), so this
+    // wait ends as soon as the slowest split has written its partial
+    __threadfence();
+    atomicAdd(a.cnt + head, 1u);
+    const uint64_t t0 = globaltimer_ns();
+    int ok = 1;
+    while (ld_acquire_gpu(a.cnt + head) < (unsigned)C) {
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        ok = 0;
+        set_status(a.status, CASSPEC_E_TIMEOUT);
+        break;
+      }
+    }
+    flags[1] = ok;
+  }
+  __syncthreads();
 
-  // ---- merge: this rank finishes rows rank, rank + C, ... from all C partials ----
-  const uint32_t o_base = smem_u32(part_o), ml_base = smem_u32(part_ml);
-  constexpr int V4 = HD / 4;
-  for (int idx = tid; idx < ((a.n + C - 1) / C) * V4; idx += kAttnThreads) {
-    const int row = rank + (idx / V4) * C, c4 = (idx % V4) * 4;
-    if (row >= a.n) continue;
-    float M = -INFINITY;
-    float2 ml[kAttnMaxCluster];
-#pragma unroll
-    for (int k = 0; k < kAttnMaxCluster; ++k) {
-      if (k < C) {
-        ml[k] = ld_dsmem_f2(map_to_rank(ml_base + row * 8, k));
-        M = fmaxf(M, ml[k].x);
+  // ---- merge: this split finishes rows rank, rank + C, ... over all C partials, in split order ----
+  if (flags[1]) {
+    __threadfence();
+    constexpr int V4 = HD / 4;
+    const float* pob = a.part_o + (size_t)head * C * 64 * HD;
+    const float2* pml = a.part_ml + (size_t)head * C * 64;
+    for (int idx = tid; idx < ((n + C - 1) / C) * V4; idx += kAttnThreads) {
+      const int row = rank + (idx / V4) * C, c4 = (idx % V4) * 4;
+      if (row >= n) continue;
+      float M = -INFINITY;
+      for (int k = 0; k < C; ++k) M = fmaxf(M, __ldcg(pml + k * 64 + row).x);
+      float L = 0.f;
+      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k = 0; k < C; ++k) {
+        const float2 ml = __ldcg(pml + k * 64 + row);
+        if (ml.x != -INFINITY) {
+          const float w = exp2f(ml.x - M);
+          const float4 ov = __ldcg(reinterpret_cast<const float4*>(pob + ((size_t)k * 64 + row) * HD + c4));
+          L += ml.y * w;
+          o.x += ov.x * w;
+          o.y += ov.y * w;
+          o.z += ov.z * w;
+          o.w += ov.w * w;
+        }
       }
+      const float inv = 1.f / L;
+      const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
+      const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
+      uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
+      hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
+      hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
+      lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
+      lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
+      *reinterpret_cast<uint2*>(a.o + (size_t)row * a.d + head * HD + c4) = hi;
+      *reinterpret_cast<uint2*>(a.o + (size_t)(64 + row) * a.d + head * HD + c4) = lo;
     }
-    float L = 0.f;
-    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int k = 0; k < kAttnMaxCluster; ++k) {
-      if (k < C && ml[k].x != -INFINITY) {
-        const float w = exp2f(ml[k].x - M);
-        const float4 ov = ld_dsmem_f4(map_to_rank(o_base + (row * HD + c4) * 4, k));
-        L += ml[k].y * w;
-        o.x += ov.x * w;
-        o.y += ov.y * w;
-        o.z += ov.z * w;
-        o.w += ov.w * w;
-      }
-    }
-    const float inv = 1.f / L;
-    const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
-    const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
-    uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
-    hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
-    hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
-    lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
-    lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
-    *reinterpret_cast<uint2*>(a.o + (size_t)row * a.d + head * HD + c4) = hi;
-    *reinterpret_cast<uint2*>(a.o + (size_t)(64 + row) * a.d + head * HD + c4) = lo;
   }
-  cluster_sync();  // no rank leaves while another still reads its shared memory
+  __syncthreads();
+  if (tid == 0) {  // the last split out (every split has stopped reading the arrival counter)
+    __threadfence();
+    if (atomicAdd(a.cnt + a.n_heads + head, 1u) == (unsigned)(C - 1)) {
+      a.cnt[head] = 0u;
+      a.cnt[a.n_heads + head] = 0u;
+    }
+  }
 }
 
-int attn_cluster(int n_heads, int num_sms) {
-  int c = (2 * num_sms) / n_heads;  // two CTAs per SM: the whole grid runs in one wave
-  if (c > kAttnMaxCluster) c = kAttnMaxCluster;
+int attn_splits(int n_heads, int num_sms) {
+  int c = (2 * num_sms) / n_heads;  // two CTAs per SM: the whole grid is resident at once
+  if (c > kAttnMaxSplits) c = kAttnMaxSplits;
   if (c < 1) c = 1;
   return c;
 }
@@ -351,24 +371,20 @@ static cudaError_t launch_hd(const CUtensorMap& tm, const AttnArgs& a, cudaStrea
     configured = dev;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.n_heads * a.cluster);
+  cfg.gridDim = dim3(a.n_heads * a.splits);
   cfg.blockDim = dim3(kAttnThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = a.cluster;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 2 : 1;
+  cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kern, tm, a);
 }
 
 cudaError_t launch_tree_attention(const CUtensorMap& tm, const AttnArgs& a, int hd, cudaStream_t stream, bool pdl) {
-  if (a.cluster < 1 || a.cluster > kAttnMaxCluster) return cudaErrorInvalidValue;
+  if (a.splits < 1 || a.splits > kAttnMaxSplits) return cudaErrorInvalidValue;
   if (hd == 128) return launch_hd<128>(tm, a, stream, pdl);
   if (hd == 64) return launch_hd<64>(tm, a, stream, pdl);
   return cudaErrorInvalidValue;

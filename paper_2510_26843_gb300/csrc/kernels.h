@@ -71,6 +71,7 @@ struct GemmI8Args {
   EpiParams ep;
 };
 
+constexpr int kAttnMaxSplits = 16;
 struct AttnArgs {
   const uint16_t* q;    // [64][d] bf16 (rotated)
   uint16_t* o;          // split attention output [128][d] bf16
@@ -78,8 +79,11 @@ struct AttnArgs {
   const int* dP;
   int T, n, ctx, d, n_heads;
   int layer;            // K/V rows of this layer in the cache tensor map: ((layer * 2 + kv) * H + h) * ctx + slot
-  int cluster;          // CTAs per head (thread-block cluster size, <= 8)
+  int splits;           // CTAs per head (split-KV), <= kAttnMaxSplits; n_heads * splits <= 2 * SMs
   float scale_log2;     // log2(e) / sqrt(hd)
+  float* part_o;        // [n_heads][splits][64][hd] fp32 unnormalised partial outputs
+  float2* part_ml;      // [n_heads][splits][64] (running max, sum) per row
+  unsigned* cnt;        // [2 * n_heads] arrival and exit counters per head, zero between launches
   int* status;
 };
 
@@ -123,7 +127,7 @@ cudaError_t launch_gemm_bf16(const CUtensorMap& tmW, const CUtensorMap& tmW2, co
 int gemm_i8_ksplit(int tiles, int K, int num_sms);
 cudaError_t launch_gemm_i8(const GemmI8Args& args, int BN, int epi, cudaStream_t stream, bool pdl);
 
-int attn_cluster(int n_heads, int num_sms);
+int attn_splits(int n_heads, int num_sms);
 cudaError_t launch_tree_attention(const CUtensorMap& tmKV, const AttnArgs& a, int hd, cudaStream_t stream, bool pdl);
 
 cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int* tdepth, unsigned long long* tanc,
