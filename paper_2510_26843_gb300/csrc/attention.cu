@@ -45,6 +45,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
   constexpr uint32_t STAGE = 2 * TILE;
   constexpr int S = kAttnStages;
   constexpr int NCH = HD / 8;  // 16-byte chunks per row
+  static_assert(64 * kAttnMaxSplits * 12 + 64 * 4 <= S * STAGE, "merge weights must fit in the K/V ring");
   extern __shared__ __align__(1024) uint8_t sm[];
   uint8_t* ring = sm;
   uint8_t* qs = sm + S * STAGE;
@@ -65,7 +66,26 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
     flags[1] = 0;
     fence_mbar_init();
   }
-  if (tid == kAttnCompute) tma_prefetch_desc(&tmKV);
+  if (tid == kAttnCompute) {
+    tma_prefetch_desc(&tmKV);
+    // Before the dependency wait: pull this split's K/V blocks into L2 while the previous kernel
+    // finishes.  The committed prefix is written only by earlier steps, and an L2 prefetch is a
+    // coherent hint, so a P read here that a predecessor is about to change can only make the
+    // prefetch miss, never change a result.
+    const int Ph = *reinterpret_cast<const volatile int*>(a.dP);
+    if (Ph >= 0 && Ph <= a.ctx) {
+      const int nb = min((Ph + a.T + a.n + kAttnBlk - 1) / kAttnBlk, a.ctx / kAttnBlk);
+      const int row_k = ((a.layer * 2 + 0) * a.n_heads + head) * a.ctx;
+      const int row_v = ((a.layer * 2 + 1) * a.n_heads + head) * a.ctx;
+      for (int b = rank * nb / C; b < (rank + 1) * nb / C; ++b) {
+#pragma unroll
+        for (int sub = 0; sub < HD / 64; ++sub) {
+          tma_prefetch_l2_2d(&tmKV, sub * 64, row_k + b * kAttnBlk);
+          tma_prefetch_l2_2d(&tmKV, sub * 64, row_v + b * kAttnBlk);
+        }
+      }
+    }
+  }
   __syncthreads();
   pdl_trigger();
   pdl_wait();
@@ -305,31 +325,49 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
   __syncthreads();
 
   // ---- merge: this split finishes rows rank, rank + C, ... over all C partials, in split order ----
+  // (the K/V ring is drained: its shared memory holds the merge weights)
   if (flags[1]) {
     __threadfence();
     constexpr int V4 = HD / 4;
     const float* pob = a.part_o + (size_t)head * C * 64 * HD;
     const float2* pml = a.part_ml + (size_t)head * C * 64;
-    for (int idx = tid; idx < ((n + C - 1) / C) * V4; idx += kAttnThreads) {
-      const int row = rank + (idx / V4) * C, c4 = (idx % V4) * 4;
-      if (row >= n) continue;
+    const int nr = rank < n ? (n - rank + C - 1) / C : 0;  // rows of this split
+    float2* ml_s = reinterpret_cast<float2*>(ring);          // [nr][C] (max, sum)
+    float* w_s = reinterpret_cast<float*>(ring + 64 * kAttnMaxSplits * 8);  // [nr][C] weights
+    float* inv_s = w_s + 64 * kAttnMaxSplits;                                // [nr] 1 / sum
+    if (tid < nr * C) ml_s[tid] = __ldcg(pml + (tid % C) * 64 + rank + (tid / C) * C);
+    __syncthreads();
+    if (tid < nr) {
       float M = -INFINITY;
-      for (int k = 0; k < C; ++k) M = fmaxf(M, __ldcg(pml + k * 64 + row).x);
+      for (int k = 0; k < C; ++k) M = fmaxf(M, ml_s[tid * C + k].x);
       float L = 0.f;
-      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int k = 0; k < C; ++k) {
-        const float2 ml = __ldcg(pml + k * 64 + row);
-        if (ml.x != -INFINITY) {
-          const float w = exp2f(ml.x - M);
-          const float4 ov = __ldcg(reinterpret_cast<const float4*>(pob + ((size_t)k * 64 + row) * HD + c4));
-          L += ml.y * w;
-          o.x += ov.x * w;
-          o.y += ov.y * w;
-          o.z += ov.z * w;
-          o.w += ov.w * w;
+        const float2 ml = ml_s[tid * C + k];
+        const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);  // an empty split weighs 0
+        w_s[tid * C + k] = w;
+        L += ml.y * w;
+      }
+      inv_s[tid] = 1.f / L;
+    }
+    __syncthreads();
+    for (int idx = tid; idx < nr * V4; idx += kAttnThreads) {
+      const int j = idx / V4, c4 = (idx % V4) * 4, row = rank + j * C;
+      float4 ov[kAttnMaxSplits];  // every partial of this element in flight at once
+#pragma unroll
+      for (int k = 0; k < kAttnMaxSplits; ++k)
+        if (k < C) ov[k] = __ldcg(reinterpret_cast<const float4*>(pob + ((size_t)k * 64 + row) * HD + c4));
+      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int k = 0; k < kAttnMaxSplits; ++k) {
+        if (k < C) {
+          const float w = w_s[j * C + k];
+          o.x += ov[k].x * w;
+          o.y += ov[k].y * w;
+          o.z += ov[k].z * w;
+          o.w += ov[k].w * w;
         }
       }
-      const float inv = 1.f / L;
+      const float inv = inv_s[j];
       const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
       const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
       uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
