@@ -37,11 +37,11 @@ __host__ __device__ constexpr int chain_w_stages(int BN) {
                                                                    : (int)((kChainSmemBudget - chain_fixed(BN)) / kWTile);
 }
 __host__ __device__ constexpr size_t chain_smem(int BN) { return chain_fixed(BN) + (size_t)chain_w_stages(BN) * kWTile; }
-// TMEM per accumulator buffer: two accumulators (alternate k-steps) of 2*BN columns (the hi and
-// lo planes stacked as one N = 2*BN operand); two buffers.
-__host__ __device__ constexpr uint32_t chain_buf_cols(int BN) { return 4u * (uint32_t)BN; }
+// TMEM per accumulator buffer: one accumulator of 2*BN columns (the hi and lo planes stacked as
+// one N = 2*BN operand); two buffers.
+__host__ __device__ constexpr uint32_t chain_buf_cols(int BN) { return 2u * (uint32_t)BN; }
 __host__ __device__ constexpr uint32_t chain_tmem_cols(int BN) {
-  return 2 * chain_buf_cols(BN) <= 128 ? 128 : (2 * chain_buf_cols(BN) <= 256 ? 256 : 512);
+  return 2 * chain_buf_cols(BN) <= 64 ? 64 : (2 * chain_buf_cols(BN) <= 128 ? 128 : 256);
 }
 
 __device__ __forceinline__ long long chain_u0(int c, long long U, int G) { return (long long)c * U / G; }
@@ -257,12 +257,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             const uint32_t sa = smem_u32(wring + ws * kWTile);
             const uint32_t sh = smem_u32(xring + xs * XS);
             // One MMA per 16-column k-step with the hi and lo planes stacked (N = 2 * BN, the X stage
-            // holds them back to back); even and odd k-steps go to two accumulators so that
-            // consecutive MMAs do not depend on each other.
+            // holds them back to back), all into one accumulator: splitting even and odd k-steps
+            // over two accumulators measured slower.
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              tc_mma_bf16(d_tmem + (uint32_t)(kk & 1) * (2u * BN), sw128_kmajor_desc(sa + kk * 32),
-                          sw128_kmajor_desc(sh + kk * 32), IDESC, (uu > u || kk >= 2) ? 1u : 0u);
+              tc_mma_bf16(d_tmem, sw128_kmajor_desc(sa + kk * 32), sw128_kmajor_desc(sh + kk * 32), IDESC,
+                          (uu > u || kk > 0) ? 1u : 0u);
             tc_commit(&wempty[ws]);
             tc_commit(&xempty[xs]);
             if (++ws == SW) {
@@ -350,15 +350,13 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         float v[BN];
         const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)buf * chain_buf_cols(BN);
 #pragma unroll
-        for (int c = 0; c < BN; c += 16) {  // (acc0 hi + acc0 lo) + (acc1 hi + acc1 lo), fixed order
-          float t1[16], t2[16], t3[16];
+        for (int c = 0; c < BN; c += 16) {  // hi-plane product + lo-plane product
+          float t1[16];
           tmem_ld_x16(taddr + c, &v[c]);
           tmem_ld_x16(taddr + BN + c, t1);
-          tmem_ld_x16(taddr + 2 * BN + c, t2);
-          tmem_ld_x16(taddr + 3 * BN + c, t3);
           tmem_ld_wait();
 #pragma unroll
-          for (int j = 0; j < 16; ++j) v[c + j] = (v[c + j] + t1[j]) + (t2[j] + t3[j]);
+          for (int j = 0; j < 16; ++j) v[c + j] += t1[j];
         }
         tc_fence_before();
         __syncwarp();
