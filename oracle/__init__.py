@@ -1,4 +1,5 @@
-"""CPU fp64 oracle of the CAS-Spec tree step -- TEST INFRASTRUCTURE ONLY.
+"""CPU fp64 oracle of the CAS-Spec tree step (casspec_oracle) and of the DyTC scheduler
+(dytc_oracle) -- TEST INFRASTRUCTURE ONLY.
 
 Imported only by tests/, __graft_entry__.smoke() and bench.py's CPU baseline / reference arm.
 The CUDA library never imports, links or runs anything here.
