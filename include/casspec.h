@@ -285,6 +285,81 @@ CASSPEC_API int casspec_rmsnorm(const float* x, const float* g, int n, int d, fl
 /* Per-row int8 quantisation of bf16 rows x [n][d] -> q [n][d], s [n] (same rule). */
 CASSPEC_API int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q_out, float* s_out, void* cuda_stream);
 
+/* ---------------------------------------------------------------------------------------------
+ * Dynamic Tree Cascade scheduling (DyTC): host code, no GPU work; thread-compatible (one scheduler
+ * per thread).  It decides which draft configuration drafts how many tokens below which node of the
+ * draft tree; the caller runs those drafts with casspec_tree_step and verifies the tree.
+ * ------------------------------------------------------------------------------------------- */
+
+/* Expected walltime improvement factors under i.i.d. Bernoulli acceptance (Sec. 3):
+ *   casspec_ewif_sd: T_SD = (1 - a^(k+1)) / ((1 - a)(c k + 1)), draft acceptance a, cost coefficient c
+ *     (draft step time / target step time), draft length k;
+ *   casspec_ewif_hc: horizontal cascade, d1 drafts k1 tokens then d2 drafts k2:
+ *     [(1 - a1^(k1+1)) / (1 - a1) + a1^k1 a2 (1 - a2^k2) / (1 - a2)] / (1 + k1 c1 + k2 c2);
+ *   casspec_ewif_vc: vertical cascade, n rounds of d2 drafting k tokens for d1:
+ *     (1 - a phi(a)^n) / ((1 - a)(1 + n c1 + n k c2)), phi(x) = 1 + (x - 1)(1 - (a12 x)^(k+1)) / (1 - a12 x),
+ *     a = acceptance of d1 by the target, a12 = acceptance of d2 by d1; phi^n is the n-th power.
+ * Return NaN for out-of-range arguments (acceptance outside [0, 1], negative lengths; a = 1 for the
+ * cascade forms). */
+CASSPEC_API double casspec_ewif_sd(double alpha, double c, int k);
+CASSPEC_API double casspec_ewif_hc(double a1, double c1, int k1, double a2, double c2, int k2);
+CASSPEC_API double casspec_ewif_vc(double alpha, double alpha12, double c1, double c2, int n, int k);
+
+/* The step objective of Eq. 5 (Sec. 4.2): T_s = (E_acc + a^k a_dn) / (c k + c_dn), with
+ * E_acc = a (1 - a^k) / (1 - a) (= k at a = 1) and (a_dn, c_dn) the bottom draft's acceptance and cost
+ * (its "least future speedup").  NaN where Algorithm 2 skips the pair (c k + c_dn ~ 0) or k < 1. */
+CASSPEC_API double casspec_dytc_objective(double alpha, double c, int k, double alpha_dn, double c_dn);
+
+#define CASSPEC_DYTC_MAX_CFG 16
+typedef struct casspec_dytc casspec_dytc;
+typedef struct {
+  int n_cfg;        /* candidate draft configurations, 1..CASSPEC_DYTC_MAX_CFG */
+  double alpha_dn;  /* bottom draft: acceptance rate ... */
+  double c_dn;      /* ... and cost coefficient (0 = free: the stop rule never fires) */
+  int k_max;        /* longest draft per expansion (Algorithm 1's k_max) */
+  double t_min;     /* stop when alpha_dn / c_dn * P_acc(leaf) < t_min (Sec. 4.2) */
+  int m_max;        /* largest tree, root included, 1..CASSPEC_MAX_TREE */
+  double lambda;    /* EMA weight of the previous estimate (the paper uses 0.7) */
+  int window;       /* outcomes per configuration in the recent mean (the paper uses H = 20) */
+} casspec_dytc_params;
+
+/* Create a scheduler over n_cfg candidate configurations with initial acceptance estimates
+ * alpha_init[n_cfg] (host, in [0, 1]; e.g. from a calibration run, App. D) and cost coefficients
+ * cost[n_cfg] (host, >= 0).  Errors: E_INVAL for out-of-range parameters, E_CAPACITY. */
+CASSPEC_API int casspec_dytc_create(const casspec_dytc_params* p, const double* alpha_init, const double* cost,
+                                    casspec_dytc** out);
+CASSPEC_API void casspec_dytc_destroy(casspec_dytc* s);
+/* Replace a configuration's cost coefficient (e.g. from measured step times). */
+CASSPEC_API int casspec_dytc_set_cost(casspec_dytc* s, int cfg, double cost);
+/* Current acceptance estimate of a configuration. */
+CASSPEC_API int casspec_dytc_alpha(const casspec_dytc* s, int cfg, double* alpha_out);
+/* Algorithm 2 (App. D) with the current estimates: the configuration and draft length k in
+ * [1, k_max] maximising Eq. 5, first maximum on ties; *cfg_out = -1 and *k_out = 0 when no pair has
+ * a positive objective.  *obj_out (may be NULL) receives the maximum. */
+CASSPEC_API int casspec_dytc_best_config(const casspec_dytc* s, int* cfg_out, int* k_out, double* obj_out);
+/* Acceptance bookkeeping (Sec. 4.2): record whether the first token that configuration cfg drafted
+ * in this round was accepted (the last `window` outcomes are kept); at the end of a round,
+ * casspec_dytc_end_step sets alpha <- lambda alpha + (1 - lambda) mean(outcomes) for every
+ * configuration recorded since the previous end of round; the others keep their estimate (App. D). */
+CASSPEC_API int casspec_dytc_record(casspec_dytc* s, int cfg, int accepted);
+CASSPEC_API int casspec_dytc_end_step(casspec_dytc* s);
+/* Algorithm 1 (Sec. 4.2) with one drafted token per position, driven by the caller:
+ *   casspec_dytc_tree_reset: the tree holds the root (node 0: the last committed token), P_acc = 1;
+ *   casspec_dytc_tree_plan: returns 1 with the active leaf of highest P_acc (lowest index on ties),
+ *     the configuration and k of Algorithm 2; returns 0 (stop) when the tree holds m_max nodes, no
+ *     leaf is active, alpha_dn / c_dn * P_acc(leaf) < t_min, or no configuration has a positive
+ *     objective (that leaf is then deactivated);
+ *   casspec_dytc_tree_extend: appends the k tokens drafted by cfg below `leaf` as a chain, each with
+ *     P_acc = P_acc(parent) * alpha(cfg); the leaf and each new node that gets a child stop being
+ *     active leaves.  Stops at m_max nodes; returns the number of nodes appended (or an error);
+ *   casspec_dytc_tree_get: the tree in node order, arrays of m_max entries (any may be NULL):
+ *     parent (-1 for the root), token (-1 for the root), cfg (-1 for the root), P_acc. */
+CASSPEC_API int casspec_dytc_tree_reset(casspec_dytc* s);
+CASSPEC_API int casspec_dytc_tree_plan(casspec_dytc* s, int* leaf_out, int* cfg_out, int* k_out);
+CASSPEC_API int casspec_dytc_tree_extend(casspec_dytc* s, int leaf, int cfg, int k, const int32_t* tokens);
+CASSPEC_API int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out, int32_t* token_out,
+                                      int32_t* cfg_out, double* p_acc_out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -30,6 +30,10 @@ EXPORTS = [
     "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_linear_bf16_static",
     "casspec_rmsnorm",
     "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
+    "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
+    "casspec_dytc_destroy", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
+    "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_get",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -38,6 +42,12 @@ class ModelConfig(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32), ("vocab", ctypes.c_int32),
                 ("rope_base", ctypes.c_float), ("rms_eps", ctypes.c_float), ("with_int8", ctypes.c_int32)]
+
+
+class DytcParams(ctypes.Structure):
+    _fields_ = [("n_cfg", ctypes.c_int32), ("alpha_dn", ctypes.c_double), ("c_dn", ctypes.c_double),
+                ("k_max", ctypes.c_int32), ("t_min", ctypes.c_double), ("m_max", ctypes.c_int32),
+                ("lambda_", ctypes.c_double), ("window", ctypes.c_int32)]
 
 
 class CasspecError(RuntimeError):
@@ -50,6 +60,7 @@ _lib = None
 _P = ctypes.c_void_p
 _I = ctypes.c_int
 _SZ = ctypes.c_size_t
+_D = ctypes.c_double
 
 
 def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
@@ -62,6 +73,22 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib = ctypes.CDLL(path)
     sig = {
         "casspec_model_bytes": (_SZ, [ctypes.POINTER(ModelConfig)]),
+        "casspec_ewif_sd": (_D, [_D, _D, _I]),
+        "casspec_ewif_hc": (_D, [_D, _D, _I, _D, _D, _I]),
+        "casspec_ewif_vc": (_D, [_D, _D, _D, _D, _I, _I]),
+        "casspec_dytc_objective": (_D, [_D, _D, _I, _D, _D]),
+        "casspec_dytc_create": (_I, [ctypes.POINTER(DytcParams), ctypes.POINTER(_D), ctypes.POINTER(_D), ctypes.POINTER(_P)]),
+        "casspec_dytc_destroy": (None, [_P]),
+        "casspec_dytc_set_cost": (_I, [_P, _I, _D]),
+        "casspec_dytc_alpha": (_I, [_P, _I, ctypes.POINTER(_D)]),
+        "casspec_dytc_best_config": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_D)]),
+        "casspec_dytc_record": (_I, [_P, _I, _I]),
+        "casspec_dytc_end_step": (_I, [_P]),
+        "casspec_dytc_tree_reset": (_I, [_P]),
+        "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+        "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
+        "casspec_dytc_tree_get": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
+                                       ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_D)]),
         "casspec_create_model": (_I, [ctypes.POINTER(ModelConfig), _P, _SZ, ctypes.POINTER(_P)]),
         "casspec_destroy_model": (None, [_P]),
         "casspec_set_stream": (_I, [_P, _P]),
@@ -277,3 +304,95 @@ def launch_count(m: int) -> int:
     c = ctypes.c_uint64()
     _check("casspec_launch_count", load_library().casspec_launch_count(m, ctypes.byref(c)))
     return c.value
+
+
+# ------------------------------------------------------------------------------------------------
+# DyTC scheduling (host code in the library; no GPU work)
+# ------------------------------------------------------------------------------------------------
+def ewif_sd(alpha: float, c: float, k: int) -> float:
+    return load_library().casspec_ewif_sd(alpha, c, k)
+
+
+def ewif_hc(a1: float, c1: float, k1: int, a2: float, c2: float, k2: int) -> float:
+    return load_library().casspec_ewif_hc(a1, c1, k1, a2, c2, k2)
+
+
+def ewif_vc(alpha: float, alpha12: float, c1: float, c2: float, n: int, k: int) -> float:
+    return load_library().casspec_ewif_vc(alpha, alpha12, c1, c2, n, k)
+
+
+def dytc_objective(alpha: float, c: float, k: int, alpha_dn: float, c_dn: float) -> float:
+    return load_library().casspec_dytc_objective(alpha, c, k, alpha_dn, c_dn)
+
+
+class Dytc:
+    """Owner of one native DyTC scheduler (casspec_dytc_*)."""
+
+    def __init__(self, alphas, costs, alpha_dn: float, c_dn: float, k_max: int, t_min: float, m_max: int,
+                 lam: float = 0.7, window: int = 20):
+        lib = load_library()
+        n = len(alphas)
+        p = DytcParams(n, alpha_dn, c_dn, k_max, t_min, m_max, lam, window)
+        a = (_D * n)(*alphas)
+        c = (_D * n)(*costs)
+        h = _P()
+        _check("casspec_dytc_create", lib.casspec_dytc_create(ctypes.byref(p), a, c, ctypes.byref(h)))
+        self.h, self.m_max, self.n_cfg = h.value, m_max, n
+
+    def close(self) -> None:
+        if self.h:
+            load_library().casspec_dytc_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def set_cost(self, cfg: int, cost: float) -> None:
+        _check("casspec_dytc_set_cost", load_library().casspec_dytc_set_cost(self.h, cfg, cost))
+
+    def alpha(self, cfg: int) -> float:
+        v = _D()
+        _check("casspec_dytc_alpha", load_library().casspec_dytc_alpha(self.h, cfg, ctypes.byref(v)))
+        return v.value
+
+    def best_config(self) -> tuple[int | None, int, float]:
+        s, k, v = _I(), _I(), _D()
+        _check("casspec_dytc_best_config",
+               load_library().casspec_dytc_best_config(self.h, ctypes.byref(s), ctypes.byref(k), ctypes.byref(v)))
+        return (None if s.value < 0 else s.value), k.value, v.value
+
+    def record(self, cfg: int, accepted: bool) -> None:
+        _check("casspec_dytc_record", load_library().casspec_dytc_record(self.h, cfg, int(bool(accepted))))
+
+    def end_step(self) -> None:
+        _check("casspec_dytc_end_step", load_library().casspec_dytc_end_step(self.h))
+
+    def tree_reset(self) -> None:
+        _check("casspec_dytc_tree_reset", load_library().casspec_dytc_tree_reset(self.h))
+
+    def tree_plan(self) -> tuple[int, int, int] | None:
+        leaf, s, k = _I(), _I(), _I()
+        rc = load_library().casspec_dytc_tree_plan(self.h, ctypes.byref(leaf), ctypes.byref(s), ctypes.byref(k))
+        if rc < 0:
+            raise CasspecError("casspec_dytc_tree_plan", rc)
+        return (leaf.value, s.value, k.value) if rc == 1 else None
+
+    def tree_extend(self, leaf: int, cfg: int, tokens) -> int:
+        t = (ctypes.c_int32 * len(tokens))(*[int(x) for x in tokens])
+        rc = load_library().casspec_dytc_tree_extend(self.h, leaf, cfg, len(tokens), t)
+        if rc < 0:
+            raise CasspecError("casspec_dytc_tree_extend", rc)
+        return rc
+
+    def tree_get(self) -> dict:
+        m = self.m_max
+        n = _I()
+        par, tok, cfg = (ctypes.c_int32 * m)(), (ctypes.c_int32 * m)(), (ctypes.c_int32 * m)()
+        pacc = (_D * m)()
+        _check("casspec_dytc_tree_get", load_library().casspec_dytc_tree_get(self.h, ctypes.byref(n), par, tok, cfg, pacc))
+        k = n.value
+        return {"parent": list(par[:k]), "token": list(tok[:k]), "cfg": list(cfg[:k]), "p_acc": list(pacc[:k])}
+

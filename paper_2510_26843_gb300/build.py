@@ -13,7 +13,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libcasspec.so")
 SOURCES = ["api.cu", "chain.cu", "gemm_tc.cu", "gemm_i8.cu", "attention.cu", "small_kernels.cu",
-           "linear_static.cu"]
+           "linear_static.cu", "dytc.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-DCASSPEC_BUILD"]
@@ -42,7 +42,7 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
 
     def compile_one(src: str) -> str:
         path = os.path.join(CSRC, src)
-        obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
+        obj = os.path.join(OUT_DIR, os.path.splitext(src)[0] + ".o")
         if _stale(obj, [path, *headers, __file__]) or extra:
             cmd = [cc, *ARCH, *FLAGS, *extra, "-c", path, "-o", obj]
             if verbose:

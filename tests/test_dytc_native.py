@@ -1,0 +1,129 @@
+"""The native DyTC scheduler (casspec_ewif_*, casspec_dytc_*: host code in the C-ABI library) against
+the DyTC oracle, on seeded random inputs.  No GPU: these entry points do no device work."""
+from __future__ import annotations
+
+import random
+
+import pytest
+
+from oracle import dytc_oracle as D
+
+
+@pytest.fixture(scope="module")
+def cs():
+    from paper_2510_26843_gb300 import build as b
+
+    b.build()
+    import paper_2510_26843_gb300 as m
+
+    m.load_library()
+    return m
+
+
+def _rng(seed):
+    return random.Random(seed)
+
+
+def test_ewif_closed_forms_match_oracle(cs):
+    r = _rng(1)
+    for _ in range(300):
+        a, a2, a12 = r.uniform(0.01, 0.99), r.uniform(0.01, 0.99), r.uniform(0.01, 0.99)
+        c, c2 = r.uniform(0.0, 1.0), r.uniform(0.0, 0.2)
+        k, k2, n = r.randint(0, 10), r.randint(0, 10), r.randint(1, 6)
+        assert cs.ewif_sd(a, c, k) == pytest.approx(D.ewif_sd(a, c, k), rel=1e-12)
+        assert cs.ewif_hc(a, c, k, a2, c2, k2) == pytest.approx(D.ewif_hc(a, c, k, a2, c2, k2), rel=1e-12)
+        assert cs.ewif_vc(a, a12, c, c2, n, k) == pytest.approx(D.ewif_vc(a, a12, c, c2, n, k), rel=1e-12)
+    assert cs.ewif_sd(1.0, 0.2, 3) == pytest.approx(4 / 1.6)  # a = 1: every draft accepted
+
+
+def test_objective_and_best_config_match_oracle(cs):
+    r = _rng(2)
+    for _ in range(200):
+        n_cfg = r.randint(1, 6)
+        alphas = [r.choice([r.uniform(0, 1), 1.0, 0.0]) if r.random() < 0.1 else r.uniform(0, 1) for _ in range(n_cfg)]
+        costs = [r.uniform(0.01, 1.0) for _ in range(n_cfg)]
+        a_dn, c_dn, k_max = r.uniform(0, 1), r.choice([0.0, r.uniform(0.0, 0.1)]), r.randint(1, 8)
+        for s in range(n_cfg):
+            for k in range(1, k_max + 1):
+                want = D.step_objective(alphas[s], costs[s], k, a_dn, c_dn)
+                got = cs.dytc_objective(alphas[s], costs[s], k, a_dn, c_dn)
+                assert (want is None and got != got) or got == pytest.approx(want, rel=1e-12)
+        sch = cs.Dytc(alphas, costs, a_dn, c_dn, k_max, 0.0, 16)
+        s_o, k_o, v_o = D.find_best_config(alphas, costs, a_dn, c_dn, k_max)
+        s_n, k_n, v_n = sch.best_config()
+        assert (s_n, k_n) == (s_o, k_o)
+        if s_o is not None:
+            assert v_n == pytest.approx(v_o, rel=1e-12)
+        sch.close()
+
+
+def test_ema_matches_oracle(cs):
+    r = _rng(3)
+    n_cfg = 4
+    init = [r.uniform(0, 1) for _ in range(n_cfg)]
+    sch = cs.Dytc(init, [0.3] * n_cfg, 0.5, 0.01, 4, 0.0, 16, lam=0.7, window=5)
+    ora = D.AlphaEstimates(init, lam=0.7, window=5)
+    for _ in range(60):
+        used = [c for c in range(n_cfg) if r.random() < 0.5]
+        for c in used:
+            for _ in range(r.randint(1, 3)):
+                acc = r.random() < 0.6
+                sch.record(c, acc)
+                ora.record(c, acc)
+        sch.end_step()
+        ora.step(used)
+        for c in range(n_cfg):
+            assert sch.alpha(c) == pytest.approx(ora.alpha[c], rel=1e-12, abs=1e-15)
+    sch.close()
+
+
+def _fake_draft(cfg, path, k):
+    base = 7 * len(path) + 13 * cfg
+    return [(base + 3 * i) % 101 for i in range(k)]
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_draft_tree_matches_oracle(cs, seed):
+    r = _rng(100 + seed)
+    n_cfg = r.randint(1, 4)
+    alphas = [r.uniform(0.3, 0.99) for _ in range(n_cfg)]
+    costs = [r.uniform(0.05, 0.8) for _ in range(n_cfg)]
+    a_dn, c_dn = r.uniform(0.1, 0.8), r.choice([0.0, r.uniform(0.01, 0.1)])
+    k_max, t_min, m_max = r.randint(1, 6), r.uniform(0.1, 10.0), r.randint(2, 64)
+    want = D.draft_tree(alphas, costs, a_dn, c_dn, k_max, t_min, m_max, _fake_draft)
+    sch = cs.Dytc(alphas, costs, a_dn, c_dn, k_max, t_min, m_max)
+    sch.tree_reset()
+    steps = []
+    while True:
+        plan = sch.tree_plan()
+        if plan is None:
+            break
+        leaf, s, k = plan
+        tr = sch.tree_get()
+        path, v = [], leaf
+        while v >= 0:
+            path.append(v)
+            v = tr["parent"][v]
+        path.reverse()
+        steps.append((leaf, s, k))
+        sch.tree_extend(leaf, s, _fake_draft(s, path, k))
+    got = sch.tree_get()
+    assert steps == want["steps"]
+    assert got["parent"] == want["parent"]
+    assert got["token"][1:] == want["token"][1:] and got["token"][0] == -1
+    assert got["cfg"] == want["cfg"]
+    assert got["p_acc"] == pytest.approx(want["p_acc"], rel=1e-12)
+    sch.close()
+
+
+def test_argument_errors(cs):
+    with pytest.raises(cs.CasspecError):
+        cs.Dytc([1.5], [0.1], 0.5, 0.01, 4, 1.0, 16)  # acceptance outside [0, 1]
+    with pytest.raises(cs.CasspecError):
+        cs.Dytc([0.5], [0.1], 0.5, 0.01, 4, 1.0, 65)  # tree larger than CASSPEC_MAX_TREE
+    sch = cs.Dytc([0.5], [0.1], 0.5, 0.01, 4, 1.0, 16)
+    with pytest.raises(cs.CasspecError):
+        sch.record(3, True)  # no such configuration
+    with pytest.raises(cs.CasspecError):
+        sch.tree_extend(5, 0, [1])  # no such leaf
+    sch.close()
