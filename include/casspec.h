@@ -360,6 +360,33 @@ CASSPEC_API int casspec_dytc_tree_extend(casspec_dytc* s, int leaf, int cfg, int
 CASSPEC_API int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out, int32_t* token_out,
                                       int32_t* cfg_out, double* p_acc_out);
 
+/* A draft configuration of the model (Sec. 4.1, DSIA): its layer mask and GEMM mode, as for
+ * casspec_tree_step (skip_mask host uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16,
+ * 1 W8A8). */
+typedef struct {
+  const uint8_t* skip_mask;
+  int quant_mode;
+} casspec_draft_cfg;
+
+/* One round of DyTC speculative decoding (Sec. 4.2: Algorithm 1, one drafted token per position,
+ * then verification by the target).  Configuration i of scheduler s runs as cfgs[i].  root_token is
+ * the last generated token, not yet in the cache (the previous round's bonus token); kv must hold a
+ * committed prefix with no tree (T = 0).
+ *   Each expansion (leaf, cfg, k) that Algorithm 1 plans runs the chosen draft over root .. leaf as one
+ *   chain and then once per further drafted token (greedy argmax), and appends the k tokens.  The
+ *   target then verifies the whole tree (casspec_tree_step, all layers, bf16), the longest matching
+ *   path is accepted (casspec_accept_greedy) and compacted into the cache (casspec_kv_compact).  For
+ *   every expansion whose leaf was accepted, whether its first drafted token was accepted is recorded,
+ *   and the estimates are updated (casspec_dytc_end_step).
+ *   dev_work: device int32 [4 * CASSPEC_MAX_TREE] (caller-owned scratch).  out_tokens (host int32
+ *   [CASSPEC_MAX_TREE]) receives the tokens this round commits after the root, the last being the
+ *   bonus token (the next root); *n_out their count (>= 1); *n_drafted_out (may be NULL) the drafted
+ *   nodes.  Synchronises the model's stream several times (it reads drafted tokens back).
+ *   Errors: E_INVAL, E_STATE (kv holds a tree), E_TREE (device-reported), errors of the calls above. */
+CASSPEC_API int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv* kv, const casspec_draft_cfg* cfgs,
+                                   int32_t root_token, int32_t* dev_work, int32_t* out_tokens, int* n_out,
+                                   int* n_drafted_out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -33,7 +33,7 @@ EXPORTS = [
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
     "casspec_dytc_destroy", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_get",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -48,6 +48,10 @@ class DytcParams(ctypes.Structure):
     _fields_ = [("n_cfg", ctypes.c_int32), ("alpha_dn", ctypes.c_double), ("c_dn", ctypes.c_double),
                 ("k_max", ctypes.c_int32), ("t_min", ctypes.c_double), ("m_max", ctypes.c_int32),
                 ("lambda_", ctypes.c_double), ("window", ctypes.c_int32)]
+
+
+class DraftCfg(ctypes.Structure):
+    _fields_ = [("skip_mask", ctypes.c_void_p), ("quant_mode", ctypes.c_int32)]
 
 
 class CasspecError(RuntimeError):
@@ -87,6 +91,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_reset": (_I, [_P]),
         "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
+        "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, ctypes.POINTER(ctypes.c_int32),
+                                    ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_get": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
                                        ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_D)]),
         "casspec_create_model": (_I, [ctypes.POINTER(ModelConfig), _P, _SZ, ctypes.POINTER(_P)]),
@@ -395,4 +401,17 @@ class Dytc:
         _check("casspec_dytc_tree_get", load_library().casspec_dytc_tree_get(self.h, ctypes.byref(n), par, tok, cfg, pacc))
         k = n.value
         return {"parent": list(par[:k]), "token": list(tok[:k]), "cfg": list(cfg[:k]), "p_acc": list(pacc[:k])}
+
+    def round(self, m: int, kv: int, cfgs, root_token: int, dev_work) -> tuple[list[int], int]:
+        """One DyTC round (casspec_dytc_round).  cfgs: list of (skip_mask or None, quant_mode) per
+        configuration; dev_work: torch int32 CUDA tensor of 4 * MAX_TREE entries.  Returns the committed
+        tokens (the last is the bonus token) and the number of drafted nodes."""
+        masks = [None if sm is None else np.ascontiguousarray(np.asarray(sm, dtype=np.uint8)) for sm, _ in cfgs]
+        arr = (DraftCfg * len(cfgs))(*[DraftCfg(None if mk is None else mk.ctypes.data, int(q))
+                                        for mk, (_, q) in zip(masks, cfgs)])
+        out = (ctypes.c_int32 * MAX_TREE)()
+        n, nd = _I(), _I()
+        _check("casspec_dytc_round", load_library().casspec_dytc_round(self.h, m, kv, arr, int(root_token), _ptr(dev_work),
+                                                                       out, ctypes.byref(n), ctypes.byref(nd)))
+        return list(out[: n.value]), nd.value
 

@@ -987,3 +987,103 @@ int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q, float* s, 
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------------
+// One DyTC round (Sec. 4.2, Algorithm 1 with one drafted token per position, then verification)
+// ---------------------------------------------------------------------------------------------
+namespace {
+int read_dev_i32(casspec_model* m, const int32_t* dev, int count, int32_t* host) {
+  CK(cudaMemcpyAsync(host, dev, (size_t)count * 4, cudaMemcpyDeviceToHost, m->stream));
+  CK(cudaStreamSynchronize(m->stream));
+  return CASSPEC_OK;
+}
+}  // namespace
+
+extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv* kv, const casspec_draft_cfg* cfgs,
+                                  int32_t root_token, int32_t* dev_work, int32_t* out_tokens, int* n_out,
+                                  int* n_drafted_out) {
+  if (s == nullptr || m == nullptr || kv == nullptr || cfgs == nullptr || dev_work == nullptr || out_tokens == nullptr ||
+      n_out == nullptr || kv->m != m)
+    return CASSPEC_E_INVAL;
+  if (kv->T != 0) return CASSPEC_E_STATE;  // a round starts from a committed prefix
+  int32_t* d_tok = dev_work;
+  int32_t* d_par = dev_work + kMaxTree;
+  int32_t* d_acc = dev_work + 2 * kMaxTree;
+  const int32_t* d_am = m->am;
+  int rc;
+  if ((rc = casspec_dytc_tree_reset(s)) != CASSPEC_OK) return rc;
+  struct Expansion {
+    int leaf, cfg, first;
+  };
+  std::vector<Expansion> exps;
+  int32_t par[kMaxTree], tok[kMaxTree], ncfg[kMaxTree];
+  int n = 1;
+  tok[0] = root_token;
+  par[0] = -1;
+  while (true) {
+    int leaf = -1, c = -1, k = 0;
+    rc = casspec_dytc_tree_plan(s, &leaf, &c, &k);
+    if (rc < 0) return rc;
+    if (rc == 0) break;
+    if ((rc = casspec_dytc_tree_get(s, &n, par, tok, ncfg, nullptr)) != CASSPEC_OK) return rc;
+    tok[0] = root_token;
+    // the chosen draft processes root .. leaf as one chain (valid for any layer mask), then each
+    // drafted token in turn; the argmax of the last processed node is the next drafted token
+    int32_t chain[kMaxTree];
+    int len = 0;
+    for (int v = leaf; v >= 0; v = par[v]) chain[len++] = v;
+    int32_t ctok[kMaxTree], cpar[kMaxTree];
+    for (int i = 0; i < len; ++i) {
+      ctok[i] = tok[chain[len - 1 - i]];
+      cpar[i] = i - 1;
+    }
+    casspec_kv_reset_tree(kv);
+    CK(cudaMemcpyAsync(d_tok, ctok, (size_t)len * 4, cudaMemcpyHostToDevice, m->stream));
+    CK(cudaMemcpyAsync(d_par, cpar, (size_t)len * 4, cudaMemcpyHostToDevice, m->stream));
+    if ((rc = casspec_tree_step(m, kv, d_tok, d_par, len, cfgs[c].skip_mask, cfgs[c].quant_mode, nullptr)) != CASSPEC_OK)
+      return rc;
+    int32_t drafted[kMaxTree];
+    if ((rc = read_dev_i32(m, d_am + (len - 1), 1, &drafted[0])) != CASSPEC_OK) return rc;
+    const int room = std::min(k, kMaxTree - len);  // physical tree slots of this expansion
+    for (int i = 1; i < room; ++i) {
+      ctok[len + i - 1] = drafted[i - 1];
+      cpar[len + i - 1] = len + i - 2;
+      CK(cudaMemcpyAsync(d_tok + len + i - 1, &ctok[len + i - 1], 4, cudaMemcpyHostToDevice, m->stream));
+      CK(cudaMemcpyAsync(d_par + len + i - 1, &cpar[len + i - 1], 4, cudaMemcpyHostToDevice, m->stream));
+      if ((rc = casspec_tree_step(m, kv, d_tok + len + i - 1, d_par + len + i - 1, 1, cfgs[c].skip_mask,
+                                  cfgs[c].quant_mode, nullptr)) != CASSPEC_OK)
+        return rc;
+      if ((rc = read_dev_i32(m, d_am, 1, &drafted[i])) != CASSPEC_OK) return rc;
+    }
+    const int first = n;
+    rc = casspec_dytc_tree_extend(s, leaf, c, room, drafted);
+    if (rc < 0) return rc;
+    if (rc > 0) exps.push_back({leaf, c, first});
+    if (rc < room) break;  // the tree is full
+  }
+  if ((rc = casspec_dytc_tree_get(s, &n, par, tok, ncfg, nullptr)) != CASSPEC_OK) return rc;
+  tok[0] = root_token;
+  // verification by the target model over the whole tree, greedy acceptance
+  casspec_kv_reset_tree(kv);
+  CK(cudaMemcpyAsync(d_tok, tok, (size_t)n * 4, cudaMemcpyHostToDevice, m->stream));
+  CK(cudaMemcpyAsync(d_par, par, (size_t)n * 4, cudaMemcpyHostToDevice, m->stream));
+  if ((rc = casspec_tree_step(m, kv, d_tok, d_par, n, nullptr, 0, nullptr)) != CASSPEC_OK) return rc;
+  if ((rc = casspec_accept_greedy(m, nullptr, d_tok, d_par, n, d_acc)) != CASSPEC_OK) return rc;
+  int32_t acc[kMaxTree + 2];
+  if ((rc = read_dev_i32(m, d_acc, n + 2, acc)) != CASSPEC_OK) return rc;
+  const int L = acc[0];
+  if (L < 1 || L > n) return CASSPEC_E_TREE;
+  std::vector<uint8_t> on_path(n, 0);
+  for (int i = 1; i <= L; ++i)
+    if (acc[i] >= 0 && acc[i] < n) on_path[acc[i]] = 1;
+  // first-draft-token outcomes of the expansions whose leaf the target accepted (Sec. 4.2)
+  for (const auto& e : exps)
+    if (on_path[e.leaf]) casspec_dytc_record(s, e.cfg, on_path[e.first]);
+  casspec_dytc_end_step(s);
+  if ((rc = casspec_kv_compact(kv, d_acc)) != CASSPEC_OK) return rc;
+  for (int i = 2; i <= L; ++i) out_tokens[i - 2] = tok[acc[i]];
+  out_tokens[L - 1] = acc[L + 1];  // the bonus token: the next round's root
+  *n_out = L;
+  if (n_drafted_out) *n_drafted_out = n - 1;
+  return CASSPEC_OK;
+}

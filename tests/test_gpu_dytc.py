@@ -1,0 +1,86 @@
+"""DyTC speculative decoding on the GPU (Sec. 4.2 Algorithm 1 with the native scheduler, drafts and
+verification as tree steps): on the tiny decoder, rounds of casspec_dytc_round must reproduce the
+oracle's greedy autoregressive output (losslessness, Sec. 5.1), except after a near-tie of greedy
+decoding itself (top-2 logit margin below 1e-3), and the acceptance estimates must follow what the
+target accepted."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+SH = synth.TINY
+SEED = 1234
+MARGIN = 1e-3
+
+
+@pytest.fixture(scope="module")
+def cs():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import paper_2510_26843_gb300 as m
+
+    m.load_library()
+    return m
+
+
+def _truth(prefix, steps):
+    ow = oracle.Weights.from_seed(SEED, SH, keep_layers=SH.n_layers)
+    okv = oracle.KVCache(SH.n_layers, SH.n_heads, SH.head_dim, 256)
+    lg = oracle.tree_step(ow, okv, prefix, synth.chain(len(prefix)))
+    oracle.kv_compact(okv, list(range(len(prefix))))
+    truth, margins = [int(oracle.argmax_lowest(lg[-1:])[0])], [oracle.top2_margin(lg[-1:])[0]]
+    while len(truth) < steps + 1:
+        lg = oracle.tree_step(ow, okv, [truth[-1]], [-1])
+        oracle.kv_compact(okv, [0])
+        truth.append(int(oracle.argmax_lowest(lg)[0]))
+        margins.append(oracle.top2_margin(lg)[0])
+    return truth, margins
+
+
+def test_dytc_rounds_are_lossless_and_learn_acceptance(cs):
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    steps = 40
+    prefix = synth.prefix_tokens(SEED, 64, SH.vocab)
+    truth, margins = _truth(prefix, steps)
+
+    dm = DeviceModel(SH, SEED, with_int8=True)
+    kv = DeviceKV(dm, 256)
+    n0 = len(prefix)
+    t = torch.tensor(np.asarray(prefix, dtype=np.int32), device="cuda")
+    p = torch.tensor(np.asarray(synth.chain(n0), dtype=np.int32), device="cuda")
+    logits = torch.empty(n0, SH.vocab, device="cuda")
+    cs.tree_step(dm.h, kv.h, t, p, n0, None, 0, logits)
+    cs.kv_compact(kv.h, torch.tensor([n0, *range(n0), 0], dtype=torch.int32, device="cuda"))
+    out = [int(torch.argmax(logits[-1]).item())]
+
+    # two draft configurations of the 2-layer model: the first layer alone (bf16), and every layer
+    # in W8A8; a notional bottom draft (alpha 0.3, cost 0.05)
+    cfgs = [(np.array([1, 0], dtype=np.uint8), 0), (None, 1)]
+    sch = cs.Dytc([0.5, 0.5], [0.5, 0.6], alpha_dn=0.3, c_dn=0.05, k_max=4, t_min=0.5, m_max=16)
+    work = torch.zeros(4 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    rounds = drafted = 0
+    while len(out) < steps:
+        toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work)
+        assert 1 <= len(toks) <= nd + 1
+        out.extend(toks)
+        drafted += nd
+        rounds += 1
+    assert cs.get_status(dm.h) == 0
+    first_diff = next((i for i in range(steps) if out[i] != truth[i]), None)
+    if first_diff is not None:
+        assert min(margins[: first_diff + 1]) < MARGIN, (first_diff, out[:steps], truth[:steps])
+    assert drafted > 0 and rounds < steps  # drafts were made and some were accepted
+    # the W8A8 draft of every layer agrees with the target far more often than the half-depth one
+    assert sch.alpha(1) > sch.alpha(0)
+    P, T = cs.kv_length(kv.h)
+    assert T == 0 and P == n0 + len(out) - 1  # every committed token but the last root is cached
+    sch.close()
+    kv.close()
+    dm.close()
