@@ -25,7 +25,15 @@ What it computes (CAS-Spec, arXiv 2510.26843):
     a_dn / c_dn * P_acc < t_min or the tree holds m_max nodes, choose (S, k) by Algorithm 2, append
     the k drafted tokens below the leaf with P_acc(child) = P_acc(parent) * a_S.
 
+  * Sec. 4.2, the hardware-aware latency prediction behind the cost coefficients: a Bayesian linear
+    regression of step latency on the bytes the step moves (a roofline: latency = w0 + w1 * bytes),
+    Gaussian prior N(mu0, diag(sd0^2)) on w and Gaussian noise; c(S) = predicted latency of draft S /
+    predicted latency of the target.
+
 Readings (the paper is silent or inconsistent; each is also listed in the design notes):
+  * the latency model's regressor is the bytes a step moves (weights of its active layers, K/V,
+    activations), the quantity the roofline of a memory-bound step is linear in; the paper names
+    only "roofline latency" and "Bayesian linear regression";
   * phi^n in T_VC is the n-th power of the generating function (n independent rounds of d2);
   * only leaves are expanded: Algorithm 1 marks every new node active and never clears the expanded
     node, which would let a node be drafted twice from the same sequence; a node that receives a
@@ -190,3 +198,21 @@ def draft_tree(alphas: list[float], costs: list[float], a_dn: float, c_dn: float
             if len(parent) >= m_max:
                 return {"parent": parent, "token": token, "cfg": cfg_of, "p_acc": p_acc, "steps": steps}
     return {"parent": parent, "token": token, "cfg": cfg_of, "p_acc": p_acc, "steps": steps}
+
+
+# ------------------------------------------------------------------------------------------------
+# Sec. 4.2: latency model (Bayesian linear regression)
+# ------------------------------------------------------------------------------------------------
+def blr_posterior(x, y, mu0, sd0, noise_sd):
+    """Posterior mean and covariance of w in y = w0 + w1 x + e, e ~ N(0, noise_sd^2), with prior
+    w ~ N(mu0, diag(sd0^2)): cov = (S0^-1 + X^T X / s^2)^-1, mean = cov (S0^-1 mu0 + X^T y / s^2)."""
+    import numpy as np
+
+    X = np.stack([np.ones(len(x)), np.asarray(x, dtype=np.float64)], axis=1) if len(x) else np.zeros((0, 2))
+    y = np.asarray(y, dtype=np.float64)
+    prec0 = np.diag(1.0 / np.asarray(sd0, dtype=np.float64) ** 2)
+    prec = prec0 + X.T @ X / noise_sd ** 2
+    cov = np.linalg.inv(prec)
+    mean = cov @ (prec0 @ np.asarray(mu0, dtype=np.float64) + X.T @ y / noise_sd ** 2)
+    return mean, cov
+
