@@ -310,6 +310,15 @@ CASSPEC_API double casspec_ewif_vc(double alpha, double alpha12, double c1, doub
  * (its "least future speedup").  NaN where Algorithm 2 skips the pair (c k + c_dn ~ 0) or k < 1. */
 CASSPEC_API double casspec_dytc_objective(double alpha, double c, int k, double alpha_dn, double c_dn);
 
+/* The latency model behind the cost coefficients (Sec. 4.2: hardware-aware latency prediction by
+ * Bayesian linear regression): latency = w0 + w1 x with x the bytes a step moves (its roofline is
+ * linear in them), prior w ~ N(mu0, diag(sd0^2)) (mu0, sd0 host [2]), Gaussian noise of standard
+ * deviation noise_sd, fitted to m measured steps (x, y host [m]; m = 0 returns the prior).  Writes the
+ * posterior mean to w_out [2] and, if non-NULL, the posterior covariance to cov_out [2][2].  A draft's
+ * cost coefficient is then (w0 + w1 x_draft) / (w0 + w1 x_target).  Errors: E_INVAL. */
+CASSPEC_API int casspec_latency_fit(const double* x, const double* y, int m, const double* mu0, const double* sd0,
+                                    double noise_sd, double* w_out, double* cov_out);
+
 #define CASSPEC_DYTC_MAX_CFG 16
 typedef struct casspec_dytc casspec_dytc;
 typedef struct {

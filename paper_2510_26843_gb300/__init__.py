@@ -33,7 +33,7 @@ EXPORTS = [
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
     "casspec_dytc_destroy", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -91,6 +91,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_reset": (_I, [_P]),
         "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
+        "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
+                                     ctypes.POINTER(_D), ctypes.POINTER(_D)]),
         "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, ctypes.POINTER(ctypes.c_int32),
                                     ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_get": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
@@ -329,6 +331,16 @@ def ewif_vc(alpha: float, alpha12: float, c1: float, c2: float, n: int, k: int) 
 
 def dytc_objective(alpha: float, c: float, k: int, alpha_dn: float, c_dn: float) -> float:
     return load_library().casspec_dytc_objective(alpha, c, k, alpha_dn, c_dn)
+
+
+def latency_fit(x, y, mu0, sd0, noise_sd: float) -> tuple[list[float], list[float]]:
+    """Posterior mean [w0, w1] and covariance (row-major 2 x 2) of latency = w0 + w1 * bytes."""
+    m = len(x)
+    xa, ya = (_D * max(m, 1))(*[float(v) for v in x]), (_D * max(m, 1))(*[float(v) for v in y])
+    mu, sd = (_D * 2)(*[float(v) for v in mu0]), (_D * 2)(*[float(v) for v in sd0])
+    w, cov = (_D * 2)(), (_D * 4)()
+    _check("casspec_latency_fit", load_library().casspec_latency_fit(xa, ya, m, mu, sd, float(noise_sd), w, cov))
+    return list(w), list(cov)
 
 
 class Dytc:

@@ -222,4 +222,41 @@ int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out
   return CASSPEC_OK;
 }
 
+int casspec_latency_fit(const double* x, const double* y, int m, const double* mu0, const double* sd0, double noise_sd,
+                        double* w_out, double* cov_out) {
+  if ((m > 0 && (x == nullptr || y == nullptr)) || m < 0 || mu0 == nullptr || sd0 == nullptr || w_out == nullptr ||
+      !(sd0[0] > 0.0) || !(sd0[1] > 0.0) || !(noise_sd > 0.0))
+    return CASSPEC_E_INVAL;
+  // Solved in the scaled regressor u = x / xs (w1 scaled to w1 xs with its prior) so that the 2 x 2
+  // system stays well conditioned whatever unit x comes in; precision = S0^-1 + U^T U / s^2,
+  // rhs = S0^-1 mu0 + U^T y / s^2.
+  double xs = 0.0;
+  for (int i = 0; i < m; ++i) xs = std::fmax(xs, std::fabs(x[i]));
+  if (!(xs > 0.0)) xs = 1.0;
+  const double is2 = 1.0 / (noise_sd * noise_sd);
+  const double sd1 = sd0[1] * xs, mu1 = mu0[1] * xs;
+  double a = 1.0 / (sd0[0] * sd0[0]), b = 0.0, d = 1.0 / (sd1 * sd1);
+  double r0 = mu0[0] * a, r1 = mu1 * d;
+  for (int i = 0; i < m; ++i) {
+    const double u = x[i] / xs;
+    a += is2;
+    b += u * is2;
+    d += u * u * is2;
+    r0 += y[i] * is2;
+    r1 += u * y[i] * is2;
+  }
+  const double det = a * d - b * b;
+  if (!(det > 0.0)) return CASSPEC_E_INVAL;
+  const double c00 = d / det, c01 = -b / det, c11 = a / det;
+  w_out[0] = c00 * r0 + c01 * r1;
+  w_out[1] = (c01 * r0 + c11 * r1) / xs;
+  if (cov_out) {
+    cov_out[0] = c00;
+    cov_out[1] = c01 / xs;
+    cov_out[2] = c01 / xs;
+    cov_out[3] = c11 / (xs * xs);
+  }
+  return CASSPEC_OK;
+}
+
 }  // extern "C"

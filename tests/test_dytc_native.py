@@ -127,3 +127,20 @@ def test_argument_errors(cs):
     with pytest.raises(cs.CasspecError):
         sch.tree_extend(5, 0, [1])  # no such leaf
     sch.close()
+
+
+def test_latency_fit_matches_oracle(cs):
+    import numpy as np
+
+    rng = np.random.default_rng(11)
+    for m in (0, 1, 5, 40):
+        x = rng.uniform(1.0, 30.0, m)  # GB moved per step
+        y = 20.0 + x * 151.5 + rng.normal(0, 50.0, m)  # microseconds (6.6 TB/s)
+        mu0, sd0, noise = [0.0, 150.0], [100.0, 100.0], 40.0
+        w, cov = cs.latency_fit(x, y, mu0, sd0, noise)
+        mean_o, cov_o = D.blr_posterior(x, y, mu0, sd0, noise)
+        assert w == pytest.approx(list(mean_o), rel=1e-9)
+        assert cov == pytest.approx(list(cov_o.reshape(-1)), rel=1e-9, abs=1e-30)
+    with pytest.raises(cs.CasspecError):
+        cs.latency_fit([1.0], [2.0], [0.0, 0.0], [0.0, 1.0], 1.0)  # zero prior spread
+

@@ -191,25 +191,25 @@ def test_blr_limits_and_sequential_updates():
     import numpy as np
 
     rng = np.random.default_rng(7)
-    x = rng.uniform(1e9, 15e9, 12)
-    y = 25.0 + x / 6.5e3 + rng.normal(0, 30.0, 12)  # microseconds: overhead + bytes at 6.5 TB/s
+    x = rng.uniform(1.0, 15.0, 12)  # GB moved per step
+    y = 25.0 + x * 153.8 + rng.normal(0, 30.0, 12)  # microseconds: overhead + bytes at 6.5 TB/s
     # a flat prior gives ordinary least squares
     mean, _ = D.blr_posterior(x, y, [0.0, 0.0], [1e12, 1e12], 30.0)
     ols = np.linalg.lstsq(np.stack([np.ones(12), x], 1), y, rcond=None)[0]
     assert mean == pytest.approx(ols, rel=1e-6)
     # no data gives the prior
-    mean0, cov0 = D.blr_posterior([], [], [5.0, 1e-4], [2.0, 1e-5], 30.0)
-    assert mean0 == pytest.approx([5.0, 1e-4]) and cov0 == pytest.approx(np.diag([4.0, 1e-10]))
+    mean0, cov0 = D.blr_posterior([], [], [5.0, 150.0], [2.0, 10.0], 30.0)
+    assert mean0 == pytest.approx([5.0, 150.0]) and cov0 == pytest.approx(np.diag([4.0, 100.0]))
     # conjugacy: one point at a time (each posterior the next prior, through its full covariance)
     # equals the batch posterior
-    mu, cov = np.array([10.0, 2e-4]), np.diag([50.0 ** 2, (1e-4) ** 2])
+    mu, cov = np.array([10.0, 140.0]), np.diag([50.0 ** 2, 40.0 ** 2])
     for xi, yi in zip(x, y):
         h = np.array([1.0, xi])
         s = h @ cov @ h + 30.0 ** 2
         gain = cov @ h / s
         mu = mu + gain * (yi - h @ mu)
         cov = cov - np.outer(gain, h @ cov)
-    mean_b, cov_b = D.blr_posterior(x, y, [10.0, 2e-4], [50.0, 1e-4], 30.0)
+    mean_b, cov_b = D.blr_posterior(x, y, [10.0, 140.0], [50.0, 40.0], 30.0)
     assert mean_b == pytest.approx(mu, rel=1e-6)
     assert cov_b == pytest.approx(cov, rel=1e-5, abs=1e-30)
 
