@@ -369,6 +369,16 @@ CASSPEC_API int casspec_dytc_tree_extend(casspec_dytc* s, int leaf, int cfg, int
 CASSPEC_API int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out, int32_t* token_out,
                                       int32_t* cfg_out, double* p_acc_out);
 
+/* Prompt-lookup bottom draft (PLD: the default bottom draft M_dn, Sec. 4.1; its match length is its
+ * confidence, Sec. 4.2).  Over the history tokens (dev int32 [L], L >= 0), find the longest n in
+ * [n_min, n_max] (1 <= n_min <= n_max <= 64) such that the last n tokens occurred earlier, ending at a
+ * position p < L - 1; among those occurrences take the latest; draft the tokens x[p+1 .. p+k] (cut at
+ * the history's end, k <= CASSPEC_MAX_TREE).  out (dev int32 [2 + k]) receives {n (0: no match),
+ * drafted count, tokens...}.  One kernel on cuda_stream; the library's models are not involved.
+ * Errors: E_INVAL (arguments), E_CUDA (launch). */
+CASSPEC_API int casspec_pld_draft(const int32_t* tokens, int L, int n_min, int n_max, int k, int32_t* out,
+                                  void* cuda_stream);
+
 /* A draft configuration of the model (Sec. 4.1, DSIA): its layer mask and GEMM mode, as for
  * casspec_tree_step (skip_mask host uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16,
  * 1 W8A8). */

@@ -33,7 +33,7 @@ EXPORTS = [
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
     "casspec_dytc_destroy", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -91,6 +91,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_reset": (_I, [_P]),
         "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
+        "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
         "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
                                      ctypes.POINTER(_D), ctypes.POINTER(_D)]),
         "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, ctypes.POINTER(ctypes.c_int32),
@@ -331,6 +332,12 @@ def ewif_vc(alpha: float, alpha12: float, c1: float, c2: float, n: int, k: int) 
 
 def dytc_objective(alpha: float, c: float, k: int, alpha_dn: float, c_dn: float) -> float:
     return load_library().casspec_dytc_objective(alpha, c, k, alpha_dn, c_dn)
+
+
+def pld_draft(tokens, L: int, n_min: int, n_max: int, k: int, out, stream=None) -> None:
+    """casspec_pld_draft: tokens dev int32 [L], out dev int32 [2 + k] = {match length, count, tokens}."""
+    _check("casspec_pld_draft", load_library().casspec_pld_draft(_ptr(tokens), L, n_min, n_max, k, _ptr(out),
+                                                                   _stream(stream)))
 
 
 def latency_fit(x, y, mu0, sd0, noise_sd: float) -> tuple[list[float], list[float]]:
