@@ -379,12 +379,14 @@ CASSPEC_API int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t
 CASSPEC_API int casspec_pld_draft(const int32_t* tokens, int L, int n_min, int n_max, int k, int32_t* out,
                                   void* cuda_stream);
 
-/* A draft configuration of the model (Sec. 4.1, DSIA): its layer mask and GEMM mode, as for
- * casspec_tree_step (skip_mask host uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16,
- * 1 W8A8). */
+/* A draft configuration: a DSIA draft of the model (Sec. 4.1), with its layer mask and GEMM mode as
+ * for casspec_tree_step (skip_mask host uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16,
+ * 1 W8A8), or, when pld_n_max > 0, the prompt-lookup bottom draft (casspec_pld_draft with n in
+ * [1, pld_n_max] over the committed history and the path to the leaf). */
 typedef struct {
   const uint8_t* skip_mask;
   int quant_mode;
+  int pld_n_max;
 } casspec_draft_cfg;
 
 /* One round of DyTC speculative decoding (Sec. 4.2: Algorithm 1, one drafted token per position,
@@ -397,14 +399,18 @@ typedef struct {
  *   path is accepted (casspec_accept_greedy) and compacted into the cache (casspec_kv_compact).  For
  *   every expansion whose leaf was accepted, whether its first drafted token was accepted is recorded,
  *   and the estimates are updated (casspec_dytc_end_step).
- *   dev_work: device int32 [4 * CASSPEC_MAX_TREE] (caller-owned scratch).  out_tokens (host int32
+ *   A prompt-lookup configuration drafts from history (dev int32, the committed tokens, the last
+ *   being root_token; hist_len entries, room for CASSPEC_MAX_TREE more, which the round overwrites);
+ *   finding no earlier occurrence counts as a rejected first token and ends the drafting.  history
+ *   may be NULL when no configuration is a prompt lookup.
+ *   dev_work: device int32 [5 * CASSPEC_MAX_TREE] (caller-owned scratch).  out_tokens (host int32
  *   [CASSPEC_MAX_TREE]) receives the tokens this round commits after the root, the last being the
  *   bonus token (the next root); *n_out their count (>= 1); *n_drafted_out (may be NULL) the drafted
  *   nodes.  Synchronises the model's stream several times (it reads drafted tokens back).
  *   Errors: E_INVAL, E_STATE (kv holds a tree), E_TREE (device-reported), errors of the calls above. */
 CASSPEC_API int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv* kv, const casspec_draft_cfg* cfgs,
-                                   int32_t root_token, int32_t* dev_work, int32_t* out_tokens, int* n_out,
-                                   int* n_drafted_out);
+                                   int32_t root_token, int32_t* history, int hist_len, int32_t* dev_work,
+                                   int32_t* out_tokens, int* n_out, int* n_drafted_out);
 
 #ifdef __cplusplus
 }

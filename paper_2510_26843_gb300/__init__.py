@@ -51,7 +51,7 @@ class DytcParams(ctypes.Structure):
 
 
 class DraftCfg(ctypes.Structure):
-    _fields_ = [("skip_mask", ctypes.c_void_p), ("quant_mode", ctypes.c_int32)]
+    _fields_ = [("skip_mask", ctypes.c_void_p), ("quant_mode", ctypes.c_int32), ("pld_n_max", ctypes.c_int32)]
 
 
 class CasspecError(RuntimeError):
@@ -94,8 +94,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
         "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
                                      ctypes.POINTER(_D), ctypes.POINTER(_D)]),
-        "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, ctypes.POINTER(ctypes.c_int32),
-                                    ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+        "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, _I, _P,
+                                    ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_get": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
                                        ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_D)]),
         "casspec_create_model": (_I, [ctypes.POINTER(ModelConfig), _P, _SZ, ctypes.POINTER(_P)]),
@@ -421,16 +421,26 @@ class Dytc:
         k = n.value
         return {"parent": list(par[:k]), "token": list(tok[:k]), "cfg": list(cfg[:k]), "p_acc": list(pacc[:k])}
 
-    def round(self, m: int, kv: int, cfgs, root_token: int, dev_work) -> tuple[list[int], int]:
-        """One DyTC round (casspec_dytc_round).  cfgs: list of (skip_mask or None, quant_mode) per
-        configuration; dev_work: torch int32 CUDA tensor of 4 * MAX_TREE entries.  Returns the committed
-        tokens (the last is the bonus token) and the number of drafted nodes."""
-        masks = [None if sm is None else np.ascontiguousarray(np.asarray(sm, dtype=np.uint8)) for sm, _ in cfgs]
-        arr = (DraftCfg * len(cfgs))(*[DraftCfg(None if mk is None else mk.ctypes.data, int(q))
-                                        for mk, (_, q) in zip(masks, cfgs)])
+    def round(self, m: int, kv: int, cfgs, root_token: int, dev_work, history=None, hist_len: int = 0) -> tuple[list[int], int]:
+        """One DyTC round (casspec_dytc_round).  cfgs: per configuration (skip_mask or None, quant_mode)
+        for a model draft, or ("pld", n_max) for the prompt-lookup draft; history: torch int32 CUDA
+        tensor of the committed tokens (hist_len valid, the last = root_token, room for MAX_TREE more);
+        dev_work: torch int32 CUDA tensor of 5 * MAX_TREE entries.  Returns the committed tokens (the
+        last is the bonus token) and the number of drafted nodes."""
+        masks, items = [], []
+        for a, b in cfgs:
+            if isinstance(a, str):
+                masks.append(None)
+                items.append(DraftCfg(None, 0, int(b)))
+            else:
+                mk = None if a is None else np.ascontiguousarray(np.asarray(a, dtype=np.uint8))
+                masks.append(mk)
+                items.append(DraftCfg(None if mk is None else mk.ctypes.data, int(b), 0))
+        arr = (DraftCfg * len(items))(*items)
         out = (ctypes.c_int32 * MAX_TREE)()
         n, nd = _I(), _I()
-        _check("casspec_dytc_round", load_library().casspec_dytc_round(self.h, m, kv, arr, int(root_token), _ptr(dev_work),
-                                                                       out, ctypes.byref(n), ctypes.byref(nd)))
+        _check("casspec_dytc_round", load_library().casspec_dytc_round(self.h, m, kv, arr, int(root_token), _ptr(history),
+                                                                       int(hist_len), _ptr(dev_work), out,
+                                                                       ctypes.byref(n), ctypes.byref(nd)))
         return list(out[: n.value]), nd.value
 

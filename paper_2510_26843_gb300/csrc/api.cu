@@ -1000,8 +1000,8 @@ int read_dev_i32(casspec_model* m, const int32_t* dev, int count, int32_t* host)
 }  // namespace
 
 extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv* kv, const casspec_draft_cfg* cfgs,
-                                  int32_t root_token, int32_t* dev_work, int32_t* out_tokens, int* n_out,
-                                  int* n_drafted_out) {
+                                  int32_t root_token, int32_t* history, int hist_len, int32_t* dev_work,
+                                  int32_t* out_tokens, int* n_out, int* n_drafted_out) {
   if (s == nullptr || m == nullptr || kv == nullptr || cfgs == nullptr || dev_work == nullptr || out_tokens == nullptr ||
       n_out == nullptr || kv->m != m)
     return CASSPEC_E_INVAL;
@@ -1009,6 +1009,7 @@ extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv*
   int32_t* d_tok = dev_work;
   int32_t* d_par = dev_work + kMaxTree;
   int32_t* d_acc = dev_work + 2 * kMaxTree;
+  int32_t* d_pld = dev_work + 3 * kMaxTree + 8;  // {match length, count, tokens...}
   const int32_t* d_am = m->am;
   int rc;
   if ((rc = casspec_dytc_tree_reset(s)) != CASSPEC_OK) return rc;
@@ -1036,6 +1037,26 @@ extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv*
     for (int i = 0; i < len; ++i) {
       ctok[i] = tok[chain[len - 1 - i]];
       cpar[i] = i - 1;
+    }
+    if (cfgs[c].pld_n_max > 0) {
+      // the prompt-lookup bottom draft: the path below the root continues the committed history
+      if (history == nullptr || hist_len < 1) return CASSPEC_E_INVAL;
+      if (len > 1)
+        CK(cudaMemcpyAsync(history + hist_len, ctok + 1, (size_t)(len - 1) * 4, cudaMemcpyHostToDevice, m->stream));
+      if ((rc = casspec_pld_draft(history, hist_len + len - 1, 1, cfgs[c].pld_n_max, k, d_pld, m->stream)) != CASSPEC_OK)
+        return rc;
+      int32_t pr[kMaxTree + 2];
+      if ((rc = read_dev_i32(m, d_pld, 2 + k, pr)) != CASSPEC_OK) return rc;
+      if (pr[1] < 1) {  // no earlier occurrence: nothing drafted, a failure of this configuration
+        casspec_dytc_record(s, c, 0);
+        break;
+      }
+      const int first = n;
+      rc = casspec_dytc_tree_extend(s, leaf, c, pr[1], pr + 2);
+      if (rc < 0) return rc;
+      if (rc > 0) exps.push_back({leaf, c, first});
+      if (rc < pr[1]) break;  // the tree is full
+      continue;
     }
     casspec_kv_reset_tree(kv);
     CK(cudaMemcpyAsync(d_tok, ctok, (size_t)len * 4, cudaMemcpyHostToDevice, m->stream));

@@ -64,7 +64,7 @@ def test_dytc_rounds_are_lossless_and_learn_acceptance(cs):
     # in W8A8; a notional bottom draft (alpha 0.3, cost 0.05)
     cfgs = [(np.array([1, 0], dtype=np.uint8), 0), (None, 1)]
     sch = cs.Dytc([0.5, 0.5], [0.5, 0.6], alpha_dn=0.3, c_dn=0.05, k_max=4, t_min=0.5, m_max=16)
-    work = torch.zeros(4 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    work = torch.zeros(5 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
     rounds = drafted = 0
     while len(out) < steps:
         toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work)
@@ -84,3 +84,49 @@ def test_dytc_rounds_are_lossless_and_learn_acceptance(cs):
     sch.close()
     kv.close()
     dm.close()
+
+
+def test_dytc_rounds_with_prompt_lookup_bottom_draft_are_lossless(cs):
+    """The same with the prompt-lookup draft (casspec_pld_draft over the committed history) as a third
+    configuration: whatever it proposes, verification keeps the output equal to greedy decoding."""
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    steps = 48
+    prefix = synth.prefix_tokens(SEED + 1, 64, SH.vocab)
+    truth, margins = _truth(prefix, steps)
+    dm = DeviceModel(SH, SEED, with_int8=True)
+    kv = DeviceKV(dm, 256)
+    n0 = len(prefix)
+    t = torch.tensor(np.asarray(prefix, dtype=np.int32), device="cuda")
+    p = torch.tensor(np.asarray(synth.chain(n0), dtype=np.int32), device="cuda")
+    logits = torch.empty(n0, SH.vocab, device="cuda")
+    cs.tree_step(dm.h, kv.h, t, p, n0, None, 0, logits)
+    cs.kv_compact(kv.h, torch.tensor([n0, *range(n0), 0], dtype=torch.int32, device="cuda"))
+    out = [int(torch.argmax(logits[-1]).item())]
+    history = torch.zeros(n0 + steps + 4 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    history[:n0] = t
+    history[n0] = out[0]
+    hist_len = n0 + 1
+
+    cfgs = [(np.array([1, 0], dtype=np.uint8), 0), (None, 1), ("pld", 4)]
+    sch = cs.Dytc([0.5, 0.5, 0.3], [0.5, 0.6, 0.02], alpha_dn=0.3, c_dn=0.02, k_max=4, t_min=0.5, m_max=16)
+    work = torch.zeros(5 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    rounds = 0
+    while len(out) < steps:
+        toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work, history, hist_len)
+        assert 1 <= len(toks) <= nd + 1
+        history[hist_len:hist_len + len(toks)] = torch.tensor(toks, dtype=torch.int32, device="cuda")
+        hist_len += len(toks)
+        out.extend(toks)
+        rounds += 1
+    assert cs.get_status(dm.h) == 0
+    first_diff = next((i for i in range(steps) if out[i] != truth[i]), None)
+    if first_diff is not None:
+        assert min(margins[: first_diff + 1]) < MARGIN, (first_diff, out[:steps], truth[:steps])
+    assert rounds < steps
+    P, T = cs.kv_length(kv.h)
+    assert T == 0 and P == n0 + len(out) - 1
+    sch.close()
+    kv.close()
+    dm.close()
+
