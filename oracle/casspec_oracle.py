@@ -402,3 +402,16 @@ def kv_compact(kv: KVCache, path: list) -> None:
             kv.valid[l][P + k] = ok[k]
     kv.P = P + len(path)
     kv.reset_tree()
+
+
+def topk_softmax(logits: np.ndarray, k: int) -> tuple[np.ndarray, np.ndarray]:
+    """K-best candidates per row for tree expansion (Sec. 4.2, Algorithm 1: top-K tokens of each drafted
+    position; their normalised probabilities rank siblings): the k largest logits of each row (ties to
+    the lower token id), and their softmax probabilities over the whole row, in fp64."""
+    x = np.asarray(logits, dtype=np.float64)
+    k = min(k, x.shape[1])
+    idx = np.argsort(-x, axis=1, kind="stable")[:, :k]
+    m = x.max(axis=1, keepdims=True)
+    z = np.exp(x - m).sum(axis=1, keepdims=True)
+    prob = np.exp(np.take_along_axis(x, idx, axis=1) - m) / z
+    return idx.astype(np.int64), prob

@@ -445,3 +445,23 @@ def test_compaction_equals_causal_cache(tiny):
         k_ref, v_ref = (t.numpy() for t in cache[l])
         np.testing.assert_allclose(kv.K[l][:, :kv.P], k_ref, rtol=1e-9, atol=1e-10)
         np.testing.assert_allclose(kv.V[l][:, :kv.P], v_ref, rtol=1e-9, atol=1e-10)
+
+
+# ------------------------------------------------------------------------------------------------
+# top-K candidates (tree expansion, Sec. 4.2)
+# ------------------------------------------------------------------------------------------------
+def test_topk_softmax_against_brute_force_and_torch():
+    rng = np.random.default_rng(3)
+    x = rng.normal(0, 3, (5, 40))
+    x[2, 7] = x[2, 3] = x[2].max() + 1.0  # an exact tie at the top: the lower id first
+    idx, prob = oracle.topk_softmax(x, 4)
+    for r in range(5):
+        order = sorted(range(40), key=lambda j: (-x[r, j], j))[:4]
+        assert list(idx[r]) == order
+    assert list(idx[2][:2]) == [3, 7]
+    ref = torch.softmax(torch.tensor(x), dim=1).numpy()
+    assert np.allclose(prob, np.take_along_axis(ref, idx, axis=1), rtol=1e-12, atol=0)
+    # k larger than the row: every token, in order
+    idx2, prob2 = oracle.topk_softmax(x[:, :3], 8)
+    assert idx2.shape == (5, 3) and np.allclose(prob2.sum(axis=1), 1.0)
+
