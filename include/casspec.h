@@ -379,6 +379,14 @@ CASSPEC_API int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t
 CASSPEC_API int casspec_pld_draft(const int32_t* tokens, int L, int n_min, int n_max, int k, int32_t* out,
                                   void* cuda_stream);
 
+/* K-best candidates per row (Sec. 4.2, Algorithm 1: the top-K tokens of each drafted position; their
+ * normalised probabilities rank the sibling candidates).  logits dev fp32 [n][V] (e.g. a tree step's
+ * logits_out); for each row, idx_out (dev int32 [n][K]) receives the K largest logits' token ids in
+ * descending order (lower id first on ties; -1 past V) and prob_out (dev fp32 [n][K]) their softmax
+ * probabilities over the whole row.  1 <= K <= 8.  One kernel on cuda_stream.  Errors: E_INVAL, E_CUDA. */
+CASSPEC_API int casspec_topk(const float* logits, int n, int V, int K, int32_t* idx_out, float* prob_out,
+                             void* cuda_stream);
+
 /* A draft configuration: a DSIA draft of the model (Sec. 4.1), with its layer mask and GEMM mode as
  * for casspec_tree_step (skip_mask host uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16,
  * 1 W8A8), or, when pld_n_max > 0, the prompt-lookup bottom draft (casspec_pld_draft with n in

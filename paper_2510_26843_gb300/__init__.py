@@ -33,7 +33,7 @@ EXPORTS = [
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
     "casspec_dytc_destroy", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft", "casspec_topk",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -92,6 +92,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
         "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
+        "casspec_topk": (_I, [_P, _I, _I, _I, _P, _P, _P]),
         "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
                                      ctypes.POINTER(_D), ctypes.POINTER(_D)]),
         "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, _I, _P,
@@ -338,6 +339,12 @@ def pld_draft(tokens, L: int, n_min: int, n_max: int, k: int, out, stream=None) 
     """casspec_pld_draft: tokens dev int32 [L], out dev int32 [2 + k] = {match length, count, tokens}."""
     _check("casspec_pld_draft", load_library().casspec_pld_draft(_ptr(tokens), L, n_min, n_max, k, _ptr(out),
                                                                    _stream(stream)))
+
+
+def topk(logits, n: int, V: int, K: int, idx_out, prob_out, stream=None) -> None:
+    """casspec_topk: logits dev fp32 [n][V] -> idx_out dev int32 [n][K], prob_out dev fp32 [n][K]."""
+    _check("casspec_topk", load_library().casspec_topk(_ptr(logits), n, V, K, _ptr(idx_out), _ptr(prob_out),
+                                                         _stream(stream)))
 
 
 def latency_fit(x, y, mu0, sd0, noise_sd: float) -> tuple[list[float], list[float]]:
