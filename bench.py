@@ -331,6 +331,25 @@ def run_reference(args) -> None:
 # ------------------------------------------------------------------------------------------------
 # the GPU arm
 # ------------------------------------------------------------------------------------------------
+def max_over_ranks(value: float) -> float:
+    """The largest value over the ranks of the default process group (the value itself without one).
+    Replicas time the same step independently; the job's step time is the slowest replica's."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return value
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(n_tree: int, step_us: float, world: int) -> float:
+    """Whole-job tree tokens per second: every replica verifies n_tree tokens per step."""
+    return n_tree / (step_us * 1e-6) * world
+
+
 def run_gpu(args) -> None:
     import torch
     import torch.distributed as dist
@@ -413,10 +432,7 @@ def run_gpu(args) -> None:
     launches = cs.launch_count(dm.h) - n0
     clk = clocks.stop()
     ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms)
     us = ms * 1e3
 
     # ---- end to end through the C ABI with host buffers ----
@@ -486,7 +502,7 @@ def run_gpu(args) -> None:
         "step_roofline": {"algorithmic_bytes": ab["total"],
                           "pct_of_8TBps": round(100 * ab["total"] / (us * 1e-6) / 8e12, 2),
                           "frac_of_hbm_peak": round(ab["total"] / (us * 1e-6) / 1e9 / peak, 4),
-                          "tokens_per_s": round(n / (us * 1e-6) * world, 1)},
+                          "tokens_per_s": round(job_tokens_per_s(n, us, world), 1)},
         "roofline": {"kernel": f"{kern}, {args.workload}", "bound": "hbm", "achieved": round(achieved, 1),
                      "peak": peak, "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback", "unit": "GB/s", "frac": round(achieved / peak, 4),
