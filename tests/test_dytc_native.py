@@ -144,3 +144,31 @@ def test_latency_fit_matches_oracle(cs):
     with pytest.raises(cs.CasspecError):
         cs.latency_fit([1.0], [2.0], [0.0, 0.0], [0.0, 1.0], 1.0)  # zero prior spread
 
+
+
+@pytest.mark.parametrize("alphas,costs,a_dn,c_dn,k_max,t_min,m_max", [
+    ([0.8], [0.3], 0.5, 0.05, 4, 1.0, 1),       # a one-node tree: nothing to expand
+    ([0.8, 0.6], [0.3, 0.2], 0.5, 0.0, 3, 1e9, 20),  # a free bottom draft: only the size limit stops
+    ([1.0, 0.5], [0.4, 0.1], 0.5, 0.05, 5, 1.0, 64),  # a draft that is always accepted (E_acc = k)
+    ([0.9], [0.3], 0.5, 0.05, 1, 0.0, 64),      # k_max = 1: one token per expansion
+    ([0.0, 0.0], [0.3, 0.3], 0.0, 0.05, 4, 0.0, 16),  # no positive objective: the root is closed
+])
+def test_draft_tree_edge_cases_match_oracle(cs, alphas, costs, a_dn, c_dn, k_max, t_min, m_max):
+    want = D.draft_tree(alphas, costs, a_dn, c_dn, k_max, t_min, m_max, _fake_draft)
+    sch = cs.Dytc(alphas, costs, a_dn, c_dn, k_max, t_min, m_max)
+    sch.tree_reset()
+    while True:
+        plan = sch.tree_plan()
+        if plan is None:
+            break
+        leaf, s, k = plan
+        tr = sch.tree_get()
+        path, v = [], leaf
+        while v >= 0:
+            path.append(v)
+            v = tr["parent"][v]
+        sch.tree_extend(leaf, s, _fake_draft(s, path[::-1], k))
+    got = sch.tree_get()
+    assert got["parent"] == want["parent"] and got["cfg"] == want["cfg"]
+    assert got["p_acc"] == pytest.approx(want["p_acc"], rel=1e-12)
+    sch.close()
