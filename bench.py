@@ -44,6 +44,8 @@ WORKLOADS = {
     "layer7b": (1, 1024, 32, 6, 4, 0.0, 0, True),
     # two layers at the verify sizes (prefix 2048, 64 nodes): a small case for kernel profiles
     "attn7b": (2, 2048, 64, 8, None, 0.0, 0, True),
+    # two W8A8 draft layers (prefix 2048, 8 nodes): a small case for profiling the int8 projections
+    "w8a8layer7b": (2, 2048, 8, 8, None, 0.0, 1, False),
     "verify13b": (40, 4096, 64, 8, None, 0.0, 0, True),
     # one cascade round: the 60%-skip W8A8 draft appends the tree level by level, the 40%-skip bf16
     # draft re-checks all 64 nodes, then the full verify, acceptance and compaction
