@@ -11,7 +11,9 @@ What it computes (CAS-Spec, arXiv 2510.26843):
     verification of different branches"; "tree-based parallel draft generation"), run by the target
     model and by its DSIA drafts (Sec. 4.1, Def. 4.1);
   * DSIA layer sparsity (Sec. 4.1, "skipping a subset of transformer layers"): a switched-off
-    layer is the identity on the residual stream and writes no K/V;
+    layer is the identity on the residual stream and writes no K/V; the same at the granularity of
+    a layer's attention or FFN sub-block (Sec. 4.1 names both granularities): a skipped attention
+    block adds nothing to the residual stream and writes no K/V, a skipped FFN block adds nothing;
   * DSIA activation quantisation (Sec. 4.1 and App. C, QSpec-style W?A? drafts): here W8A8, per
     output channel symmetric int8 weights and per-token dynamic symmetric int8 activations on the
     inputs of Wqkv, Wo, Wgate/Wup and Wdown; attention, K/V and the LM head stay in floating point;
@@ -290,13 +292,28 @@ def tree_attention(q: np.ndarray, kv: KVCache, layer: int, slots: list, anc: lis
     return out
 
 
+SKIP_ATTN = 0x2  # skip-mask flag: the layer's attention block is skipped
+SKIP_FFN = 0x4  # skip-mask flag: the layer's FFN block is skipped
+
+
+def layer_blocks(code: int) -> tuple[bool, bool]:
+    """(attention on, FFN on) for one skip-mask byte: 0 switches the whole layer off; otherwise
+    each sub-block runs unless its flag is set."""
+    code = int(code)
+    if code == 0:
+        return False, False
+    return not code & SKIP_ATTN, not code & SKIP_FFN
+
+
 def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
               skip_mask: np.ndarray | None = None, quant_mode: int = 0,
               trace: dict | None = None, attn_bf16: bool = False) -> np.ndarray:
     """One draft/verify pass over n new tree nodes; returns logits [n, V] (fp64).
 
     The nodes occupy tree slots T .. T+n-1 (cache slots P+T .. P+T+n-1); each active layer writes
-    their K/V there.  skip_mask[l] == 0 switches layer l off (Sec. 4.1 layer sparsity).
+    their K/V there.  skip_mask[l] == 0 switches layer l off (Sec. 4.1 layer sparsity); a non-zero
+    byte keeps it on except for the sub-blocks whose flag it carries: SKIP_ATTN (the attention
+    block: no residual update, no K/V written) and SKIP_FFN (the FFN block).
     quant_mode 1 runs the W8A8 draft (App. C).  `trace`, if given, receives per-layer intermediates.
     attn_bf16 rounds q and the K/V written to the cache to bf16 (a bf16 cache and bf16 attention
     operands).  It is a perturbation of the size of bf16 storage, used by tests to measure how far
@@ -306,7 +323,6 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
     tokens = np.asarray(tokens, dtype=np.int64)
     parent = np.asarray(parent, dtype=np.int64)
     n = len(tokens)
-    d, H, h = sh.d_model, sh.n_heads, sh.head_dim
     if kv.P + kv.T + n > kv.capacity:
         raise ValueError("KV capacity exceeded")
     depth, anc = tree_topology(parent, kv.T, kv.depth, kv.anc)
@@ -318,33 +334,44 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
 
     x = w.f64("embed")[tokens]  # [n, d]
     for l in range(sh.n_layers):
-        if not mask[l]:
-            continue
-        xn = rmsnorm(x, w.gain("attn_norm", l), sh.rms_eps)
-        qkv = _linear(xn, w, "wqkv", l, quant)
-        q = rope(qkv[:, :d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
-        k = rope(qkv[:, d:2 * d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
-        v = qkv[:, 2 * d:].reshape(n, H, h)
-        if attn_bf16:
-            q, k, v = round_bf16(q), round_bf16(k), round_bf16(v)
-        for i, s in enumerate(slots):
-            kv.K[l][:, s] = k[i]
-            kv.V[l][:, s] = v[i]
-            kv.valid[l][s] = True
-        o = tree_attention(q, kv, l, slots, [all_anc[kv.T + i] for i in range(n)]).reshape(n, d)
-        x = x + _linear(o, w, "wo", l, quant)
-        xn2 = rmsnorm(x, w.gain("ffn_norm", l), sh.rms_eps)
-        g = _linear(xn2, w, "wg", l, quant)
-        u = _linear(xn2, w, "wu", l, quant)
-        x = x + _linear(silu(g) * u, w, "wd", l, quant)
-        if trace is not None:
-            trace[l] = {"xn": xn, "q": q, "k": k, "v": v, "o": o, "x": x.copy()}
+        attn_on, ffn_on = layer_blocks(mask[l])
+        if attn_on:
+            x = _attention_block(x, w, kv, l, quant, pos, slots, all_anc, n, attn_bf16, trace)
+        if ffn_on:
+            xn2 = rmsnorm(x, w.gain("ffn_norm", l), sh.rms_eps)
+            g = _linear(xn2, w, "wg", l, quant)
+            u = _linear(xn2, w, "wu", l, quant)
+            x = x + _linear(silu(g) * u, w, "wd", l, quant)
+        if trace is not None and (attn_on or ffn_on):
+            trace.setdefault(l, {})["x"] = x.copy()
     xf = rmsnorm(x, w.gain("final_norm"), sh.rms_eps)
     logits = xf @ w.f64("lm_head").T
     kv.depth = kv.depth + depth
     kv.anc = kv.anc + anc
     kv.T += n
     return logits
+
+
+def _attention_block(x, w, kv, l, quant, pos, slots, all_anc, n, attn_bf16, trace):
+    """x + Wo . TreeAttention(RoPE(Wq xn), RoPE(Wk xn), Wv xn) with xn = RMSNorm(x); writes the
+    nodes' K/V of layer l."""
+    sh = w.shape
+    d, H, h = sh.d_model, sh.n_heads, sh.head_dim
+    xn = rmsnorm(x, w.gain("attn_norm", l), sh.rms_eps)
+    qkv = _linear(xn, w, "wqkv", l, quant)
+    q = rope(qkv[:, :d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
+    k = rope(qkv[:, d:2 * d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
+    v = qkv[:, 2 * d:].reshape(n, H, h)
+    if attn_bf16:
+        q, k, v = round_bf16(q), round_bf16(k), round_bf16(v)
+    for i, s in enumerate(slots):
+        kv.K[l][:, s] = k[i]
+        kv.V[l][:, s] = v[i]
+        kv.valid[l][s] = True
+    o = tree_attention(q, kv, l, slots, [all_anc[kv.T + i] for i in range(n)]).reshape(n, d)
+    if trace is not None:
+        trace[l] = {"xn": xn, "q": q, "k": k, "v": v, "o": o}
+    return x + _linear(o, w, "wo", l, quant)
 
 
 # ----------------------------------------------------------------------------------------------

@@ -317,6 +317,80 @@ def test_skip_one_layer_equals_model_without_it(tiny):
                                   oracle.tree_step(w, kv2, toks, parent))
 
 
+def _gains(name, layer):
+    """Distinct seeded RMSNorm gains per (norm, layer)."""
+    kind = {"attn_norm": 1, "ffn_norm": 2, "final_norm": 3}[name]
+    return np.random.default_rng(100 * max(layer, 0) + kind).uniform(0.5, 1.5, SH.d_model)
+
+
+def _weights_with(zero: tuple | None = None):
+    """Tiny weights with the gains above, optionally with one matrix (name, layer) zeroed."""
+    def get(name, layer):
+        bits = synth.weight_bf16(SEED, SH, name, layer)
+        return np.zeros_like(bits) if zero == (name, layer) else bits
+
+    return oracle.Weights(SH, get, _gains, keep_layers=SH.n_layers)
+
+
+@pytest.mark.parametrize("mask,blocks", [
+    ([1, 1], [(True, True), (True, True)]),
+    ([1 | 2, 1], [(False, True), (True, True)]),  # layer 0 without attention
+    ([1, 1 | 4], [(True, True), (True, False)]),  # layer 1 without FFN
+    ([1 | 4, 1 | 2], [(True, False), (False, True)]),
+])
+def test_gains_and_sub_blocks_match_causal_forward(tiny, mask, blocks):
+    """Chain prefill with non-unit gains (each norm its own) and sub-block masks against the
+    textbook causal forward given the same gains and sub-block switches: the RMSNorm of each block
+    uses that block's gains and a skipped block is dropped from the residual stream."""
+    _, _, prefix = tiny
+    ref = CausalLM(SH, SEED, gains=_gains)
+    kv = oracle.KVCache(SH.n_layers, SH.n_heads, SH.head_dim, 128)
+    got = oracle.tree_step(_weights_with(), kv, prefix[:40], synth.chain(40), skip_mask=np.array(mask, np.uint8))
+    want = ref.forward(prefix[:40], blocks=blocks)
+    assert np.max(np.abs(got - want) / np.ptp(want, axis=1, keepdims=True)) < 1e-10
+
+
+@pytest.mark.parametrize("layer", [0, 1])
+@pytest.mark.parametrize("block", ["attn", "ffn"])
+def test_skipped_sub_block_equals_zeroed_output_matrix(tiny, layer, block):
+    """Skipping a layer's attention (FFN) block gives exactly the model whose output projection Wo
+    (down projection Wd) of that layer is zero: the block adds nothing to the residual stream.  The
+    gains differ per norm, so running the other block with the wrong norm would show.  A skipped
+    attention block writes no K/V in that layer."""
+    _, _, prefix = tiny
+    flag, name = (oracle.SKIP_ATTN, "wo") if block == "attn" else (oracle.SKIP_FFN, "wd")
+    mask = np.ones(SH.n_layers, np.uint8)
+    mask[layer] |= flag
+    w_skip, w_zero = _weights_with(), _weights_with((name, layer))
+    kv_s, pre_s = _prefilled(w_skip, prefix, mask=mask)
+    kv_z, pre_z = _prefilled(w_zero, prefix)
+    np.testing.assert_array_equal(pre_s, pre_z)
+    toks, parent = synth.tokens(21, 8, SH.vocab), synth.tree(21, 8, 4)
+    got = oracle.tree_step(w_skip, kv_s, toks, parent, skip_mask=mask)
+    want = oracle.tree_step(w_zero, kv_z, toks, parent)
+    np.testing.assert_array_equal(got, want)
+    P = len(prefix)
+    for l in range(SH.n_layers):
+        written = bool(kv_s.valid[l][P:P + 8].all())
+        assert written == (l != layer or block == "ffn")
+        assert not kv_s.valid[l][P:P + 8].any() or written
+    # and the skipped block changes the result (the pin is not vacuous)
+    kv_f, _ = _prefilled(w_skip, prefix)
+    assert np.max(np.abs(oracle.tree_step(w_skip, kv_f, toks, parent) - got)) > 1e-3
+
+
+def test_both_sub_blocks_skipped_is_the_layer_off(tiny):
+    w, _, prefix = tiny
+    toks, parent = synth.tokens(22, 6, SH.vocab), synth.tree(22, 6, 3)
+    both = np.array([1 | oracle.SKIP_ATTN | oracle.SKIP_FFN, 1], np.uint8)
+    off = np.array([0, 1], np.uint8)
+    kv1, _ = _prefilled(w, prefix, mask=off)
+    kv2, _ = _prefilled(w, prefix, mask=off)
+    np.testing.assert_array_equal(oracle.tree_step(w, kv1, toks, parent, skip_mask=both),
+                                  oracle.tree_step(w, kv2, toks, parent, skip_mask=off))
+    assert oracle.layer_blocks(1) == (True, True) and oracle.layer_blocks(0) == (False, False)
+
+
 def test_int8_mode_close_to_bf16_mode(tiny):
     """W8A8 draft logits stay within the quantisation error of the full-precision model."""
     w, ref, prefix = tiny

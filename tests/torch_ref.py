@@ -16,8 +16,13 @@ import synth
 
 
 class CausalLM:
-    def __init__(self, shape: synth.ModelShape, seed: int):
+    def __init__(self, shape: synth.ModelShape, seed: int, gains=None):
+        """gains(name, layer) -> [d] RMSNorm gains ("attn_norm", "ffn_norm", "final_norm"); ones
+        if None."""
         self.sh = shape
+        one = lambda name, layer: np.ones(shape.d_model)  # noqa: E731
+        self.gain = lambda name, layer=-1: torch.as_tensor(  # noqa: E731
+            np.asarray((gains or one)(name, layer), dtype=np.float64))
         get = lambda name, layer=0: torch.from_numpy(  # noqa: E731
             synth.bf16_to_f32(synth.weight_bf16(seed, shape, name, layer)).astype(np.float64))
         self.embed = get("embed")
@@ -38,29 +43,39 @@ class CausalLM:
         z = torch.complex(x[..., :half], x[..., half:]) * rot
         return torch.cat([z.real, z.imag], dim=-1)
 
-    def forward(self, tokens, layers_on=None, return_kv: bool = False):
-        """Logits [S, V] of a causal forward over `tokens` (positions 0..S-1)."""
+    def forward(self, tokens, layers_on=None, return_kv: bool = False, blocks=None):
+        """Logits [S, V] of a causal forward over `tokens` (positions 0..S-1).  layers_on[l] false
+        drops layer l; blocks[l] = (attention on, FFN on) drops single sub-blocks."""
         sh = self.sh
-        d, H, h = sh.d_model, sh.n_heads, sh.head_dim
+        d = sh.d_model
         toks = torch.as_tensor(np.asarray(tokens), dtype=torch.long)
         S = len(toks)
         pos = torch.arange(S)
         x = self.embed[toks]
-        ones = torch.ones(d, dtype=torch.float64)
         kv = []
         for l, W in enumerate(self.layers):
+            attn, ffn = (True, True) if blocks is None else blocks[l]
             if layers_on is not None and not layers_on[l]:
+                attn = ffn = False
+            if not attn:
                 kv.append(None)
-                continue
-            xn = F.rms_norm(x, (d,), ones, sh.rms_eps)
-            q = F.linear(xn, W["wq"]).view(S, H, h).transpose(0, 1)
-            k = F.linear(xn, W["wk"]).view(S, H, h).transpose(0, 1)
-            v = F.linear(xn, W["wv"]).view(S, H, h).transpose(0, 1)
-            q, k = self._rope(q, pos), self._rope(k, pos)
-            kv.append((k, v))
-            a = F.scaled_dot_product_attention(q[None], k[None], v[None], is_causal=True)[0]
-            x = x + F.linear(a.transpose(0, 1).reshape(S, d), W["wo"])
-            xn = F.rms_norm(x, (d,), ones, sh.rms_eps)
-            x = x + F.linear(F.silu(F.linear(xn, W["wg"])) * F.linear(xn, W["wu"]), W["wd"])
-        logits = F.linear(F.rms_norm(x, (d,), ones, sh.rms_eps), self.lm_head)
+            if attn:
+                x = self._attention(x, W, l, pos, kv)
+            if ffn:
+                xn = F.rms_norm(x, (d,), self.gain("ffn_norm", l), sh.rms_eps)
+                x = x + F.linear(F.silu(F.linear(xn, W["wg"])) * F.linear(xn, W["wu"]), W["wd"])
+        logits = F.linear(F.rms_norm(x, (d,), self.gain("final_norm"), sh.rms_eps), self.lm_head)
         return (logits.numpy(), kv) if return_kv else logits.numpy()
+
+    def _attention(self, x, W, l, pos, kv):
+        sh = self.sh
+        d, H, h = sh.d_model, sh.n_heads, sh.head_dim
+        S = x.shape[0]
+        xn = F.rms_norm(x, (d,), self.gain("attn_norm", l), sh.rms_eps)
+        q = F.linear(xn, W["wq"]).view(S, H, h).transpose(0, 1)
+        k = F.linear(xn, W["wk"]).view(S, H, h).transpose(0, 1)
+        v = F.linear(xn, W["wv"]).view(S, H, h).transpose(0, 1)
+        q, k = self._rope(q, pos), self._rope(k, pos)
+        kv.append((k, v))
+        a = F.scaled_dot_product_attention(q[None], k[None], v[None], is_causal=True)[0]
+        return x + F.linear(a.transpose(0, 1).reshape(S, d), W["wo"])
