@@ -38,6 +38,8 @@ extern "C" {
 #define CASSPEC_API __attribute__((visibility("default")))
 
 #define CASSPEC_MAX_TREE 64 /* tree slots per round; also the largest n of one call */
+#define CASSPEC_SKIP_ATTN 0x2u /* skip-mask flag: the layer's attention block is skipped */
+#define CASSPEC_SKIP_FFN 0x4u  /* skip-mask flag: the layer's FFN block is skipped */
 
 typedef enum casspec_status {
   CASSPEC_OK = 0,
@@ -176,9 +178,14 @@ CASSPEC_API int casspec_kv_length(casspec_kv* kv, int* P_out, int* T_out);
  *                               plus exactly its ancestors and itself.
  *   n           1 .. 64, T + n <= 64, P + T + n <= max_ctx
  *   skip_mask   host uint8 [n_layers] or NULL (all layers on); 0 switches layer l off: the layer
- *               is the identity on the residual stream and writes no K/V (layer-sparsity DSIA).
- *               Rule: every active layer must hold K/V for all T existing tree slots (nested
- *               masks, as in a layer-sparsity cascade); otherwise E_STATE.
+ *               is the identity on the residual stream and writes no K/V (layer-sparsity DSIA,
+ *               Sec. 4.1).  A non-zero byte keeps the layer on except for the sub-blocks whose
+ *               flag it carries (Sec. 4.1 also names attention / FFN sub-blocks as the unit):
+ *               CASSPEC_SKIP_ATTN drops the attention block (no residual update, no K/V
+ *               written), CASSPEC_SKIP_FFN the FFN block; both flags equal 0.  Other bits are
+ *               ignored.
+ *               Rule: every layer whose attention runs must hold K/V for all T existing tree
+ *               slots (nested masks, as in a layer-sparsity cascade); otherwise E_STATE.
  *   quant_mode  0: bf16 weights, fp32 accumulation.  1: W8A8 GEMMs for WQKV, WO, WG/WU, WD with
  *               per-token dynamic int8 activations (activation-quantisation DSIA); attention, K/V
  *               and the LM head stay bf16.  Mode 1 needs casspec_quantize_weights first.

@@ -17,6 +17,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libcasspec.so")
 
 OK, E_INVAL, E_SHAPE, E_CAPACITY, E_CUDA, E_TREE, E_TIMEOUT, E_STATE = 0, -1, -2, -3, -4, -5, -6, -7
 MAX_TREE = 64
+SKIP_ATTN, SKIP_FFN = 0x2, 0x4  # skip-mask flags on a non-zero byte: drop the attention / FFN block
 OPT_PDL, OPT_GRAPHS = 1, 2
 
 (T_EMBED, T_LM_HEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WG, T_WU, T_WD,

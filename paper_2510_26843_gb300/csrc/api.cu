@@ -268,6 +268,17 @@ cudaEvent_t prof_begin(casspec_model* m, int kind, cudaStream_t s) {
 //   layer] -> for each active layer: attention, chain[Wo, Wgate/Wup, Wdown, next layer's QKV or the
 //   LM head] -> argmax merge.  RMSNorm is folded into the chain phases that consume it.
 //   int8 mode: per-projection W8A8 kernels with RMSNorm / quantisation kernels, then chain[LM head].
+// Sub-blocks of a layer that a step runs (from a skip-mask byte).
+constexpr uint8_t kBlockAttn = 1, kBlockFfn = 2;
+uint8_t layer_blocks(uint8_t code) {
+  if (code == 0) return 0;
+  return (uint8_t)(((code & CASSPEC_SKIP_ATTN) ? 0 : kBlockAttn) | ((code & CASSPEC_SKIP_FFN) ? 0 : kBlockFfn));
+}
+enum { IT_QKV, IT_ATTN, IT_WO, IT_GU, IT_DOWN, IT_LM };
+struct StepItem {
+  int kind, l;
+};
+
 int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent, int n,
                  const std::vector<uint8_t>& on, int mode, float* logits, cudaStream_t s, bool prof, int& count) {
   const auto& c = m->cfg;
@@ -278,11 +289,31 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   std::vector<int> act;
   for (int l = 0; l < c.n_layers; ++l)
     if (on[l]) act.push_back(l);
+  // The step as a list of projections and attentions: per active layer QKV, attention and Wo when
+  // its attention block is on, gate/up and down when its FFN block is on; the LM head last.
+  // Every residual projection (Wo, down) is followed by a projection that reads x.
+  std::vector<StepItem> items;
+  for (int l : act) {
+    if (on[l] & kBlockAttn) {
+      items.push_back({IT_QKV, l});
+      items.push_back({IT_ATTN, l});
+      items.push_back({IT_WO, l});
+    }
+    if (on[l] & kBlockFfn) {
+      items.push_back({IT_GU, l});
+      items.push_back({IT_DOWN, l});
+    }
+  }
+  items.push_back({IT_LM, -1});
+  // gains of the RMSNorm that a projection reading x applies
+  auto reader_gain = [&](const StepItem& it) -> const float* {
+    return it.kind == IT_QKV ? m->layers[it.l].attn_norm : it.kind == IT_GU ? m->layers[it.l].ffn_norm : m->final_norm;
+  };
 
   LAUNCH(CASSPEC_K_OTHER, launch_tree_prep(parent, n, T, kv->dP, kv->tdepth, kv->tanc, m->pos, m->anc, m->status, s,
                                            pdl));
   // the first projection that reads x normalises it with these gains (null: an int8 layer does)
-  const float* g_first = act.empty() ? m->final_norm : (mode == 0 ? m->layers[act[0]].attn_norm : nullptr);
+  const float* g_first = (mode == 0 || act.empty()) ? reader_gain(items[0]) : nullptr;
   LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, g_first, m->x, m->ssp, m->xa, s, pdl));
   const int bi = BN / 16 - 1;  // tensor maps of the split activations for this BN
 
@@ -329,14 +360,14 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.xa_out = m->xa;
     p.ep.g_next = g_next;
   };
-  auto ph_gu = [&](PhaseDesc& p) {
+  auto ph_gu = [&](int ss_tiles, PhaseDesc& p) {
     p = PhaseDesc{};
     p.epi = EPI_GLU;
     p.tiles = cdiv(F, 64);
     p.kblocks = cdiv(d, 64);
     p.K = d;
     p.ss = m->ssp;
-    p.ss_tiles = d / 128;
+    p.ss_tiles = ss_tiles;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = F;
@@ -392,40 +423,62 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   };
 
   if (mode == 0) {
+    // Consecutive projections share one chain launch (up to kMaxPhases phases); every attention
+    // ends the current chain.  With all blocks on this gives [QKV], then [Wo, gate/up, down,
+    // next QKV or LM head] after each attention.
     ChainArgs ca = {};
     ChainMaps cm = {};
+    int nph = 0, nchains = 0;
+    auto flush = [&]() -> int {
+      if (nph == 0) return CASSPEC_OK;
+      ca.nphases = nph;
+      const int kind = (nph == 1 && ca.ph[0].epi == EPI_LMHEAD) ? CASSPEC_K_LMHEAD
+                       : (nchains == 0 && ca.ph[0].epi == EPI_QKV) ? CASSPEC_K_QKV
+                                                                   : CASSPEC_K_GATEUP;
+      const int rc = chain(ca, cm, kind);
+      ca = ChainArgs{};
+      cm = ChainMaps{};
+      nph = 0;
+      ++nchains;
+      return rc;
+    };
     int rc;
-    ca.nphases = 1;
-    if (act.empty()) {
-      ph_lm(1, ca.ph[0], cm.w[0], cm.x[0]);
-      if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
-    } else {
-      ph_qkv(act[0], 1, ca.ph[0], cm.w[0], cm.x[0]);
-      if ((rc = chain(ca, cm, CASSPEC_K_QKV)) != CASSPEC_OK) return rc;
-      for (size_t i = 0; i < act.size(); ++i) {
-        const int l = act[i];
-        const bool last = i + 1 == act.size();
-        if ((rc = attention(l)) != CASSPEC_OK) return rc;
-        ChainArgs cb = {};
-        ChainMaps cn = {};
-        cb.nphases = 4;
-        ph_resid(d, m->layers[l].ffn_norm, cb.ph[0]);
-        cn.w[0] = m->layers[l].tm_o;
-        cn.x[0] = m->tm_o[bi];
-        ph_gu(cb.ph[1]);
-        cn.w[1] = m->layers[l].tm_g;
-        cn.w2[1] = m->layers[l].tm_u;
-        cn.x[1] = m->tm_xa[bi];
-        ph_resid(F, last ? m->final_norm : m->layers[act[i + 1]].attn_norm, cb.ph[2]);
-        cn.w[2] = m->layers[l].tm_d;
-        cn.x[2] = m->tm_u[bi];
-        if (!last)
-          ph_qkv(act[i + 1], d / 128, cb.ph[3], cn.w[3], cn.x[3]);
-        else
-          ph_lm(d / 128, cb.ph[3], cn.w[3], cn.x[3]);
-        if ((rc = chain(cb, cn, CASSPEC_K_GATEUP)) != CASSPEC_OK) return rc;
+    for (size_t i = 0; i < items.size(); ++i) {
+      const StepItem& it = items[i];
+      if (it.kind == IT_ATTN) {
+        if ((rc = flush()) != CASSPEC_OK || (rc = attention(it.l)) != CASSPEC_OK) return rc;
+        continue;
       }
+      if (nph == kMaxPhases && (rc = flush()) != CASSPEC_OK) return rc;
+      const int ss_tiles = i == 0 ? 1 : d / 128;  // the embedding leaves one partial, a residual d/128
+      PhaseDesc& p = ca.ph[nph];
+      switch (it.kind) {
+        case IT_QKV:
+          ph_qkv(it.l, ss_tiles, p, cm.w[nph], cm.x[nph]);
+          break;
+        case IT_WO:
+          ph_resid(d, reader_gain(items[i + 1]), p);
+          cm.w[nph] = m->layers[it.l].tm_o;
+          cm.x[nph] = m->tm_o[bi];
+          break;
+        case IT_GU:
+          ph_gu(ss_tiles, p);
+          cm.w[nph] = m->layers[it.l].tm_g;
+          cm.w2[nph] = m->layers[it.l].tm_u;
+          cm.x[nph] = m->tm_xa[bi];
+          break;
+        case IT_DOWN:
+          ph_resid(F, reader_gain(items[i + 1]), p);
+          cm.w[nph] = m->layers[it.l].tm_d;
+          cm.x[nph] = m->tm_u[bi];
+          break;
+        default:
+          ph_lm(ss_tiles, p, cm.w[nph], cm.x[nph]);
+          break;
+      }
+      ++nph;
     }
+    if ((rc = flush()) != CASSPEC_OK) return rc;
   } else {
     auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
                      int epi, const EpiParams& e) -> cudaError_t {
@@ -446,45 +499,55 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       g8.ep = e;
       return launch_gemm_i8(g8, BN, epi, s, pdl);
     };
-    for (size_t i = 0; i < act.size(); ++i) {
-      const int l = act[i];
-      LayerPtrs& Lp = m->layers[l];
-      LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
-      EpiParams e = base;
-      e.N = 3 * d;
-      e.q_out = m->q;
-      e.kc = kv_layer_k(kv, l);
-      e.vc = kv_layer_v(kv, l);
-      LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+    EpiParams er = base;  // residual projections
+    er.N = d;
+    er.y = m->x;
+    er.ldy = d;
+    for (size_t i = 0; i < items.size(); ++i) {
+      const StepItem& it = items[i];
       int rc;
-      if ((rc = attention(l)) != CASSPEC_OK) return rc;
-      EpiParams er = base;
-      er.N = d;
-      er.y = m->x;
-      er.ldy = d;
-      // W8A8 activations are the bf16 values: the hi plane of the split output
-      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
-      LAUNCH(CASSPEC_K_WO, gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, er));
-      LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
-      EpiParams eg = base;
-      eg.N = F;
-      eg.u_out = m->u;
-      LAUNCH(CASSPEC_K_GATEUP, gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
-      LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
+      if (it.kind == IT_LM) {
+        ChainArgs ca = {};
+        ChainMaps cm = {};
+        ca.nphases = 1;
+        ph_lm(i == 0 ? 1 : d / 128, ca.ph[0], cm.w[0], cm.x[0]);
+        if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
+        continue;
+      }
+      if (it.kind == IT_ATTN) {
+        if ((rc = attention(it.l)) != CASSPEC_OK) return rc;
+        continue;
+      }
+      LayerPtrs& Lp = m->layers[it.l];
       EpiParams ed = er;
-      if (i + 1 == act.size()) {  // the LM head's RMSNorm scale and operand
-        ed.ss_out = m->ssp;
+      if ((it.kind == IT_WO || it.kind == IT_DOWN) && items[i + 1].kind == IT_LM) {
+        ed.ss_out = m->ssp;  // the last residual projection leaves the LM head's RMSNorm inputs
         ed.xa_out = m->xa;
         ed.g_next = m->final_norm;
       }
-      LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
+      if (it.kind == IT_QKV) {
+        LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
+        EpiParams e = base;
+        e.N = 3 * d;
+        e.q_out = m->q;
+        e.kc = kv_layer_k(kv, it.l);
+        e.vc = kv_layer_v(kv, it.l);
+        LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+      } else if (it.kind == IT_WO) {
+        // W8A8 activations are the bf16 values: the hi plane of the split output
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
+        LAUNCH(CASSPEC_K_WO, gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
+      } else if (it.kind == IT_GU) {
+        LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
+        EpiParams eg = base;
+        eg.N = F;
+        eg.u_out = m->u;
+        LAUNCH(CASSPEC_K_GATEUP, gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
+      } else {
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
+        LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
+      }
     }
-    ChainArgs ca = {};
-    ChainMaps cm = {};
-    ca.nphases = 1;
-    ph_lm(act.empty() ? 1 : d / 128, ca.ph[0], cm.w[0], cm.x[0]);
-    int rc;
-    if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
   }
   LAUNCH(CASSPEC_K_OTHER, launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, m->lay.lm_tiles, n, m->am, m->margin, s, pdl));
   return CASSPEC_OK;
@@ -791,11 +854,11 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
   if (n < 1 || n > kMaxTree) return CASSPEC_E_SHAPE;
   if (kv->T + n > kMaxTree || kv->P_upper + kv->T + n > kv->ctx) return CASSPEC_E_CAPACITY;
   const int NL = m->cfg.n_layers;
-  std::vector<uint8_t> on(NL, 1);
+  std::vector<uint8_t> on(NL, kBlockAttn | kBlockFfn);
   if (skip_mask)
-    for (int l = 0; l < NL; ++l) on[l] = skip_mask[l] != 0;
-  for (int l = 0; l < NL; ++l)
-    if (on[l] && kv->layer_valid[l] != kv->T) return CASSPEC_E_STATE;
+    for (int l = 0; l < NL; ++l) on[l] = layer_blocks(skip_mask[l]);
+  for (int l = 0; l < NL; ++l)  // attention reads the K/V of the existing tree slots
+    if ((on[l] & kBlockAttn) && kv->layer_valid[l] != kv->T) return CASSPEC_E_STATE;
 
   std::lock_guard<std::mutex> lock(m->mu);
   int rc = CASSPEC_OK;
@@ -830,7 +893,7 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
   }
   const int Tn = kv->T + n;
   for (int l = 0; l < NL; ++l)
-    if (on[l]) kv->layer_valid[l] = Tn;
+    if (on[l] & kBlockAttn) kv->layer_valid[l] = Tn;
   kv->T = Tn;
   return CASSPEC_OK;
 }

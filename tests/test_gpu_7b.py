@@ -44,9 +44,10 @@ def rel_err(got, ref):
     return np.max(np.abs(got - ref) / np.ptp(ref, axis=1, keepdims=True), axis=1)
 
 
-def oracle_cache(shape, P, extra):
+def oracle_cache(shape, P, extra, layers=None):
+    """Oracle cache holding the stand-in prefix K/V of `layers` (default: all)."""
     okv = oracle.KVCache(shape.n_layers, shape.n_heads, shape.head_dim, P + extra)
-    for l in range(shape.n_layers):
+    for l in range(shape.n_layers) if layers is None else layers:
         k = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, shape, l, "k", P)).astype(np.float64)
         v = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, shape, l, "v", P)).astype(np.float64)
         okv.load_prefix(l, k, v)
@@ -211,4 +212,34 @@ def test_7b_int8_one_layer(cs, dm7, ow7):
     ref = oracle.tree_step(ow7, oracle_cache(SH7, P, n), toks, parent, skip_mask=mask, quant_mode=1)
     err = rel_err(got, ref)
     assert np.all(err < TOL_INT8), err.max()
+    kv.close()
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_7b_sub_block_skip(cs, dm7, ow7, mode):
+    """Attention / FFN sub-block skipping at the 7B shapes.  The mask (layer 0 attention only,
+    layers 1, 2 and 4 FFN only, layer 3 whole, the rest off) makes the projection chain run
+    [QKV], [Wo, gate/up, down, gate/up], [down, QKV], [Wo, gate/up, down, gate/up], [down, LM head]:
+    a chain that starts with a down projection, two chains in a row, and gate/up right after
+    another layer's down projection.  Tolerances as in test_7b_draft_steps."""
+    from paper_2510_26843_gb300.workload import DeviceKV
+
+    P, n = 2048, 8
+    kv = DeviceKV(dm7, P + 64)
+    kv.load_random_prefix(SEED, P)
+    parent = synth.tree(SEED + 3, n, 8)
+    toks = synth.tokens(SEED + 3, n, SH7.vocab)
+    mask = np.zeros(SH7.n_layers, dtype=np.uint8)
+    mask[:5] = [1 | cs.SKIP_FFN, 1 | cs.SKIP_ATTN, 1 | cs.SKIP_ATTN, 1, 1 | cs.SKIP_ATTN]
+    got, _, _ = gpu_step(cs, dm7, kv, toks, parent, SH7.vocab, mask=mask, mode=mode)
+    assert cs.get_status(dm7.h) == 0
+    attending = [0, 3]  # the layers whose attention runs read the prefix
+    ref = oracle.tree_step(ow7, oracle_cache(SH7, P, n, attending), toks, parent, skip_mask=mask, quant_mode=mode)
+    err = rel_err(got, ref)
+    if mode == 0:
+        assert np.all(err < TOL_BF16), err.max()
+    else:
+        pert = oracle.tree_step(ow7, oracle_cache(SH7, P, n, attending), toks, parent, skip_mask=mask,
+                                quant_mode=mode, attn_bf16=True)
+        assert err.max() <= max(TOL_INT8, 2.0 * rel_err(pert, ref).max()), err.max()
     kv.close()

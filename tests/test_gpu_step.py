@@ -187,6 +187,40 @@ def test_appended_draft_levels_and_skip_mask(cs, dev_model, ow, prefix):
     kv.close()
 
 
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("mask", [(1 | 2, 1), (1, 1 | 4), (1 | 4, 1 | 2), (1 | 2, 1 | 2), (1 | 2 | 4, 1 | 4)])
+def test_sub_block_skip(cs, dev_model, ow, prefix, mask, mode):
+    """Attention (flag 2) / FFN (flag 4) sub-block skipping against the oracle, in both GEMM modes;
+    (2, 2) runs no attention at all (gate/up, down, gate/up, down, LM head: two chains in a row)."""
+    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
+    parent = synth.tree(30, 8, 4)
+    toks = synth.tokens(30, 8, SH.vocab)
+    m = np.array(mask, np.uint8)
+    got = gpu_step(cs, dev_model, kv, toks, parent, mask=m, mode=mode)
+    assert cs.get_status(dev_model.h) == 0
+    ref = oracle.tree_step(ow, okv, toks, parent, skip_mask=m, quant_mode=mode)
+    err = rel_err(got, ref)
+    assert np.all(err < (TOL_BF16 if mode == 0 else TOL_INT8)), err
+    kv.close()
+
+
+def test_sub_block_skip_kv_rule(cs, dev_model, ow, prefix):
+    """A draft whose layer 0 runs only its FFN writes no K/V there: a later level may again skip
+    that attention block, but not run it."""
+    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
+    ffn_only = np.array([1 | cs.SKIP_ATTN, 1], np.uint8)
+    got = gpu_step(cs, dev_model, kv, [3, 4], [-1, 0], mask=ffn_only)
+    ref = oracle.tree_step(ow, okv, [3, 4], [-1, 0], skip_mask=ffn_only)
+    assert np.all(rel_err(got, ref) < TOL_BF16)
+    got = gpu_step(cs, dev_model, kv, [5], [1], mask=ffn_only)  # T = 2: layer 1 attends its own slots
+    ref = oracle.tree_step(ow, okv, [5], [1], skip_mask=ffn_only)
+    assert np.all(rel_err(got, ref) < TOL_BF16)
+    rc = cs.tree_step(dev_model.h, kv.h, _i32([6]), _i32([2]), 1, np.array([1, 1], np.uint8), 0, None, check=False)
+    assert rc == cs.E_STATE
+    assert cs.get_status(dev_model.h) == 0
+    kv.close()
+
+
 def test_all_layers_off_closed_form(cs, dev_model, ow, prefix):
     kv, okv = fresh_pair(cs, dev_model, ow, prefix)
     toks, parent = np.array([3, 4, 5]), np.array([-1, 0, 1])
