@@ -327,6 +327,7 @@ CASSPEC_API int casspec_latency_fit(const double* x, const double* y, int m, con
                                     double noise_sd, double* w_out, double* cov_out);
 
 #define CASSPEC_DYTC_MAX_CFG 16
+#define CASSPEC_TOPK_MAX 8 /* largest K of casspec_topk and of the DyTC tree */
 typedef struct casspec_dytc casspec_dytc;
 typedef struct {
   int n_cfg;        /* candidate draft configurations, 1..CASSPEC_DYTC_MAX_CFG */
@@ -337,6 +338,8 @@ typedef struct {
   int m_max;        /* largest tree, root included, 1..CASSPEC_MAX_TREE */
   double lambda;    /* EMA weight of the previous estimate (the paper uses 0.7) */
   int window;       /* outcomes per configuration in the recent mean (the paper uses H = 20) */
+  int topk;         /* Algorithm 1's K: candidates per drafted position, 1..CASSPEC_TOPK_MAX (1: a chain) */
+  double p_tree;    /* Algorithm 1's P_tree: top-P mass of the kept candidates, (0, 1] */
 } casspec_dytc_params;
 
 /* Create a scheduler over n_cfg candidate configurations with initial acceptance estimates
@@ -345,6 +348,8 @@ typedef struct {
 CASSPEC_API int casspec_dytc_create(const casspec_dytc_params* p, const double* alpha_init, const double* cost,
                                     casspec_dytc** out);
 CASSPEC_API void casspec_dytc_destroy(casspec_dytc* s);
+/* The parameters a scheduler was created with. */
+CASSPEC_API int casspec_dytc_get_params(const casspec_dytc* s, casspec_dytc_params* out);
 /* Replace a configuration's cost coefficient (e.g. from measured step times). */
 CASSPEC_API int casspec_dytc_set_cost(casspec_dytc* s, int cfg, double cost);
 /* Current acceptance estimate of a configuration. */
@@ -375,6 +380,23 @@ CASSPEC_API int casspec_dytc_tree_plan(casspec_dytc* s, int* leaf_out, int* cfg_
 CASSPEC_API int casspec_dytc_tree_extend(casspec_dytc* s, int leaf, int cfg, int k, const int32_t* tokens);
 CASSPEC_API int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out, int32_t* token_out,
                                       int32_t* cfg_out, double* p_acc_out);
+/* Algorithm 1 with K candidates per drafted position and sibling-parallel drafting (Sec. 4.2):
+ *   casspec_dytc_tree_begin: the branches of an expansion of `leaf` (planned by casspec_dytc_tree_plan):
+ *     the leaf and, when `siblings` is non-zero and the leaf is not the root, every active sibling of
+ *     the leaf (same parent) in node order; branches_out (host int32 [CASSPEC_MAX_TREE]), *nb_out their
+ *     number.  A neural draft passes siblings = 1 and extends every branch in the same draft steps; a
+ *     retrieval draft passes 0.
+ *   casspec_dytc_tree_add: one drafted position below `node` (a branch's current node): tokens and
+ *     probabilities (host [kc], rank order, kc in 1..CASSPEC_TOPK_MAX; e.g. casspec_topk of the draft's
+ *     logits row of `node`) are normalised over the kc; candidates are kept in rank order, the first
+ *     always and each further one while the normalised mass kept before it is below p_tree; each
+ *     becomes a child of `node` with P_acc = P_acc(node) * alpha(cfg) * its normalised probability;
+ *     `node` stops being an active leaf.  Returns the index of the top-1 child (the branch's next
+ *     node), 0 when the tree already holds m_max nodes (nothing added), or an error.  Stops adding at
+ *     m_max nodes.  With kc = 1 it appends one node with P_acc(node) * alpha(cfg), like tree_extend. */
+CASSPEC_API int casspec_dytc_tree_begin(casspec_dytc* s, int leaf, int siblings, int32_t* branches_out, int* nb_out);
+CASSPEC_API int casspec_dytc_tree_add(casspec_dytc* s, int node, int cfg, const int32_t* tokens, const float* probs,
+                                      int kc);
 
 /* Prompt-lookup bottom draft (PLD: the default bottom draft M_dn, Sec. 4.1; its match length is its
  * confidence, Sec. 4.2).  Over the history tokens (dev int32 [L], L >= 0), find the longest n in
@@ -404,28 +426,34 @@ typedef struct {
   int pld_n_max;
 } casspec_draft_cfg;
 
-/* One round of DyTC speculative decoding (Sec. 4.2: Algorithm 1, one drafted token per position,
- * then verification by the target).  Configuration i of scheduler s runs as cfgs[i].  root_token is
- * the last generated token, not yet in the cache (the previous round's bonus token); kv must hold a
- * committed prefix with no tree (T = 0).
- *   Each expansion (leaf, cfg, k) that Algorithm 1 plans runs the chosen draft over root .. leaf as one
- *   chain and then once per further drafted token (greedy argmax), and appends the k tokens.  The
- *   target then verifies the whole tree (casspec_tree_step, all layers, bf16), the longest matching
+/* One round of DyTC speculative decoding (Sec. 4.2: Algorithm 1, then verification by the target).
+ * Configuration i of scheduler s runs as cfgs[i].  root_token is the last generated token, not yet
+ * in the cache (the previous round's bonus token); kv must hold a committed prefix with no tree (T = 0).
+ *   K = 1 (the scheduler's topk): each expansion (leaf, cfg, k) that Algorithm 1 plans runs the chosen
+ *   draft over root .. leaf as one chain and then once per further drafted token (greedy argmax), and
+ *   appends the k tokens.
+ *   K > 1 with a neural draft: the draft runs over root .. leaf plus the leaf's active siblings (the
+ *   branches, casspec_dytc_tree_begin) in one tree step, then once per further position over the
+ *   branches' top-1 children; at each position casspec_topk of each branch's logits row gives the
+ *   candidates that casspec_dytc_tree_add keeps.  dev_logits (device fp32 [CASSPEC_MAX_TREE][vocab])
+ *   receives the draft's logits; it may be NULL when K = 1.
+ *   The target then verifies the whole tree (casspec_tree_step, all layers, bf16), the longest matching
  *   path is accepted (casspec_accept_greedy) and compacted into the cache (casspec_kv_compact).  For
- *   every expansion whose leaf was accepted, whether its first drafted token was accepted is recorded,
- *   and the estimates are updated (casspec_dytc_end_step).
+ *   every branch of an expansion whose node was accepted, whether its top-1 child was accepted is
+ *   recorded (the first drafted token's outcome), and the estimates are updated (casspec_dytc_end_step).
  *   A prompt-lookup configuration drafts from history (dev int32, the committed tokens, the last
  *   being root_token; hist_len entries, room for CASSPEC_MAX_TREE more, which the round overwrites);
  *   finding no earlier occurrence counts as a rejected first token and ends the drafting.  history
  *   may be NULL when no configuration is a prompt lookup.
- *   dev_work: device int32 [5 * CASSPEC_MAX_TREE] (caller-owned scratch).  out_tokens (host int32
+ *   dev_work: device int32 [CASSPEC_DYTC_WORK] (caller-owned scratch).  out_tokens (host int32
  *   [CASSPEC_MAX_TREE]) receives the tokens this round commits after the root, the last being the
  *   bonus token (the next root); *n_out their count (>= 1); *n_drafted_out (may be NULL) the drafted
  *   nodes.  Synchronises the model's stream several times (it reads drafted tokens back).
  *   Errors: E_INVAL, E_STATE (kv holds a tree), E_TREE (device-reported), errors of the calls above. */
 CASSPEC_API int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv* kv, const casspec_draft_cfg* cfgs,
                                    int32_t root_token, int32_t* history, int hist_len, int32_t* dev_work,
-                                   int32_t* out_tokens, int* n_out, int* n_drafted_out);
+                                   float* dev_logits, int32_t* out_tokens, int* n_out, int* n_drafted_out);
+#define CASSPEC_DYTC_WORK (24 * CASSPEC_MAX_TREE) /* int32 entries of casspec_dytc_round's dev_work */
 
 #ifdef __cplusplus
 }

@@ -40,6 +40,17 @@ Readings (the paper is silent or inconsistent; each is also listed in the design
     child is no longer an active leaf;
   * ties: Algorithm 2 keeps the first (S, k) reaching the maximum (strict >); among active leaves of
     equal P_acc the lowest node index is expanded;
+  * Algorithm 1 with K > 1 (`draft_tree_topk`; the printed loop, its function names and the shape
+    of y disagree with one another): at every drafted position the draft's K best tokens, their
+    probabilities normalised over the K, are candidate children of the branch's current node; the
+    first candidate is always kept and each further one while the normalised mass kept before it
+    is below P_tree (top-P); the top-1 child continues the branch.  The token-level refinement of
+    P_acc (Sec. 4.2, "normalized probability" of a drafted token) is
+    P_acc(child) = P_acc(parent) * a_S * p_norm(child), which is Algorithm 1's a_S product at K = 1.
+    Sibling-parallel drafting: expanding a leaf with a neural draft extends, in the same draft
+    steps and by the same k, every active sibling of that leaf (same parent), each as a branch of
+    its own; branches are processed in node order, and within a branch candidates in rank order,
+    until the tree holds m_max nodes;
   * "a ~ 1" and "c k + c_dn ~ 0" in Algorithm 2 are |1 - a| < 1e-9 and |c k + c_dn| < 1e-12.
 """
 from __future__ import annotations
@@ -198,6 +209,87 @@ def draft_tree(alphas: list[float], costs: list[float], a_dn: float, c_dn: float
             if len(parent) >= m_max:
                 return {"parent": parent, "token": token, "cfg": cfg_of, "p_acc": p_acc, "steps": steps}
     return {"parent": parent, "token": token, "cfg": cfg_of, "p_acc": p_acc, "steps": steps}
+
+
+def topp_keep(probs: list[float], p_tree: float) -> list[float]:
+    """Normalised probabilities of the candidates kept from one position's K best (rank order):
+    the first always, each further one while the normalised mass before it is below p_tree."""
+    total = sum(probs)
+    kept, mass = [], 0.0
+    for j, p in enumerate(probs):
+        if j > 0 and mass >= p_tree:
+            break
+        q = p / total
+        kept.append(q)
+        mass += q
+    return kept
+
+
+def draft_tree_topk(alphas: list[float], costs: list[float], a_dn: float, c_dn: float, k_max: int,
+                    t_min: float, m_max: int, p_tree: float, cands, chain_cfgs=()) -> dict:
+    """Algorithm 1 with K candidates per drafted position and sibling-parallel drafting.
+
+    ``cands(cfg, path)`` returns configuration ``cfg``'s K best next tokens after the node sequence
+    ``path`` (root first), as (token, probability) pairs in rank order.  Configurations in
+    ``chain_cfgs`` (a retrieval bottom draft) give one candidate per position and draft no
+    siblings; an empty candidate list ends that branch, and at an expansion's first position it
+    ends the drafting (nothing to propose).  Returns the tree like ``draft_tree``; ``steps`` holds
+    (leaf, cfg, k, branches)."""
+    parent, token, cfg_of, p_acc, active = [-1], [None], [-1], [1.0], [True]
+    steps = []
+
+    def out():
+        return {"parent": parent, "token": token, "cfg": cfg_of, "p_acc": p_acc, "steps": steps}
+
+    def path_to(v):
+        path = []
+        while v >= 0:
+            path.append(v)
+            v = parent[v]
+        return path[::-1]
+
+    while len(parent) < m_max:
+        open_leaves = [i for i in range(len(parent)) if active[i]]
+        if not open_leaves:
+            break
+        leaf = max(open_leaves, key=lambda i: (p_acc[i], -i))
+        if c_dn > 0.0 and a_dn / c_dn * p_acc[leaf] < t_min:
+            break
+        s, k, _ = find_best_config(alphas, costs, a_dn, c_dn, k_max)
+        if s is None:
+            active[leaf] = False
+            break
+        branches = [leaf]
+        if s not in chain_cfgs and leaf != 0:
+            branches += [j for j in range(len(parent)) if j != leaf and active[j] and parent[j] == parent[leaf]]
+        steps.append((leaf, s, k, list(branches)))
+        cur = list(branches)
+        for pos in range(k):
+            nxt = []
+            for c in cur:
+                pairs = cands(s, path_to(c))
+                if s in chain_cfgs:
+                    pairs = pairs[:1]
+                if not pairs:
+                    if pos == 0 and c == leaf:
+                        return out()
+                    continue
+                kept = topp_keep([p for _, p in pairs], 1.0 if s in chain_cfgs else p_tree)
+                active[c] = False  # c receives children: no longer a leaf
+                first = None
+                for (tok, _), q in zip(pairs, kept):
+                    parent.append(c)
+                    token.append(tok)
+                    cfg_of.append(s)
+                    p_acc.append(p_acc[c] * alphas[s] * q)
+                    active.append(True)
+                    if first is None:
+                        first = len(parent) - 1
+                    if len(parent) >= m_max:
+                        return out()
+                nxt.append(first)
+            cur = nxt
+    return out()
 
 
 # ------------------------------------------------------------------------------------------------

@@ -17,6 +17,8 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libcasspec.so")
 
 OK, E_INVAL, E_SHAPE, E_CAPACITY, E_CUDA, E_TREE, E_TIMEOUT, E_STATE = 0, -1, -2, -3, -4, -5, -6, -7
 MAX_TREE = 64
+TOPK_MAX = 8
+DYTC_WORK = 24 * MAX_TREE  # int32 entries of casspec_dytc_round's device scratch
 SKIP_ATTN, SKIP_FFN = 0x2, 0x4  # skip-mask flags on a non-zero byte: drop the attention / FFN block
 OPT_PDL, OPT_GRAPHS = 1, 2
 
@@ -32,9 +34,9 @@ EXPORTS = [
     "casspec_rmsnorm",
     "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
-    "casspec_dytc_destroy", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
+    "casspec_dytc_destroy", "casspec_dytc_get_params", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft", "casspec_topk",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_begin", "casspec_dytc_tree_add", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft", "casspec_topk",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -48,7 +50,8 @@ class ModelConfig(ctypes.Structure):
 class DytcParams(ctypes.Structure):
     _fields_ = [("n_cfg", ctypes.c_int32), ("alpha_dn", ctypes.c_double), ("c_dn", ctypes.c_double),
                 ("k_max", ctypes.c_int32), ("t_min", ctypes.c_double), ("m_max", ctypes.c_int32),
-                ("lambda_", ctypes.c_double), ("window", ctypes.c_int32)]
+                ("lambda_", ctypes.c_double), ("window", ctypes.c_int32), ("topk", ctypes.c_int32),
+                ("p_tree", ctypes.c_double)]
 
 
 class DraftCfg(ctypes.Structure):
@@ -84,6 +87,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_objective": (_D, [_D, _D, _I, _D, _D]),
         "casspec_dytc_create": (_I, [ctypes.POINTER(DytcParams), ctypes.POINTER(_D), ctypes.POINTER(_D), ctypes.POINTER(_P)]),
         "casspec_dytc_destroy": (None, [_P]),
+        "casspec_dytc_get_params": (_I, [_P, ctypes.POINTER(DytcParams)]),
         "casspec_dytc_set_cost": (_I, [_P, _I, _D]),
         "casspec_dytc_alpha": (_I, [_P, _I, ctypes.POINTER(_D)]),
         "casspec_dytc_best_config": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_D)]),
@@ -92,11 +96,13 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_reset": (_I, [_P]),
         "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
+        "casspec_dytc_tree_begin": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_I)]),
+        "casspec_dytc_tree_add": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_float), _I]),
         "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
         "casspec_topk": (_I, [_P, _I, _I, _I, _P, _P, _P]),
         "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
                                      ctypes.POINTER(_D), ctypes.POINTER(_D)]),
-        "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, _I, _P,
+        "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, _I, _P, _P,
                                     ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_get": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
                                        ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_D)]),
@@ -362,10 +368,10 @@ class Dytc:
     """Owner of one native DyTC scheduler (casspec_dytc_*)."""
 
     def __init__(self, alphas, costs, alpha_dn: float, c_dn: float, k_max: int, t_min: float, m_max: int,
-                 lam: float = 0.7, window: int = 20):
+                 lam: float = 0.7, window: int = 20, topk: int = 1, p_tree: float = 1.0):
         lib = load_library()
         n = len(alphas)
-        p = DytcParams(n, alpha_dn, c_dn, k_max, t_min, m_max, lam, window)
+        p = DytcParams(n, alpha_dn, c_dn, k_max, t_min, m_max, lam, window, topk, p_tree)
         a = (_D * n)(*alphas)
         c = (_D * n)(*costs)
         h = _P()
@@ -420,6 +426,23 @@ class Dytc:
             raise CasspecError("casspec_dytc_tree_extend", rc)
         return rc
 
+    def tree_begin(self, leaf: int, siblings: bool = True) -> list[int]:
+        br, nb = (ctypes.c_int32 * MAX_TREE)(), _I()
+        _check("casspec_dytc_tree_begin",
+               load_library().casspec_dytc_tree_begin(self.h, leaf, int(bool(siblings)), br, ctypes.byref(nb)))
+        return list(br[: nb.value])
+
+    def tree_add(self, node: int, cfg: int, tokens, probs) -> int:
+        """Candidates (rank order) of one drafted position below `node`; returns the top-1 child,
+        0 when the tree is full."""
+        kc = len(tokens)
+        t = (ctypes.c_int32 * kc)(*[int(x) for x in tokens])
+        p = (ctypes.c_float * kc)(*[float(x) for x in probs])
+        rc = load_library().casspec_dytc_tree_add(self.h, node, cfg, t, p, kc)
+        if rc < 0:
+            raise CasspecError("casspec_dytc_tree_add", rc)
+        return rc
+
     def tree_get(self) -> dict:
         m = self.m_max
         n = _I()
@@ -429,12 +452,14 @@ class Dytc:
         k = n.value
         return {"parent": list(par[:k]), "token": list(tok[:k]), "cfg": list(cfg[:k]), "p_acc": list(pacc[:k])}
 
-    def round(self, m: int, kv: int, cfgs, root_token: int, dev_work, history=None, hist_len: int = 0) -> tuple[list[int], int]:
+    def round(self, m: int, kv: int, cfgs, root_token: int, dev_work, history=None, hist_len: int = 0,
+              dev_logits=None) -> tuple[list[int], int]:
         """One DyTC round (casspec_dytc_round).  cfgs: per configuration (skip_mask or None, quant_mode)
         for a model draft, or ("pld", n_max) for the prompt-lookup draft; history: torch int32 CUDA
         tensor of the committed tokens (hist_len valid, the last = root_token, room for MAX_TREE more);
-        dev_work: torch int32 CUDA tensor of 5 * MAX_TREE entries.  Returns the committed tokens (the
-        last is the bonus token) and the number of drafted nodes."""
+        dev_work: torch int32 CUDA tensor of DYTC_WORK entries; dev_logits: torch fp32 CUDA tensor of
+        MAX_TREE x vocab (needed when topk > 1).  Returns the committed tokens (the last is the bonus
+        token) and the number of drafted nodes."""
         masks, items = [], []
         for a, b in cfgs:
             if isinstance(a, str):
@@ -448,7 +473,7 @@ class Dytc:
         out = (ctypes.c_int32 * MAX_TREE)()
         n, nd = _I(), _I()
         _check("casspec_dytc_round", load_library().casspec_dytc_round(self.h, m, kv, arr, int(root_token), _ptr(history),
-                                                                       int(hist_len), _ptr(dev_work), out,
+                                                                       int(hist_len), _ptr(dev_work), _ptr(dev_logits), out,
                                                                        ctypes.byref(n), ctypes.byref(nd)))
         return list(out[: n.value]), nd.value
 

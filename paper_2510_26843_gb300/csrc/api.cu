@@ -1052,7 +1052,7 @@ int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q, float* s, 
 }  // extern "C"
 
 // ---------------------------------------------------------------------------------------------
-// One DyTC round (Sec. 4.2, Algorithm 1 with one drafted token per position, then verification)
+// One DyTC round (Sec. 4.2, Algorithm 1, then verification)
 // ---------------------------------------------------------------------------------------------
 namespace {
 int read_dev_i32(casspec_model* m, const int32_t* dev, int count, int32_t* host) {
@@ -1064,20 +1064,27 @@ int read_dev_i32(casspec_model* m, const int32_t* dev, int count, int32_t* host)
 
 extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv* kv, const casspec_draft_cfg* cfgs,
                                   int32_t root_token, int32_t* history, int hist_len, int32_t* dev_work,
-                                  int32_t* out_tokens, int* n_out, int* n_drafted_out) {
+                                  float* dev_logits, int32_t* out_tokens, int* n_out, int* n_drafted_out) {
   if (s == nullptr || m == nullptr || kv == nullptr || cfgs == nullptr || dev_work == nullptr || out_tokens == nullptr ||
       n_out == nullptr || kv->m != m)
     return CASSPEC_E_INVAL;
   if (kv->T != 0) return CASSPEC_E_STATE;  // a round starts from a committed prefix
+  casspec_dytc_params prm;
+  if (casspec_dytc_get_params(s, &prm) != CASSPEC_OK) return CASSPEC_E_INVAL;
+  const int K = prm.topk;
+  if (K > 1 && dev_logits == nullptr) return CASSPEC_E_INVAL;
+  const int V = m->cfg.vocab;
   int32_t* d_tok = dev_work;
   int32_t* d_par = dev_work + kMaxTree;
   int32_t* d_acc = dev_work + 2 * kMaxTree;
   int32_t* d_pld = dev_work + 3 * kMaxTree + 8;  // {match length, count, tokens...}
+  int32_t* d_tki = dev_work + 5 * kMaxTree;      // top-K ids [64][8]
+  float* d_tkp = reinterpret_cast<float*>(dev_work + 13 * kMaxTree);  // top-K probabilities [64][8]
   const int32_t* d_am = m->am;
   int rc;
   if ((rc = casspec_dytc_tree_reset(s)) != CASSPEC_OK) return rc;
   struct Expansion {
-    int leaf, cfg, first;
+    int leaf, cfg, first;  // a branch node of an expansion and its top-1 child
   };
   std::vector<Expansion> exps;
   int32_t par[kMaxTree], tok[kMaxTree], ncfg[kMaxTree];
@@ -1121,6 +1128,71 @@ extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv*
       if (rc < pr[1]) break;  // the tree is full
       continue;
     }
+    if (K > 1) {
+      // the branches: the leaf and its active siblings; the draft runs over root .. leaf plus the
+      // siblings (children of the leaf's parent, slot len - 2), so the branches' rows are contiguous
+      int32_t br[kMaxTree];
+      int nb = 0;
+      if ((rc = casspec_dytc_tree_begin(s, leaf, 1, br, &nb)) != CASSPEC_OK) return rc;
+      for (int b = 1; b < nb; ++b) {
+        ctok[len + b - 1] = tok[br[b]];
+        cpar[len + b - 1] = len - 2;
+      }
+      int n_dev = len + nb - 1;  // tree slots the draft holds (distinct nodes of the tree)
+      casspec_kv_reset_tree(kv);
+      CK(cudaMemcpyAsync(d_tok, ctok, (size_t)n_dev * 4, cudaMemcpyHostToDevice, m->stream));
+      CK(cudaMemcpyAsync(d_par, cpar, (size_t)n_dev * 4, cudaMemcpyHostToDevice, m->stream));
+      if ((rc = casspec_tree_step(m, kv, d_tok, d_par, n_dev, cfgs[c].skip_mask, cfgs[c].quant_mode, dev_logits)) !=
+          CASSPEC_OK)
+        return rc;
+      int slot[kMaxTree], cur[kMaxTree];
+      for (int b = 0; b < nb; ++b) {
+        slot[b] = len - 1 + b;
+        cur[b] = br[b];
+      }
+      const float* rows = dev_logits + (size_t)(len - 1) * V;
+      bool full = false;
+      for (int pos = 0; pos < k && !full; ++pos) {
+        if ((rc = casspec_topk(rows, nb, V, K, d_tki, d_tkp, m->stream)) != CASSPEC_OK) return rc;
+        int32_t ids[kMaxTree * CASSPEC_TOPK_MAX];
+        float pr[kMaxTree * CASSPEC_TOPK_MAX];
+        CK(cudaMemcpyAsync(pr, d_tkp, (size_t)nb * K * 4, cudaMemcpyDeviceToHost, m->stream));
+        if ((rc = read_dev_i32(m, d_tki, nb * K, ids)) != CASSPEC_OK) return rc;
+        int nxt = 0;
+        for (int b = 0; b < nb; ++b) {
+          const int child = casspec_dytc_tree_add(s, cur[b], c, ids + b * K, pr + b * K, K);
+          if (child < 0) return child;
+          if (child == 0) {  // the tree is full
+            full = true;
+            break;
+          }
+          if (pos == 0) exps.push_back({cur[b], c, child});
+          cur[nxt] = child;
+          slot[nxt] = slot[b];
+          ctok[nxt] = ids[b * K];
+          ++nxt;
+        }
+        if (full || pos + 1 == k) break;
+        int tree_n = 0;
+        if ((rc = casspec_dytc_tree_get(s, &tree_n, nullptr, nullptr, nullptr, nullptr)) != CASSPEC_OK) return rc;
+        if (tree_n >= prm.m_max) break;
+        // the next position: the branches' top-1 children, one tree step over all of them
+        nb = nxt;
+        for (int b = 0; b < nb; ++b) {
+          cpar[n_dev + b] = slot[b];
+          slot[b] = n_dev + b;
+        }
+        CK(cudaMemcpyAsync(d_tok + n_dev, ctok, (size_t)nb * 4, cudaMemcpyHostToDevice, m->stream));
+        CK(cudaMemcpyAsync(d_par + n_dev, cpar + n_dev, (size_t)nb * 4, cudaMemcpyHostToDevice, m->stream));
+        if ((rc = casspec_tree_step(m, kv, d_tok + n_dev, d_par + n_dev, nb, cfgs[c].skip_mask, cfgs[c].quant_mode,
+                                    dev_logits)) != CASSPEC_OK)
+          return rc;
+        n_dev += nb;
+        rows = dev_logits;
+      }
+      if (full) break;
+      continue;
+    }
     casspec_kv_reset_tree(kv);
     CK(cudaMemcpyAsync(d_tok, ctok, (size_t)len * 4, cudaMemcpyHostToDevice, m->stream));
     CK(cudaMemcpyAsync(d_par, cpar, (size_t)len * 4, cudaMemcpyHostToDevice, m->stream));
@@ -1160,11 +1232,13 @@ extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv*
   std::vector<uint8_t> on_path(n, 0);
   for (int i = 1; i <= L; ++i)
     if (acc[i] >= 0 && acc[i] < n) on_path[acc[i]] = 1;
-  // first-draft-token outcomes of the expansions whose leaf the target accepted (Sec. 4.2)
+  // first-draft-token outcomes of the expansion branches the target accepted (Sec. 4.2)
   for (const auto& e : exps)
     if (on_path[e.leaf]) casspec_dytc_record(s, e.cfg, on_path[e.first]);
   casspec_dytc_end_step(s);
+  const long long p_upper = kv->P_upper;
   if ((rc = casspec_kv_compact(kv, d_acc)) != CASSPEC_OK) return rc;
+  kv->P_upper = p_upper + L;  // the accepted length is known here: keep the capacity bound exact
   for (int i = 2; i <= L; ++i) out_tokens[i - 2] = tok[acc[i]];
   out_tokens[L - 1] = acc[L + 1];  // the bonus token: the next round's root
   *n_out = L;

@@ -7,9 +7,14 @@
 //     configurations used in a step (App. D);
 //   * Eq. 5 / App. D Algorithm 2: the (configuration, draft length) maximising the local speedup plus
 //     the least future speedup of the bottom draft;
-//   * Algorithm 1 with one drafted token per position: expand the active leaf of highest accumulated
-//     acceptance until the stop rule (alpha_dn / c_dn * P_acc < t_min) or the tree size limit, the
-//     drafted tokens coming from the caller (the tree steps of the chosen draft configuration).
+//   * Algorithm 1: expand the active leaf of highest accumulated acceptance until the stop rule
+//     (alpha_dn / c_dn * P_acc < t_min) or the tree size limit, the drafted tokens coming from the
+//     caller (the tree steps of the chosen draft configuration).  With K candidates per drafted
+//     position (top-K), the candidates are normalised over the K and kept in rank order while the
+//     mass kept before them is below P_tree (top-P, the first always); each child gets
+//     P_acc(parent) * alpha(cfg) * its normalised probability (the token-level refinement of
+//     Sec. 4.2), and the top-1 child continues the branch.  Expanding a leaf with a neural draft
+//     also extends its active siblings in the same draft steps (tree-based parallel drafting).
 // An expanded node stops being an active leaf (Algorithm 1 as printed never clears it, which would
 // let the same sequence be drafted twice).  Ties keep the first maximum and the lowest node index.
 #include <cmath>
@@ -82,7 +87,8 @@ double casspec_dytc_objective(double alpha, double c, int k, double alpha_dn, do
 int casspec_dytc_create(const casspec_dytc_params* p, const double* alpha_init, const double* cost, casspec_dytc** out) {
   if (p == nullptr || alpha_init == nullptr || cost == nullptr || out == nullptr) return CASSPEC_E_INVAL;
   if (p->n_cfg < 1 || p->n_cfg > CASSPEC_DYTC_MAX_CFG || p->k_max < 1 || p->m_max < 1 || p->m_max > CASSPEC_MAX_TREE ||
-      p->window < 1 || !(p->lambda >= 0.0 && p->lambda <= 1.0) || bad_alpha(p->alpha_dn) || p->c_dn < 0.0)
+      p->window < 1 || !(p->lambda >= 0.0 && p->lambda <= 1.0) || bad_alpha(p->alpha_dn) || p->c_dn < 0.0 ||
+      p->topk < 1 || p->topk > CASSPEC_TOPK_MAX || !(p->p_tree > 0.0 && p->p_tree <= 1.0))
     return CASSPEC_E_INVAL;
   for (int i = 0; i < p->n_cfg; ++i)
     if (bad_alpha(alpha_init[i]) || !(cost[i] >= 0.0)) return CASSPEC_E_INVAL;
@@ -98,6 +104,12 @@ int casspec_dytc_create(const casspec_dytc_params* p, const double* alpha_init, 
 }
 
 void casspec_dytc_destroy(casspec_dytc* s) { delete s; }
+
+int casspec_dytc_get_params(const casspec_dytc* s, casspec_dytc_params* out) {
+  if (s == nullptr || out == nullptr) return CASSPEC_E_INVAL;
+  *out = s->p;
+  return CASSPEC_OK;
+}
 
 int casspec_dytc_set_cost(casspec_dytc* s, int cfg, double cost) {
   if (s == nullptr || cfg < 0 || cfg >= s->p.n_cfg || !(cost >= 0.0)) return CASSPEC_E_INVAL;
@@ -208,6 +220,48 @@ int casspec_dytc_tree_extend(casspec_dytc* s, int leaf, int cfg, int k, const in
     ++added;
   }
   return added;
+}
+
+int casspec_dytc_tree_begin(casspec_dytc* s, int leaf, int siblings, int32_t* branches_out, int* nb_out) {
+  if (s == nullptr || branches_out == nullptr || nb_out == nullptr) return CASSPEC_E_INVAL;
+  const int n = (int)s->parent.size();
+  if (leaf < 0 || leaf >= n || !s->active[leaf]) return CASSPEC_E_INVAL;
+  int nb = 0;
+  branches_out[nb++] = leaf;
+  if (siblings && leaf != 0)
+    for (int j = 0; j < n; ++j)
+      if (j != leaf && s->active[j] && s->parent[j] == s->parent[leaf]) branches_out[nb++] = j;
+  *nb_out = nb;
+  return CASSPEC_OK;
+}
+
+int casspec_dytc_tree_add(casspec_dytc* s, int node, int cfg, const int32_t* tokens, const float* probs, int kc) {
+  if (s == nullptr || tokens == nullptr || probs == nullptr || cfg < 0 || cfg >= s->p.n_cfg || kc < 1 ||
+      kc > CASSPEC_TOPK_MAX)
+    return CASSPEC_E_INVAL;
+  const int n0 = (int)s->parent.size();
+  if (node < 0 || node >= n0) return CASSPEC_E_INVAL;
+  if (n0 >= s->p.m_max) return 0;
+  double total = 0.0;
+  for (int j = 0; j < kc; ++j) {
+    if (!(probs[j] >= 0.0f)) return CASSPEC_E_INVAL;
+    total += (double)probs[j];
+  }
+  if (!(total > 0.0)) return CASSPEC_E_INVAL;
+  s->active[node] = 0;  // it receives children
+  const double base = s->p_acc[node] * s->alpha[cfg];
+  double mass = 0.0;
+  for (int j = 0; j < kc && (int)s->parent.size() < s->p.m_max; ++j) {
+    if (j > 0 && mass >= s->p.p_tree) break;
+    const double q = (double)probs[j] / total;
+    s->parent.push_back(node);
+    s->token.push_back(tokens[j]);
+    s->cfg.push_back(cfg);
+    s->p_acc.push_back(base * q);
+    s->active.push_back(1);
+    mass += q;
+  }
+  return n0;  // the top-1 child
 }
 
 int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out, int32_t* token_out, int32_t* cfg_out,

@@ -172,3 +172,95 @@ def test_draft_tree_edge_cases_match_oracle(cs, alphas, costs, a_dn, c_dn, k_max
     assert got["parent"] == want["parent"] and got["cfg"] == want["cfg"]
     assert got["p_acc"] == pytest.approx(want["p_acc"], rel=1e-12)
     sch.close()
+
+
+def _cands_f32(K):
+    """Seeded fake candidates: K distinct tokens with float32-exact decreasing probabilities."""
+    import numpy as np
+
+    def cands(cfg, path):
+        h = (7 * len(path) + 13 * cfg + 5 * path[-1] + 3) % 89
+        w = np.sort(np.random.default_rng(h).uniform(0.01, 1.0, K).astype(np.float32))[::-1]
+        return [((h + 17 * j) % 211, float(w[j])) for j in range(K)]
+    return cands
+
+
+def _native_topk_tree(cs, sch, cands, chain_cfgs=()):
+    """Algorithm 1 with K candidates, driven through tree_plan / tree_begin / tree_add as the GPU
+    round drives it; returns the steps (leaf, cfg, k, branches)."""
+    sch.tree_reset()
+    steps = []
+    while True:
+        plan = sch.tree_plan()
+        if plan is None:
+            break
+        leaf, s, k = plan
+        branches = sch.tree_begin(leaf, siblings=s not in chain_cfgs)
+        steps.append((leaf, s, k, list(branches)))
+        cur, full = list(branches), False
+        for _ in range(k):
+            tr = sch.tree_get()
+            nxt = []
+            for c in cur:
+                path, v = [], c
+                while v >= 0:
+                    path.append(v)
+                    v = tr["parent"][v]
+                pairs = cands(s, path[::-1])
+                if s in chain_cfgs:
+                    pairs = pairs[:1]
+                child = sch.tree_add(c, s, [t for t, _ in pairs], [p for _, p in pairs])
+                if child == 0:
+                    full = True
+                    break
+                nxt.append(child)
+            if full:
+                break
+            cur = nxt
+            if len(sch.tree_get()["parent"]) >= sch.m_max:
+                break
+        if full:
+            break
+    return steps
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_topk_tree_matches_oracle(cs, seed):
+    r = _rng(500 + seed)
+    n_cfg = r.randint(1, 4)
+    alphas = [r.uniform(0.3, 0.99) for _ in range(n_cfg)]
+    costs = [r.uniform(0.05, 0.8) for _ in range(n_cfg)]
+    a_dn, c_dn = r.uniform(0.1, 0.8), r.choice([0.0, r.uniform(0.01, 0.1)])
+    k_max, t_min, m_max = r.randint(1, 5), r.uniform(0.05, 3.0), r.randint(2, 64)
+    K, p_tree = r.randint(1, 8), r.choice([1.0, r.uniform(0.3, 0.99)])
+    chain = (n_cfg - 1,) if n_cfg > 1 and r.random() < 0.5 else ()
+    cands = _cands_f32(K)
+    want = D.draft_tree_topk(alphas, costs, a_dn, c_dn, k_max, t_min, m_max, p_tree, cands, chain_cfgs=chain)
+    sch = cs.Dytc(alphas, costs, a_dn, c_dn, k_max, t_min, m_max, topk=K, p_tree=p_tree)
+    steps = _native_topk_tree(cs, sch, cands, chain)
+    got = sch.tree_get()
+    assert steps == want["steps"]
+    assert got["parent"] == want["parent"] and got["cfg"] == want["cfg"]
+    assert got["token"][1:] == want["token"][1:]
+    assert got["p_acc"] == pytest.approx(want["p_acc"], rel=1e-12)
+    sch.close()
+
+
+def test_topk_tree_argument_errors(cs):
+    for kw in ({"topk": 0}, {"topk": 9}, {"p_tree": 0.0}, {"p_tree": 1.5}):
+        with pytest.raises(cs.CasspecError):
+            cs.Dytc([0.5], [0.1], 0.5, 0.01, 4, 1.0, 16, **kw)
+    sch = cs.Dytc([0.5], [0.1], 0.5, 0.01, 4, 1.0, 16, topk=3, p_tree=0.9)
+    with pytest.raises(cs.CasspecError):
+        sch.tree_begin(4)  # no such node
+    with pytest.raises(cs.CasspecError):
+        sch.tree_add(0, 0, [], [])  # no candidate
+    with pytest.raises(cs.CasspecError):
+        sch.tree_add(0, 0, [1, 2], [0.0, 0.0])  # no probability mass
+    with pytest.raises(cs.CasspecError):
+        sch.tree_add(0, 1, [1], [1.0])  # no such configuration
+    assert sch.tree_add(0, 0, [5, 6, 7], [0.5, 0.3, 0.2]) == 1
+    assert sch.tree_get()["parent"] == [-1, 0, 0, 0]  # mass 0.5, then 0.8, both below 0.9: all three kept
+    assert sch.tree_add(1, 0, [8, 9], [0.95, 0.05]) == 4
+    assert sch.tree_get()["parent"] == [-1, 0, 0, 0, 1]  # 0.95 reaches 0.9: the second is dropped
+    sch.close()

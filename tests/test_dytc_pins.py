@@ -213,3 +213,101 @@ def test_blr_limits_and_sequential_updates():
     assert mean_b == pytest.approx(mu, rel=1e-6)
     assert cov_b == pytest.approx(cov, rel=1e-5, abs=1e-30)
 
+
+
+# ------------------------------------------------------------------------------------------------
+# Algorithm 1 with K candidates per drafted position (top-K / top-P) and sibling-parallel drafting
+# ------------------------------------------------------------------------------------------------
+def test_topp_keep_hand_cases():
+    assert D.topp_keep([0.5, 0.25, 0.25], 0.75) == [0.5, 0.25]  # mass 0.75 reached: the third is dropped
+    assert D.topp_keep([0.5, 0.25, 0.25], 0.76) == [0.5, 0.25, 0.25]
+    assert D.topp_keep([0.5, 0.25, 0.25], 0.5) == [0.5]
+    assert D.topp_keep([0.5, 0.25, 0.25], 0.25) == [0.5]  # the first is always kept
+    assert D.topp_keep([2.0, 1.0, 1.0], 1.0) == [0.5, 0.25, 0.25]  # normalised over the K
+    assert D.topp_keep([0.3], 0.1) == [1.0]
+
+
+def test_topk_tree_worked_example():
+    """Hand-traced: one configuration (a = 0.8, k = 2), candidates (token 1, p 0.6), (token 2, p 0.4)
+    after every path, P_tree = 0.9 (both kept), m_max = 12.
+      expansion 1: root -> n1 (1, 0.48), n2 (2, 0.32); n1 -> n3 (1, 0.2304), n4 (2, 0.1536);
+      expansion 2: leaf n2 (0.32 is the highest active P_acc; its sibling n1 is expanded already):
+                   n2 -> n5 (1, 0.1536), n6 (2, 0.1024); n5 -> n7 (1, 0.073728), n8 (2, 0.049152);
+      expansion 3: leaf n3 (0.2304) with its active sibling n4 as a second branch:
+                   n3 -> n9 (1, 0.110592), n10 (2, 0.073728); n4 -> n11 (1, 0.073728): 12 nodes, full."""
+    s, k, _ = D.find_best_config([0.8], [0.05], 0.5, 0.2, 2)  # Eq. 5: 5.87 at k = 2 against 4.8 at k = 1
+    assert (s, k) == (0, 2)
+    tr = D.draft_tree_topk([0.8], [0.05], 0.5, 0.2, 2, 0.0, 12, 0.9, lambda cfg, path: [(1, 0.6), (2, 0.4)])
+    assert tr["parent"] == [-1, 0, 0, 1, 1, 2, 2, 5, 5, 3, 3, 4]
+    assert tr["token"] == [None, 1, 2, 1, 2, 1, 2, 1, 2, 1, 2, 1]
+    assert tr["p_acc"] == pytest.approx([1.0, 0.48, 0.32, 0.2304, 0.1536, 0.1536, 0.1024, 0.073728, 0.049152,
+                                         0.110592, 0.073728, 0.073728], rel=1e-12)
+    assert tr["steps"] == [(0, 0, 2, [0]), (2, 0, 2, [2]), (3, 0, 2, [3, 4])]
+
+
+def _fake_cands(K):
+    def cands(cfg, path):
+        base = (7 * len(path) + 13 * cfg + 5 * path[-1]) % 97
+        w = [1.0 / (j + 1 + (base % 3)) for j in range(K)]
+        return [((base + 11 * j) % 101, w[j]) for j in range(K)]
+    return cands
+
+
+def _depth_token(cfg, depth):
+    return (7 * depth + 13 * cfg) % 101
+
+
+@pytest.mark.parametrize("alphas,costs,a_dn,c_dn,k_max,t_min,m_max", [
+    ([0.9, 0.8], [0.4, 0.3], 0.5, 0.05, 4, 1.0, 16),
+    ([0.7, 0.6, 0.95], [0.3, 0.1, 0.6], 0.4, 0.02, 3, 0.5, 64),
+    ([0.5], [0.2], 0.3, 0.05, 5, 4.0, 32),
+])
+def test_topk_tree_with_one_candidate_is_algorithm_1(alphas, costs, a_dn, c_dn, k_max, t_min, m_max):
+    """K = 1: the top-K expansion is the chain expansion of draft_tree, node for node (a draft
+    whose token depends on the configuration and the depth, given in both forms)."""
+    want = D.draft_tree(alphas, costs, a_dn, c_dn, k_max, t_min, m_max,
+                        lambda cfg, path, k: [_depth_token(cfg, len(path) + i) for i in range(k)])
+    got = D.draft_tree_topk(alphas, costs, a_dn, c_dn, k_max, t_min, m_max, 0.5,
+                            lambda cfg, path: [(_depth_token(cfg, len(path)), 0.37)])
+    assert got["parent"] == want["parent"] and got["token"] == want["token"] and got["cfg"] == want["cfg"]
+    assert got["p_acc"] == pytest.approx(want["p_acc"], rel=1e-12)
+    assert [st[:3] for st in got["steps"]] == want["steps"]
+    assert all(st[3] == [st[0]] for st in got["steps"])  # one branch: no siblings exist at K = 1
+
+
+@pytest.mark.parametrize("K,p_tree,m_max", [(2, 0.9, 24), (3, 0.6, 64), (4, 1.0, 40), (3, 0.2, 64)])
+def test_topk_tree_invariants(K, p_tree, m_max):
+    alphas, costs = [0.85, 0.7], [0.35, 0.15]
+    cands = _fake_cands(K)
+    tr = D.draft_tree_topk(alphas, costs, 0.5, 0.02, 3, 0.2, m_max, p_tree, cands)
+    par, tok, pacc, cfg = tr["parent"], tr["token"], tr["p_acc"], tr["cfg"]
+    n = len(par)
+    assert n <= m_max and par[0] == -1 and pacc[0] == 1.0
+
+    def path_to(v):
+        p = []
+        while v >= 0:
+            p.append(v)
+            v = par[v]
+        return p[::-1]
+
+    kids = {}
+    for i in range(1, n):
+        assert 0 <= par[i] < i
+        kids.setdefault(par[i], []).append(i)
+    for v, ch in kids.items():
+        # the children of a node are the kept prefix of its candidates, in rank order (each node
+        # receives candidates from one drafted position only)
+        pairs = cands(cfg[ch[0]], path_to(v))
+        kept = D.topp_keep([p for _, p in pairs], p_tree)
+        assert len(ch) <= len(kept)
+        if ch[-1] != n - 1:  # not cut by the size limit
+            assert len(ch) == len(kept)
+        for j, c in enumerate(ch):
+            assert tok[c] == pairs[j][0]
+            assert pacc[c] == pytest.approx(pacc[v] * alphas[cfg[c]] * kept[j], rel=1e-12)
+    for leaf, s, k, branches in tr["steps"]:
+        assert branches[0] == leaf
+        assert all(par[b] == par[leaf] for b in branches)  # the leaf and its siblings
+    if p_tree <= 1.0 / K:  # the top-1 alone reaches the mass: a chain per expansion, no siblings
+        assert all(len(ch) == 1 for ch in kids.values())

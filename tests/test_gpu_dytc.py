@@ -64,7 +64,7 @@ def test_dytc_rounds_are_lossless_and_learn_acceptance(cs):
     # in W8A8; a notional bottom draft (alpha 0.3, cost 0.05)
     cfgs = [(np.array([1, 0], dtype=np.uint8), 0), (None, 1)]
     sch = cs.Dytc([0.5, 0.5], [0.5, 0.6], alpha_dn=0.3, c_dn=0.05, k_max=4, t_min=0.5, m_max=16)
-    work = torch.zeros(5 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    work = torch.zeros(cs.DYTC_WORK, dtype=torch.int32, device="cuda")
     rounds = drafted = 0
     while len(out) < steps:
         toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work)
@@ -110,7 +110,7 @@ def test_dytc_rounds_with_prompt_lookup_bottom_draft_are_lossless(cs):
 
     cfgs = [(np.array([1, 0], dtype=np.uint8), 0), (None, 1), ("pld", 4)]
     sch = cs.Dytc([0.5, 0.5, 0.3], [0.5, 0.6, 0.02], alpha_dn=0.3, c_dn=0.02, k_max=4, t_min=0.5, m_max=16)
-    work = torch.zeros(5 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    work = torch.zeros(cs.DYTC_WORK, dtype=torch.int32, device="cuda")
     rounds = 0
     while len(out) < steps:
         toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work, history, hist_len)
@@ -130,3 +130,60 @@ def test_dytc_rounds_with_prompt_lookup_bottom_draft_are_lossless(cs):
     kv.close()
     dm.close()
 
+
+
+def test_dytc_rounds_with_top_k_siblings_are_lossless(cs):
+    """K = 3 candidates per drafted position with top-P 0.9 (Algorithm 1's tree expansion) and
+    sibling-parallel drafting, with the two model drafts and the prompt-lookup draft: the output
+    stays greedy decoding, and the trees branch."""
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    steps = 48
+    prefix = synth.prefix_tokens(SEED + 2, 64, SH.vocab)
+    truth, margins = _truth(prefix, steps)
+    dm = DeviceModel(SH, SEED, with_int8=True)
+    kv = DeviceKV(dm, 256)
+    n0 = len(prefix)
+    t = torch.tensor(np.asarray(prefix, dtype=np.int32), device="cuda")
+    p = torch.tensor(np.asarray(synth.chain(n0), dtype=np.int32), device="cuda")
+    logits = torch.empty(n0, SH.vocab, device="cuda")
+    cs.tree_step(dm.h, kv.h, t, p, n0, None, 0, logits)
+    cs.kv_compact(kv.h, torch.tensor([n0, *range(n0), 0], dtype=torch.int32, device="cuda"))
+    out = [int(torch.argmax(logits[-1]).item())]
+    history = torch.zeros(n0 + steps + 4 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    history[:n0] = t
+    history[n0] = out[0]
+    hist_len = n0 + 1
+
+    # the W8A8 draft starts as Algorithm 2's choice (Eq. 5: 10.3 against 9.75 for the prompt lookup);
+    # the tiny drafts' distributions are flat (normalised top-1 of three about 0.35), so its
+    # expansions keep all three candidates and the tree branches from the first position
+    cfgs = [(np.array([1, 0], dtype=np.uint8), 0), (None, 1), ("pld", 4)]
+    sch = cs.Dytc([0.6, 0.95, 0.3], [0.5, 0.1, 0.02], alpha_dn=0.3, c_dn=0.02, k_max=3, t_min=0.3, m_max=32,
+                  topk=3, p_tree=0.9)
+    work = torch.zeros(cs.DYTC_WORK, dtype=torch.int32, device="cuda")
+    dlog = torch.empty(cs.MAX_TREE, SH.vocab, device="cuda")
+    rounds = branched = 0
+    while len(out) < steps:
+        toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work, history, hist_len, dev_logits=dlog)
+        assert 1 <= len(toks) <= nd + 1
+        tr = sch.tree_get()
+        kids = np.bincount(np.asarray(tr["parent"][1:], dtype=np.int64), minlength=len(tr["parent"]))
+        branched += int(kids.max(initial=0) > 1)
+        history[hist_len:hist_len + len(toks)] = torch.tensor(toks, dtype=torch.int32, device="cuda")
+        hist_len += len(toks)
+        out.extend(toks)
+        rounds += 1
+    assert cs.get_status(dm.h) == 0
+    first_diff = next((i for i in range(steps) if out[i] != truth[i]), None)
+    if first_diff is not None:
+        assert min(margins[: first_diff + 1]) < MARGIN, (first_diff, out[:steps], truth[:steps])
+    assert branched > 0 and rounds < steps
+    P, T = cs.kv_length(kv.h)
+    assert T == 0 and P == n0 + len(out) - 1
+    # a round with K > 1 needs the logits buffer
+    with pytest.raises(cs.CasspecError):
+        sch.round(dm.h, kv.h, cfgs, out[-1], work, history, hist_len)
+    sch.close()
+    kv.close()
+    dm.close()
