@@ -292,6 +292,20 @@ def draft_tree_topk(alphas: list[float], costs: list[float], a_dn: float, c_dn: 
     return out()
 
 
+def vc_accept(proposals: list[int], argmax: list[int]) -> list[int]:
+    """One holistic round of the vertical cascade VC(d_i, d_n) (Sec. 4.2: its draft length follows
+    from how many low-level tokens d_i accepts): d_n proposed `proposals` below the leaf; d_i's
+    greedy choices are argmax[0] at the leaf and argmax[r] after the r-th proposal.  Returns d_i's
+    drafted tokens: the proposals it accepts in order, then its own next token."""
+    out = []
+    for r, q in enumerate(proposals):
+        if q != argmax[r]:
+            break
+        out.append(q)
+    out.append(argmax[len(out)])
+    return out
+
+
 # ------------------------------------------------------------------------------------------------
 # Sec. 4.2: latency model (Bayesian linear regression)
 # ------------------------------------------------------------------------------------------------

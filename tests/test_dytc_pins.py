@@ -311,3 +311,33 @@ def test_topk_tree_invariants(K, p_tree, m_max):
         assert all(par[b] == par[leaf] for b in branches)  # the leaf and its siblings
     if p_tree <= 1.0 / K:  # the top-1 alone reaches the mass: a chain per expansion, no siblings
         assert all(len(ch) == 1 for ch in kids.values())
+
+
+# ------------------------------------------------------------------------------------------------
+# Sec. 4.2 vertical cascade VC(d_i, d_n) as one holistic round
+# ------------------------------------------------------------------------------------------------
+def test_vc_accept_hand_cases():
+    assert D.vc_accept([], [7]) == [7]  # nothing proposed: d_i drafts one token
+    assert D.vc_accept([5, 6, 9], [5, 6, 8, 1]) == [5, 6, 8]  # two accepted, then d_i's correction
+    assert D.vc_accept([5, 6, 9], [5, 6, 9, 4]) == [5, 6, 9, 4]  # all accepted plus d_i's next token
+    assert D.vc_accept([3, 6], [5, 6, 2]) == [5]  # the first rejected: later matches do not count
+
+
+def test_vc_accept_equals_greedy_chain_prefix():
+    """Whatever d_n proposes, the round's tokens are a prefix of d_i's own greedy chain: brute force
+    over proposals against a fixed greedy continuation g (d_i's argmax after g[:r] is g[r])."""
+    import itertools
+
+    g = [4, 1, 3, 3, 0]
+    for j in range(4):
+        for prop in itertools.product(range(5), repeat=j):
+            # d_i's argmax after each proposal prefix: g continues only while the proposals follow g
+            am, ok = [], True
+            for r in range(j + 1):
+                am.append(g[r] if ok else (r * 7 + 2) % 5)
+                ok = ok and r < j and prop[r] == g[r]
+            got = D.vc_accept(list(prop), am)
+            a = 0
+            while a < j and prop[a] == g[a]:
+                a += 1
+            assert got == g[:a + 1]
