@@ -416,14 +416,26 @@ CASSPEC_API int casspec_pld_draft(const int32_t* tokens, int L, int n_min, int n
 CASSPEC_API int casspec_topk(const float* logits, int n, int V, int K, int32_t* idx_out, float* prob_out,
                              void* cuda_stream);
 
-/* A draft configuration: a DSIA draft of the model (Sec. 4.1), with its layer mask and GEMM mode as
- * for casspec_tree_step (skip_mask host uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16,
- * 1 W8A8), or, when pld_n_max > 0, the prompt-lookup bottom draft (casspec_pld_draft with n in
- * [1, pld_n_max] over the committed history and the path to the leaf). */
+/* One holistic round of the vertical cascade VC(d_i, d_n) (Sec. 4.2; its draft length depends on how
+ * many low-level tokens are accepted): d_n proposed proposals[j] (host) below a leaf, and d_i's greedy
+ * choices are argmax[0] at the leaf and argmax[r] after the r-th proposal (host [j + 1]).  out (host
+ * [j + 1]) receives the proposals d_i accepts, in order up to the first mismatch, then d_i's own next
+ * token.  Returns their count (1 .. j + 1) or E_INVAL. */
+CASSPEC_API int casspec_vc_accept(const int32_t* proposals, int j, const int32_t* argmax, int32_t* out);
+
+/* A draft configuration (Sec. 4.1), one of:
+ *   - a DSIA draft of the model: layer mask and GEMM mode as for casspec_tree_step (skip_mask host
+ *     uint8 [n_layers], NULL = all layers on; quant_mode 0 bf16, 1 W8A8), pld_n_max = 0;
+ *   - the prompt-lookup bottom draft: pld_n_max > 0, vc = 0 (casspec_pld_draft with n in
+ *     [1, pld_n_max] over the committed history and the path to the leaf);
+ *   - the vertical cascade VC(model draft, prompt lookup): pld_n_max > 0, vc != 0; the prompt lookup
+ *     proposes up to k tokens below the leaf and the model draft checks them in one tree step
+ *     (casspec_vc_accept).  Its acceptance estimate is that of the model draft's tokens (App. D). */
 typedef struct {
   const uint8_t* skip_mask;
   int quant_mode;
   int pld_n_max;
+  int vc;
 } casspec_draft_cfg;
 
 /* One round of DyTC speculative decoding (Sec. 4.2: Algorithm 1, then verification by the target).
@@ -443,8 +455,10 @@ typedef struct {
  *   recorded (the first drafted token's outcome), and the estimates are updated (casspec_dytc_end_step).
  *   A prompt-lookup configuration drafts from history (dev int32, the committed tokens, the last
  *   being root_token; hist_len entries, room for CASSPEC_MAX_TREE more, which the round overwrites);
- *   finding no earlier occurrence counts as a rejected first token and ends the drafting.  history
- *   may be NULL when no configuration is a prompt lookup.
+ *   finding no earlier occurrence counts as a rejected first token and ends the drafting.  A vertical
+ *   cascade configuration runs its model draft once over root .. leaf plus the lookup's proposals
+ *   (none when nothing matches) and appends the tokens casspec_vc_accept gives.  history may be NULL
+ *   when no configuration uses the prompt lookup.
  *   dev_work: device int32 [CASSPEC_DYTC_WORK] (caller-owned scratch).  out_tokens (host int32
  *   [CASSPEC_MAX_TREE]) receives the tokens this round commits after the root, the last being the
  *   bonus token (the next root); *n_out their count (>= 1); *n_drafted_out (may be NULL) the drafted

@@ -36,7 +36,7 @@ EXPORTS = [
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
     "casspec_dytc_destroy", "casspec_dytc_get_params", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_begin", "casspec_dytc_tree_add", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft", "casspec_topk",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_begin", "casspec_dytc_tree_add", "casspec_vc_accept", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft", "casspec_topk",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -55,7 +55,8 @@ class DytcParams(ctypes.Structure):
 
 
 class DraftCfg(ctypes.Structure):
-    _fields_ = [("skip_mask", ctypes.c_void_p), ("quant_mode", ctypes.c_int32), ("pld_n_max", ctypes.c_int32)]
+    _fields_ = [("skip_mask", ctypes.c_void_p), ("quant_mode", ctypes.c_int32), ("pld_n_max", ctypes.c_int32),
+                ("vc", ctypes.c_int32)]
 
 
 class CasspecError(RuntimeError):
@@ -96,6 +97,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_reset": (_I, [_P]),
         "casspec_dytc_tree_plan": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_extend": (_I, [_P, _I, _I, _I, ctypes.POINTER(ctypes.c_int32)]),
+        "casspec_vc_accept": (_I, [ctypes.POINTER(ctypes.c_int32), _I, ctypes.POINTER(ctypes.c_int32),
+                                   ctypes.POINTER(ctypes.c_int32)]),
         "casspec_dytc_tree_begin": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(_I)]),
         "casspec_dytc_tree_add": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_float), _I]),
         "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
@@ -342,6 +345,18 @@ def dytc_objective(alpha: float, c: float, k: int, alpha_dn: float, c_dn: float)
     return load_library().casspec_dytc_objective(alpha, c, k, alpha_dn, c_dn)
 
 
+def vc_accept(proposals, argmax) -> list[int]:
+    """casspec_vc_accept: d_i's drafted tokens of one vertical-cascade round (host lists)."""
+    j = len(proposals)
+    p = (ctypes.c_int32 * max(j, 1))(*[int(x) for x in proposals])
+    a = (ctypes.c_int32 * (j + 1))(*[int(x) for x in argmax[: j + 1]])
+    out = (ctypes.c_int32 * (j + 1))()
+    rc = load_library().casspec_vc_accept(p, j, a, out)
+    if rc < 0:
+        raise CasspecError("casspec_vc_accept", rc)
+    return list(out[:rc])
+
+
 def pld_draft(tokens, L: int, n_min: int, n_max: int, k: int, out, stream=None) -> None:
     """casspec_pld_draft: tokens dev int32 [L], out dev int32 [2 + k] = {match length, count, tokens}."""
     _check("casspec_pld_draft", load_library().casspec_pld_draft(_ptr(tokens), L, n_min, n_max, k, _ptr(out),
@@ -362,6 +377,25 @@ def latency_fit(x, y, mu0, sd0, noise_sd: float) -> tuple[list[float], list[floa
     w, cov = (_D * 2)(), (_D * 4)()
     _check("casspec_latency_fit", load_library().casspec_latency_fit(xa, ya, m, mu, sd, float(noise_sd), w, cov))
     return list(w), list(cov)
+
+
+def draft_cfgs(cfgs):
+    """casspec_draft_cfg array for casspec_dytc_round, and the mask arrays it points into (keep them
+    alive for the call).  Each entry: (skip_mask or None, quant_mode) for a model draft,
+    ("pld", n_max) for the prompt lookup, ("vc", skip_mask or None, quant_mode, n_max) for the
+    vertical cascade of that model draft over the prompt lookup."""
+    masks, items = [], []
+    for cfg in cfgs:
+        kind = cfg[0] if isinstance(cfg[0], str) else None
+        if kind == "pld":
+            masks.append(None)
+            items.append(DraftCfg(None, 0, int(cfg[1]), 0))
+            continue
+        a, b, n_vc = (cfg[1], cfg[2], int(cfg[3])) if kind == "vc" else (cfg[0], cfg[1], 0)
+        mk = None if a is None else np.ascontiguousarray(np.asarray(a, dtype=np.uint8))
+        masks.append(mk)
+        items.append(DraftCfg(None if mk is None else mk.ctypes.data, int(b), n_vc, int(n_vc > 0)))
+    return (DraftCfg * len(items))(*items), masks
 
 
 class Dytc:
@@ -455,21 +489,13 @@ class Dytc:
     def round(self, m: int, kv: int, cfgs, root_token: int, dev_work, history=None, hist_len: int = 0,
               dev_logits=None) -> tuple[list[int], int]:
         """One DyTC round (casspec_dytc_round).  cfgs: per configuration (skip_mask or None, quant_mode)
-        for a model draft, or ("pld", n_max) for the prompt-lookup draft; history: torch int32 CUDA
+        for a model draft, ("pld", n_max) for the prompt-lookup draft, or ("vc", skip_mask, quant_mode,
+        n_max) for the vertical cascade of that model draft over the prompt lookup; history: torch int32 CUDA
         tensor of the committed tokens (hist_len valid, the last = root_token, room for MAX_TREE more);
         dev_work: torch int32 CUDA tensor of DYTC_WORK entries; dev_logits: torch fp32 CUDA tensor of
         MAX_TREE x vocab (needed when topk > 1).  Returns the committed tokens (the last is the bonus
         token) and the number of drafted nodes."""
-        masks, items = [], []
-        for a, b in cfgs:
-            if isinstance(a, str):
-                masks.append(None)
-                items.append(DraftCfg(None, 0, int(b)))
-            else:
-                mk = None if a is None else np.ascontiguousarray(np.asarray(a, dtype=np.uint8))
-                masks.append(mk)
-                items.append(DraftCfg(None if mk is None else mk.ctypes.data, int(b), 0))
-        arr = (DraftCfg * len(items))(*items)
+        arr, masks = draft_cfgs(cfgs)
         out = (ctypes.c_int32 * MAX_TREE)()
         n, nd = _I(), _I()
         _check("casspec_dytc_round", load_library().casspec_dytc_round(self.h, m, kv, arr, int(root_token), _ptr(history),

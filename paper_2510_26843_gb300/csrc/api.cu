@@ -1108,6 +1108,44 @@ extern "C" int casspec_dytc_round(casspec_dytc* s, casspec_model* m, casspec_kv*
       ctok[i] = tok[chain[len - 1 - i]];
       cpar[i] = i - 1;
     }
+    if (cfgs[c].pld_n_max > 0 && cfgs[c].vc) {
+      // the vertical cascade VC(model draft, prompt lookup), one holistic round: the lookup proposes
+      // up to k tokens after history + path, the model draft runs once over root .. leaf plus the
+      // proposals (a chain), and its greedy prefix match plus its own next token are appended
+      if (history == nullptr || hist_len < 1) return CASSPEC_E_INVAL;
+      const int kq = std::min(k, kMaxTree - len);
+      int j = 0;
+      int32_t pr[kMaxTree + 2];
+      if (kq > 0) {
+        if (len > 1)
+          CK(cudaMemcpyAsync(history + hist_len, ctok + 1, (size_t)(len - 1) * 4, cudaMemcpyHostToDevice, m->stream));
+        if ((rc = casspec_pld_draft(history, hist_len + len - 1, 1, cfgs[c].pld_n_max, kq, d_pld, m->stream)) !=
+            CASSPEC_OK)
+          return rc;
+        if ((rc = read_dev_i32(m, d_pld, 2 + kq, pr)) != CASSPEC_OK) return rc;
+        j = std::min(std::max(pr[1], 0), kq);
+      }
+      for (int i = 0; i < j; ++i) {
+        ctok[len + i] = pr[2 + i];
+        cpar[len + i] = len + i - 1;
+      }
+      casspec_kv_reset_tree(kv);
+      CK(cudaMemcpyAsync(d_tok, ctok, (size_t)(len + j) * 4, cudaMemcpyHostToDevice, m->stream));
+      CK(cudaMemcpyAsync(d_par, cpar, (size_t)(len + j) * 4, cudaMemcpyHostToDevice, m->stream));
+      if ((rc = casspec_tree_step(m, kv, d_tok, d_par, len + j, cfgs[c].skip_mask, cfgs[c].quant_mode, nullptr)) !=
+          CASSPEC_OK)
+        return rc;
+      int32_t am[kMaxTree + 1], drafted[kMaxTree + 1];
+      if ((rc = read_dev_i32(m, d_am + (len - 1), j + 1, am)) != CASSPEC_OK) return rc;
+      const int cnt = casspec_vc_accept(pr + 2, j, am, drafted);
+      if (cnt < 0) return cnt;
+      const int first = n;
+      rc = casspec_dytc_tree_extend(s, leaf, c, cnt, drafted);
+      if (rc < 0) return rc;
+      if (rc > 0) exps.push_back({leaf, c, first});
+      if (rc < cnt) break;  // the tree is full
+      continue;
+    }
     if (cfgs[c].pld_n_max > 0) {
       // the prompt-lookup bottom draft: the path below the root continues the committed history
       if (history == nullptr || hist_len < 1) return CASSPEC_E_INVAL;

@@ -264,6 +264,17 @@ int casspec_dytc_tree_add(casspec_dytc* s, int node, int cfg, const int32_t* tok
   return n0;  // the top-1 child
 }
 
+int casspec_vc_accept(const int32_t* proposals, int j, const int32_t* argmax, int32_t* out) {
+  if (j < 0 || (j > 0 && proposals == nullptr) || argmax == nullptr || out == nullptr) return CASSPEC_E_INVAL;
+  int a = 0;
+  while (a < j && proposals[a] == argmax[a]) {
+    out[a] = proposals[a];
+    ++a;
+  }
+  out[a] = argmax[a];  // d_i's own next token after the accepted prefix
+  return a + 1;
+}
+
 int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out, int32_t* token_out, int32_t* cfg_out,
                           double* p_acc_out) {
   if (s == nullptr || n_out == nullptr) return CASSPEC_E_INVAL;

@@ -264,3 +264,23 @@ def test_topk_tree_argument_errors(cs):
     assert sch.tree_add(1, 0, [8, 9], [0.95, 0.05]) == 4
     assert sch.tree_get()["parent"] == [-1, 0, 0, 0, 1]  # 0.95 reaches 0.9: the second is dropped
     sch.close()
+
+
+def test_vc_accept_matches_oracle(cs):
+    r = _rng(900)
+    for _ in range(500):
+        j = r.randint(0, 6)
+        g = [r.randint(0, 4) for _ in range(j + 1)]
+        prop = [g[i] if r.random() < 0.7 else r.randint(0, 4) for i in range(j)]
+        assert cs.vc_accept(prop, g) == D.vc_accept(prop, g)
+    assert cs.load_library().casspec_vc_accept(None, -1, None, None) == cs.E_INVAL
+
+
+def test_draft_cfg_marshalling(cs):
+    import numpy as np
+
+    mask = np.array([1, 0, 1], dtype=np.uint8)
+    arr, keep = cs.draft_cfgs([(mask, 0), (None, 1), ("pld", 4), ("vc", mask, 1, 3), ("vc", None, 0, 2)])
+    got = [(a.skip_mask is not None, a.quant_mode, a.pld_n_max, a.vc) for a in arr]
+    assert got == [(True, 0, 0, 0), (False, 1, 0, 0), (False, 0, 4, 0), (True, 1, 3, 1), (False, 0, 2, 1)]
+    assert arr[0].skip_mask == keep[0].ctypes.data and list(keep[3]) == [1, 0, 1]

@@ -187,3 +187,68 @@ def test_dytc_rounds_with_top_k_siblings_are_lossless(cs):
     sch.close()
     kv.close()
     dm.close()
+
+
+def test_dytc_rounds_with_vertical_cascade(cs):
+    """VC(first-layer draft, prompt lookup) as a configuration (Sec. 4.2: one holistic round per
+    expansion): every node it drafts is the first-layer draft's own greedy token at its parent
+    (checked against the oracle's draft, except at near-ties), and the output stays greedy decoding.
+    The prefix repeats a 16-token segment so that the lookup has matches to propose."""
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    steps = 40
+    seg = synth.prefix_tokens(SEED + 3, 16, SH.vocab)
+    prefix = np.concatenate([seg] * 4)
+    truth, margins = _truth(prefix, steps)
+    ow = oracle.Weights.from_seed(SEED, SH, keep_layers=SH.n_layers)
+    dm = DeviceModel(SH, SEED, with_int8=True)
+    kv = DeviceKV(dm, 256)
+    n0 = len(prefix)
+    t = torch.tensor(np.asarray(prefix, dtype=np.int32), device="cuda")
+    p = torch.tensor(np.asarray(synth.chain(n0), dtype=np.int32), device="cuda")
+    logits = torch.empty(n0, SH.vocab, device="cuda")
+    cs.tree_step(dm.h, kv.h, t, p, n0, None, 0, logits)
+    cs.kv_compact(kv.h, torch.tensor([n0, *range(n0), 0], dtype=torch.int32, device="cuda"))
+    out = [int(torch.argmax(logits[-1]).item())]
+    history = torch.zeros(n0 + steps + 4 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    history[:n0] = t
+    history[n0] = out[0]
+    hist_len = n0 + 1
+
+    d1 = np.array([1, 0], dtype=np.uint8)
+    cfgs = [("vc", d1, 0, 4), (None, 1)]
+    # Eq. 5 picks the cascade with k = 3 at these estimates
+    sch = cs.Dytc([0.8, 0.9], [0.2, 0.6], alpha_dn=0.3, c_dn=0.3, k_max=4, t_min=0.3, m_max=24)
+    assert sch.best_config()[:2] == (0, 3)
+    work = torch.zeros(cs.DYTC_WORK, dtype=torch.int32, device="cuda")
+    rounds = checked = 0
+    while len(out) < steps:
+        committed, root = list(prefix) + out[:-1], out[-1]
+        toks, nd = sch.round(dm.h, kv.h, cfgs, root, work, history, hist_len)
+        tr = sch.tree_get()
+        vc_nodes = [v for v in range(1, len(tr["parent"])) if tr["cfg"][v] == 0]
+        if vc_nodes:
+            okv = oracle.KVCache(SH.n_layers, SH.n_heads, SH.head_dim, 256)
+            oracle.tree_step(ow, okv, committed, synth.chain(len(committed)), skip_mask=d1)
+            oracle.kv_compact(okv, list(range(len(committed))))
+            ttoks = [root] + tr["token"][1:]
+            lg = oracle.tree_step(ow, okv, ttoks, tr["parent"], skip_mask=d1)
+            am, mg = oracle.argmax_lowest(lg), oracle.top2_margin(lg)
+            for v in vc_nodes:
+                if mg[tr["parent"][v]] >= MARGIN:
+                    assert tr["token"][v] == am[tr["parent"][v]], (rounds, v)
+                    checked += 1
+        history[hist_len:hist_len + len(toks)] = torch.tensor(toks, dtype=torch.int32, device="cuda")
+        hist_len += len(toks)
+        out.extend(toks)
+        rounds += 1
+    assert cs.get_status(dm.h) == 0
+    first_diff = next((i for i in range(steps) if out[i] != truth[i]), None)
+    if first_diff is not None:
+        assert min(margins[: first_diff + 1]) < MARGIN, (first_diff, out[:steps], truth[:steps])
+    assert checked > 0 and rounds < steps
+    P, T = cs.kv_length(kv.h)
+    assert T == 0 and P == n0 + len(out) - 1
+    sch.close()
+    kv.close()
+    dm.close()
