@@ -364,7 +364,8 @@ CASSPEC_API int casspec_dytc_best_config(const casspec_dytc* s, int* cfg_out, in
  * configuration recorded since the previous end of round; the others keep their estimate (App. D). */
 CASSPEC_API int casspec_dytc_record(casspec_dytc* s, int cfg, int accepted);
 CASSPEC_API int casspec_dytc_end_step(casspec_dytc* s);
-/* Algorithm 1 (Sec. 4.2) with one drafted token per position, driven by the caller:
+/* Algorithm 1 (Sec. 4.2), driven by the caller (one drafted token per position here; K candidates per
+ * position with casspec_dytc_tree_begin / casspec_dytc_tree_add below):
  *   casspec_dytc_tree_reset: the tree holds the root (node 0: the last committed token), P_acc = 1;
  *   casspec_dytc_tree_plan: returns 1 with the active leaf of highest P_acc (lowest index on ties),
  *     the configuration and k of Algorithm 2; returns 0 (stop) when the tree holds m_max nodes, no

@@ -20,10 +20,13 @@ What it computes (CAS-Spec, arXiv 2510.26843):
       T_s(S, k) = (E_acc + a_S^k a_dn) / (c_S k + c_dn),  E_acc = a_S (1 - a_S^k) / (1 - a_S)
     (E_acc = k when a_S is 1), the local speedup of the step plus the least future speedup of the
     bottom draft d_n;
-  * Sec. 4.2 Algorithm 1 (draft tree generation) with one token per drafted position (K = 1): expand
-    the active leaf with the highest accumulated acceptance P_acc, stop when
-    a_dn / c_dn * P_acc < t_min or the tree holds m_max nodes, choose (S, k) by Algorithm 2, append
-    the k drafted tokens below the leaf with P_acc(child) = P_acc(parent) * a_S.
+  * Sec. 4.2 Algorithm 1 (draft tree generation): expand the active leaf with the highest
+    accumulated acceptance P_acc, stop when a_dn / c_dn * P_acc < t_min or the tree holds m_max
+    nodes, choose (S, k) by Algorithm 2; with one token per drafted position (K = 1, `draft_tree`)
+    append the k drafted tokens below the leaf with P_acc(child) = P_acc(parent) * a_S; with K
+    candidates per position and sibling-parallel drafting, `draft_tree_topk` (readings below);
+  * Sec. 4.2 vertical cascade VC(d_i, d_n) as one holistic round (`vc_accept`): d_i's drafted tokens
+    are the low-level proposals it accepts in order, then its own next token.
 
   * Sec. 4.2, the hardware-aware latency prediction behind the cost coefficients: a Bayesian linear
     regression of step latency on the bytes the step moves (a roofline: latency = w0 + w1 * bytes),
