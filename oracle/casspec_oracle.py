@@ -14,9 +14,11 @@ What it computes (CAS-Spec, arXiv 2510.26843):
     layer is the identity on the residual stream and writes no K/V; the same at the granularity of
     a layer's attention or FFN sub-block (Sec. 4.1 names both granularities): a skipped attention
     block adds nothing to the residual stream and writes no K/V, a skipped FFN block adds nothing;
-  * DSIA activation quantisation (Sec. 4.1 and App. C, QSpec-style W?A? drafts): here W8A8, per
-    output channel symmetric int8 weights and per-token dynamic symmetric int8 activations on the
-    inputs of Wqkv, Wo, Wgate/Wup and Wdown; attention, K/V and the LM head stay in floating point;
+  * DSIA activation quantisation (Sec. 4.1 and App. C, QSpec-style W?A? drafts): W8A8 and W4A4,
+    per output channel symmetric weights and per-token dynamic symmetric activations on the inputs
+    of Wqkv, Wo, Wgate/Wup and Wdown; attention, K/V and the LM head stay in floating point;
+  * DSIA activation sparsity (Sec. 4.1 and App. C, TEAL): the smallest-magnitude share of each
+    projection input is zeroed per token;
   * lossless greedy verification (Sec. 5.1: output identical to autoregressive decoding): the
     longest root-to-leaf path whose tokens equal the target's argmax, plus the bonus token;
   * compaction of the accepted path's K/V into the committed cache.
@@ -82,33 +84,49 @@ def silu(x: np.ndarray) -> np.ndarray:
 # ----------------------------------------------------------------------------------------------
 
 
-def quantize_rows_f32(x: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
-    """Symmetric per-row int8 quantisation evaluated in fp32.
+def quantize_rows_f32(x: np.ndarray, qmax: int = 127) -> tuple[np.ndarray, np.ndarray]:
+    """Symmetric per-row quantisation evaluated in fp32 (qmax 127: int8; 7: int4).
 
     x: fp32 rows [r, c] (bf16 inputs widened exactly).  Returns (q int8 [r, c], scale fp32 [r]).
-    inv = 127 / amax (fp32 division), t = x * inv (fp32 multiply), q = rint(t) (ties to even),
-    clamp to +-127; scale = amax / 127 (fp32 division).  amax = 0 -> q = 0, scale = 0.
+    inv = qmax / amax (fp32 division), t = x * inv (fp32 multiply), q = rint(t) (ties to even),
+    clamp to +-qmax; scale = amax / qmax (fp32 division).  amax = 0 -> q = 0, scale = 0.
     """
     x = np.asarray(x, dtype=np.float32)
+    qm = np.float32(qmax)
     amax = np.max(np.abs(x), axis=-1)
     safe = np.where(amax > 0, amax, np.float32(1.0)).astype(np.float32)
-    inv = (np.float32(127.0) / safe).astype(np.float32)
+    inv = (qm / safe).astype(np.float32)
     t = (x * inv[:, None]).astype(np.float32)
-    q = np.clip(np.rint(t), -127, 127).astype(np.int8)
+    q = np.clip(np.rint(t), -qmax, qmax).astype(np.int8)
     q[amax == 0] = 0
-    scale = np.where(amax > 0, (amax / np.float32(127.0)).astype(np.float32), np.float32(0.0)).astype(np.float32)
+    scale = np.where(amax > 0, (amax / qm).astype(np.float32), np.float32(0.0)).astype(np.float32)
     return q, scale
 
 
-def quantize_rows_f64(x: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+def quantize_rows_f64(x: np.ndarray, qmax: int = 127) -> tuple[np.ndarray, np.ndarray]:
     """The same rule evaluated in fp64 (end-to-end oracle activations)."""
     x = np.asarray(x, dtype=np.float64)
     amax = np.max(np.abs(x), axis=-1)
     safe = np.where(amax > 0, amax, 1.0)
-    q = np.clip(np.rint(x * (127.0 / safe)[:, None]), -127, 127).astype(np.int8)
+    q = np.clip(np.rint(x * (qmax / safe)[:, None]), -qmax, qmax).astype(np.int8)
     q[amax == 0] = 0
-    scale = np.where(amax > 0, amax / 127.0, 0.0)
+    scale = np.where(amax > 0, amax / qmax, 0.0)
     return q, scale
+
+
+def sparsify_rows(x: np.ndarray, s: float) -> np.ndarray:
+    """Activation sparsity by magnitude (the TEAL DSIA of App. C): per row of length K, the
+    floor(s * K) entries of smallest magnitude become 0 and the others are kept; among equal
+    magnitudes the lower index is kept."""
+    x = np.array(x, dtype=np.float64, copy=True)
+    K = x.shape[-1]
+    z = int(math.floor(s * K + 1e-9))
+    if z <= 0:
+        return x
+    for r in range(x.shape[0]):
+        order = sorted(range(K), key=lambda c: (-abs(x[r, c]), c))
+        x[r, order[K - z:]] = 0.0
+    return x
 
 
 def linear_w8a8(qx: np.ndarray, sx: np.ndarray, qw: np.ndarray, sw: np.ndarray) -> np.ndarray:
@@ -168,8 +186,12 @@ class Weights:
 
     def int8(self, name: str, layer: int) -> tuple[np.ndarray, np.ndarray]:
         """Per-output-channel int8 weights and fp32 scales (quantize_rows_f32 of the bf16 rows)."""
-        return self._cached(("i8", layer, name),
-                            lambda: quantize_rows_f32(synth.bf16_to_f32(self.bits(name, layer))))
+        return self.intq(name, layer, 127)
+
+    def intq(self, name: str, layer: int, qmax: int) -> tuple[np.ndarray, np.ndarray]:
+        """Per-output-channel weights with codes in [-qmax, qmax] (127: int8, 7: int4) and scales."""
+        return self._cached((f"i{qmax}", layer, name),
+                            lambda: quantize_rows_f32(synth.bf16_to_f32(self.bits(name, layer)), qmax))
 
     def gain(self, name: str, layer: int = -1) -> np.ndarray:
         return np.asarray(self._gain(name, layer), dtype=np.float64)
@@ -253,12 +275,20 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
     return u.view(np.float32)
 
 
-def _linear(x: np.ndarray, w: Weights, name: str, layer: int, quant: bool) -> np.ndarray:
-    if quant:
+QMAX = {1: 127, 2: 7}  # quant_mode -> largest code: W8A8, W4A4
+
+
+def _linear(x: np.ndarray, w: Weights, name: str, layer: int, lin: tuple) -> np.ndarray:
+    """One projection of a draft: lin = (quant_mode, activation sparsity).  The sparsity rule
+    applies to the projection's input first; a quantised mode then quantises that input."""
+    mode, sparsity = lin
+    if sparsity > 0.0:
+        x = sparsify_rows(x, sparsity)
+    if mode in QMAX:
         # The quantiser's integer decisions are taken on the activation as the draft stores it
         # (bf16) with the fp32 rule, i.e. in the kernel's precision.
-        qx, sx = quantize_rows_f32(round_bf16(x))
-        qw, sw = w.int8(name, layer)
+        qx, sx = quantize_rows_f32(round_bf16(x), QMAX[mode])
+        qw, sw = w.intq(name, layer, QMAX[mode])
         return linear_w8a8(qx, sx, qw, sw)
     return x @ w.f64(name, layer).T
 
@@ -307,14 +337,17 @@ def layer_blocks(code: int) -> tuple[bool, bool]:
 
 def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
               skip_mask: np.ndarray | None = None, quant_mode: int = 0,
-              trace: dict | None = None, attn_bf16: bool = False) -> np.ndarray:
+              trace: dict | None = None, attn_bf16: bool = False, act_sparsity: float = 0.0) -> np.ndarray:
     """One draft/verify pass over n new tree nodes; returns logits [n, V] (fp64).
 
     The nodes occupy tree slots T .. T+n-1 (cache slots P+T .. P+T+n-1); each active layer writes
     their K/V there.  skip_mask[l] == 0 switches layer l off (Sec. 4.1 layer sparsity); a non-zero
     byte keeps it on except for the sub-blocks whose flag it carries: SKIP_ATTN (the attention
     block: no residual update, no K/V written) and SKIP_FFN (the FFN block).
-    quant_mode 1 runs the W8A8 draft (App. C).  `trace`, if given, receives per-layer intermediates.
+    quant_mode 1 runs the W8A8 draft, 2 the W4A4 draft (App. C: QSpec's bit width; codes +-7 with the
+    same rule); act_sparsity s > 0 zeroes the floor(s K) smallest-magnitude inputs of every projection
+    (App. C: TEAL activation sparsity), before any quantisation.  `trace`, if given, receives
+    per-layer intermediates.
     attn_bf16 rounds q and the K/V written to the cache to bf16 (a bf16 cache and bf16 attention
     operands).  It is a perturbation of the size of bf16 storage, used by tests to measure how far
     the method's own output moves under it; the reference result keeps it off.
@@ -330,18 +363,20 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
     slots = [kv.P + kv.T + i for i in range(n)]
     all_anc = kv.anc + anc
     mask = np.ones(sh.n_layers, dtype=np.uint8) if skip_mask is None else np.asarray(skip_mask)
-    quant = quant_mode == 1
+    if quant_mode not in (0, 1, 2) or not 0.0 <= act_sparsity < 1.0:
+        raise ValueError("quant_mode must be 0, 1 or 2 and act_sparsity in [0, 1)")
+    lin = (quant_mode, float(act_sparsity))
 
     x = w.f64("embed")[tokens]  # [n, d]
     for l in range(sh.n_layers):
         attn_on, ffn_on = layer_blocks(mask[l])
         if attn_on:
-            x = _attention_block(x, w, kv, l, quant, pos, slots, all_anc, n, attn_bf16, trace)
+            x = _attention_block(x, w, kv, l, lin, pos, slots, all_anc, n, attn_bf16, trace)
         if ffn_on:
             xn2 = rmsnorm(x, w.gain("ffn_norm", l), sh.rms_eps)
-            g = _linear(xn2, w, "wg", l, quant)
-            u = _linear(xn2, w, "wu", l, quant)
-            x = x + _linear(silu(g) * u, w, "wd", l, quant)
+            g = _linear(xn2, w, "wg", l, lin)
+            u = _linear(xn2, w, "wu", l, lin)
+            x = x + _linear(silu(g) * u, w, "wd", l, lin)
         if trace is not None and (attn_on or ffn_on):
             trace.setdefault(l, {})["x"] = x.copy()
     xf = rmsnorm(x, w.gain("final_norm"), sh.rms_eps)
@@ -352,13 +387,13 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
     return logits
 
 
-def _attention_block(x, w, kv, l, quant, pos, slots, all_anc, n, attn_bf16, trace):
+def _attention_block(x, w, kv, l, lin, pos, slots, all_anc, n, attn_bf16, trace):
     """x + Wo . TreeAttention(RoPE(Wq xn), RoPE(Wk xn), Wv xn) with xn = RMSNorm(x); writes the
     nodes' K/V of layer l."""
     sh = w.shape
     d, H, h = sh.d_model, sh.n_heads, sh.head_dim
     xn = rmsnorm(x, w.gain("attn_norm", l), sh.rms_eps)
-    qkv = _linear(xn, w, "wqkv", l, quant)
+    qkv = _linear(xn, w, "wqkv", l, lin)
     q = rope(qkv[:, :d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
     k = rope(qkv[:, d:2 * d].reshape(n, H, h).transpose(1, 0, 2), pos, sh.rope_base).transpose(1, 0, 2)
     v = qkv[:, 2 * d:].reshape(n, H, h)
@@ -371,7 +406,7 @@ def _attention_block(x, w, kv, l, quant, pos, slots, all_anc, n, attn_bf16, trac
     o = tree_attention(q, kv, l, slots, [all_anc[kv.T + i] for i in range(n)]).reshape(n, d)
     if trace is not None:
         trace[l] = {"xn": xn, "q": q, "k": k, "v": v, "o": o}
-    return x + _linear(o, w, "wo", l, quant)
+    return x + _linear(o, w, "wo", l, lin)
 
 
 # ----------------------------------------------------------------------------------------------

@@ -129,6 +129,51 @@ def test_quantizer_properties_random():
     assert np.all(np.abs(q - x / s[:, None].astype(np.float64)) <= 0.5 + 1e-4)
 
 
+def test_int4_quantizer_golden_rows_and_properties():
+    for line in open(os.path.join(GOLDEN, "quant4_rows.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        xs, qs = line.split("|")
+        x = np.array([[float(v) for v in xs.split()]], dtype=np.float32)
+        want = [int(v) for v in qs.split()]
+        for fn in (oracle.quantize_rows_f32, oracle.quantize_rows_f64):
+            q, s = fn(x, 7)
+            assert q[0].tolist() == want
+            assert s[0] == float(np.max(np.abs(x))) / 7
+    rng = np.random.default_rng(13)
+    x = (rng.standard_normal((40, 200)) * rng.uniform(0.01, 10, (40, 1))).astype(np.float32)
+    q, s = oracle.quantize_rows_f32(x, 7)
+    i = np.argmax(np.abs(x), axis=1)
+    assert np.all(np.abs(q[np.arange(40), i]) == 7) and np.abs(q).max() == 7
+    assert np.all(np.abs(q - x / s[:, None].astype(np.float64)) <= 0.5 + 1e-5)
+
+
+def test_sparsify_rows_bruteforce():
+    """The floor(s K) smallest magnitudes become 0 (ties: the higher index goes first), checked against
+    a plain selection loop on rows with many ties."""
+    rng = np.random.default_rng(17)
+    for _ in range(60):
+        K = int(rng.integers(1, 24))
+        x = rng.integers(-4, 5, (3, K)).astype(np.float64) * 0.5
+        s = float(rng.choice([0.0, 0.25, 0.4, 0.5, 0.9]))
+        got = oracle.sparsify_rows(x, s)
+        z = int(math.floor(s * K + 1e-9))
+        for r in range(3):
+            kept = []
+            for _ in range(K - z):  # repeatedly take the largest magnitude, lowest index on ties
+                best = None
+                for c in range(K):
+                    if c in kept:
+                        continue
+                    if best is None or abs(x[r, c]) > abs(x[r, best]):
+                        best = c
+                kept.append(best)
+            want = np.zeros(K)
+            want[kept] = x[r, kept]
+            assert np.array_equal(got[r], want), (x[r], s, got[r], want)
+    assert np.array_equal(oracle.sparsify_rows(x, 0.0), x)
+
+
 def test_w8a8_linear_bruteforce():
     rng = np.random.default_rng(4)
     qx = rng.integers(-127, 128, (3, 37), dtype=np.int64).astype(np.int8)
@@ -401,6 +446,34 @@ def test_int8_mode_close_to_bf16_mode(tiny):
     b = oracle.tree_step(w, kv2, toks, parent, quant_mode=1)
     err = np.max(np.abs(a - b) / np.ptp(a, axis=1, keepdims=True))
     assert 1e-5 < err < 0.1, err
+
+
+def test_w4a4_and_activation_sparsity_modes(tiny):
+    """W4A4 (App. C, QSpec's bit width) and TEAL activation sparsity: sparsity 0 is the dense
+    model exactly; one projection with a single kept input is that input times one weight column;
+    W4A4 moves the logits more than W8A8 and less than the whole logit range."""
+    w, ref, prefix = tiny
+    toks, parent = synth.tokens(3, 8, SH.vocab), synth.tree(3, 8, 4)
+    runs = {}
+    for key, kw in {"bf16": {}, "s0": {"act_sparsity": 0.0}, "w8": {"quant_mode": 1}, "w4": {"quant_mode": 2},
+                    "s50": {"act_sparsity": 0.5}, "w4s50": {"quant_mode": 2, "act_sparsity": 0.5}}.items():
+        kv, _ = _prefilled(w, prefix)
+        runs[key] = oracle.tree_step(w, kv, toks, parent, **kw)
+    np.testing.assert_array_equal(runs["s0"], runs["bf16"])
+
+    def err(a):
+        return np.max(np.abs(a - runs["bf16"]) / np.ptp(runs["bf16"], axis=1, keepdims=True))
+
+    assert err(runs["w8"]) < err(runs["w4"]) < 1.0
+    assert err(runs["s50"]) > 1e-3 and err(runs["w4s50"]) > 1e-3
+    x = np.zeros((1, SH.d_model))
+    x[0, 5], x[0, 9] = -3.0, 0.25
+    from oracle import casspec_oracle
+
+    y = casspec_oracle._linear(x, w, "wo", 0, (0, 1.0 - 1.0 / SH.d_model))  # keep one input of d
+    np.testing.assert_allclose(y[0], -3.0 * w.f64("wo", 0)[:, 5], rtol=0, atol=0)
+    with pytest.raises(ValueError):
+        oracle.tree_step(w, oracle.KVCache(SH.n_layers, SH.n_heads, SH.head_dim, 128), toks, parent, quant_mode=3)
 
 
 def test_attn_bf16_rounds_only_the_attention_operands(tiny):
