@@ -333,7 +333,7 @@ typedef struct {
   int n_cfg;        /* candidate draft configurations, 1..CASSPEC_DYTC_MAX_CFG */
   double alpha_dn;  /* bottom draft: acceptance rate ... */
   double c_dn;      /* ... and cost coefficient (0 = free: the stop rule never fires) */
-  int k_max;        /* longest draft per expansion (Algorithm 1's k_max) */
+  int k_max;        /* longest draft per expansion (Algorithm 1's k_max), 1..CASSPEC_MAX_TREE */
   double t_min;     /* stop when alpha_dn / c_dn * P_acc(leaf) < t_min (Sec. 4.2) */
   int m_max;        /* largest tree, root included, 1..CASSPEC_MAX_TREE */
   double lambda;    /* EMA weight of the previous estimate (the paper uses 0.7) */

@@ -86,7 +86,8 @@ double casspec_dytc_objective(double alpha, double c, int k, double alpha_dn, do
 
 int casspec_dytc_create(const casspec_dytc_params* p, const double* alpha_init, const double* cost, casspec_dytc** out) {
   if (p == nullptr || alpha_init == nullptr || cost == nullptr || out == nullptr) return CASSPEC_E_INVAL;
-  if (p->n_cfg < 1 || p->n_cfg > CASSPEC_DYTC_MAX_CFG || p->k_max < 1 || p->m_max < 1 || p->m_max > CASSPEC_MAX_TREE ||
+  if (p->n_cfg < 1 || p->n_cfg > CASSPEC_DYTC_MAX_CFG || p->k_max < 1 || p->k_max > CASSPEC_MAX_TREE || p->m_max < 1 ||
+      p->m_max > CASSPEC_MAX_TREE ||
       p->window < 1 || !(p->lambda >= 0.0 && p->lambda <= 1.0) || bad_alpha(p->alpha_dn) || p->c_dn < 0.0 ||
       p->topk < 1 || p->topk > CASSPEC_TOPK_MAX || !(p->p_tree > 0.0 && p->p_tree <= 1.0))
     return CASSPEC_E_INVAL;

@@ -121,6 +121,8 @@ def test_argument_errors(cs):
         cs.Dytc([1.5], [0.1], 0.5, 0.01, 4, 1.0, 16)  # acceptance outside [0, 1]
     with pytest.raises(cs.CasspecError):
         cs.Dytc([0.5], [0.1], 0.5, 0.01, 4, 1.0, 65)  # tree larger than CASSPEC_MAX_TREE
+    with pytest.raises(cs.CasspecError):
+        cs.Dytc([0.5], [0.1], 0.5, 0.01, 65, 1.0, 16)  # draft longer than any tree
     sch = cs.Dytc([0.5], [0.1], 0.5, 0.01, 4, 1.0, 16)
     with pytest.raises(cs.CasspecError):
         sch.record(3, True)  # no such configuration
