@@ -262,23 +262,25 @@ cudaEvent_t prof_begin(casspec_model* m, int kind, cudaStream_t s) {
     ++count;                                                                 \
   } while (0)
 
-// Enqueue one tree step on stream s (argument checks already done).  `count` receives the number
-// of kernels enqueued; profiling events are recorded only when `prof` is set.
-//   bf16 mode: tree prep -> embedding (+ row sums of squares) -> chain[QKV of the first active
-//   layer] -> for each active layer: attention, chain[Wo, Wgate/Wup, Wdown, next layer's QKV or the
-//   LM head] -> argmax merge.  RMSNorm is folded into the chain phases that consume it.
-//   int8 mode: per-projection W8A8 kernels with RMSNorm / quantisation kernels, then chain[LM head].
 // Sub-blocks of a layer that a step runs (from a skip-mask byte).
 constexpr uint8_t kBlockAttn = 1, kBlockFfn = 2;
 uint8_t layer_blocks(uint8_t code) {
   if (code == 0) return 0;
   return (uint8_t)(((code & CASSPEC_SKIP_ATTN) ? 0 : kBlockAttn) | ((code & CASSPEC_SKIP_FFN) ? 0 : kBlockFfn));
 }
+// One projection or attention of a step (`l`: its layer, -1 for the LM head).
 enum { IT_QKV, IT_ATTN, IT_WO, IT_GU, IT_DOWN, IT_LM };
 struct StepItem {
   int kind, l;
 };
 
+// Enqueue one tree step on stream s (argument checks already done).  `count` receives the number
+// of kernels enqueued; profiling events are recorded only when `prof` is set.
+//   bf16 mode: tree prep -> embedding (+ row sums of squares) -> chain launches of consecutive
+//   projections, each attention ending one (with every block on: chain[QKV of the first layer],
+//   then per layer attention and chain[Wo, Wgate/Wup, Wdown, next layer's QKV or the LM head]) ->
+//   argmax merge.  RMSNorm is folded into the chain phases that consume it.
+//   int8 mode: per-projection W8A8 kernels with RMSNorm / quantisation kernels, then chain[LM head].
 int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const int32_t* parent, int n,
                  const std::vector<uint8_t>& on, int mode, float* logits, cudaStream_t s, bool prof, int& count) {
   const auto& c = m->cfg;
