@@ -58,3 +58,35 @@ def test_status_strings_without_gpu(lib_path):
     cs.load_library(lib_path)
     assert cs.status_string(cs.E_TREE) == "invalid tree or accepted path"
     assert cs.status_string(cs.OK) == "ok"
+
+
+def _header_constants() -> dict:
+    """Every `#define CASSPEC_X <int>` and every `CASSPEC_X = <int>` enumerator of the header."""
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    out = {}
+    for name, val in re.findall(r"#define\s+CASSPEC_([A-Z0-9_]+)\s+(0x[0-9A-Fa-f]+|-?\d+)u?\b", src):
+        out[name] = int(val, 0)
+    for name, val in re.findall(r"\bCASSPEC_([A-Z0-9_]+)\s*=\s*(-?\d+)", src):
+        out[name] = int(val)
+    for name, expr in re.findall(r"#define\s+CASSPEC_([A-Z0-9_]+)\s+\((\d+)\s*\*\s*CASSPEC_MAX_TREE\)", src):
+        out[name] = int(expr) * out["MAX_TREE"]
+    return out
+
+
+def test_binding_constants_match_the_header():
+    """The binding's copies of the header's constants (status codes, capacities, skip flags, option
+    bits, tensor ids, profiling kinds) are the header's values."""
+    import paper_2510_26843_gb300 as cs
+
+    h = _header_constants()
+    pairs = {"MAX_TREE": "MAX_TREE", "TOPK_MAX": "TOPK_MAX", "DYTC_WORK": "DYTC_WORK", "SKIP_ATTN": "SKIP_ATTN",
+             "SKIP_FFN": "SKIP_FFN", "OPT_PDL": "OPT_PDL", "OPT_GRAPHS": "OPT_GRAPHS", "OK": "OK"}
+    for key in list(h):
+        if key.startswith(("E_", "T_", "K_")):
+            pairs[key] = key
+    checked = 0
+    for hname, pname in pairs.items():
+        if hname in h and hasattr(cs, pname):
+            assert getattr(cs, pname) == h[hname], (hname, getattr(cs, pname), h[hname])
+            checked += 1
+    assert checked >= 40, checked  # status codes, tensor ids and profiling kinds are all covered
