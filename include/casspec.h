@@ -323,6 +323,13 @@ CASSPEC_API double casspec_dytc_objective(double alpha, double c, int k, double 
  * deviation noise_sd, fitted to m measured steps (x, y host [m]; m = 0 returns the prior).  Writes the
  * posterior mean to w_out [2] and, if non-NULL, the posterior covariance to cov_out [2][2].  A draft's
  * cost coefficient is then (w0 + w1 x_draft) / (w0 + w1 x_target).  Errors: E_INVAL. */
+/* Algorithmic bytes of one tree step (the regressor of the latency model): for every layer whose
+ * attention block runs (skip_mask as for casspec_tree_step, NULL = all on) its Wqkv and Wo, the prefix
+ * K/V of P slots read and the n new K/V written; for every FFN block that runs its Wg, Wu and Wd; the
+ * LM head read and the n rows of fp32 logits written.  Weights count 2 bytes in bf16 (quant_mode 0),
+ * 1 byte plus 4 per output row in W8A8 (quant_mode 1).  Host only.  Returns -1 on bad arguments. */
+CASSPEC_API double casspec_step_bytes(const casspec_model_config* cfg, const uint8_t* skip_mask, int quant_mode, int n,
+                                      int P);
 CASSPEC_API int casspec_latency_fit(const double* x, const double* y, int m, const double* mu0, const double* sd0,
                                     double noise_sd, double* w_out, double* cov_out);
 
@@ -352,8 +359,20 @@ CASSPEC_API void casspec_dytc_destroy(casspec_dytc* s);
 CASSPEC_API int casspec_dytc_get_params(const casspec_dytc* s, casspec_dytc_params* out);
 /* Replace a configuration's cost coefficient (e.g. from measured step times). */
 CASSPEC_API int casspec_dytc_set_cost(casspec_dytc* s, int cfg, double cost);
-/* Current acceptance estimate of a configuration. */
+/* The latency model fed by measured steps (Sec. 4.2, hardware-aware latency prediction):
+ *   casspec_dytc_observe records one measured step (bytes it moved, microseconds; the scheduler keeps
+ *   the most recent 512);
+ *   casspec_dytc_fit_costs fits casspec_latency_fit to the recorded steps (prior mu0, sd0, noise_sd)
+ *   and sets every configuration's cost coefficient to its predicted latency over the target's,
+ *   c = max(w0 + w1 cfg_bytes[i], 0) / (w0 + w1 target_bytes) (cfg_bytes host [n_cfg], e.g. from
+ *   casspec_step_bytes).  w_out (host [2], may be NULL) receives the fitted w.  Errors: E_INVAL (bad
+ *   arguments, a non-positive predicted target latency). */
+CASSPEC_API int casspec_dytc_observe(casspec_dytc* s, double bytes, double us);
+CASSPEC_API int casspec_dytc_fit_costs(casspec_dytc* s, const double* cfg_bytes, double target_bytes, const double* mu0,
+                                       const double* sd0, double noise_sd, double* w_out);
+/* Current acceptance estimate and cost coefficient of a configuration. */
 CASSPEC_API int casspec_dytc_alpha(const casspec_dytc* s, int cfg, double* alpha_out);
+CASSPEC_API int casspec_dytc_cost(const casspec_dytc* s, int cfg, double* cost_out);
 /* Algorithm 2 (App. D) with the current estimates: the configuration and draft length k in
  * [1, k_max] maximising Eq. 5, first maximum on ties; *cfg_out = -1 and *k_out = 0 when no pair has
  * a positive objective.  *obj_out (may be NULL) receives the maximum. */

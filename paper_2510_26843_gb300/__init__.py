@@ -34,9 +34,9 @@ EXPORTS = [
     "casspec_rmsnorm",
     "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
-    "casspec_dytc_destroy", "casspec_dytc_get_params", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_best_config",
+    "casspec_dytc_destroy", "casspec_dytc_get_params", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_cost", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
-    "casspec_dytc_tree_extend", "casspec_dytc_tree_begin", "casspec_dytc_tree_add", "casspec_vc_accept", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_pld_draft", "casspec_topk",
+    "casspec_dytc_tree_extend", "casspec_dytc_tree_begin", "casspec_dytc_tree_add", "casspec_vc_accept", "casspec_dytc_tree_get", "casspec_dytc_round", "casspec_latency_fit", "casspec_step_bytes", "casspec_dytc_observe", "casspec_dytc_fit_costs", "casspec_pld_draft", "casspec_topk",
 ]
 K_QKV, K_ATTN, K_WO, K_GATEUP, K_DOWN, K_LMHEAD, K_OTHER, K_COUNT = range(8)
 
@@ -91,6 +91,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_get_params": (_I, [_P, ctypes.POINTER(DytcParams)]),
         "casspec_dytc_set_cost": (_I, [_P, _I, _D]),
         "casspec_dytc_alpha": (_I, [_P, _I, ctypes.POINTER(_D)]),
+        "casspec_dytc_cost": (_I, [_P, _I, ctypes.POINTER(_D)]),
         "casspec_dytc_best_config": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_D)]),
         "casspec_dytc_record": (_I, [_P, _I, _I]),
         "casspec_dytc_end_step": (_I, [_P]),
@@ -103,6 +104,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_dytc_tree_add": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_float), _I]),
         "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
         "casspec_topk": (_I, [_P, _I, _I, _I, _P, _P, _P]),
+        "casspec_step_bytes": (_D, [ctypes.POINTER(ModelConfig), _P, _I, _I, _I]),
+        "casspec_dytc_observe": (_I, [_P, _D, _D]),
+        "casspec_dytc_fit_costs": (_I, [_P, ctypes.POINTER(_D), _D, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
+                                        ctypes.POINTER(_D)]),
         "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
                                      ctypes.POINTER(_D), ctypes.POINTER(_D)]),
         "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, _I, _P, _P,
@@ -379,6 +384,16 @@ def latency_fit(x, y, mu0, sd0, noise_sd: float) -> tuple[list[float], list[floa
     return list(w), list(cov)
 
 
+def step_bytes(cfg: ModelConfig, skip_mask=None, quant_mode: int = 0, n: int = 1, P: int = 0) -> float:
+    """casspec_step_bytes: algorithmic bytes of one tree step of this configuration."""
+    mk = None if skip_mask is None else np.ascontiguousarray(np.asarray(skip_mask, dtype=np.uint8))
+    v = load_library().casspec_step_bytes(ctypes.byref(cfg), None if mk is None else mk.ctypes.data, int(quant_mode),
+                                          int(n), int(P))
+    if v < 0:
+        raise CasspecError("casspec_step_bytes", E_INVAL)
+    return v
+
+
 def draft_cfgs(cfgs):
     """casspec_draft_cfg array for casspec_dytc_round, and the mask arrays it points into (keep them
     alive for the call).  Each entry: (skip_mask or None, quant_mode) for a model draft,
@@ -431,6 +446,11 @@ class Dytc:
         _check("casspec_dytc_alpha", load_library().casspec_dytc_alpha(self.h, cfg, ctypes.byref(v)))
         return v.value
 
+    def cost(self, cfg: int) -> float:
+        v = _D()
+        _check("casspec_dytc_cost", load_library().casspec_dytc_cost(self.h, cfg, ctypes.byref(v)))
+        return v.value
+
     def best_config(self) -> tuple[int | None, int, float]:
         s, k, v = _I(), _I(), _D()
         _check("casspec_dytc_best_config",
@@ -459,6 +479,17 @@ class Dytc:
         if rc < 0:
             raise CasspecError("casspec_dytc_tree_extend", rc)
         return rc
+
+    def observe(self, bytes_moved: float, us: float) -> None:
+        _check("casspec_dytc_observe", load_library().casspec_dytc_observe(self.h, float(bytes_moved), float(us)))
+
+    def fit_costs(self, cfg_bytes, target_bytes: float, mu0, sd0, noise_sd: float) -> list[float]:
+        """Refit the latency model to the observed steps and reset every configuration's cost; returns w."""
+        cb = (_D * self.n_cfg)(*[float(v) for v in cfg_bytes])
+        mu, sd, w = (_D * 2)(*[float(v) for v in mu0]), (_D * 2)(*[float(v) for v in sd0]), (_D * 2)()
+        _check("casspec_dytc_fit_costs",
+               load_library().casspec_dytc_fit_costs(self.h, cb, float(target_bytes), mu, sd, float(noise_sd), w))
+        return list(w)
 
     def tree_begin(self, leaf: int, siblings: bool = True) -> list[int]:
         br, nb = (ctypes.c_int32 * MAX_TREE)(), _I()

@@ -53,7 +53,13 @@ struct casspec_dytc {
   std::vector<int32_t> parent, token, cfg;
   std::vector<double> p_acc;
   std::vector<uint8_t> active;
+  // measured steps for the latency model: bytes moved and microseconds (the most recent kObs)
+  std::vector<double> obs_x, obs_y;
 };
+
+namespace {
+constexpr size_t kObs = 512;
+}
 
 extern "C" {
 
@@ -121,6 +127,12 @@ int casspec_dytc_set_cost(casspec_dytc* s, int cfg, double cost) {
 int casspec_dytc_alpha(const casspec_dytc* s, int cfg, double* alpha_out) {
   if (s == nullptr || alpha_out == nullptr || cfg < 0 || cfg >= s->p.n_cfg) return CASSPEC_E_INVAL;
   *alpha_out = s->alpha[cfg];
+  return CASSPEC_OK;
+}
+
+int casspec_dytc_cost(const casspec_dytc* s, int cfg, double* cost_out) {
+  if (s == nullptr || cost_out == nullptr || cfg < 0 || cfg >= s->p.n_cfg) return CASSPEC_E_INVAL;
+  *cost_out = s->cost[cfg];
   return CASSPEC_OK;
 }
 
@@ -285,6 +297,57 @@ int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out
   if (token_out) std::memcpy(token_out, s->token.data(), n * sizeof(int32_t));
   if (cfg_out) std::memcpy(cfg_out, s->cfg.data(), n * sizeof(int32_t));
   if (p_acc_out) std::memcpy(p_acc_out, s->p_acc.data(), n * sizeof(double));
+  return CASSPEC_OK;
+}
+
+double casspec_step_bytes(const casspec_model_config* c, const uint8_t* skip_mask, int quant_mode, int n, int P) {
+  if (c == nullptr || c->n_layers < 1 || c->d_model < 1 || c->ffn < 1 || c->vocab < 1 || n < 0 || P < 0 ||
+      quant_mode < 0 || quant_mode > 1)
+    return -1.0;
+  const double d = c->d_model, F = c->ffn, V = c->vocab;
+  const double wb = quant_mode == 1 ? 1.0 : 2.0;  // bytes per weight
+  const double sb = quant_mode == 1 ? 4.0 : 0.0;  // bytes per row scale
+  double bytes = V * d * 2.0 + (double)n * V * 4.0;  // LM head read, fp32 logits written
+  for (int l = 0; l < c->n_layers; ++l) {
+    const uint8_t code = skip_mask ? skip_mask[l] : 1;
+    if (code == 0) continue;
+    if (!(code & CASSPEC_SKIP_ATTN))  // Wqkv, Wo (+ scales), the prefix K/V read, the new K/V written
+      bytes += 4.0 * d * d * wb + 4.0 * d * sb + 2.0 * P * d * 2.0 + 2.0 * n * d * 2.0;
+    if (!(code & CASSPEC_SKIP_FFN))  // Wg, Wu, Wd (+ scales)
+      bytes += 3.0 * d * F * wb + (2.0 * F + d) * sb;
+  }
+  return bytes;
+}
+
+int casspec_dytc_observe(casspec_dytc* s, double bytes, double us) {
+  if (s == nullptr || !(bytes >= 0.0) || !(us > 0.0)) return CASSPEC_E_INVAL;
+  if (s->obs_x.size() == kObs) {
+    s->obs_x.erase(s->obs_x.begin());
+    s->obs_y.erase(s->obs_y.begin());
+  }
+  s->obs_x.push_back(bytes);
+  s->obs_y.push_back(us);
+  return CASSPEC_OK;
+}
+
+int casspec_dytc_fit_costs(casspec_dytc* s, const double* cfg_bytes, double target_bytes, const double* mu0,
+                           const double* sd0, double noise_sd, double* w_out) {
+  if (s == nullptr || cfg_bytes == nullptr || !(target_bytes > 0.0)) return CASSPEC_E_INVAL;
+  double w[2];
+  const int m = (int)s->obs_x.size();
+  const int rc = casspec_latency_fit(m ? s->obs_x.data() : nullptr, m ? s->obs_y.data() : nullptr, m, mu0, sd0,
+                                     noise_sd, w, nullptr);
+  if (rc != CASSPEC_OK) return rc;
+  const double t_target = w[0] + w[1] * target_bytes;
+  if (!(t_target > 0.0)) return CASSPEC_E_INVAL;
+  for (int c = 0; c < s->p.n_cfg; ++c) {
+    if (!(cfg_bytes[c] >= 0.0)) return CASSPEC_E_INVAL;
+  }
+  for (int c = 0; c < s->p.n_cfg; ++c) s->cost[c] = std::fmax(w[0] + w[1] * cfg_bytes[c], 0.0) / t_target;
+  if (w_out) {
+    w_out[0] = w[0];
+    w_out[1] = w[1];
+  }
   return CASSPEC_OK;
 }
 

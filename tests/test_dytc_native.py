@@ -286,3 +286,66 @@ def test_draft_cfg_marshalling(cs):
     got = [(a.skip_mask is not None, a.quant_mode, a.pld_n_max, a.vc) for a in arr]
     assert got == [(True, 0, 0, 0), (False, 1, 0, 0), (False, 0, 4, 0), (True, 1, 3, 1), (False, 0, 2, 1)]
     assert arr[0].skip_mask == keep[0].ctypes.data and list(keep[3]) == [1, 0, 1]
+
+
+def _cfg7b(cs):
+    import synth
+
+    s = synth.LLAMA7B
+    return cs.config(s.n_layers, s.d_model, s.n_heads, s.head_dim, s.ffn, s.vocab)
+
+
+def test_step_bytes_match_the_bench_byte_model(cs):
+    """casspec_step_bytes (the latency model's regressor) equals the benchmark's algorithmic bytes for
+    the 7B verify, a 50% layer-skip draft and a W8A8 draft; sub-block masks drop exactly their block."""
+    import numpy as np
+
+    import bench
+    import synth
+
+    sh = bench._shape()
+    cfg = _cfg7b(cs)
+    assert cs.step_bytes(cfg, None, 0, 64, 2048) == bench.algorithmic_bytes(sh, 64, 2048)["total"]
+    mask = synth.skip_masks(7, sh.n_layers, [0.5])[0]
+    assert cs.step_bytes(cfg, mask, 0, 8, 2048) == bench.algorithmic_bytes(sh, 8, 2048, 16)["total"]
+    assert cs.step_bytes(cfg, None, 1, 8, 2048) == bench.algorithmic_bytes(sh, 8, 2048, None, 1)["total"]
+    d, F, V, L = sh.d_model, sh.ffn, sh.vocab, sh.n_layers
+    head = V * d * 2 + 8 * V * 4
+    assert cs.step_bytes(cfg, np.zeros(L, np.uint8), 0, 8, 2048) == head
+    no_attn = np.full(L, 1 | cs.SKIP_ATTN, np.uint8)
+    assert cs.step_bytes(cfg, no_attn, 0, 8, 2048) == head + L * 3 * d * F * 2  # no K/V either
+    no_ffn = np.full(L, 1 | cs.SKIP_FFN, np.uint8)
+    assert cs.step_bytes(cfg, no_ffn, 0, 8, 2048) == head + L * (4 * d * d * 2 + 2 * 2048 * d * 2 + 2 * 8 * d * 2)
+    with pytest.raises(cs.CasspecError):
+        cs.step_bytes(cfg, None, 2, 8, 2048)
+
+
+def test_costs_fitted_from_measured_steps(cs):
+    """Steps measured on a roofline (20 us + bytes at 6.5 TB/s, noise 20 us) give the cost coefficients
+    of the fitted model, the same as the oracle's posterior mean predicts, and near the true ratios."""
+    import numpy as np
+
+    rng = np.random.default_rng(5)
+    x = rng.uniform(1e9, 1.5e10, 60)
+    y = 20.0 + x / 6.5e6 + rng.normal(0, 20.0, 60)
+    mu0, sd0, noise = [0.0, 1.0 / 6e6], [100.0, 1e-6], 20.0
+    sch = cs.Dytc([0.6, 0.7, 0.3], [0.5, 0.5, 0.5], 0.3, 0.02, 4, 1.0, 16)
+    for a, b in zip(x, y):
+        sch.observe(a, b)
+    cfg_bytes, target = [7.3e9, 7.8e9, 4.0e9], 1.433e10
+    w = sch.fit_costs(cfg_bytes, target, mu0, sd0, noise)
+    mean, _ = D.blr_posterior(x, y, mu0, sd0, noise)
+    assert w == pytest.approx(list(mean), rel=1e-9)
+    costs = [sch.cost(c) for c in range(3)]
+    pred = [(mean[0] + mean[1] * b) / (mean[0] + mean[1] * target) for b in cfg_bytes]
+    assert costs == pytest.approx(pred, rel=1e-9)
+    true = [(20.0 + b / 6.5e6) / (20.0 + target / 6.5e6) for b in cfg_bytes]
+    assert costs == pytest.approx(true, rel=0.02)
+    # Algorithm 2 now runs on the fitted costs
+    s_o, k_o, _ = D.find_best_config([0.6, 0.7, 0.3], pred, 0.3, 0.02, 4)
+    assert sch.best_config()[:2] == (s_o, k_o)
+    with pytest.raises(cs.CasspecError):
+        sch.fit_costs(cfg_bytes, 0.0, mu0, sd0, noise)
+    with pytest.raises(cs.CasspecError):
+        sch.observe(1e9, 0.0)
+    sch.close()
