@@ -528,6 +528,101 @@ def run_gpu(args) -> None:
         dist.destroy_process_group()
 
 
+def run_dytc(args) -> None:
+    """DyTC speculative rounds (Sec. 4.2: Algorithm 1 with K = 2 candidates and top-P 0.8, Algorithm 2,
+    the EMA estimates) on the 7B shape through casspec_dytc_round: a 50%-layer-skip bf16 draft, a W8A8
+    draft and the prompt-lookup bottom draft, the full model verifying.  The prompt is 512 seeded
+    tokens run through the model, so the cache and the lookup history agree.  Rounds synchronise the
+    host (it reads drafted tokens back), so they are timed by wall clock after warm-up; the value is
+    committed tokens per second.  Weights are random: acceptance here measures the machinery, not a
+    trained model's agreement."""
+    import torch
+
+    import synth
+    import paper_2510_26843_gb300 as cs
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    cs.load_library()
+    sh = _shape()
+    P0, rounds = 512, args.warmup + args.steps
+    dm = DeviceModel(sh, SEED, with_int8=True)
+    kv = DeviceKV(dm, P0 + 65 * rounds + 192)
+    stream = torch.cuda.current_stream()
+    cs.set_stream(dm.h, stream)
+    cs.set_options(dm.h, cs.OPT_PDL)
+    prompt = synth.prefix_tokens(SEED, P0, sh.vocab)
+    logits = torch.empty(64, sh.vocab, dtype=torch.float32, device="cuda")
+    for a in range(0, P0, 64):  # prefill in 64-token chains
+        t = torch.tensor(prompt[a:a + 64], dtype=torch.int32, device="cuda")
+        p = torch.tensor(synth.chain(64), dtype=torch.int32, device="cuda")
+        cs.tree_step(dm.h, kv.h, t, p, 64, None, 0, logits)
+        cs.kv_compact(kv.h, torch.tensor([64, *range(64), 0], dtype=torch.int32, device="cuda"))
+    out = [int(torch.argmax(logits[63]).item())]
+    history = torch.zeros(P0 + 65 * rounds + 4 * cs.MAX_TREE, dtype=torch.int32, device="cuda")
+    history[:P0] = torch.tensor(prompt, dtype=torch.int32, device="cuda")
+    history[P0] = out[0]
+    hist_len = P0 + 1
+
+    mask = synth.skip_masks(SEED, sh.n_layers, [0.5])[0]
+    cfg = cs.config(sh.n_layers, sh.d_model, sh.n_heads, sh.head_dim, sh.ffn, sh.vocab)
+    full = cs.step_bytes(cfg, None, 0, 64, P0)
+    costs = [cs.step_bytes(cfg, mask, 0, 8, P0) / full, cs.step_bytes(cfg, None, 1, 8, P0) / full, 0.02]
+    cfgs = [(mask, 0), (None, 1), ("pld", 4)]
+    sch = cs.Dytc([0.5, 0.8, 0.3], costs, alpha_dn=0.3, c_dn=0.02, k_max=4, t_min=0.5, m_max=64, topk=2, p_tree=0.8)
+    work = torch.zeros(cs.DYTC_WORK, dtype=torch.int32, device="cuda")
+    dlog = torch.empty(cs.MAX_TREE, sh.vocab, dtype=torch.float32, device="cuda")
+
+    def one_round():
+        nonlocal hist_len
+        toks, nd = sch.round(dm.h, kv.h, cfgs, out[-1], work, history, hist_len, dev_logits=dlog)
+        history[hist_len:hist_len + len(toks)] = torch.tensor(toks, dtype=torch.int32, device="cuda")
+        hist_len += len(toks)
+        out.extend(toks)
+        return len(toks), nd
+
+    for _ in range(args.warmup):
+        one_round()
+    torch.cuda.synchronize()
+    st = cs.get_status(dm.h)
+    if st != 0:
+        raise RuntimeError(f"device status after warm-up: {st} ({cs.status_string(st)})")
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    time.sleep(0.2)
+    n0 = cs.launch_count(dm.h)
+    committed = drafted = 0
+    clocks.mark(True)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        c, nd = one_round()
+        committed += c
+        drafted += nd
+    torch.cuda.synchronize()
+    t1 = time.perf_counter()
+    clocks.mark(False)
+    launches = cs.launch_count(dm.h) - n0
+    st = cs.get_status(dm.h)
+    if st != 0:
+        raise RuntimeError(f"device status after the timed rounds: {st} ({cs.status_string(st)})")
+    us = (t1 - t0) * 1e6 / args.steps
+    line = {
+        "metric": "DyTC speculative rounds, 7B shape: committed tokens per second", "impl": "ours",
+        "value": round(committed / (t1 - t0), 1), "unit": "tok/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "higher_is_better": True, "dtype": "bf16 + int8 drafts",
+        "data": "synthetic (seeded N(0,0.02) weights, seeded 512-token prompt)",
+        "config": {"workload": "dytc7b: llama7b-shape 32 layers, prompt 512; drafts 50%-skip bf16, W8A8, "
+                               "prompt lookup (n <= 4); K = 2, top-P 0.8, k_max 4, m_max 64",
+                   "l2": "no flush: every round streams the weights of several steps (GBs)"},
+        "us_per_round": round(us, 1), "tokens_per_round": round(committed / args.steps, 3),
+        "drafted_per_round": round(drafted / args.steps, 2),
+        "alpha": [round(sch.alpha(c), 4) for c in range(3)], "costs": [round(c, 4) for c in costs],
+        "gpu_launches": int(launches), "clocks": clocks.stop(),
+    }
+    print(json.dumps(line), flush=True)
+    sch.close()
+    kv.close()
+    dm.close()
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -537,9 +632,15 @@ def main() -> None:
     ap.add_argument("--no-graphs", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
-    ap.add_argument("--workload", default="verify7b", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="verify7b", choices=sorted(WORKLOADS) + ["dytc7b"])
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.workload == "dytc7b":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable": "the oracle's 7B-shape DyTC round takes minutes of "
+                                                                  "CPU per round"}), flush=True)
+        else:
+            run_dytc(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)
