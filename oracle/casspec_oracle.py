@@ -130,8 +130,14 @@ def sparsify_rows(x: np.ndarray, s: float) -> np.ndarray:
 
 
 def linear_w8a8(qx: np.ndarray, sx: np.ndarray, qw: np.ndarray, sw: np.ndarray) -> np.ndarray:
-    """y[t, o] = (sum_k qx[t, k] * qw[o, k]) * sx[t] * sw[o]; the integer sum is exact (int64)."""
-    acc = qx.astype(np.int64) @ qw.astype(np.int64).T
+    """y[t, o] = (sum_k qx[t, k] * qw[o, k]) * sx[t] * sw[o]; the integer sum is exact.
+
+    The codes are integers of magnitude <= 127, so every partial sum of the dot product is an integer
+    below K * 127^2 < 2^53: the fp64 matrix product returns the exact integer sum in any summation
+    order (the same value as an int64 sum; pinned against an int64 brute force)."""
+    K = qx.shape[-1]
+    assert K * 127 * 127 < 2 ** 53
+    acc = qx.astype(np.float64) @ qw.astype(np.float64).T
     return acc.astype(np.float64) * np.asarray(sx, dtype=np.float64)[:, None] * np.asarray(sw, dtype=np.float64)[None, :]
 
 
@@ -337,7 +343,8 @@ def layer_blocks(code: int) -> tuple[bool, bool]:
 
 def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
               skip_mask: np.ndarray | None = None, quant_mode: int = 0,
-              trace: dict | None = None, attn_bf16: bool = False, act_sparsity: float = 0.0) -> np.ndarray:
+              trace: dict | None = None, attn_bf16: bool = False, act_sparsity: float = 0.0,
+              x0: np.ndarray | None = None) -> np.ndarray:
     """One draft/verify pass over n new tree nodes; returns logits [n, V] (fp64).
 
     The nodes occupy tree slots T .. T+n-1 (cache slots P+T .. P+T+n-1); each active layer writes
@@ -351,6 +358,8 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
     attn_bf16 rounds q and the K/V written to the cache to bf16 (a bf16 cache and bf16 attention
     operands).  It is a perturbation of the size of bf16 storage, used by tests to measure how far
     the method's own output moves under it; the reference result keeps it off.
+    x0 [n, d], if given, is the residual stream entering the first layer in place of the tokens'
+    embedding rows (a test feeds one layer the input another implementation gave it).
     """
     sh = w.shape
     tokens = np.asarray(tokens, dtype=np.int64)
@@ -367,7 +376,7 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
         raise ValueError("quant_mode must be 0, 1 or 2 and act_sparsity in [0, 1)")
     lin = (quant_mode, float(act_sparsity))
 
-    x = w.f64("embed")[tokens]  # [n, d]
+    x = w.f64("embed")[tokens] if x0 is None else np.array(x0, dtype=np.float64).reshape(n, sh.d_model)  # [n, d]
     for l in range(sh.n_layers):
         attn_on, ffn_on = layer_blocks(mask[l])
         if attn_on:
@@ -376,7 +385,10 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
             xn2 = rmsnorm(x, w.gain("ffn_norm", l), sh.rms_eps)
             g = _linear(xn2, w, "wg", l, lin)
             u = _linear(xn2, w, "wu", l, lin)
-            x = x + _linear(silu(g) * u, w, "wd", l, lin)
+            hgu = silu(g) * u
+            if trace is not None:
+                trace.setdefault(l, {})["u"] = hgu
+            x = x + _linear(hgu, w, "wd", l, lin)
         if trace is not None and (attn_on or ffn_on):
             trace.setdefault(l, {})["x"] = x.copy()
     xf = rmsnorm(x, w.gain("final_norm"), sh.rms_eps)
@@ -405,7 +417,7 @@ def _attention_block(x, w, kv, l, lin, pos, slots, all_anc, n, attn_bf16, trace)
         kv.valid[l][s] = True
     o = tree_attention(q, kv, l, slots, [all_anc[kv.T + i] for i in range(n)]).reshape(n, d)
     if trace is not None:
-        trace[l] = {"xn": xn, "q": q, "k": k, "v": v, "o": o}
+        trace.setdefault(l, {}).update({"xn": xn, "q": q, "k": k, "v": v, "o": o})
     return x + _linear(o, w, "wo", l, lin)
 
 

@@ -183,6 +183,17 @@ def test_w8a8_linear_bruteforce():
     for t, o in itertools.product(range(3), range(5)):
         acc = sum(int(qx[t, k]) * int(qw[o, k]) for k in range(37))
         assert y[t, o] == pytest.approx(acc * sx[t] * sw[o], rel=1e-15)
+    # the integer sums are exact at the longest rows of the 13B shape, extreme codes included
+    K = 13824
+    qx = rng.integers(-127, 128, (4, K), dtype=np.int64)
+    qx[0] = 127
+    qw = rng.integers(-127, 128, (6, K), dtype=np.int64)
+    qw[0] = 127
+    qw[1] = -127
+    y = oracle.linear_w8a8(qx.astype(np.int8), np.ones(4), qw.astype(np.int8), np.ones(6))
+    exact = np.array([[int(np.dot(qx[t], qw[o])) for o in range(6)] for t in range(4)], dtype=np.int64)
+    assert exact[0, 0] == K * 127 * 127
+    assert np.array_equal(y, exact.astype(np.float64)) and np.array_equal(y.astype(np.int64), exact)
 
 
 # ------------------------------------------------------------------------------------------------
@@ -360,6 +371,27 @@ def test_skip_one_layer_equals_model_without_it(tiny):
     kv2, _ = _prefilled(w, prefix)
     np.testing.assert_array_equal(oracle.tree_step(w, kv1, toks, parent, skip_mask=np.ones(2, np.uint8)),
                                   oracle.tree_step(w, kv2, toks, parent))
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_layer_input_override_composes(tiny, mode):
+    """x0 replaces the embedding as the first layer's input: the embedding rows themselves give the
+    default result bit for bit, and layer 1 run alone from the residual layer 0 left (traced) gives
+    the two-layer result (same caches), in bf16 and W8A8 mode."""
+    w, ref, prefix = tiny
+    toks, parent = synth.tokens(21, 6, SH.vocab), synth.tree(21, 6, 3)
+    kv1, _ = _prefilled(w, prefix)
+    kv2, _ = _prefilled(w, prefix)
+    tr = {}
+    full = oracle.tree_step(w, kv1, toks, parent, quant_mode=mode, trace=tr)
+    same = oracle.tree_step(w, kv2, toks, parent, quant_mode=mode, x0=w.f64("embed")[toks])
+    np.testing.assert_array_equal(full, same)
+    kv3, _ = _prefilled(w, prefix)
+    only1 = np.array([0, 1], dtype=np.uint8)
+    tail = oracle.tree_step(w, kv3, toks, parent, skip_mask=only1, quant_mode=mode, x0=tr[0]["x"])
+    np.testing.assert_array_equal(full, tail)
+    np.testing.assert_array_equal(kv3.K[1], kv1.K[1])  # layer 1 wrote the same K/V
+    assert "u" in tr[1] and tr[1]["u"].shape == (6, SH.ffn)
 
 
 def _gains(name, layer):
