@@ -76,7 +76,14 @@ typedef struct casspec_kv casspec_kv;       /* opaque host handle */
  *   ATTN_NORM [d] fp32, FFN_NORM [d] fp32 (RMSNorm gains)
  *   WQKV [3d][d] bf16 (rows: Wq, then Wk, then Wv), WO [d][d], WG [F][d], WU [F][d], WD [d][F] bf16
  * The int8 copies (written by casspec_quantize_weights) are WQKV_Q .. WD_Q int8 with the same
- * shapes and WQKV_S .. WD_S fp32 per-output-row scales. */
+ * shapes and WQKV_S .. WD_S fp32 per-output-row scales.
+ * Step state (read-only views of the model's scratch, valid until the next step on the model; layer
+ * ignored; for tests and for callers that want the hidden state):
+ *   RESIDUAL [64][d] fp32: the residual stream after the step's last active layer (before the final
+ *     RMSNorm), rows 0 .. n-1 valid;
+ *   ACT_Q [64][K] int8 and ACT_S [64] fp32: codes and per-token scales of the latest quantised
+ *     projection input of a W8A8 step (the down projection's input, K = ffn, when the last active
+ *     layer ran its FFN block). */
 enum casspec_tensor_id {
   CASSPEC_T_EMBED = 0,
   CASSPEC_T_LM_HEAD = 1,
@@ -97,12 +104,21 @@ enum casspec_tensor_id {
   CASSPEC_T_WO_S = 16,
   CASSPEC_T_WG_S = 17,
   CASSPEC_T_WU_S = 18,
-  CASSPEC_T_WD_S = 19
+  CASSPEC_T_WD_S = 19,
+  CASSPEC_T_RESIDUAL = 20,
+  CASSPEC_T_ACT_Q = 21,
+  CASSPEC_T_ACT_S = 22
 };
 
 /* Option bits for casspec_set_options. */
 #define CASSPEC_OPT_PDL 1u    /* programmatic dependent launch between the step's kernels (default on) */
 #define CASSPEC_OPT_GRAPHS 2u /* replay a captured CUDA graph per (call shape, pointers) (default off) */
+/* Test hook for the failure path (default off): while set, a bf16 tree step with two or more
+ * projections in one chain launch makes that launch's second phase wait for an arrival that never
+ * comes; the bounded wait expires (2 s), the step reports CASSPEC_E_TIMEOUT through
+ * casspec_get_status, and the model stays usable once the bit is cleared.  Such steps run
+ * eagerly (never captured into a graph). */
+#define CASSPEC_OPT_TEST_STALL 4u
 
 /* ---------------------------------------------------------------------------------------------
  * Model
@@ -216,8 +232,9 @@ CASSPEC_API int casspec_accept_greedy(casspec_model* m, const float* logits, con
 /* Move the K/V of the accepted path (accepted_out as written by casspec_accept_greedy, dev) from
  * tree slots to committed slots P .. P+L-1 in every layer, then P += L and T = 0.  All layers must
  * hold the tree's K/V (the verify pass ran with every layer on), else E_STATE.  A path that is
- * inconsistent with the current tree (L < 1, L > T, an index >= T, non-increasing indices) sets
- * E_TREE on the status word and leaves the cache unchanged. */
+ * inconsistent with the current tree (L < 1, L > T, an index >= T, a first node other than the
+ * root, slot 0, or a node whose parent is not the node before it) sets E_TREE on the status word
+ * and leaves the cache unchanged. */
 CASSPEC_API int casspec_kv_compact(casspec_kv* kv, const int32_t* accepted_out);
 
 /* ---------------------------------------------------------------------------------------------
@@ -262,8 +279,11 @@ CASSPEC_API size_t casspec_linear_workspace_bytes(int N, int K, int n);
 /* Y[i][o] = sum_k X[i][k] * W[o][k] (fp32 accumulation on the tensor cores) for i < n, o < N.
  *   W dev bf16 [N][K], X dev bf16 [n][K] (row stride K), Y dev fp32 [n][ldy], ldy >= N.
  *   1 <= n <= 64, K % 8 == 0, N >= 1; W and X 16-byte aligned.
+ *   N <= 130,944 (1023 tiles of 128 rows).
  *   workspace dev, >= casspec_linear_workspace_bytes(N, K, n) bytes; its first 4 KB must be zero
- *   before the first call and are left zero by every call that completes. */
+ *   before the first call and are left zero by every call that completes.  A call whose bounded
+ *   device wait expired leaves CASSPEC_E_TIMEOUT in the int32 at byte offset 4092 of the workspace
+ *   (its status word; Y is then incomplete) and the 4 KB must be zeroed again before the next call. */
 CASSPEC_API int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int n, float* Y, int ldy,
                         void* workspace, size_t workspace_bytes, void* cuda_stream);
 
@@ -277,9 +297,15 @@ CASSPEC_API int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint1
  *   The scratch is shared by all calls on a device: calls that overlap in time (other streams or
  *   threads) race on it and must be serialised by the caller.
  *   Returns CASSPEC_E_CAPACITY when ceil(N / 128) + min(ceil(N/128) * ceil(K/64), SM count) > 256
- *   (N up to 13,312 on a 152-SM GB300); other errors as casspec_linear_bf16. */
+ *   (N up to 13,312 on a 152-SM GB300); other errors as casspec_linear_bf16.
+ *   A bounded device wait of the kernel that expires leaves CASSPEC_E_TIMEOUT in the scratch's
+ *   status word (Y is then incomplete); casspec_linear_bf16_static_status reads it. */
 CASSPEC_API int casspec_linear_bf16_static(const uint16_t* W, int N, int K, const uint16_t* X, int n, float* Y, int ldy,
                                void* cuda_stream);
+/* Status word of the latest casspec_linear_bf16_static call on the current device (0 or
+ * CASSPEC_E_TIMEOUT): waits for cuda_stream, then copies the word to *status_out (no allocation).
+ * Each call clears the word when it starts. */
+CASSPEC_API int casspec_linear_bf16_static_status(void* cuda_stream, int* status_out);
 
 /* RMSNorm of n rows (Llama pre-norm): y = x / sqrt(mean(x^2) + eps) * g, fp32 arithmetic.
  *   x dev fp32 [n][d]; g dev fp32 [d]; y_bf16 dev bf16 [n][d] (may be NULL if q is given).
@@ -323,6 +349,9 @@ CASSPEC_API double casspec_dytc_objective(double alpha, double c, int k, double 
  * deviation noise_sd, fitted to m measured steps (x, y host [m]; m = 0 returns the prior).  Writes the
  * posterior mean to w_out [2] and, if non-NULL, the posterior covariance to cov_out [2][2].  A draft's
  * cost coefficient is then (w0 + w1 x_draft) / (w0 + w1 x_target).  Errors: E_INVAL. */
+CASSPEC_API int casspec_latency_fit(const double* x, const double* y, int m, const double* mu0, const double* sd0,
+                                    double noise_sd, double* w_out, double* cov_out);
+
 /* Algorithmic bytes of one tree step (the regressor of the latency model): for every layer whose
  * attention block runs (skip_mask as for casspec_tree_step, NULL = all on) its Wqkv and Wo, the prefix
  * K/V of P slots read and the n new K/V written; for every FFN block that runs its Wg, Wu and Wd; the
@@ -330,8 +359,6 @@ CASSPEC_API double casspec_dytc_objective(double alpha, double c, int k, double 
  * 1 byte plus 4 per output row in W8A8 (quant_mode 1).  Host only.  Returns -1 on bad arguments. */
 CASSPEC_API double casspec_step_bytes(const casspec_model_config* cfg, const uint8_t* skip_mask, int quant_mode, int n,
                                       int P);
-CASSPEC_API int casspec_latency_fit(const double* x, const double* y, int m, const double* mu0, const double* sd0,
-                                    double noise_sd, double* w_out, double* cov_out);
 
 #define CASSPEC_DYTC_MAX_CFG 16
 #define CASSPEC_TOPK_MAX 8 /* largest K of casspec_topk and of the DyTC tree */
@@ -359,17 +386,24 @@ CASSPEC_API void casspec_dytc_destroy(casspec_dytc* s);
 CASSPEC_API int casspec_dytc_get_params(const casspec_dytc* s, casspec_dytc_params* out);
 /* Replace a configuration's cost coefficient (e.g. from measured step times). */
 CASSPEC_API int casspec_dytc_set_cost(casspec_dytc* s, int cfg, double cost);
-/* The latency model fed by measured steps (Sec. 4.2, hardware-aware latency prediction):
- *   casspec_dytc_observe records one measured step (bytes it moved, microseconds; the scheduler keeps
- *   the most recent 512);
- *   casspec_dytc_fit_costs fits casspec_latency_fit to the recorded steps (prior mu0, sd0, noise_sd)
- *   and sets every configuration's cost coefficient to its predicted latency over the target's,
- *   c = max(w0 + w1 cfg_bytes[i], 0) / (w0 + w1 target_bytes) (cfg_bytes host [n_cfg], e.g. from
- *   casspec_step_bytes).  w_out (host [2], may be NULL) receives the fitted w.  Errors: E_INVAL (bad
- *   arguments, a non-positive predicted target latency). */
-CASSPEC_API int casspec_dytc_observe(casspec_dytc* s, double bytes, double us);
-CASSPEC_API int casspec_dytc_fit_costs(casspec_dytc* s, const double* cfg_bytes, double target_bytes, const double* mu0,
-                                       const double* sd0, double noise_sd, double* w_out);
+/* The latency model fed by measured steps (Sec. 4.2, hardware-aware latency prediction).  Steps of
+ * different arithmetic (bf16, W8A8, W4A4) do not share one bytes-to-time line -- the quantised
+ * projections are limited by their integer or conversion work, not only by the bytes they stream --
+ * so each class (CASSPEC_DYTC_MAX_CLASS of them; use the step's quant_mode) has its own regression:
+ *   casspec_dytc_observe records one measured step of class cls (bytes it moved, microseconds; the
+ *   scheduler keeps the most recent 512 per class);
+ *   casspec_dytc_fit_costs fits casspec_latency_fit to each class's recorded steps (prior mu0, sd0,
+ *   noise_sd; a class without steps keeps the prior) and sets every configuration's cost coefficient
+ *   to its predicted latency over the target's, c = max(w0 + w1 cfg_bytes[i], 0) / (v0 + v1 target_bytes),
+ *   with w the fit of the configuration's class cfg_class[i] and v that of class 0, the target's
+ *   (cfg_class, cfg_bytes host [n_cfg]; bytes e.g. from casspec_step_bytes).  w_out (host
+ *   [CASSPEC_DYTC_MAX_CLASS][2], may be NULL) receives every class's fitted w.  Errors: E_INVAL (bad
+ *   arguments, a class out of range, a non-positive predicted target latency). */
+#define CASSPEC_DYTC_MAX_CLASS 4
+CASSPEC_API int casspec_dytc_observe(casspec_dytc* s, int cls, double bytes, double us);
+CASSPEC_API int casspec_dytc_fit_costs(casspec_dytc* s, const int* cfg_class, const double* cfg_bytes,
+                                       double target_bytes, const double* mu0, const double* sd0, double noise_sd,
+                                       double* w_out);
 /* Current acceptance estimate and cost coefficient of a configuration. */
 CASSPEC_API int casspec_dytc_alpha(const casspec_dytc* s, int cfg, double* alpha_out);
 CASSPEC_API int casspec_dytc_cost(const casspec_dytc* s, int cfg, double* cost_out);

@@ -18,19 +18,21 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libcasspec.so")
 OK, E_INVAL, E_SHAPE, E_CAPACITY, E_CUDA, E_TREE, E_TIMEOUT, E_STATE = 0, -1, -2, -3, -4, -5, -6, -7
 MAX_TREE = 64
 TOPK_MAX = 8
+DYTC_MAX_CLASS = 4  # latency-model classes (one regression per step arithmetic)
 DYTC_WORK = 24 * MAX_TREE  # int32 entries of casspec_dytc_round's device scratch
 SKIP_ATTN, SKIP_FFN = 0x2, 0x4  # skip-mask flags on a non-zero byte: drop the attention / FFN block
-OPT_PDL, OPT_GRAPHS = 1, 2
+OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL = 1, 2, 4
 
 (T_EMBED, T_LM_HEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WG, T_WU, T_WD,
- T_WQKV_Q, T_WO_Q, T_WG_Q, T_WU_Q, T_WD_Q, T_WQKV_S, T_WO_S, T_WG_S, T_WU_S, T_WD_S) = range(20)
+ T_WQKV_Q, T_WO_Q, T_WG_Q, T_WU_Q, T_WD_Q, T_WQKV_S, T_WO_S, T_WG_S, T_WU_S, T_WD_S,
+ T_RESIDUAL, T_ACT_Q, T_ACT_S) = range(23)
 
 EXPORTS = [
     "casspec_model_bytes", "casspec_create_model", "casspec_destroy_model", "casspec_set_stream",
     "casspec_set_options", "casspec_tensor", "casspec_quantize_weights", "casspec_kv_bytes", "casspec_kv_create",
     "casspec_kv_destroy", "casspec_kv_layer", "casspec_kv_set_prefix", "casspec_kv_reset_tree", "casspec_kv_length",
     "casspec_tree_step", "casspec_argmax", "casspec_accept_greedy", "casspec_kv_compact", "casspec_get_status",
-    "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_linear_bf16_static",
+    "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_linear_bf16_static", "casspec_linear_bf16_static_status",
     "casspec_rmsnorm",
     "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
@@ -105,9 +107,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_pld_draft": (_I, [_P, _I, _I, _I, _I, _P, _P]),
         "casspec_topk": (_I, [_P, _I, _I, _I, _P, _P, _P]),
         "casspec_step_bytes": (_D, [ctypes.POINTER(ModelConfig), _P, _I, _I, _I]),
-        "casspec_dytc_observe": (_I, [_P, _D, _D]),
-        "casspec_dytc_fit_costs": (_I, [_P, ctypes.POINTER(_D), _D, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
-                                        ctypes.POINTER(_D)]),
+        "casspec_dytc_observe": (_I, [_P, _I, _D, _D]),
+        "casspec_dytc_fit_costs": (_I, [_P, ctypes.POINTER(_I), ctypes.POINTER(_D), _D, ctypes.POINTER(_D),
+                                        ctypes.POINTER(_D), _D, ctypes.POINTER(_D)]),
         "casspec_latency_fit": (_I, [ctypes.POINTER(_D), ctypes.POINTER(_D), _I, ctypes.POINTER(_D), ctypes.POINTER(_D), _D,
                                      ctypes.POINTER(_D), ctypes.POINTER(_D)]),
         "casspec_dytc_round": (_I, [_P, _P, _P, ctypes.POINTER(DraftCfg), ctypes.c_int32, _P, _I, _P, _P,
@@ -136,6 +138,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_linear_workspace_bytes": (_SZ, [_I, _I, _I]),
         "casspec_linear_bf16": (_I, [_P, _I, _I, _P, _I, _P, _I, _P, _SZ, _P]),
         "casspec_linear_bf16_static": (_I, [_P, _I, _I, _P, _I, _P, _I, _P]),
+        "casspec_linear_bf16_static_status": (_I, [_P, ctypes.POINTER(_I)]),
         "casspec_rmsnorm": (_I, [_P, _P, _I, _I, ctypes.c_float, _P, _P, _P, _P]),
         "casspec_quantize_rows": (_I, [_P, _I, _I, _P, _P, _P]),
         "casspec_profile": (_I, [_P, _I]),
@@ -303,6 +306,14 @@ def linear_bf16(W, N: int, K: int, X, n: int, Y, ldy: int, workspace, stream=Non
 def linear_bf16_static(W, N: int, K: int, X, n: int, Y, ldy: int, stream=None) -> None:
     _check("casspec_linear_bf16_static",
            load_library().casspec_linear_bf16_static(_ptr(W), N, K, _ptr(X), n, _ptr(Y), ldy, _stream(stream)))
+
+
+def linear_bf16_static_status(stream=None) -> int:
+    """Status word of the latest casspec_linear_bf16_static call on the current device (syncs)."""
+    st = _I()
+    _check("casspec_linear_bf16_static_status",
+           load_library().casspec_linear_bf16_static_status(_stream(stream), ctypes.byref(st)))
+    return st.value
 
 
 def rmsnorm(x, g, n: int, d: int, eps: float, y=None, q=None, s=None, stream=None) -> None:
@@ -480,16 +491,21 @@ class Dytc:
             raise CasspecError("casspec_dytc_tree_extend", rc)
         return rc
 
-    def observe(self, bytes_moved: float, us: float) -> None:
-        _check("casspec_dytc_observe", load_library().casspec_dytc_observe(self.h, float(bytes_moved), float(us)))
+    def observe(self, cls: int, bytes_moved: float, us: float) -> None:
+        """Record one measured step of arithmetic class `cls` (its quant_mode)."""
+        _check("casspec_dytc_observe",
+               load_library().casspec_dytc_observe(self.h, int(cls), float(bytes_moved), float(us)))
 
-    def fit_costs(self, cfg_bytes, target_bytes: float, mu0, sd0, noise_sd: float) -> list[float]:
-        """Refit the latency model to the observed steps and reset every configuration's cost; returns w."""
+    def fit_costs(self, cfg_class, cfg_bytes, target_bytes: float, mu0, sd0, noise_sd: float) -> list[list[float]]:
+        """Refit each class's latency model to its observed steps and reset every configuration's cost;
+        returns the fitted w of every class."""
+        cc = (_I * self.n_cfg)(*[int(v) for v in cfg_class])
         cb = (_D * self.n_cfg)(*[float(v) for v in cfg_bytes])
-        mu, sd, w = (_D * 2)(*[float(v) for v in mu0]), (_D * 2)(*[float(v) for v in sd0]), (_D * 2)()
+        mu, sd = (_D * 2)(*[float(v) for v in mu0]), (_D * 2)(*[float(v) for v in sd0])
+        w = (_D * (2 * DYTC_MAX_CLASS))()
         _check("casspec_dytc_fit_costs",
-               load_library().casspec_dytc_fit_costs(self.h, cb, float(target_bytes), mu, sd, float(noise_sd), w))
-        return list(w)
+               load_library().casspec_dytc_fit_costs(self.h, cc, cb, float(target_bytes), mu, sd, float(noise_sd), w))
+        return [[w[2 * k], w[2 * k + 1]] for k in range(DYTC_MAX_CLASS)]
 
     def tree_begin(self, leaf: int, siblings: bool = True) -> list[int]:
         br, nb = (ctypes.c_int32 * MAX_TREE)(), _I()

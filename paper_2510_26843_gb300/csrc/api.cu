@@ -26,6 +26,7 @@ struct LayerPtrs {
   int8_t *qkv_q, *wo_q, *wg_q, *wu_q, *wd_q;
   float *qkv_s, *wo_s, *wg_s, *wu_s, *wd_s;
   CUtensorMap tm_qkv, tm_o, tm_g, tm_u, tm_d;
+  uint8_t *wqkv_p, *wo_p, *wgu_p, *wd_p;  // the projections packed per CTA for the chain (pack_rows_kernel)
 };
 
 // Byte layout of a model's device memory (weights, int8 copies, step scratch).
@@ -34,8 +35,10 @@ struct Layout {
   size_t embed, lm_head, final_norm;
   std::vector<size_t> attn_norm, ffn_norm, wqkv, wo, wg, wu, wd;
   std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
+  std::vector<size_t> wqkv_p, wo_p, wgu_p, wd_p;
+  size_t lm_p;
   size_t x, q, o, u, xa, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
-  size_t gemm_part, gemm_cnt, chain_cnt, chain_bar, i8_part, i8_cnt, attn_part, attn_ml, attn_cnt, status;
+  size_t gemm_part, gemm_cnt, chain_ready, chain_done, i8_part, i8_cnt, attn_part, attn_ml, attn_cnt, status;
   size_t scratch_begin;
   int max_tiles, lm_tiles;
 };
@@ -47,12 +50,13 @@ bool config_ok(const casspec_model_config* c) {
   if (c->n_heads < 1 || c->d_model != c->n_heads * c->head_dim) return false;
   if (c->d_model % 128 != 0 || c->d_model > 16384) return false;
   if (c->ffn < 16 || c->ffn % 16 != 0 || c->ffn > 65536) return false;
-  if (c->vocab < 1 || c->vocab % 8 != 0 || c->vocab > 131072) return false;
+  if (c->vocab < 16 || c->vocab % 8 != 0 || c->vocab > 131072) return false;
   if (!(c->rope_base > 0.f) || !(c->rms_eps >= 0.f)) return false;
   return true;
 }
 
 int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
+int roundup16(int n) { return (n + 15) / 16 * 16; }
 
 Layout make_layout(const casspec_model_config& c) {
   Layout L;
@@ -76,6 +80,15 @@ Layout make_layout(const casspec_model_config& c) {
     L.wu.push_back(take(F * d * 2));
     L.wd.push_back(take(d * F * 2));
   }
+  // the bf16 projections once more, packed per CTA in the order the projection chain streams them
+  // (the row-major tensors stay for filling, export, quantisation and the stand-alone GEMM)
+  for (size_t l = 0; l < NL; ++l) {
+    L.wqkv_p.push_back(take(pack_rows_bytes((int)(3 * d), (int)d, PACK_QKV)));
+    L.wo_p.push_back(take(pack_rows_bytes((int)d, (int)d, PACK_PLAIN)));
+    L.wgu_p.push_back(take(pack_rows_bytes((int)F, (int)d, PACK_GLU)));
+    L.wd_p.push_back(take(pack_rows_bytes((int)d, (int)F, PACK_PLAIN)));
+  }
+  L.lm_p = take(pack_rows_bytes(roundup16((int)V), (int)d, PACK_PLAIN));
   if (c.with_int8) {
     for (size_t l = 0; l < NL; ++l) {
       L.qkv_q.push_back(take(3 * d * d));
@@ -101,19 +114,19 @@ Layout make_layout(const casspec_model_config& c) {
   L.xa = take(2 * T * d * 2);
   L.xq = take(T * std::max(d, F));
   L.xs = take(T * 4);
-  L.ssp = take((size_t)std::max<size_t>(d / 128, 1) * T * 4);
+  L.ssp = take((size_t)std::max<size_t>(d / 128, kSmsBound) * T * 4);  // per-slice partial sums of squares
   L.pos = take(T * 4);
   L.anc = take(T * 8);
-  L.am_v1 = take((size_t)L.lm_tiles * T * 4);
-  L.am_i1 = take((size_t)L.lm_tiles * T * 4);
-  L.am_v2 = take((size_t)L.lm_tiles * T * 4);
+  L.am_v1 = take((size_t)kSmsBound * T * 4);  // per-slice LM-head (max, argmax, second max)
+  L.am_i1 = take((size_t)kSmsBound * T * 4);
+  L.am_v2 = take((size_t)kSmsBound * T * 4);
   L.am = take(T * 4);
   L.margin = take(T * 4);
   L.am2 = take(T * 4);
   L.gemm_part = take(gemm_partials_floats(L.max_tiles, kSmsBound) * 4);
   L.gemm_cnt = take((size_t)L.max_tiles * 4);
-  L.chain_cnt = take((size_t)kMaxPhases * 1024 * 4);
-  L.chain_bar = take(256);
+  L.chain_ready = take((size_t)kMaxPhases * kReadyPerPhase * 4);
+  L.chain_done = take(256);
   {  // int32 partial tiles of the W8A8 projections: tiles x ksplit slots of 64 x 128
     const size_t kq = (size_t)(cdiv(d, 128) + 3) / 4, kf = (size_t)(cdiv(F, 128) + 3) / 4;
     const size_t slots = std::max(std::max((size_t)cdiv(3 * d, 128) * kq, (size_t)cdiv(F, 64) * kq),
@@ -135,8 +148,6 @@ int num_sms_of_current_device() {
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
   return sms;
 }
-
-int roundup16(int n) { return (n + 15) / 16 * 16; }
 
 }  // namespace
 
@@ -170,7 +181,9 @@ struct casspec_model {
   CUtensorMap tm_o[4], tm_u[4], tm_xa[4];  // their 64 x BN boxes, BN = 16, 32, 48, 64
   int8_t* xq;
   float* xs;
-  unsigned *chain_cnt, *chain_bar;
+  unsigned *chain_ready, *chain_done;
+  uint8_t* lm_p = nullptr;   // the LM head packed for the chain
+  bool pack_dirty = true;    // the row-major weights may have changed since the last packing
   int* pos;
   unsigned long long* anc;
   float *am_v1, *am_v2, *margin;
@@ -262,6 +275,26 @@ cudaEvent_t prof_begin(casspec_model* m, int kind, cudaStream_t s) {
     ++count;                                                                 \
   } while (0)
 
+// Refresh the chain's packed weight copies from the row-major tensors (on the model's stream).
+int pack_weights(casspec_model* m, int& count) {
+  const auto& c = m->cfg;
+  const int d = c.d_model, F = c.ffn, V = c.vocab, hd = c.head_dim;
+  const int G = chain_grid(m->num_sms);
+  for (int l = 0; l < c.n_layers; ++l) {
+    LayerPtrs& p = m->layers[l];
+    CK(launch_pack_rows(p.wqkv, nullptr, 3 * d, 3 * d, d, G, PACK_QKV, d, hd, d / kRowGroup, p.wqkv_p, m->stream));
+    CK(launch_pack_rows(p.wo, nullptr, d, d, d, G, PACK_PLAIN, d, hd, d / kRowGroup, p.wo_p, m->stream));
+    CK(launch_pack_rows(p.wg, p.wu, F, F, d, G, PACK_GLU, d, hd, d / kRowGroup, p.wgu_p, m->stream));
+    CK(launch_pack_rows(p.wd, nullptr, d, d, F, G, PACK_PLAIN, d, hd, F / kRowGroup, p.wd_p, m->stream));
+    count += 4;
+  }
+  CK(launch_pack_rows(m->lm_head, nullptr, roundup16(V), V, d, G, PACK_PLAIN, d, hd, d / kRowGroup, m->lm_p,
+                      m->stream));
+  ++count;
+  m->pack_dirty = false;
+  return CASSPEC_OK;
+}
+
 // Sub-blocks of a layer that a step runs (from a skip-mask byte).
 constexpr uint8_t kBlockAttn = 1, kBlockFfn = 2;
 uint8_t layer_blocks(uint8_t code) {
@@ -329,31 +362,36 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   base.pos = m->pos;
   base.rope = kv->rope;
 
-  // ---- phase descriptors of the projection chain ----
-  auto ph_qkv = [&](int l, int ss_tiles, PhaseDesc& p, CUtensorMap& w, CUtensorMap& x) {
-    p = PhaseDesc{};
+  // ---- phases of the projection chain ----
+  const int G = chain_grid(m->num_sms);
+  const int resid_parts = std::min(d / kRowGroup, G);  // partial sums of squares a residual phase leaves
+  auto ph_qkv = [&](int l, int ss_parts, ChainPhase& p, CUtensorMap& x) {
+    p = ChainPhase{};
     p.epi = EPI_QKV;
-    p.tiles = 3 * d / 128;
-    p.kblocks = cdiv(d, 64);
+    p.N = 3 * d;
     p.K = d;
+    p.kb = cdiv(d, 64);
+    p.wp = m->layers[l].wqkv_p;
+    p.rot_groups = d / kRowGroup;
     p.ss = m->ssp;
-    p.ss_tiles = ss_tiles;
+    p.ss_parts = ss_parts;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = 3 * d;
     p.ep.q_out = m->q;
     p.ep.kc = kv_layer_k(kv, l);
     p.ep.vc = kv_layer_v(kv, l);
-    w = m->layers[l].tm_qkv;
     x = m->tm_xa[bi];
   };
   // residual projection; g_next: gains of the RMSNorm that the next projection applies to x
-  auto ph_resid = [&](int K, const float* g_next, PhaseDesc& p) {
-    p = PhaseDesc{};
+  auto ph_resid = [&](int K, const uint8_t* wp, int rot_groups, const float* g_next, ChainPhase& p) {
+    p = ChainPhase{};
     p.epi = EPI_RESID;
-    p.tiles = d / 128;
-    p.kblocks = cdiv(K, 64);
+    p.N = d;
     p.K = K;
+    p.kb = cdiv(K, 64);
+    p.wp = wp;
+    p.rot_groups = rot_groups;
     p.ep = base;
     p.ep.N = d;
     p.ep.y = m->x;
@@ -362,27 +400,31 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.xa_out = m->xa;
     p.ep.g_next = g_next;
   };
-  auto ph_gu = [&](int ss_tiles, PhaseDesc& p) {
-    p = PhaseDesc{};
+  auto ph_gu = [&](int l, int ss_parts, ChainPhase& p) {
+    p = ChainPhase{};
     p.epi = EPI_GLU;
-    p.tiles = cdiv(F, 64);
-    p.kblocks = cdiv(d, 64);
+    p.N = F;
     p.K = d;
+    p.kb = cdiv(d, 64);
+    p.wp = m->layers[l].wgu_p;
+    p.rot_groups = d / kRowGroup;
     p.ss = m->ssp;
-    p.ss_tiles = ss_tiles;
+    p.ss_parts = ss_parts;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = F;
     p.ep.u_out = m->u;
   };
-  auto ph_lm = [&](int ss_tiles, PhaseDesc& p, CUtensorMap& w, CUtensorMap& x) {
-    p = PhaseDesc{};
+  auto ph_lm = [&](int ss_parts, ChainPhase& p, CUtensorMap& x) {
+    p = ChainPhase{};
     p.epi = EPI_LMHEAD;
-    p.tiles = m->lay.lm_tiles;
-    p.kblocks = cdiv(d, 64);
+    p.N = roundup16(V);
     p.K = d;
+    p.kb = cdiv(d, 64);
+    p.wp = m->lm_p;
+    p.rot_groups = d / kRowGroup;
     p.ss = m->ssp;
-    p.ss_tiles = ss_tiles;
+    p.ss_parts = ss_parts;
     p.eps = c.rms_eps;
     p.ep = base;
     p.ep.N = V;
@@ -390,16 +432,25 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.am_v1 = m->am_v1;
     p.ep.am_i1 = m->am_i1;
     p.ep.am_v2 = m->am_v2;
-    w = m->tm_lm;
     x = m->tm_xa[bi];
   };
-  const int cgrid = chain_grid(m->num_sms);
+  bool stall_pending = (m->flags & CASSPEC_OPT_TEST_STALL) != 0;
   auto chain = [&](ChainArgs& ca, ChainMaps& cm, int kind) -> int {
-    ca.partials = m->gemm_part;
-    ca.counters = m->chain_cnt;
-    ca.bar = m->chain_bar;
+    ca.bn = BN;
+    ca.ready = m->chain_ready;
+    ca.done = m->chain_done;
     ca.status = m->status;
-    LAUNCH(kind, launch_chain(cm, ca, BN, cgrid, s, pdl));
+    ca.stall_phase = -1;
+    if (stall_pending && ca.nphases >= 2) {  // test hook: the first multi-phase launch of the step
+      ca.stall_phase = 1;
+      stall_pending = false;
+    }
+    for (int p = 0; p < ca.nphases; ++p) {  // consecutive phases feed each other
+      ca.ph[p].in_phase = p - 1;
+      ca.ph[p].in_N = p > 0 ? ca.ph[p - 1].N : 0;
+      ca.ph[p].publish = p + 1 < ca.nphases ? 1 : 0;
+    }
+    LAUNCH(kind, launch_chain(cm, ca, G, s, pdl));
     return CASSPEC_OK;
   };
   auto attention = [&](int l) -> int {
@@ -452,30 +503,26 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         continue;
       }
       if (nph == kMaxPhases && (rc = flush()) != CASSPEC_OK) return rc;
-      const int ss_tiles = i == 0 ? 1 : d / 128;  // the embedding leaves one partial, a residual d/128
-      PhaseDesc& p = ca.ph[nph];
+      const int ss_parts = i == 0 ? 1 : resid_parts;  // the embedding leaves one partial, a residual phase one per slice
+      ChainPhase& p = ca.ph[nph];
       switch (it.kind) {
         case IT_QKV:
-          ph_qkv(it.l, ss_tiles, p, cm.w[nph], cm.x[nph]);
+          ph_qkv(it.l, ss_parts, p, cm.x[nph]);
           break;
         case IT_WO:
-          ph_resid(d, reader_gain(items[i + 1]), p);
-          cm.w[nph] = m->layers[it.l].tm_o;
+          ph_resid(d, m->layers[it.l].wo_p, d / kRowGroup, reader_gain(items[i + 1]), p);
           cm.x[nph] = m->tm_o[bi];
           break;
         case IT_GU:
-          ph_gu(ss_tiles, p);
-          cm.w[nph] = m->layers[it.l].tm_g;
-          cm.w2[nph] = m->layers[it.l].tm_u;
+          ph_gu(it.l, ss_parts, p);
           cm.x[nph] = m->tm_xa[bi];
           break;
         case IT_DOWN:
-          ph_resid(F, reader_gain(items[i + 1]), p);
-          cm.w[nph] = m->layers[it.l].tm_d;
+          ph_resid(F, m->layers[it.l].wd_p, F / kRowGroup, reader_gain(items[i + 1]), p);
           cm.x[nph] = m->tm_u[bi];
           break;
         default:
-          ph_lm(ss_tiles, p, cm.w[nph], cm.x[nph]);
+          ph_lm(ss_parts, p, cm.x[nph]);
           break;
       }
       ++nph;
@@ -508,11 +555,11 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     for (size_t i = 0; i < items.size(); ++i) {
       const StepItem& it = items[i];
       int rc;
-      if (it.kind == IT_LM) {
+      if (it.kind == IT_LM) {  // the LM head stays bf16: the chain, after the W8A8 layers' residual tiles
         ChainArgs ca = {};
         ChainMaps cm = {};
         ca.nphases = 1;
-        ph_lm(i == 0 ? 1 : d / 128, ca.ph[0], cm.w[0], cm.x[0]);
+        ph_lm(i == 0 ? 1 : d / 128, ca.ph[0], cm.x[0]);
         if ((rc = chain(ca, cm, CASSPEC_K_LMHEAD)) != CASSPEC_OK) return rc;
         continue;
       }
@@ -551,7 +598,8 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       }
     }
   }
-  LAUNCH(CASSPEC_K_OTHER, launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, m->lay.lm_tiles, n, m->am, m->margin, s, pdl));
+  LAUNCH(CASSPEC_K_OTHER, launch_argmax_reduce(m->am_v1, m->am_i1, m->am_v2, std::min(roundup16(V) / kRowGroup, G), n,
+                                               m->am, m->margin, s, pdl));
   return CASSPEC_OK;
 }
 
@@ -596,6 +644,13 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   if (bytes < L.total) return CASSPEC_E_CAPACITY;
   const int sms = num_sms_of_current_device();
   if (sms <= 0 || sms > kSmsBound) return CASSPEC_E_CUDA;
+  {  // the projection chain's per-CTA slices must fit one MMA (and a residual slice the epilogue)
+    const int G = chain_grid(sms), d = cfg->d_model, F = cfg->ffn;
+    if (chain_slice_rows(d, G, false) > 64 || chain_slice_rows(3 * d, G, false) > 256 ||
+        chain_slice_rows(F, G, true) > 256 || chain_slice_rows(roundup16(cfg->vocab), G, false) > 256 ||
+        cdiv(F, 64) > kReadyPerPhase || cdiv(d, 64) > kReadyPerPhase)
+      return CASSPEC_E_SHAPE;
+  }
   casspec_model* m = new (std::nothrow) casspec_model();
   if (m == nullptr) return CASSPEC_E_CAPACITY;
   m->cfg = *cfg;
@@ -617,6 +672,10 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
     p.wg = reinterpret_cast<uint16_t*>(b + L.wg[l]);
     p.wu = reinterpret_cast<uint16_t*>(b + L.wu[l]);
     p.wd = reinterpret_cast<uint16_t*>(b + L.wd[l]);
+    p.wqkv_p = b + L.wqkv_p[l];
+    p.wo_p = b + L.wo_p[l];
+    p.wgu_p = b + L.wgu_p[l];
+    p.wd_p = b + L.wd_p[l];
     if (cfg->with_int8) {
       p.qkv_q = reinterpret_cast<int8_t*>(b + L.qkv_q[l]);
       p.wo_q = reinterpret_cast<int8_t*>(b + L.wo_q[l]);
@@ -636,8 +695,9 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   m->u = reinterpret_cast<uint16_t*>(b + L.u);
   m->xa = reinterpret_cast<uint16_t*>(b + L.xa);
   m->ssp = reinterpret_cast<float*>(b + L.ssp);
-  m->chain_cnt = reinterpret_cast<unsigned*>(b + L.chain_cnt);
-  m->chain_bar = reinterpret_cast<unsigned*>(b + L.chain_bar);
+  m->chain_ready = reinterpret_cast<unsigned*>(b + L.chain_ready);
+  m->chain_done = reinterpret_cast<unsigned*>(b + L.chain_done);
+  m->lm_p = b + L.lm_p;
   m->xq = reinterpret_cast<int8_t*>(b + L.xq);
   m->xs = reinterpret_cast<float*>(b + L.xs);
   m->pos = reinterpret_cast<int*>(b + L.pos);
@@ -697,7 +757,8 @@ int casspec_set_stream(casspec_model* m, void* stream) {
 }
 
 int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
-  if (m == nullptr || (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS)) != 0) return CASSPEC_E_INVAL;
+  if (m == nullptr || (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS | CASSPEC_OPT_TEST_STALL)) != 0)
+    return CASSPEC_E_INVAL;
   if (old_flags) *old_flags = m->flags;
   if (flags != m->flags) {
     for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second.first);
@@ -709,11 +770,13 @@ int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
 
 int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size_t* bytes) {
   if (m == nullptr || dev_ptr == nullptr) return CASSPEC_E_INVAL;
+  if (tensor <= CASSPEC_T_WD) m->pack_dirty = true;  // the caller may write through the pointer
   const auto& c = m->cfg;
   const size_t d = c.d_model, F = c.ffn, V = c.vocab;
-  const bool per_layer = tensor >= CASSPEC_T_ATTN_NORM;
+  const bool state = tensor >= CASSPEC_T_RESIDUAL;
+  const bool per_layer = tensor >= CASSPEC_T_ATTN_NORM && !state;
   if (per_layer && (layer < 0 || layer >= c.n_layers)) return CASSPEC_E_INVAL;
-  if (tensor >= CASSPEC_T_WQKV_Q && !c.with_int8) return CASSPEC_E_INVAL;
+  if (tensor >= CASSPEC_T_WQKV_Q && !state && !c.with_int8) return CASSPEC_E_INVAL;
   void* p = nullptr;
   size_t nb = 0;
   const LayerPtrs* L = per_layer ? &m->layers[layer] : nullptr;
@@ -738,6 +801,9 @@ int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size
     case CASSPEC_T_WG_S: p = L->wg_s; nb = F * 4; break;
     case CASSPEC_T_WU_S: p = L->wu_s; nb = F * 4; break;
     case CASSPEC_T_WD_S: p = L->wd_s; nb = d * 4; break;
+    case CASSPEC_T_RESIDUAL: p = m->x; nb = (size_t)kMaxTree * d * 4; break;
+    case CASSPEC_T_ACT_Q: p = m->xq; nb = (size_t)kMaxTree * std::max(d, F); break;
+    case CASSPEC_T_ACT_S: p = m->xs; nb = (size_t)kMaxTree * 4; break;
     default: return CASSPEC_E_INVAL;
   }
   *dev_ptr = p;
@@ -864,7 +930,12 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
 
   std::lock_guard<std::mutex> lock(m->mu);
   int rc = CASSPEC_OK;
-  if (m->flags & CASSPEC_OPT_GRAPHS) {
+  if (m->pack_dirty) {  // outside any capture: a graph never holds the packing
+    int count = 0;
+    if ((rc = pack_weights(m, count)) != CASSPEC_OK) return rc;
+    m->launches += (uint64_t)count;
+  }
+  if ((m->flags & CASSPEC_OPT_GRAPHS) && !(m->flags & CASSPEC_OPT_TEST_STALL)) {
     GraphKey key{kv, tokens, parent_idx, logits_out, n, kv->T, quant_mode, on};
     auto it = m->graphs.find(key);
     if (it == m->graphs.end()) {
@@ -929,8 +1000,8 @@ int casspec_kv_compact(casspec_kv* kv, const int32_t* accepted_out) {
     if (v != kv->T) return CASSPEC_E_STATE;
   casspec_model* m = kv->m;
   const auto& c = m->cfg;
-  CK(launch_kv_compact(kv->base, c.n_layers, c.n_heads, kv->ctx, c.head_dim, accepted_out, kv->T, kv->dP,
-                       kv->compact_cnt, m->status, m->stream));
+  CK(launch_kv_compact(kv->base, c.n_layers, c.n_heads, kv->ctx, c.head_dim, accepted_out, kv->tanc, kv->T,
+                       kv->dP, kv->compact_cnt, m->status, m->stream));
   m->launches++;
   kv->P_upper += kv->T;
   kv->T = 0;
@@ -976,8 +1047,8 @@ int casspec_get_status(casspec_model* m, int* status_out) {
     CK(cudaMemset(m->status, 0, 4));
     CK(cudaMemset(m->gemm_cnt, 0, (size_t)m->lay.max_tiles * 4));
     CK(cudaMemset(m->i8_cnt, 0, (size_t)m->lay.max_tiles * 4));
-    CK(cudaMemset(m->chain_cnt, 0, (size_t)kMaxPhases * 1024 * 4));
-    CK(cudaMemset(m->chain_bar, 0, 256));
+    CK(cudaMemset(m->chain_ready, 0, (size_t)kMaxPhases * kReadyPerPhase * 4));
+    CK(cudaMemset(m->chain_done, 0, 256));
     CK(cudaMemset(m->attn_cnt, 0, (size_t)2 * m->cfg.n_heads * 4));
   }
   if (status_out) *status_out = st;
@@ -1010,7 +1081,7 @@ int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int 
   if (n < 1 || n > kMaxTree || N < 1 || K < 8 || K % 8 != 0 || ldy < N) return CASSPEC_E_SHAPE;
   if (((uintptr_t)W & 15) || ((uintptr_t)X & 15) || ((uintptr_t)ws & 15)) return CASSPEC_E_INVAL;
   const int tiles = cdiv(N, 128);
-  if (tiles > 1024) return CASSPEC_E_SHAPE;
+  if (tiles > 1023) return CASSPEC_E_SHAPE;  // counters [0, tiles) and the status word at byte 4092
   if (ws_bytes < casspec_linear_workspace_bytes(N, K, n)) return CASSPEC_E_CAPACITY;
   const int sms = num_sms_of_current_device();
   if (sms <= 0) return CASSPEC_E_CUDA;
@@ -1025,7 +1096,7 @@ int casspec_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int 
   a.kblocks = kb;
   a.counters = static_cast<unsigned*>(ws);
   a.partials = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + 4096);
-  a.status = nullptr;
+  a.status = reinterpret_cast<int*>(static_cast<uint8_t*>(ws) + 4092);
   a.ep.n = n;
   a.ep.N = N;
   a.ep.y = Y;

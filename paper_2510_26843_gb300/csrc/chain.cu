@@ -1,54 +1,52 @@
-// Persistent projection chain on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+// Persistent projection chain on the 5th-generation tensor cores (tcgen05 + TMEM, bulk copies + TMA).
 //
 // One launch runs a list of dependent projections of a tree step -- e.g. Wo (+residual), Wgate/Wup
-// (+SwiGLU), Wdown (+residual), and the next layer's Wqkv (+rotary, K/V write) -- with a grid-wide
-// barrier between phases.  Only the activations depend on the previous phase; the weights do not,
-// so the weight stream runs on across phase boundaries and the HBM pipeline never drains between
-// projections.  Per CTA (one per SM):
-//   * warp 0 -- weight producer: streams the CTA's weight tiles (128 x 64 bf16, 128-byte swizzle,
-//     L2 evict-first) of every phase through a deep mbarrier ring, never waiting on activations;
-//   * warp 6 -- activation producer: after the phase barrier, streams the B operand tiles (BN x 64
-//     of the hi plane and of the lo plane of the split activation, 128-byte swizzle) by TMA;
-//   * warp 1 -- TMEM owner and single-thread MMA issuer: D += W hi^T + W lo^T (tcgen05.mma
-//     kind::f16, M = 128 channels, N = BN tokens), double-buffered accumulators in TMEM;
-//   * warps 2-5 -- epilogue: TMEM -> registers, stream-K fix-up (last CTA of a tile sums the partials
-//     in CTA order), the per-token RMSNorm factor, fused epilogue; then the CTA's arrival at the
-//     phase barrier.
-// Work of each phase is split stream-K over (tile, k-block) units so all SMs stream equal bytes.
-// Every wait is bounded (2 s) and reports CASSPEC_E_TIMEOUT instead of hanging.
+// (+SwiGLU), Wdown (+residual) and the next layer's Wqkv (+rotary, K/V write) or the LM head
+// (+argmax) -- with one CTA per SM.
+//
+// Work split: every projection Y[token][row] = sum_k X[token][k] W[row][k] is divided among the CTAs
+// by OUTPUT ROWS only.  CTA c owns a contiguous slice of 16-row groups (row_slice) and runs the whole
+// K range for it, so no output element is shared between CTAs: there are no partial sums, no fix-up
+// round trips, and each output is reduced in one fixed order (results do not depend on timing).
+//
+// MMA shape: the tokens are on M.  A = the split activation of one 64-column k-block, the hi plane in
+// rows 0..63 and the lo plane in rows 64..127 (16 KB, 128-byte swizzle, TMA); B = the CTA's weight
+// rows of that k-block (N = slice rows <= 256); D in TMEM, lane = plane row, column = output row.  The
+// epilogue adds the lo-plane lane to the hi-plane lane of each token, so 16 significant bits of the
+// activation reach the fp32 accumulation.
+//
+// Weights are stored pre-packed per CTA (pack_rows_kernel) as the 128-byte-swizzled shared-memory
+// image of the slice's k-blocks, in the order the CTA consumes them, so the weight producer streams
+// them with plain bulk copies into a ring of 32 KB stages and never waits on activations: the weight
+// stream runs on across phase boundaries.
+//
+// Phases are linked by per-k-block readiness counters instead of a grid barrier: a CTA counts the
+// rows it finished into the counter of every 64-column block its slice touches, and a consumer loads
+// k-block k once its counter holds all of the block's rows.  Each CTA walks its k-blocks starting
+// from the block that its own slice of the producing projection feeds (rotated order, baked into the
+// packed weights), so the first loads of a phase wait only on the CTA itself and its neighbours.
+//
+// Warps: 0 weight producer, 1 MMA issuer and TMEM owner, 2-5 epilogue (warps 4, 5 hold the hi-plane
+// lanes and run the per-token epilogue; warps 2, 3 hand over the lo-plane lanes through shared
+// memory), 6 activation producer.  Every wait is bounded (2 s) and reports CASSPEC_E_TIMEOUT instead
+// of hanging.
 #include "common.cuh"
-#include "epilogue.cuh"
 #include "kernels.h"
 
 namespace casspec {
 
 constexpr int kChainThreads = 224;
-constexpr uint32_t kWTile = 128 * 128;  // 128 rows x 64 bf16
-constexpr int kXStages = 4;
-constexpr uint32_t kChainSmemBudget = 232448u;  // 227 KB per CTA
+constexpr uint32_t kWStage = 32768;  // weight ring stage: whole k-blocks of the CTA's slice
+constexpr int kWStages = 5;
+constexpr uint32_t kXStage = 16384;  // one k-block of the split activation: 128 rows x 128 B
+constexpr int kXStages = 3;
+constexpr int kStgFloats = 2048;     // epilogue hand-over buffer: 32 rows x 64 tokens fp32 (two of them)
+constexpr uint32_t kTmemCols = 512;  // two accumulator buffers of up to 256 columns
 
-__host__ __device__ constexpr uint32_t chain_x_stage(int BN) { return 2u * (uint32_t)BN * 128u; }
-__host__ __device__ constexpr uint32_t chain_staging(int BN) { return (uint32_t)epi_staging_floats(BN) * 4u; }
-__host__ __device__ constexpr uint32_t chain_fixed(int BN) {
-  return 1024u + kXStages * chain_x_stage(BN) + chain_staging(BN) + 64u * 4u + 512u;
-}
-__host__ __device__ constexpr int chain_w_stages(int BN) {
-  return (int)((kChainSmemBudget - chain_fixed(BN)) / kWTile) > 12 ? 12
-                                                                   : (int)((kChainSmemBudget - chain_fixed(BN)) / kWTile);
-}
-__host__ __device__ constexpr size_t chain_smem(int BN) { return chain_fixed(BN) + (size_t)chain_w_stages(BN) * kWTile; }
-// TMEM per accumulator buffer: one accumulator of 2*BN columns (the hi and lo planes stacked as
-// one N = 2*BN operand); two buffers.
-__host__ __device__ constexpr uint32_t chain_buf_cols(int BN) { return 2u * (uint32_t)BN; }
-__host__ __device__ constexpr uint32_t chain_tmem_cols(int BN) {
-  return 2 * chain_buf_cols(BN) <= 64 ? 64 : (2 * chain_buf_cols(BN) <= 128 ? 128 : 256);
+__host__ __device__ constexpr size_t chain_smem() {
+  return 1024 + (size_t)kWStages * kWStage + (size_t)kXStages * kXStage + 2 * kStgFloats * 4 + 128 * 4 + 256;
 }
 
-__device__ __forceinline__ long long chain_u0(int c, long long U, int G) { return (long long)c * U / G; }
-// CTA that owns unit x when U units are split into G contiguous ranges [c U / G, (c + 1) U / G)
-__device__ __forceinline__ int chain_cta_of(long long x, long long U, int G) {
-  return (int)(((x + 1) * (long long)G - 1) / U);
-}
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -57,44 +55,47 @@ __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
 // generic-proxy global writes <-> async-proxy (TMA) reads of the split activations
 __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
-template <int BN, typename Bar>
-__device__ __forceinline__ void chain_epilogue(int epi, const EpiParams& e, int tile, int r, const float* v, float* stg,
-                                               Bar bar, int i0, int i1) {
-  switch (epi) {
-    case EPI_RESID: run_epilogue<BN, EPI_RESID>(e, tile, r, v, stg, bar, i0, i1); break;
-    case EPI_QKV: run_epilogue<BN, EPI_QKV>(e, tile, r, v, stg, bar, i0, i1); break;
-    case EPI_GLU: run_epilogue<BN, EPI_GLU>(e, tile, r, v, stg, bar, i0, i1); break;
-    case EPI_LMHEAD: run_epilogue<BN, EPI_LMHEAD>(e, tile, r, v, stg, bar, i0, i1); break;
-    default: run_epilogue<BN, EPI_STORE>(e, tile, r, v, stg, bar, i0, i1); break;
+// Wait until *p >= target (bounded; gives up on the CTA's abort flag).
+__device__ __forceinline__ bool wait_count(const unsigned* p, unsigned target, volatile int* abort) {
+  if (ld_acquire_u32(p) >= target) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (ld_acquire_u32(p) < target) {
+    if (*abort) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
   }
+  return true;
 }
 
-template <int BN>
+// 8 fp32 -> 8 bf16 of the hi plane (bf16(x)) or of the lo plane (bf16(x - bf16(x)))
+__device__ __forceinline__ uint4 split_pack8(const float* x, bool lo) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float a = x[2 * i], b = x[2 * i + 1];
+    const uint16_t ha = f2bf(a), hb = f2bf(b);
+    w[i] = lo ? pack_bf16x2(a - bf2f(ha), b - bf2f(hb)) : ((uint32_t)ha | ((uint32_t)hb << 16));
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 __global__ void __launch_bounds__(kChainThreads, 1)
     chain_kernel(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainArgs a) {
-  constexpr int SW = chain_w_stages(BN);
-  constexpr int SX = kXStages;
-  constexpr uint32_t XT = (uint32_t)BN * 128u;  // one hi or lo tile
-  constexpr uint32_t XS = 2 * XT;
-  constexpr uint32_t TMEM_COLS = chain_tmem_cols(BN);
-  constexpr uint32_t IDESC = idesc_bf16_f32(128, 2 * BN);  // B = [hi; lo], N = 2 * BN
-
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* wring = smem;
-  uint8_t* xring = smem + SW * kWTile;
-  float* stg = reinterpret_cast<float*>(xring + SX * XS);
-  float* rs = stg + epi_staging_floats(BN);
-  uint64_t* wfull = reinterpret_cast<uint64_t*>(rs + 64);
-  uint64_t* wempty = wfull + SW;
-  uint64_t* xfull = wempty + SW;
-  uint64_t* xempty = xfull + SX;
-  uint64_t* tfull = xempty + SX;
+  uint8_t* xring = wring + kWStages * kWStage;
+  float* stg = reinterpret_cast<float*>(xring + kXStages * kXStage);  // [2][32][64]
+  float* rs = stg + 2 * kStgFloats;                                   // [64] RMSNorm factors
+  float* rs2 = rs + 64;                                               // [64] second half of the sums
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(rs2 + 64);
+  uint64_t* wempty = wfull + kWStages;
+  uint64_t* xfull = wempty + kWStages;
+  uint64_t* xempty = xfull + kXStages;
+  uint64_t* tfull = xempty + kXStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
-  // [0] abort, [1] fix-up wait result, [2..9] per-warp accumulator-ready votes (two segments),
-  // [2] after the main loops: this CTA is the last out
+  // [0] abort, [1] wait result, [2..5] accumulator-ready votes, [6] last CTA out
   volatile int* flags = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -102,31 +103,26 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   const int np = a.nphases;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < SW; ++s) {
+    for (int s = 0; s < kWStages; ++s) {
       mbar_init(&wfull[s], 1);
       mbar_init(&wempty[s], 1);
     }
-    for (int s = 0; s < SX; ++s) {
+    for (int s = 0; s < kXStages; ++s) {
       mbar_init(&xfull[s], 1);
       mbar_init(&xempty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 4);
+      mbar_init(&tempty[b], 1);
     }
     mbar_init(drain, 1);
-    for (int f = 0; f < 10; ++f) flags[f] = 0;
+    for (int f = 0; f < 8; ++f) flags[f] = 0;
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) {
-    for (int p = 0; p < np; ++p) {
-      tma_prefetch_desc(&maps.w[p]);
-      if (a.ph[p].epi == EPI_GLU) tma_prefetch_desc(&maps.w2[p]);
-      tma_prefetch_desc(&maps.x[p]);
-    }
-  }
+  if (warp == 6 && lane == 0)
+    for (int p = 0; p < np; ++p) tma_prefetch_desc(&maps.x[p]);
   if (warp == 1) {
-    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -143,86 +139,88 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       uint32_t phase = 0;
       uint32_t armed = 0, armed_parity = 0;
       for (int p = 0; p < np && !flags[0]; ++p) {
-        const int kb = a.ph[p].kblocks;
-        const bool glu = a.ph[p].epi == EPI_GLU;
-        const long long U = (long long)a.ph[p].tiles * kb;
-        const long long u1 = chain_u0(cta + 1, U, G);
-        for (long long u = chain_u0(cta, U, G); u < u1; ++u) {
+        const int mult = a.ph[p].epi == EPI_GLU ? 2 : 1;
+        const int kb = a.ph[p].kb;
+        const RowSlice s = row_slice(cta, a.ph[p].N / kRowGroup, G);
+        if (s.ng == 0) continue;
+        const uint32_t chunk = (uint32_t)(s.ng * kRowGroup * mult) * 128u;  // one k-block of the slice
+        const int kpb = (int)(kWStage / chunk);
+        const uint8_t* src = a.ph[p].wp + (size_t)s.g0 * kRowGroup * mult * kb * 128;
+        for (int j0 = 0; j0 < kb; j0 += kpb) {
+          const int nk = min(kpb, kb - j0);
           if (!mbar_wait_bounded(&wempty[stage], phase ^ 1, flags)) {
             flags[0] = 1;
             set_status(a.status, CASSPEC_E_TIMEOUT);
             break;
           }
-          const int t = (int)(u / kb), k = (int)(u % kb);
-          mbar_expect_tx(&wfull[stage], kWTile);
+          const uint32_t bytes = (uint32_t)nk * chunk;
+          mbar_expect_tx(&wfull[stage], bytes);
           armed |= 1u << stage;
           armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
-          uint8_t* sa = wring + stage * kWTile;
-          if (glu) {
-            tma_load_2d(sa, &maps.w[p], &wfull[stage], k * 64, t * 64, pol);
-            tma_load_2d(sa + kWTile / 2, &maps.w2[p], &wfull[stage], k * 64, t * 64, pol);
-          } else {
-            tma_load_2d(sa, &maps.w[p], &wfull[stage], k * 64, t * 128, pol);
-          }
-          if (++stage == SW) {
+          bulk_load_hint(wring + stage * kWStage, src + (size_t)j0 * chunk, bytes, &wfull[stage], pol);
+          if (++stage == kWStages) {
             stage = 0;
             phase ^= 1;
           }
         }
       }
       if (flags[0]) {  // abort: let the copies already issued land before the CTA exits
-        for (int s = 0; s < SW; ++s)
+        for (int s = 0; s < kWStages; ++s)
           if (armed & (1u << s)) mbar_wait_bounded(&wfull[s], (armed_parity >> s) & 1, nullptr);
       }
     }
   } else if (warp == 6) {
     if (lane == 0) {
-      // ---------------- activation producer (waits for the phase barrier) ----------------
+      // ---------------- activation producer ----------------
+      // Inputs of a phase that reads an earlier kernel's output, and the readiness counters (reset by
+      // the previous launch's last CTA), are valid only once the preceding kernels have completed.
+      pdl_wait();
       const uint64_t pol = policy_evict_last();
+      const uint32_t xbytes = 2u * (uint32_t)a.bn * 128u;
       int stage = 0;
       uint32_t phase = 0;
       uint32_t armed = 0, armed_parity = 0;
       for (int p = 0; p < np && !flags[0]; ++p) {
-        if (p == 0) {
-          pdl_wait();  // inputs of the first phase come from the previous kernel
-        } else {       // ... of the others from phase p - 1 of every CTA (one counter per phase:
-                       // a CTA with no work may run ahead and arrive at later phases early)
-          const uint64_t t0 = globaltimer_ns();
-          while (ld_acquire_u32(a.bar + (p - 1)) < (unsigned)G) {
-            if (flags[0]) break;
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        const RowSlice s = row_slice(cta, a.ph[p].N / kRowGroup, G);
+        if (s.ng == 0) continue;
+        const int kb = a.ph[p].kb;
+        const int in_phase = a.ph[p].in_phase, in_N = a.ph[p].in_N;
+        const int rot = a.ph[p].rot_groups;
+        int k0 = 0;
+        if (rot > 0) k0 = (row_slice(cta, rot, G).g0 * kRowGroup / 64) % kb;
+        const unsigned* rdy = in_phase >= 0 ? a.ready + in_phase * kReadyPerPhase : nullptr;
+        const unsigned extra = p == a.stall_phase ? 1u : 0u;  // test hook: a count that never completes
+        for (int j = 0; j < kb; ++j) {
+          int k = k0 + j;
+          if (k >= kb) k -= kb;
+          if (rdy != nullptr) {
+            const unsigned target = (unsigned)min(64, in_N - 64 * k) + extra;
+            if (!wait_count(rdy + k, target, flags)) {
               flags[0] = 1;
               set_status(a.status, CASSPEC_E_TIMEOUT);
               break;
             }
+            fence_proxy_async_global();
           }
-          if (flags[0]) break;
-        }
-        fence_proxy_async_global();
-        const int kb = a.ph[p].kblocks;
-        const long long U = (long long)a.ph[p].tiles * kb;
-        const long long u1 = chain_u0(cta + 1, U, G);
-        for (long long u = chain_u0(cta, U, G); u < u1; ++u) {
           if (!mbar_wait_bounded(&xempty[stage], phase ^ 1, flags)) {
             flags[0] = 1;
             set_status(a.status, CASSPEC_E_TIMEOUT);
             break;
           }
-          const int k = (int)(u % kb);
-          mbar_expect_tx(&xfull[stage], XS);
+          mbar_expect_tx(&xfull[stage], xbytes);
           armed |= 1u << stage;
           armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
-          uint8_t* sx = xring + stage * XS;
-          tma_load_2d(sx, &maps.x[p], &xfull[stage], k * 64, 0, pol);        // hi plane, tokens 0..BN-1
-          tma_load_2d(sx + XT, &maps.x[p], &xfull[stage], k * 64, 64, pol);  // lo plane
-          if (++stage == SX) {
+          uint8_t* sx = xring + stage * kXStage;
+          tma_load_2d(sx, &maps.x[p], &xfull[stage], k * 64, 0, pol);          // hi plane -> rows 0..bn-1
+          tma_load_2d(sx + 8192, &maps.x[p], &xfull[stage], k * 64, 64, pol);  // lo plane -> rows 64..
+          if (++stage == kXStages) {
             stage = 0;
             phase ^= 1;
           }
         }
       }
       if (flags[0]) {
-        for (int s = 0; s < SX; ++s)
+        for (int s = 0; s < kXStages; ++s)
           if (armed & (1u << s)) mbar_wait_bounded(&xfull[s], (armed_parity >> s) & 1, nullptr);
       }
     }
@@ -232,54 +230,60 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       int ws = 0, xs = 0;
       uint32_t wph = 0, xph = 0;
       uint32_t used[2] = {0, 0};
-      int buf = 0;
+      int pc = 0;
       bool ok = true;
       for (int p = 0; p < np && ok; ++p) {
-        const int kb = a.ph[p].kblocks;
-        const long long U = (long long)a.ph[p].tiles * kb;
-        const long long u1 = chain_u0(cta + 1, U, G);
-        long long u = chain_u0(cta, U, G);
-        while (u < u1 && ok) {
-          const int t = (int)(u / kb);
-          const long long seg_end = ((long long)(t + 1) * kb < u1) ? (long long)(t + 1) * kb : u1;
-          if (!mbar_wait_bounded(&tempty[buf], (used[buf] & 1) ^ 1, flags)) {
+        const int mult = a.ph[p].epi == EPI_GLU ? 2 : 1;
+        const int kb = a.ph[p].kb;
+        const RowSlice s = row_slice(cta, a.ph[p].N / kRowGroup, G);
+        if (s.ng == 0) continue;
+        const int ncols = s.ng * kRowGroup * mult;
+        const uint32_t chunk = (uint32_t)ncols * 128u;
+        const int kpb = (int)(kWStage / chunk);
+        const uint32_t idesc = idesc_bf16_f32(128, ncols);
+        const int buf = pc & 1;
+        if (!mbar_wait_bounded(&tempty[buf], (used[buf] & 1) ^ 1, flags)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)buf * 256u;
+        int j = 0;
+        for (int j0 = 0; j0 < kb && ok; j0 += kpb) {
+          const int nk = min(kpb, kb - j0);
+          if (!mbar_wait_bounded(&wfull[ws], wph, flags)) {
             ok = false;
             break;
           }
-          tc_fence_after();
-          const uint32_t d_tmem = tmem_base + (uint32_t)buf * chain_buf_cols(BN);
-          for (long long uu = u; uu < seg_end; ++uu) {
-            if (!mbar_wait_bounded(&wfull[ws], wph, flags) || !mbar_wait_bounded(&xfull[xs], xph, flags)) {
+          for (int jj = 0; jj < nk; ++jj, ++j) {
+            if (!mbar_wait_bounded(&xfull[xs], xph, flags)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_u32(wring + ws * kWTile);
-            const uint32_t sh = smem_u32(xring + xs * XS);
-            // One MMA per 16-column k-step with the hi and lo planes stacked (N = 2 * BN, the X stage
-            // holds them back to back), all into one accumulator: splitting even and odd k-steps
-            // over two accumulators measured slower.
+            const uint32_t sa = smem_u32(xring + xs * kXStage);
+            const uint32_t sb = smem_u32(wring + ws * kWStage) + (uint32_t)jj * chunk;
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              tc_mma_bf16(d_tmem, sw128_kmajor_desc(sa + kk * 32), sw128_kmajor_desc(sh + kk * 32), IDESC,
-                          (uu > u || kk > 0) ? 1u : 0u);
-            tc_commit(&wempty[ws]);
+              tc_mma_bf16(d_tmem, sw128_kmajor_desc(sa + kk * 32), sw128_kmajor_desc(sb + kk * 32), idesc,
+                          (j > 0 || kk > 0) ? 1u : 0u);
             tc_commit(&xempty[xs]);
-            if (++ws == SW) {
-              ws = 0;
-              wph ^= 1;
-            }
-            if (++xs == SX) {
+            if (++xs == kXStages) {
               xs = 0;
               xph ^= 1;
             }
           }
           if (!ok) break;
-          tc_commit(&tfull[buf]);
-          used[buf]++;
-          buf ^= 1;
-          u = seg_end;
+          tc_commit(&wempty[ws]);
+          if (++ws == kWStages) {
+            ws = 0;
+            wph ^= 1;
+          }
         }
+        if (!ok) break;
+        tc_commit(&tfull[buf]);
+        used[buf]++;
+        ++pc;
       }
       if (!ok) {
         flags[0] = 1;
@@ -292,222 +296,276 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     // ---------------- epilogue warps 2..5 ----------------
     // Control flow is identical in the four warps (every decision that follows a bounded wait is
     // voted through shared memory), so their named barriers always match, even after a timeout.
-    const int q = warp & 3;
-    const int r = q * 32 + lane;
+    const int q = warp & 3;             // TMEM lane quarter of this warp
+    const bool hi = q < 2;              // lanes 0..63 hold the hi-plane rows, 64..127 the lo-plane rows
+    const int t = (q & 1) * 32 + lane;  // token of this thread
+    const int et = threadIdx.x - 64;    // 0..127
     auto bar = [] { named_bar_sync(1, 128); };
-    // The phase-barrier counters belong to the previous launch until it has completed (its last
-    // CTA resets them); a CTA without units could otherwise arrive before that reset.
     pdl_wait();
     uint32_t used[2] = {0, 0};
-    int buf = 0, seg = 0;
+    int pc = 0;
     for (int p = 0; p < np; ++p) {
-      // The phase descriptor sits in parameter space behind a runtime index: copy what the loops
-      // use into registers once, so no load of it is ordered behind the epilogue's stores.
+      // The phase descriptor sits in parameter space behind a runtime index: copy what the loops use.
       const EpiParams ep = a.ph[p].ep;
-      const int epi = a.ph[p].epi, kb = a.ph[p].kblocks, Kp = a.ph[p].K, n = ep.n;
+      const int epi = a.ph[p].epi;
+      const int mult = epi == EPI_GLU ? 2 : 1;
+      const RowSlice s = row_slice(cta, a.ph[p].N / kRowGroup, G);
+      if (s.ng == 0) continue;
+      const int R = s.ng * kRowGroup;  // output rows (EPI_GLU: channels) of this CTA
+      const int r0 = s.g0 * kRowGroup;
+      const int n = ep.n;
       const float* ss = a.ph[p].ss;
-      const int ss_tiles = a.ph[p].ss_tiles;
-      const float eps = a.ph[p].eps;
-      const long long U = (long long)a.ph[p].tiles * kb;
-      const long long u1 = chain_u0(cta + 1, U, G);
-      unsigned* counters = a.counters + p * 1024;
-      bool have_rs = false;
-      long long u = chain_u0(cta, U, G);
-      while (u < u1) {
-        const int t = (int)(u / kb);
-        const long long seg_end = ((long long)(t + 1) * kb < u1) ? (long long)(t + 1) * kb : u1;
-        const bool got = mbar_wait_bounded(&tfull[buf], used[buf] & 1, flags);
-        if (lane == 0) flags[2 + (seg & 1) * 4 + q] = got ? 1 : 0;
+      const int buf = pc & 1;
+      ++pc;
+
+      // (1) the RMSNorm factor of this phase's tokens, once every producer has counted in (overlaps
+      // this phase's MMAs): rs[t] = rsqrt(sum of the producers' partial sums of squares / K + eps)
+      if (ss != nullptr) {
+        const int in_phase = a.ph[p].in_phase;
+        if (et == 0) {
+          int ok = 1;
+          if (in_phase >= 0) {
+            const unsigned target = (unsigned)min(a.ph[in_phase].N / kRowGroup, G);
+            ok = wait_count(a.done + in_phase, target, flags) ? 1 : 0;
+            if (!ok) {
+              flags[0] = 1;
+              set_status(a.status, CASSPEC_E_TIMEOUT);
+            }
+          }
+          flags[1] = ok;
+        }
         bar();
-        const int vote = (seg & 1) * 4;
-        const bool ready = flags[2 + vote] && flags[3 + vote] && flags[4 + vote] && flags[5 + vote];
-        ++seg;
-        used[buf]++;
-        if (!ready) {  // the accumulator never arrived: give up on the rest (uniformly)
+        const bool ok = flags[1] != 0;
+        if (ok) {
+          const int parts = a.ph[p].ss_parts;
+          const int tt = et & 63, half = et >> 6;
+          const int c0 = half * (parts / 2), c1 = half ? parts : parts / 2;
+          float acc = 0.f;
+          for (int c = c0; c < c1; c += 16) {  // 16 loads in flight, summed in a fixed order
+            float v16[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) v16[k] = c + k < c1 ? __ldcg(ss + (size_t)(c + k) * 64 + tt) : 0.f;
+#pragma unroll
+            for (int k = 0; k < 16; ++k) acc += v16[k];
+          }
+          (half ? rs2 : rs)[tt] = acc;
+        }
+        bar();
+        if (ok && et < 64) rs[et] = rsqrtf((rs[et] + rs2[et]) / (float)a.ph[p].K + a.ph[p].eps);
+        bar();
+      }
+
+      // residual epilogue: this CTA's slice of the residual rows (written by this CTA's own earlier
+      // phases, same slicing, or by an earlier kernel) is loaded while the MMAs run
+      float4 xo[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) xo[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (epi == EPI_RESID && hi && t < n) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+          if (4 * k < R) xo[k] = __ldcg(reinterpret_cast<const float4*>(ep.y + (size_t)t * ep.ldy + r0) + k);
+      }
+      int pos_t = 0, P = 0;
+      if (epi == EPI_QKV) {
+        P = __ldcg(ep.dP);
+        pos_t = t < n ? __ldcg(ep.pos + t) : 0;
+      }
+
+      // (2) the accumulator of this phase
+      const bool got = mbar_wait_bounded(&tfull[buf], used[buf] & 1, flags);
+      if (lane == 0) flags[2 + q] = got ? 1 : 0;
+      bar();
+      const bool ready = flags[2] && flags[3] && flags[4] && flags[5];
+      used[buf]++;
+      bar();  // every warp has read the votes before they are rewritten
+      if (!ready) {
+        if (et == 0) {
           flags[0] = 1;
           set_status(a.status, CASSPEC_E_TIMEOUT);
-          u = seg_end;
-          buf ^= 1;
-          continue;
         }
-        if (ss != nullptr && !have_rs) {
-          // the phase's inputs are visible here: this accumulator was computed from them
-          if (r < 64) {
-            float ssum = 0.f;  // fixed summation order; loads issued 8 at a time
-            for (int j0 = 0; j0 < ss_tiles; j0 += 8) {
-              float t8[8];
-#pragma unroll
-              for (int k = 0; k < 8; ++k) t8[k] = j0 + k < ss_tiles ? __ldcg(ss + (j0 + k) * 64 + r) : 0.f;
-#pragma unroll
-              for (int k = 0; k < 8; ++k) ssum += t8[k];
-            }
-            rs[r] = rsqrtf(ssum / (float)Kp + eps);
-          }
-          bar();
-          have_rs = true;
-        }
-        tc_fence_after();
-        float v[BN];
-        const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)buf * chain_buf_cols(BN);
-#pragma unroll
-        for (int c = 0; c < BN; c += 16) {  // hi-plane product + lo-plane product
-          float t1[16];
-          tmem_ld_x16(taddr + c, &v[c]);
-          tmem_ld_x16(taddr + BN + c, t1);
+        continue;
+      }
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)buf * 256u;
+
+      // (3) 16 output rows (EPI_GLU: 16 channels, gate and up) at a time: the lo-plane warps hand
+      // their lanes to the hi-plane warps through a double-buffered staging area
+      float ssq = 0.f;                       // EPI_RESID: sum of squares of the updated rows
+      float m1 = -INFINITY, m2 = -INFINITY;  // EPI_LMHEAD: max, second max
+      int i1 = 0x7fffffff;                   //            argmax
+      const float rsv = (ss != nullptr) ? rs[t] : 1.f;
+      const int nchunks = R / 16;
+      for (int c = 0; c < nchunks; ++c) {
+        float* sb = stg + (c & 1) * kStgFloats;
+        float v[32];
+        if (!hi) {
+          tmem_ld_x16(tbase + (uint32_t)(c * 16), v);
+          if (mult == 2) tmem_ld_x16(tbase + (uint32_t)(R + c * 16), v + 16);
           tmem_ld_wait();
 #pragma unroll
-          for (int j = 0; j < 16; ++j) v[c + j] += t1[j];
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[buf]);
-        buf ^= 1;
-
-        // Stream-K fix-up.  Every owner of a shared tile deposits its partial ([token][row] slot
-        // t + cta) and counts itself in.  The owners for which the tile is their last segment of
-        // the phase (all but possibly the one that holds the tile's tail at the start of its range)
-        // reach it together at the end of the phase: each waits for every deposit, sums one slice
-        // of the tokens over the owners in CTA order (deterministic) and runs the epilogue on it.
-        // CTAs with no unit at all (phases with fewer units than CTAs) are not owners.
-        const int c_first = chain_cta_of((long long)t * kb, U, G);
-        const int c_last = chain_cta_of((long long)(t + 1) * kb - 1, U, G);
-        int i0 = 0, i1 = n;
-        bool finish = true;
-        if (c_first != c_last) {
-          const long long tile_end = (long long)(t + 1) * kb;
-          int owners = 0, parts = 0, rank = 0;
-          int own_list[6];  // the first 6 owners in CTA order
-          for (int cc = c_first; cc <= c_last; ++cc) {
-            const long long b0 = chain_u0(cc, U, G), b1 = chain_u0(cc + 1, U, G);
-            if (b1 <= b0) continue;
+          for (int i = 0; i < 16; ++i) sb[i * 64 + t] = v[i];
+          if (mult == 2) {
 #pragma unroll
-            for (int o = 0; o < 6; ++o)
-              if (o == owners) own_list[o] = cc;
-            ++owners;
-            if (b1 <= tile_end) {
-              if (cc == cta) rank = parts;
-              ++parts;
-            }
-          }
-          // own partial token-major in shared memory ([token][row], the slot layout), then coalesced
-          // 16-byte stores of the valid tokens into slot t + cta
-#pragma unroll
-          for (int i = 0; i < BN; ++i) stg[i * 128 + r] = v[i];
-          bar();
-          const int nf4 = n * 32;
-          const float4* own4 = reinterpret_cast<const float4*>(stg);
-          {
-            float4* mine4 = reinterpret_cast<float4*>(a.partials + (size_t)(t + cta) * (64 * 128));
-#pragma unroll
-            for (int j = 0; j < BN / 4; ++j)
-              if (r + 128 * j < nf4) __stcg(mine4 + r + 128 * j, own4[r + 128 * j]);
-          }
-          bar();  // then one gpu-scope fence (cumulative over the CTA's stores) before counting in
-          if (threadIdx.x == 64) {
-            __threadfence();
-            atomicAdd(&counters[t], 1u);
-          }
-          finish = seg_end == u1;  // a participant: this is the CTA's last segment of the phase
-          if (finish) {
-            if (threadIdx.x == 64) {
-              const uint64_t t0 = globaltimer_ns();
-              int ok = 1;
-              while (ld_acquire_u32(counters + t) < (unsigned)owners) {
-                if (flags[0] || globaltimer_ns() - t0 > kWaitLimitNs) {
-                  ok = 0;
-                  flags[0] = 1;
-                  set_status(a.status, CASSPEC_E_TIMEOUT);
-                  break;
-                }
-              }
-              flags[1] = ok;
-            }
-            bar();
-            finish = flags[1] != 0;
-            i0 = rank * n / parts;
-            i1 = (rank + 1) * n / parts;
-          }
-          if (finish && i1 > i0) {
-            __threadfence();
-            const int f0 = i0 * 32, f1 = i1 * 32;  // float4s of the slice
-            float4 acc[BN / 4];
-#pragma unroll
-            for (int j = 0; j < BN / 4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-            auto add4 = [](float4& x, const float4& y) {
-              x.x += y.x;
-              x.y += y.y;
-              x.z += y.z;
-              x.w += y.w;
-            };
-            if (owners <= 6 && f1 - f0 <= 4 * 128) {
-              // a small slice (at most 4 float4s per thread) from at most 6 owners: every load in
-              // flight together; sums in CTA order
-              float4 t4[6][4];
-#pragma unroll
-              for (int o = 0; o < 6; ++o) {
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                  const int f = f0 + r + 128 * j;
-                  float4 val = make_float4(0.f, 0.f, 0.f, 0.f);
-                  if (o < owners && f < f1) {
-                    const int cc = own_list[o];
-                    val = cc == cta ? own4[f]
-                                    : __ldcg(reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128)) + f);
-                  }
-                  t4[o][j] = val;
-                }
-              }
-#pragma unroll
-              for (int o = 0; o < 6; ++o) {
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                  if (j < BN / 4) add4(acc[j], t4[o][j]);
-              }
-            } else {  // larger slices or many owners: one owner at a time, all its loads in flight
-              for (int cc = c_first; cc <= c_last; ++cc) {
-                if (cc != cta && chain_u0(cc + 1, U, G) <= chain_u0(cc, U, G)) continue;
-                const float4* src = cc == cta ? own4
-                                              : reinterpret_cast<const float4*>(a.partials + (size_t)(t + cc) * (64 * 128));
-                float4 t4[BN / 4];
-#pragma unroll
-                for (int j = 0; j < BN / 4; ++j) {
-                  const int f = f0 + r + 128 * j;
-                  t4[j] = f < f1 ? (cc == cta ? src[f] : __ldcg(src + f)) : make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-#pragma unroll
-                for (int j = 0; j < BN / 4; ++j) add4(acc[j], t4[j]);
-              }
-            }
-            bar();
-            float4* st4 = reinterpret_cast<float4*>(stg);
-#pragma unroll
-            for (int j = 0; j < BN / 4; ++j) {
-              const int f = f0 + r + 128 * j;
-              if (f < f1) st4[f] = acc[j];
-            }
-            bar();
-#pragma unroll
-            for (int i = 0; i < BN; ++i) v[i] = stg[i * 128 + r];
+            for (int i = 0; i < 16; ++i) sb[(16 + i) * 64 + t] = v[16 + i];
           }
         }
-        if (finish && i1 > i0) {
-          if (ss != nullptr) {
-#pragma unroll
-            for (int i = 0; i < BN; ++i) v[i] *= rs[i];
-          }
-          chain_epilogue<BN>(epi, ep, t, r, v, stg, bar, i0, i1);
-        }
-        u = seg_end;
-      }
-      if (have_rs) bar();  // rs is rewritten by the next phase only after every thread used it
-      if (p + 1 < np) {  // this CTA's writes of phase p are done: arrive at the phase barrier
-        fence_proxy_async_global();
-        __threadfence();
         bar();
-        if (threadIdx.x == 64) {
-          __threadfence();
-          atomicAdd(&a.bar[p], 1u);
+        if (hi) {
+          tmem_ld_x16(tbase + (uint32_t)(c * 16), v);
+          if (mult == 2) tmem_ld_x16(tbase + (uint32_t)(R + c * 16), v + 16);
+          tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] = (v[i] + sb[i * 64 + t]) * rsv;
+          if (mult == 2) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[16 + i] = (v[16 + i] + sb[(16 + i) * 64 + t]) * rsv;
+          }
+          const int col = r0 + c * 16;  // first output row (channel) of the chunk
+          if (t < n) {
+            if (epi == EPI_RESID) {
+              float nv[16];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                float4 o4 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int kk = 0; kk < 16; ++kk)
+                  if (kk == 4 * c + k) o4 = xo[kk];  // register-resident old values (compile-time index)
+                nv[4 * k + 0] = o4.x + v[4 * k + 0];
+                nv[4 * k + 1] = o4.y + v[4 * k + 1];
+                nv[4 * k + 2] = o4.z + v[4 * k + 2];
+                nv[4 * k + 3] = o4.w + v[4 * k + 3];
+              }
+              float4* dst = reinterpret_cast<float4*>(ep.y + (size_t)t * ep.ldy + col);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) dst[k] = make_float4(nv[4 * k], nv[4 * k + 1], nv[4 * k + 2], nv[4 * k + 3]);
+#pragma unroll
+              for (int i = 0; i < 16; ++i) ssq += nv[i] * nv[i];
+              if (ep.xa_out != nullptr) {
+                float g[16];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const float4 g4 = __ldg(reinterpret_cast<const float4*>(ep.g_next + col) + k);
+                  g[4 * k] = nv[4 * k] * g4.x;
+                  g[4 * k + 1] = nv[4 * k + 1] * g4.y;
+                  g[4 * k + 2] = nv[4 * k + 2] * g4.z;
+                  g[4 * k + 3] = nv[4 * k + 3] * g4.w;
+                }
+                uint4* xh = reinterpret_cast<uint4*>(ep.xa_out + (size_t)t * ep.ldy + col);
+                uint4* xl = reinterpret_cast<uint4*>(ep.xa_out + (size_t)(64 + t) * ep.ldy + col);
+                xh[0] = split_pack8(g, false);
+                xh[1] = split_pack8(g + 8, false);
+                xl[0] = split_pack8(g, true);
+                xl[1] = split_pack8(g + 8, true);
+              }
+            } else if (epi == EPI_GLU) {
+              float u[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const float gt = v[i];
+                // fast exponential and division: ~1e-6 relative error, below the 16-bit split
+                u[i] = __fdividef(gt, 1.f + __expf(-gt)) * v[16 + i];
+              }
+              uint4* uh = reinterpret_cast<uint4*>(ep.u_out + (size_t)t * ep.N + col);
+              uint4* ul = reinterpret_cast<uint4*>(ep.u_out + (size_t)(64 + t) * ep.N + col);
+              uh[0] = split_pack8(u, false);
+              uh[1] = split_pack8(u + 8, false);
+              ul[0] = split_pack8(u, true);
+              ul[1] = split_pack8(u + 8, true);
+            } else if (epi == EPI_QKV) {
+              // a 16-row group holds 8 rotary pairs: rows 0..7 are dims a0..a0+7 of one head of q, k
+              // or v, rows 8..15 their partners a0+hd/2 .. (the packing order, qkv_src_row)
+              const int g = col / kRowGroup;
+              const int gpp = ep.d / kRowGroup;  // groups per part (q, k, v)
+              const int part = g / gpp;
+              const int gp = g - part * gpp;
+              const int gph = ep.hd / kRowGroup;  // groups per head
+              const int head = gp / gph;
+              const int a0 = (gp - head * gph) * 8;
+              const int half = ep.hd >> 1;
+              float o[16];
+              if (part < 2) {
+                const float4* cs = reinterpret_cast<const float4*>(ep.rope + (size_t)pos_t * half + a0);
+                float cv[8], sv[8];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const float4 c4 = __ldg(cs + k);  // (cos, sin) of two frequencies
+                  cv[2 * k] = c4.x;
+                  sv[2 * k] = c4.y;
+                  cv[2 * k + 1] = c4.z;
+                  sv[2 * k + 1] = c4.w;
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                  const float x = v[i], y = v[8 + i];
+                  o[i] = x * cv[i] - y * sv[i];
+                  o[8 + i] = y * cv[i] + x * sv[i];
+                }
+              } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) o[i] = v[i];
+              }
+              const uint4 first = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]),
+                                             pack_bf16x2(o[4], o[5]), pack_bf16x2(o[6], o[7]));
+              const uint4 second = make_uint4(pack_bf16x2(o[8], o[9]), pack_bf16x2(o[10], o[11]),
+                                              pack_bf16x2(o[12], o[13]), pack_bf16x2(o[14], o[15]));
+              uint16_t* base;
+              if (part == 0)
+                base = ep.q_out + (size_t)t * ep.d + head * ep.hd;
+              else
+                base = (part == 1 ? ep.kc : ep.vc) + ((size_t)head * ep.ctx + (P + ep.T + t)) * ep.hd;
+              *reinterpret_cast<uint4*>(base + a0) = first;
+              *reinterpret_cast<uint4*>(base + half + a0) = second;
+            } else {  // EPI_LMHEAD
+              // ep.N = vocabulary size (a multiple of 8); rows beyond it are zero padding of the last group
+              if (ep.logits != nullptr) {
+                float4* dst = reinterpret_cast<float4*>(ep.logits + (size_t)t * ep.N + col);
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                  if (col + 4 * k < ep.N) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+              }
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {  // increasing vocabulary id: ties keep the lowest
+                if (col + i >= ep.N) break;
+                if (v[i] > m1) {
+                  m2 = m1;
+                  m1 = v[i];
+                  i1 = col + i;
+                } else if (v[i] > m2) {
+                  m2 = v[i];
+                }
+              }
+            }
+          }
         }
+      }
+      // every TMEM read of this buffer is complete: hand it back to the MMA issuer
+      tc_fence_before();
+      bar();
+      if (et == 0) mbar_arrive(&tempty[buf]);
+      // per-slice partial results (slice index = CTA index)
+      if (hi) {
+        if (epi == EPI_RESID && ep.ss_out != nullptr) ep.ss_out[(size_t)cta * 64 + t] = t < n ? ssq : 0.f;
+        if (epi == EPI_LMHEAD) {
+          ep.am_v1[(size_t)cta * 64 + t] = m1;
+          ep.am_i1[(size_t)cta * 64 + t] = i1 == 0x7fffffff ? r0 : i1;
+          ep.am_v2[(size_t)cta * 64 + t] = m2;
+        }
+      }
+      // (4) publish: the slice's rows into the readiness counters of the 64-column blocks they
+      // belong to, and the CTA into the phase's completion count
+      fence_proxy_async_global();
+      __threadfence();
+      bar();
+      if (et == 0) {
+        __threadfence();
+        if (a.ph[p].publish) {
+          unsigned* rdy = a.ready + p * kReadyPerPhase;
+          for (int k = r0 / 64; k * 64 < r0 + R; ++k) {
+            const int lo = max(r0, 64 * k), hi_ = min(r0 + R, 64 * k + 64);
+            atomicAdd(rdy + k, (unsigned)(hi_ - lo));
+          }
+        }
+        atomicAdd(a.done + p, 1u);
       }
     }
   }
@@ -516,39 +574,121 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    tmem_dealloc(tmem_base, kTmemCols);
   }
-  // The last CTA out returns the phase-barrier, exit and fix-up counters to zero for the next
-  // launch (they belong to the previous launch until it completes, hence the dependency wait).
+  // The last CTA out returns the readiness and completion counters to zero for the next launch
+  // (they belong to the previous launch until it completes, hence the dependency wait).
   if (threadIdx.x == 0) {
     pdl_wait();
     __threadfence();
-    flags[2] = atomicAdd(&a.bar[kMaxPhases], 1u) == (unsigned)(G - 1) ? 1 : 0;
+    flags[6] = atomicAdd(a.done + kMaxPhases, 1u) == (unsigned)(G - 1) ? 1 : 0;
   }
   __syncthreads();
-  if (flags[2]) {
+  if (flags[6]) {
     __threadfence();
-    for (int p = threadIdx.x; p <= kMaxPhases; p += blockDim.x) a.bar[p] = 0u;
-    for (int p = 0; p < np; ++p)
-      for (int t = threadIdx.x; t < a.ph[p].tiles; t += blockDim.x) a.counters[p * 1024 + t] = 0u;
+    for (int i = threadIdx.x; i < np * kReadyPerPhase; i += blockDim.x) a.ready[i] = 0u;
+    if (threadIdx.x <= kMaxPhases) a.done[threadIdx.x] = 0u;
   }
+}
+
+// ---------------------------------------------------------------------------------------------
+// packing of a projection's weights into the per-CTA stream the chain consumes
+// ---------------------------------------------------------------------------------------------
+// Source row of packed row `row` of a QKV projection: each 16-row group holds dims a0..a0+7 and
+// a0+hd/2 .. a0+hd/2+7 of one head of q, k or v (8 rotary pairs), a0 = 8 * (group within the head).
+__host__ __device__ inline int qkv_src_row(int row, int d, int hd) {
+  const int g = row / kRowGroup, i = row % kRowGroup;
+  const int gpp = d / kRowGroup, part = g / gpp, gp = g - part * gpp;
+  const int gph = hd / kRowGroup, head = gp / gph, a0 = (gp - head * gph) * 8;
+  return part * d + head * hd + (i < 8 ? a0 + i : hd / 2 + a0 + (i - 8));
+}
+
+// One thread per 16-byte chunk of the packed image.  Logical rows `ch` (0 .. N-1; PACK_GLU: gate
+// channels, each packed twice: gate row in the slice's first half, up row in its second half);
+// source rows at or beyond `rows` (N rounded up to whole groups) are packed as zeros.
+// CTA c's slice is packed contiguously: for its j-th consumed k-block (k = (k0 + j) mod kb) the
+// slice's rows (128 bytes each, zero beyond K) in the 128-byte-swizzled image (16-byte chunk index
+// XOR row % 8), so one bulk copy lands a k-block exactly as a swizzled TMA box would.
+__global__ void pack_rows_kernel(const uint16_t* __restrict__ W, const uint16_t* __restrict__ W2, int N, int rows,
+                                 int K, int kb, int G, int kind, int d, int hd, int rot_groups, long long chunks,
+                                 uint8_t* __restrict__ out) {
+  const int mult = kind == PACK_GLU ? 2 : 1;
+  for (long long it = blockIdx.x * (long long)blockDim.x + threadIdx.x; it < chunks;
+       it += (long long)gridDim.x * blockDim.x) {
+    const int cch = (int)(it & 7);
+    const long long rk = it >> 3;
+    const int k = (int)(rk % kb);  // source k-block
+    const long long lr = rk / kb;  // logical row x half
+    const int h = (int)(lr % mult);
+    const int ch = (int)(lr / mult);
+    const int NG = N / kRowGroup;
+    const int c = row_slice_owner(ch / kRowGroup, NG, G);
+    const RowSlice s = row_slice(c, NG, G);
+    const int R = s.ng * kRowGroup;
+    const int r = h * R + (ch - s.g0 * kRowGroup);  // row within the slice's packed k-block
+    int k0 = 0;
+    if (rot_groups > 0) k0 = (row_slice(c, rot_groups, G).g0 * kRowGroup / 64) % kb;
+    const int j = (k - k0 + kb) % kb;  // consumption index of k-block k
+    int src_row = ch;
+    const uint16_t* src = W;
+    if (kind == PACK_GLU) {
+      src = h == 0 ? W : W2;
+    } else if (kind == PACK_QKV) {
+      src_row = qkv_src_row(ch, d, hd);
+    }
+    const int col = k * 64 + cch * 8;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (col < K && src_row < rows) v = *reinterpret_cast<const uint4*>(src + (size_t)src_row * K + col);
+    const size_t slice_base = (size_t)s.g0 * kRowGroup * mult * kb * 128;
+    const size_t off = slice_base + ((size_t)j * R * mult + r) * 128 + (size_t)((cch ^ (r & 7)) << 4);
+    *reinterpret_cast<uint4*>(out + off) = v;
+  }
+}
+
+size_t pack_rows_bytes(int N, int K, int kind) {
+  return (size_t)N * (kind == PACK_GLU ? 2 : 1) * (size_t)((K + 63) / 64) * 128;
+}
+
+cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int rows, int K, int G, int kind, int d,
+                             int hd, int rot_groups, uint8_t* out, cudaStream_t s) {
+  if (W == nullptr || out == nullptr || N < kRowGroup || N % kRowGroup != 0 || rows < 1 || rows > N || K < 8 ||
+      K % 8 != 0 || G < 1)
+    return cudaErrorInvalidValue;
+  if (kind == PACK_GLU && W2 == nullptr) return cudaErrorInvalidValue;
+  if (kind == PACK_QKV && (N != 3 * d || hd % kRowGroup != 0 || d % hd != 0)) return cudaErrorInvalidValue;
+  const int kb = (K + 63) / 64;
+  const long long chunks = (long long)N * (kind == PACK_GLU ? 2 : 1) * kb * 8;
+  const int threads = 256;
+  long long blocks = (chunks + threads - 1) / threads;
+  if (blocks > 65535LL * 16) blocks = 65535LL * 16;
+  pack_rows_kernel<<<(unsigned)blocks, threads, 0, s>>>(W, W2, N, rows, K, kb, G, kind, d, hd, rot_groups, chunks,
+                                                         out);
+  return cudaGetLastError();
 }
 
 int chain_grid(int num_sms) { return num_sms; }
 
-size_t chain_smem_bytes(int BN) {
-  switch (BN) {
-    case 16: return chain_smem(16);
-    case 32: return chain_smem(32);
-    case 48: return chain_smem(48);
-    default: return chain_smem(64);
-  }
+size_t chain_smem_bytes() { return chain_smem(); }
+
+int chain_slice_rows(int N, int G, bool glu) {
+  const int NG = N / kRowGroup;
+  return (NG / G + (NG % G ? 1 : 0)) * kRowGroup * (glu ? 2 : 1);
 }
 
-template <int BN>
-static cudaError_t launch_bn(const ChainMaps& maps, const ChainArgs& args, int grid, cudaStream_t stream, bool pdl) {
-  auto kern = chain_kernel<BN>;
-  constexpr size_t smem = chain_smem(BN);
+cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int grid, cudaStream_t stream, bool pdl) {
+  if (args.nphases < 1 || args.nphases > kMaxPhases || args.bn < 16 || args.bn > 64 || args.bn % 16 != 0)
+    return cudaErrorInvalidValue;
+  for (int p = 0; p < args.nphases; ++p) {
+    const ChainPhase& ph = args.ph[p];
+    if (ph.wp == nullptr || (reinterpret_cast<uintptr_t>(ph.wp) & 15) != 0 || ph.N % kRowGroup != 0 || ph.kb < 1)
+      return cudaErrorInvalidValue;
+    if (chain_slice_rows(ph.N, grid, ph.epi == EPI_GLU) > 256) return cudaErrorInvalidValue;
+    if (ph.epi == EPI_RESID && chain_slice_rows(ph.N, grid, false) > 64) return cudaErrorInvalidValue;
+    if (ph.in_phase >= p || (ph.in_phase >= 0 && (ph.in_N + 63) / 64 > kReadyPerPhase)) return cudaErrorInvalidValue;
+    if (ph.publish && (ph.N + 63) / 64 > kReadyPerPhase) return cudaErrorInvalidValue;
+  }
+  auto kern = chain_kernel;
+  constexpr size_t smem = chain_smem();
   static int configured = -1;
   int dev = 0;
   cudaGetDevice(&dev);
@@ -568,17 +708,6 @@ static cudaError_t launch_bn(const ChainMaps& maps, const ChainArgs& args, int g
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kern, maps, args);
-}
-
-cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int BN, int grid, cudaStream_t stream, bool pdl) {
-  if (args.nphases < 1 || args.nphases > kMaxPhases) return cudaErrorInvalidValue;
-  switch (BN) {
-    case 16: return launch_bn<16>(maps, args, grid, stream, pdl);
-    case 32: return launch_bn<32>(maps, args, grid, stream, pdl);
-    case 48: return launch_bn<48>(maps, args, grid, stream, pdl);
-    case 64: return launch_bn<64>(maps, args, grid, stream, pdl);
-  }
-  return cudaErrorInvalidValue;
 }
 
 }  // namespace casspec

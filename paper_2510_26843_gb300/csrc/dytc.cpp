@@ -53,8 +53,9 @@ struct casspec_dytc {
   std::vector<int32_t> parent, token, cfg;
   std::vector<double> p_acc;
   std::vector<uint8_t> active;
-  // measured steps for the latency model: bytes moved and microseconds (the most recent kObs)
-  std::vector<double> obs_x, obs_y;
+  // measured steps for the latency model, one regression per arithmetic class: bytes moved and
+  // microseconds (the most recent kObs of each class)
+  std::vector<double> obs_x[CASSPEC_DYTC_MAX_CLASS], obs_y[CASSPEC_DYTC_MAX_CLASS];
 };
 
 namespace {
@@ -319,35 +320,44 @@ double casspec_step_bytes(const casspec_model_config* c, const uint8_t* skip_mas
   return bytes;
 }
 
-int casspec_dytc_observe(casspec_dytc* s, double bytes, double us) {
-  if (s == nullptr || !(bytes >= 0.0) || !(us > 0.0)) return CASSPEC_E_INVAL;
-  if (s->obs_x.size() == kObs) {
-    s->obs_x.erase(s->obs_x.begin());
-    s->obs_y.erase(s->obs_y.begin());
+int casspec_dytc_observe(casspec_dytc* s, int cls, double bytes, double us) {
+  if (s == nullptr || cls < 0 || cls >= CASSPEC_DYTC_MAX_CLASS || !(bytes >= 0.0) || !(us > 0.0))
+    return CASSPEC_E_INVAL;
+  std::vector<double>& x = s->obs_x[cls];
+  std::vector<double>& y = s->obs_y[cls];
+  if (x.size() == kObs) {
+    x.erase(x.begin());
+    y.erase(y.begin());
   }
-  s->obs_x.push_back(bytes);
-  s->obs_y.push_back(us);
+  x.push_back(bytes);
+  y.push_back(us);
   return CASSPEC_OK;
 }
 
-int casspec_dytc_fit_costs(casspec_dytc* s, const double* cfg_bytes, double target_bytes, const double* mu0,
-                           const double* sd0, double noise_sd, double* w_out) {
-  if (s == nullptr || cfg_bytes == nullptr || !(target_bytes > 0.0)) return CASSPEC_E_INVAL;
-  double w[2];
-  const int m = (int)s->obs_x.size();
-  const int rc = casspec_latency_fit(m ? s->obs_x.data() : nullptr, m ? s->obs_y.data() : nullptr, m, mu0, sd0,
-                                     noise_sd, w, nullptr);
-  if (rc != CASSPEC_OK) return rc;
-  const double t_target = w[0] + w[1] * target_bytes;
+int casspec_dytc_fit_costs(casspec_dytc* s, const int* cfg_class, const double* cfg_bytes, double target_bytes,
+                           const double* mu0, const double* sd0, double noise_sd, double* w_out) {
+  if (s == nullptr || cfg_class == nullptr || cfg_bytes == nullptr || !(target_bytes > 0.0)) return CASSPEC_E_INVAL;
+  for (int c = 0; c < s->p.n_cfg; ++c)
+    if (!(cfg_bytes[c] >= 0.0) || cfg_class[c] < 0 || cfg_class[c] >= CASSPEC_DYTC_MAX_CLASS) return CASSPEC_E_INVAL;
+  // one posterior per class (a class without measured steps keeps the prior)
+  double w[CASSPEC_DYTC_MAX_CLASS][2];
+  for (int k = 0; k < CASSPEC_DYTC_MAX_CLASS; ++k) {
+    const int m = (int)s->obs_x[k].size();
+    const int rc = casspec_latency_fit(m ? s->obs_x[k].data() : nullptr, m ? s->obs_y[k].data() : nullptr, m, mu0,
+                                       sd0, noise_sd, w[k], nullptr);
+    if (rc != CASSPEC_OK) return rc;
+  }
+  const double t_target = w[0][0] + w[0][1] * target_bytes;
   if (!(t_target > 0.0)) return CASSPEC_E_INVAL;
   for (int c = 0; c < s->p.n_cfg; ++c) {
-    if (!(cfg_bytes[c] >= 0.0)) return CASSPEC_E_INVAL;
+    const double* wc = w[cfg_class[c]];
+    s->cost[c] = std::fmax(wc[0] + wc[1] * cfg_bytes[c], 0.0) / t_target;
   }
-  for (int c = 0; c < s->p.n_cfg; ++c) s->cost[c] = std::fmax(w[0] + w[1] * cfg_bytes[c], 0.0) / t_target;
-  if (w_out) {
-    w_out[0] = w[0];
-    w_out[1] = w[1];
-  }
+  if (w_out)
+    for (int k = 0; k < CASSPEC_DYTC_MAX_CLASS; ++k) {
+      w_out[2 * k] = w[k][0];
+      w_out[2 * k + 1] = w[k][1];
+    }
   return CASSPEC_OK;
 }
 

@@ -87,33 +87,61 @@ struct AttnArgs {
   int* status;
 };
 
-// One phase of the persistent projection chain: Y = W (hi + lo)^T over a split activation matrix
-// (tensor map ChainMaps::x), optionally scaled per token by an RMSNorm factor: when `ss` is set the
-// activation is x * g (gains already applied by its producer) and the token's result is multiplied
-// by rsqrt(sum(ss) / K + eps), which equals projecting RMSNorm(x) * g.
+// ---- the persistent projection chain (chain.cu) ----
+// A projection of N output rows is split among the G CTAs of a launch by 16-row groups: CTA c owns
+// groups [g0, g0 + ng) of the balanced split below (the first N/16 % G CTAs take one group more).
+constexpr int kRowGroup = 16;
+struct RowSlice {
+  int g0, ng;
+};
+__host__ __device__ inline RowSlice row_slice(int c, int NG, int G) {
+  const int base = NG / G, extra = NG % G;
+  return RowSlice{c * base + (c < extra ? c : extra), base + (c < extra ? 1 : 0)};
+}
+// CTA that owns group g under row_slice
+__host__ __device__ inline int row_slice_owner(int g, int NG, int G) {
+  const int base = NG / G, extra = NG % G;
+  return g < extra * (base + 1) ? g / (base + 1) : extra + (g - extra * (base + 1)) / (base > 0 ? base : 1);
+}
+
+// How the rows of a projection's weights are packed (pack_rows_kernel).
+enum PackKind : int {
+  PACK_PLAIN = 0,  // rows in order
+  PACK_GLU = 1,    // gate and up rows of the same channels in one slice (gate first)
+  PACK_QKV = 2,    // [Wq; Wk; Wv] with each 16-row group holding 8 rotary pairs of one head
+};
+
+// One phase: Y = RMSNorm?(X) W^T with X the split activation of tensor map ChainMaps::x; when `ss` is
+// set X holds x * g (gains applied by its producer) and each token's result is multiplied by
+// rsqrt(sum(ss partials) / K + eps), which equals projecting RMSNorm(x) * g.
 constexpr int kMaxPhases = 4;
-struct PhaseDesc {
-  int epi;           // EPI_QKV, EPI_RESID, EPI_GLU or EPI_LMHEAD
-  int tiles;         // 128-row output tiles (EPI_GLU: 64 gate + 64 up rows per tile)
-  int kblocks;       // ceil(K / 64)
-  int K;             // input width
-  const float* ss;   // per-tile partial sums of squares [ss_tiles][64] of x (null: no norm)
-  int ss_tiles;
+constexpr int kReadyPerPhase = 256;  // readiness counters per phase (64-column blocks of its output)
+struct ChainPhase {
+  int epi;            // EPI_RESID, EPI_GLU, EPI_QKV or EPI_LMHEAD
+  int N;              // output rows (EPI_GLU: F channels; the packed slice holds gate then up rows)
+  int K, kb;          // input width and its 64-column blocks
+  const uint8_t* wp;  // packed weights (pack_rows_kernel with this launch's G)
+  int rot_groups;     // 16-row groups of the split that produced the input (the CTA's first k-block is
+                      // the one holding its own slice of that split); must match the packing
+  int in_phase;       // phase of this launch that produces the input, -1: an earlier kernel
+  int in_N;           // output rows of that phase (the readiness targets)
+  int publish;        // a later phase of this launch reads this phase's output
+  const float* ss;    // partial sums of squares [ss_parts][64] of the normalised input (null: none)
+  int ss_parts;
   float eps;
-  EpiParams ep;
+  EpiParams ep;       // outputs; ss_out and the argmax partials are [G][64], indexed by CTA
 };
 struct ChainArgs {
   int nphases;
-  PhaseDesc ph[kMaxPhases];
-  float* partials;     // stream-K partial tiles (shared by the phases)
-  unsigned* counters;  // [kMaxPhases][1024] fix-up counters, zero between launches
-  unsigned* bar;       // [kMaxPhases + 1] phase-barrier arrival counters + exit counter, zero between launches
+  int bn;              // token rows loaded per plane: n rounded up to 16
+  ChainPhase ph[kMaxPhases];
+  unsigned* ready;     // [kMaxPhases][kReadyPerPhase], zero between launches
+  unsigned* done;      // [kMaxPhases + 1] CTAs finished per phase + exit counter, zero between launches
   int* status;
+  int stall_phase;     // test hook: this phase's first readiness wait needs one row more than ever come (-1: off)
 };
 struct ChainMaps {
-  CUtensorMap w[kMaxPhases];   // weights (EPI_GLU: gate), 64 x 128 boxes (EPI_GLU: 64 x 64)
-  CUtensorMap w2[kMaxPhases];  // EPI_GLU: up
-  CUtensorMap x[kMaxPhases];   // split activations [128][K] bf16, 64 x BN boxes
+  CUtensorMap x[kMaxPhases];  // split activations [128][K] bf16, 64 x bn boxes
 };
 
 // ---- launchers (return cudaSuccess or the launch error) ----
@@ -135,8 +163,12 @@ cudaError_t launch_tree_prep(const int* parent, int n, int T, const int* dP, int
 cudaError_t launch_embed(const uint16_t* E, const int* tokens, int n, int d, int vocab, const float* g, float* x,
                          float* ss, uint16_t* xa, cudaStream_t s, bool pdl);
 int chain_grid(int num_sms);
-size_t chain_smem_bytes(int BN);
-cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int BN, int grid, cudaStream_t stream, bool pdl);
+size_t chain_smem_bytes();
+int chain_slice_rows(int N, int G, bool glu);
+cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int grid, cudaStream_t stream, bool pdl);
+size_t pack_rows_bytes(int N, int K, int kind);
+cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int rows, int K, int G, int kind, int d,
+                             int hd, int rot_groups, uint8_t* out, cudaStream_t s);
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
                            cudaStream_t s, bool pdl);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
@@ -146,8 +178,9 @@ cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2
 cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s);
 cudaError_t launch_accept(const int* am, const int* tokens, const int* parent, int n, int* acc, int* status,
                           cudaStream_t s);
-cudaError_t launch_kv_compact(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* acc, int T,
-                              int* dP, unsigned* counter, int* status, cudaStream_t s);
+cudaError_t launch_kv_compact(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* acc,
+                              const unsigned long long* tanc, int T, int* dP, unsigned* counter, int* status,
+                              cudaStream_t s);
 cudaError_t launch_set_int(int* p, int v, cudaStream_t s);
 
 }  // namespace casspec

@@ -15,9 +15,10 @@
 namespace casspec {
 namespace {
 
-// Counters (first 4 KB) + partial slots of 64 x 128 fp32 (32 KB each).  A call needs
-// ceil(N/128) + grid slots, grid <= number of SMs (152 on GB300).
+// Counters (first 4 KB; the last int of it is the call's status word) + partial slots of 64 x 128
+// fp32 (32 KB each).  A call needs ceil(N/128) + grid slots, grid <= number of SMs (152 on GB300).
 constexpr size_t kStaticCounterBytes = 4096;
+constexpr size_t kStaticStatusOffset = kStaticCounterBytes - 4;
 constexpr size_t kStaticSlots = 256;
 constexpr size_t kStaticScratchBytes = kStaticCounterBytes + kStaticSlots * 64 * 128 * 4;  // 8 MB + 4 KB
 constexpr int kMaxDevices = 64;
@@ -82,11 +83,26 @@ extern "C" int casspec_linear_bf16_static(const uint16_t* W, int N, int K, const
   a.kblocks = kb;
   a.counters = static_cast<unsigned*>(s.ptr);
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(s.ptr) + kStaticCounterBytes);
-  a.status = nullptr;
+  a.status = reinterpret_cast<int*>(static_cast<unsigned char*>(s.ptr) + kStaticStatusOffset);
   a.ep.n = n;
   a.ep.N = N;
   a.ep.y = Y;
   a.ep.ldy = ldy;
   if (launch_gemm_bf16(tw, tw, tx, BN, EPI_STORE, a, grid, stream, false) != cudaSuccess) return CASSPEC_E_CUDA;
+  return CASSPEC_OK;
+}
+
+extern "C" int casspec_linear_bf16_static_status(void* cuda_stream, int* status_out) {
+  if (status_out == nullptr) return CASSPEC_E_INVAL;
+  DeviceScratch s;
+  const int rc = scratch_of_current_device(&s);
+  if (rc != CASSPEC_OK) return rc;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  int st = 0;
+  if (cudaMemcpyAsync(&st, static_cast<unsigned char*>(s.ptr) + kStaticStatusOffset, 4, cudaMemcpyDeviceToHost,
+                      stream) != cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess)
+    return CASSPEC_E_CUDA;
+  *status_out = st;
   return CASSPEC_OK;
 }

@@ -427,16 +427,25 @@ cudaError_t launch_accept(const int* am, const int* tokens, const int* parent, i
 // advances P (all CTAs read P before any of them can finish).
 // ---------------------------------------------------------------------------------------------
 __global__ void kv_compact_kernel(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* __restrict__ acc,
-                                  int T, int* dP, unsigned* counter, int* status) {
+                                  const unsigned long long* __restrict__ tanc, int T, int* dP, unsigned* counter,
+                                  int* status) {
   __shared__ int s_path[kMaxTree];
   __shared__ int s_ok, s_last;
   const int P = __ldcg(dP);
   if (threadIdx.x == 0) {
     const int L = __ldcg(acc);
+    // a root-first chain of the current tree: the root (slot 0), then each node a child of the one
+    // before it (ancestor sets include the node itself, so anc(j) == anc(prev) | {j} <=> parent(j) == prev)
     bool ok = L >= 1 && L <= T;
+    unsigned long long prev_anc = 0ull;
     for (int k = 0; ok && k < L; ++k) {
       const int j = __ldcg(acc + 1 + k);
       ok = j >= 0 && j < T && (k == 0 ? j == 0 : j > s_path[k - 1]);
+      if (ok) {
+        const unsigned long long an = __ldcg(tanc + j);
+        ok = an == (prev_anc | (1ull << j));
+        prev_anc = an;
+      }
       s_path[k] = j;
     }
     s_ok = ok ? L : 0;
@@ -470,12 +479,13 @@ __global__ void kv_compact_kernel(uint16_t* kv, int n_layers, int n_heads, int c
   }
 }
 
-cudaError_t launch_kv_compact(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* acc, int T, int* dP,
-                              unsigned* counter, int* status, cudaStream_t s) {
+cudaError_t launch_kv_compact(uint16_t* kv, int n_layers, int n_heads, int ctx, int hd, const int* acc,
+                              const unsigned long long* tanc, int T, int* dP, unsigned* counter, int* status,
+                              cudaStream_t s) {
   const long long items = (long long)n_layers * 2 * n_heads * (hd / 8);
   long long blocks = (items + 255) / 256;
   if (blocks > 1024) blocks = 1024;
-  kv_compact_kernel<<<(int)blocks, 256, 0, s>>>(kv, n_layers, n_heads, ctx, hd, acc, T, dP, counter, status);
+  kv_compact_kernel<<<(int)blocks, 256, 0, s>>>(kv, n_layers, n_heads, ctx, hd, acc, tanc, T, dP, counter, status);
   return cudaGetLastError();
 }
 

@@ -79,8 +79,8 @@ def test_binding_constants_match_the_header():
     import paper_2510_26843_gb300 as cs
 
     h = _header_constants()
-    pairs = {"MAX_TREE": "MAX_TREE", "TOPK_MAX": "TOPK_MAX", "DYTC_WORK": "DYTC_WORK", "SKIP_ATTN": "SKIP_ATTN",
-             "SKIP_FFN": "SKIP_FFN", "OPT_PDL": "OPT_PDL", "OPT_GRAPHS": "OPT_GRAPHS", "OK": "OK"}
+    pairs = {"MAX_TREE": "MAX_TREE", "TOPK_MAX": "TOPK_MAX", "DYTC_WORK": "DYTC_WORK", "DYTC_MAX_CLASS": "DYTC_MAX_CLASS", "SKIP_ATTN": "SKIP_ATTN",
+             "SKIP_FFN": "SKIP_FFN", "OPT_PDL": "OPT_PDL", "OPT_GRAPHS": "OPT_GRAPHS", "OPT_TEST_STALL": "OPT_TEST_STALL", "OK": "OK"}
     for key in list(h):
         if key.startswith(("E_", "T_", "K_")):
             pairs[key] = key

@@ -331,11 +331,13 @@ def test_costs_fitted_from_measured_steps(cs):
     mu0, sd0, noise = [0.0, 1.0 / 6e6], [100.0, 1e-6], 20.0
     sch = cs.Dytc([0.6, 0.7, 0.3], [0.5, 0.5, 0.5], 0.3, 0.02, 4, 1.0, 16)
     for a, b in zip(x, y):
-        sch.observe(a, b)
+        sch.observe(0, a, b)
     cfg_bytes, target = [7.3e9, 7.8e9, 4.0e9], 1.433e10
-    w = sch.fit_costs(cfg_bytes, target, mu0, sd0, noise)
+    w = sch.fit_costs([0, 0, 0], cfg_bytes, target, mu0, sd0, noise)
     mean, _ = D.blr_posterior(x, y, mu0, sd0, noise)
-    assert w == pytest.approx(list(mean), rel=1e-9)
+    assert w[0] == pytest.approx(list(mean), rel=1e-9)
+    prior, _ = D.blr_posterior([], [], mu0, sd0, noise)  # classes without steps keep the prior
+    assert w[1] == pytest.approx(list(prior), rel=1e-12)
     costs = [sch.cost(c) for c in range(3)]
     pred = [(mean[0] + mean[1] * b) / (mean[0] + mean[1] * target) for b in cfg_bytes]
     assert costs == pytest.approx(pred, rel=1e-9)
@@ -345,7 +347,49 @@ def test_costs_fitted_from_measured_steps(cs):
     s_o, k_o, _ = D.find_best_config([0.6, 0.7, 0.3], pred, 0.3, 0.02, 4)
     assert sch.best_config()[:2] == (s_o, k_o)
     with pytest.raises(cs.CasspecError):
-        sch.fit_costs(cfg_bytes, 0.0, mu0, sd0, noise)
+        sch.fit_costs([0, 0, 0], cfg_bytes, 0.0, mu0, sd0, noise)
     with pytest.raises(cs.CasspecError):
-        sch.observe(1e9, 0.0)
+        sch.fit_costs([0, 0, cs.DYTC_MAX_CLASS], cfg_bytes, target, mu0, sd0, noise)
+    with pytest.raises(cs.CasspecError):
+        sch.observe(0, 1e9, 0.0)
+    with pytest.raises(cs.CasspecError):
+        sch.observe(-1, 1e9, 10.0)
+    sch.close()
+
+
+def test_costs_fitted_per_arithmetic_class(cs):
+    """A W8A8 step moves half the bytes of a bf16 step but is slower per byte (its integer MMA work,
+    not its bytes, sets its time).  One line over the mixed observations predicts neither draft's
+    cost; fitted per class, each class follows its own line (the oracle's posterior on that class's
+    steps alone) and the costs come out near their true values and in their true order."""
+    import numpy as np
+
+    rng = np.random.default_rng(9)
+    xb = rng.uniform(4e9, 1.5e10, 40)            # bf16 steps: 20 us + bytes at 6.5 TB/s
+    yb = 20.0 + xb / 6.5e6 + rng.normal(0, 10.0, 40)
+    xq = rng.uniform(2e9, 8e9, 40)               # W8A8 steps: 30 us + bytes at 1.8 TB/s
+    yq = 30.0 + xq / 1.8e6 + rng.normal(0, 10.0, 40)
+    mu0, sd0, noise = [0.0, 1.0 / 6e6], [100.0, 1e-5], 10.0
+    sch = cs.Dytc([0.6, 0.8], [0.5, 0.5], 0.3, 0.02, 4, 1.0, 16)
+    for a, b in zip(xb, yb):
+        sch.observe(0, a, b)
+    for a, b in zip(xq, yq):
+        sch.observe(1, a, b)
+    skip_bytes, int8_bytes, target = 7.3e9, 7.8e9, 1.433e10
+    w = sch.fit_costs([0, 1], [skip_bytes, int8_bytes], target, mu0, sd0, noise)
+    mb, _ = D.blr_posterior(xb, yb, mu0, sd0, noise)
+    mq, _ = D.blr_posterior(xq, yq, mu0, sd0, noise)
+    assert w[0] == pytest.approx(list(mb), rel=1e-9) and w[1] == pytest.approx(list(mq), rel=1e-9)
+    t_target = mb[0] + mb[1] * target
+    c_skip, c_int8 = sch.cost(0), sch.cost(1)
+    assert c_skip == pytest.approx((mb[0] + mb[1] * skip_bytes) / t_target, rel=1e-9)
+    assert c_int8 == pytest.approx((mq[0] + mq[1] * int8_bytes) / t_target, rel=1e-9)
+    true_skip = (20.0 + skip_bytes / 6.5e6) / (20.0 + target / 6.5e6)
+    true_int8 = (30.0 + int8_bytes / 1.8e6) / (20.0 + target / 6.5e6)
+    assert c_skip == pytest.approx(true_skip, rel=0.03) and c_int8 == pytest.approx(true_int8, rel=0.03)
+    assert c_int8 > 1.0 > c_skip  # the W8A8 draft costs more than the verify it serves
+    # one line over both classes predicts neither draft's cost
+    m1, _ = D.blr_posterior(np.r_[xb, xq], np.r_[yb, yq], mu0, sd0, noise)
+    one = [(m1[0] + m1[1] * b) / (m1[0] + m1[1] * target) for b in (skip_bytes, int8_bytes)]
+    assert abs(one[0] / true_skip - 1) > 0.2 and abs(one[1] / true_int8 - 1) > 0.2
     sch.close()

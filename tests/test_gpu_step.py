@@ -339,6 +339,51 @@ def test_device_reports_bad_parent_and_bad_path(cs, dev_model, ow, prefix):
     assert cs.get_status(dev_model.h) == cs.E_TREE
     assert int(acc[0]) == 0
     kv.close()
+    # a path that starts at the root with increasing indices but is not a chain of the tree
+    # (nodes 1 and 2 are siblings): rejected from the ancestor sets, nothing moved
+    kv, _ = fresh_pair(cs, dev_model, ow, prefix)
+    gpu_step(cs, dev_model, kv, [1, 2, 3], [-1, 0, 0])
+    assert cs.get_status(dev_model.h) == 0
+    P_before = cs.kv_length(kv.h)[0]
+    cs.kv_compact(kv.h, _i32([3, 0, 1, 2, 0]))
+    assert cs.get_status(dev_model.h) == cs.E_TREE
+    assert cs.kv_length(kv.h)[0] == P_before
+    # the same tree with a real chain compacts
+    kv2, _ = fresh_pair(cs, dev_model, ow, prefix)
+    gpu_step(cs, dev_model, kv2, [1, 2, 3], [-1, 0, 0])
+    cs.kv_compact(kv2.h, _i32([2, 0, 2, 0]))
+    assert cs.get_status(dev_model.h) == 0
+    assert cs.kv_length(kv2.h)[0] == P_before + 2
+    kv.close()
+    kv2.close()
+
+
+def test_bounded_wait_expires_and_the_model_recovers(cs, dev_model, ow, prefix):
+    """Failure detection without a GPU fault: with the test hook set, the step's chain launch waits
+    at its second phase for an arrival that never comes.  The bounded wait gives up after its 2 s
+    limit, every CTA of the launch leaves through the abort path (copies in flight drained, tensor
+    memory freed), and the status word reports CASSPEC_E_TIMEOUT.  With the hook cleared, the next
+    step on the same model and cache is clean and matches the oracle."""
+    import time
+
+    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
+    toks, parent = synth.tokens(41, 8, SH.vocab), synth.tree(41, 8, 4)
+    old = cs.set_options(dev_model.h, cs.OPT_PDL | cs.OPT_TEST_STALL)
+    try:
+        t0 = time.perf_counter()
+        gpu_step(cs, dev_model, kv, toks, parent)
+        waited = time.perf_counter() - t0
+        assert cs.get_status(dev_model.h) == cs.E_TIMEOUT
+        assert waited > 1.5, waited  # the wait ran to its limit
+    finally:
+        cs.set_options(dev_model.h, old)
+    assert cs.get_status(dev_model.h) == 0  # read and cleared
+    cs.kv_reset_tree(kv.h)
+    got = gpu_step(cs, dev_model, kv, toks, parent)
+    assert cs.get_status(dev_model.h) == 0
+    ref = oracle.tree_step(ow, okv, toks, parent)
+    assert np.all(rel_err(got, ref) < TOL_BF16), rel_err(got, ref).max()
+    kv.close()
 
 
 def test_host_argument_errors(cs, dev_model):

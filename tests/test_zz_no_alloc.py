@@ -3,7 +3,8 @@
 Collected last (file name) so that it also runs after every other GPU test in one process; it must
 pass on its own in a fresh process too.  Both entry points run the same stream-K tcgen05 kernel
 with a fixed fix-up order, so they agree within the linear op's tolerance (and in practice
-bitwise), on two calls in a row.
+bitwise), on two calls in a row; each call is also held to the fp64 product of the bf16 operands,
+and its status word must report no expired wait.
 """
 from __future__ import annotations
 
@@ -43,15 +44,18 @@ def test_static_matches_workspace_entry_point(cs, N, K, n):
     ws = torch.zeros(cs.linear_workspace_bytes(N, K, n), dtype=torch.uint8, device="cuda")
     ref = torch.full((n, N), float("nan"), dtype=torch.float32, device="cuda")
     cs.linear_bf16(Wd, N, K, Xd, n, ref, N, ws)
-    scale = torch.from_numpy(np.abs(synth.bf16_to_f32(X)).astype(np.float64) @
-                             np.abs(synth.bf16_to_f32(W)).astype(np.float64).T)
+    Xf, Wf = synth.bf16_to_f32(X).astype(np.float64), synth.bf16_to_f32(W).astype(np.float64)
+    scale = torch.from_numpy(np.abs(Xf) @ np.abs(Wf).T)
+    exact = torch.from_numpy(Xf @ Wf.T)  # the fp64 product of the bf16 operands
     for _ in range(2):  # two calls in a row through the same static scratch
         got = torch.full((n, N), float("nan"), dtype=torch.float32, device="cuda")
         cs.linear_bf16_static(Wd, N, K, Xd, n, got, N)
+        assert cs.linear_bf16_static_status() == 0  # no bounded wait expired
         torch.cuda.synchronize()
         g, r = got.cpu().double(), ref.cpu().double()
         assert torch.isfinite(g).all()
         assert float(((g - r).abs() / (scale + 1e-30)).max()) < 2e-4
+        assert float(((g - exact).abs() / (scale + 1e-30)).max()) < 2e-4
 
 
 def test_static_rejects_sizes_beyond_its_scratch(cs):
