@@ -178,11 +178,14 @@ struct casspec_model {
   CUtensorMap tm_lm;
   float *x, *ssp;
   uint16_t *q, *o, *u, *xa;       // o, u, xa: split activations [128][K] bf16 (hi, lo planes)
-  CUtensorMap tm_o[4], tm_u[4], tm_xa[4];  // their 64 x BN boxes, BN = 16, 32, 48, 64
+  // their 64 x BN boxes, BN = 16, 32, 48, 64, and [4]: 64 x 128 boxes (both planes of all 64 tokens
+  // in one load, used when n > 48)
+  CUtensorMap tm_o[5], tm_u[5], tm_xa[5];
   int8_t* xq;
   float* xs;
   unsigned *chain_ready, *chain_done;
   uint8_t* lm_p = nullptr;   // the LM head packed for the chain
+  int resid_split = 1;       // 2: the chain runs as CTA pairs and the residual projections split K in two
   bool pack_dirty = true;    // the row-major weights may have changed since the last packing
   int* pos;
   unsigned long long* anc;
@@ -282,13 +285,14 @@ int pack_weights(casspec_model* m, int& count) {
   const int G = chain_grid(m->num_sms);
   for (int l = 0; l < c.n_layers; ++l) {
     LayerPtrs& p = m->layers[l];
-    CK(launch_pack_rows(p.wqkv, nullptr, 3 * d, 3 * d, d, G, PACK_QKV, d, hd, d / kRowGroup, p.wqkv_p, m->stream));
-    CK(launch_pack_rows(p.wo, nullptr, d, d, d, G, PACK_PLAIN, d, hd, d / kRowGroup, p.wo_p, m->stream));
-    CK(launch_pack_rows(p.wg, p.wu, F, F, d, G, PACK_GLU, d, hd, d / kRowGroup, p.wgu_p, m->stream));
-    CK(launch_pack_rows(p.wd, nullptr, d, d, F, G, PACK_PLAIN, d, hd, F / kRowGroup, p.wd_p, m->stream));
+    const int Sr = m->resid_split;  // the residual projections' split (CTA pairs: 2)
+    CK(launch_pack_rows(p.wqkv, nullptr, 3 * d, 3 * d, d, G, 1, PACK_QKV, d, hd, d / kRowGroup, p.wqkv_p, m->stream));
+    CK(launch_pack_rows(p.wo, nullptr, d, d, d, G, Sr, PACK_PLAIN, d, hd, d / kRowGroup, p.wo_p, m->stream));
+    CK(launch_pack_rows(p.wg, p.wu, F, F, d, G, 1, PACK_GLU, d, hd, d / kRowGroup, p.wgu_p, m->stream));
+    CK(launch_pack_rows(p.wd, nullptr, d, d, F, G, Sr, PACK_PLAIN, d, hd, F / kRowGroup, p.wd_p, m->stream));
     count += 4;
   }
-  CK(launch_pack_rows(m->lm_head, nullptr, roundup16(V), V, d, G, PACK_PLAIN, d, hd, d / kRowGroup, m->lm_p,
+  CK(launch_pack_rows(m->lm_head, nullptr, roundup16(V), V, d, G, 1, PACK_PLAIN, d, hd, d / kRowGroup, m->lm_p,
                       m->stream));
   ++count;
   m->pack_dirty = false;
@@ -351,6 +355,7 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
   const float* g_first = (mode == 0 || act.empty()) ? reader_gain(items[0]) : nullptr;
   LAUNCH(CASSPEC_K_OTHER, launch_embed(m->embed, tokens, n, d, V, g_first, m->x, m->ssp, m->xa, s, pdl));
   const int bi = BN / 16 - 1;  // tensor maps of the split activations for this BN
+  const int cx = BN == 64 ? 4 : bi;  // the chain loads both planes in one box at BN = 64
 
   EpiParams base = {};
   base.n = n;
@@ -364,7 +369,8 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
 
   // ---- phases of the projection chain ----
   const int G = chain_grid(m->num_sms);
-  const int resid_parts = std::min(d / kRowGroup, G);  // partial sums of squares a residual phase leaves
+  const int Sr = m->resid_split;
+  const int resid_parts = std::min(d / kRowGroup, G / Sr);  // partial sums of squares a residual phase leaves
   auto ph_qkv = [&](int l, int ss_parts, ChainPhase& p, CUtensorMap& x) {
     p = ChainPhase{};
     p.epi = EPI_QKV;
@@ -381,12 +387,13 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.q_out = m->q;
     p.ep.kc = kv_layer_k(kv, l);
     p.ep.vc = kv_layer_v(kv, l);
-    x = m->tm_xa[bi];
+    x = m->tm_xa[cx];
   };
   // residual projection; g_next: gains of the RMSNorm that the next projection applies to x
   auto ph_resid = [&](int K, const uint8_t* wp, int rot_groups, const float* g_next, ChainPhase& p) {
     p = ChainPhase{};
     p.epi = EPI_RESID;
+    p.S = Sr;
     p.N = d;
     p.K = K;
     p.kb = cdiv(K, 64);
@@ -432,7 +439,7 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     p.ep.am_v1 = m->am_v1;
     p.ep.am_i1 = m->am_i1;
     p.ep.am_v2 = m->am_v2;
-    x = m->tm_xa[bi];
+    x = m->tm_xa[cx];
   };
   bool stall_pending = (m->flags & CASSPEC_OPT_TEST_STALL) != 0;
   auto chain = [&](ChainArgs& ca, ChainMaps& cm, int kind) -> int {
@@ -441,13 +448,16 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     ca.done = m->chain_done;
     ca.status = m->status;
     ca.stall_phase = -1;
+    ca.pairs = Sr == 2 ? 1 : 0;
     if (stall_pending && ca.nphases >= 2) {  // test hook: the first multi-phase launch of the step
       ca.stall_phase = 1;
       stall_pending = false;
     }
     for (int p = 0; p < ca.nphases; ++p) {  // consecutive phases feed each other
+      if (ca.ph[p].S == 0) ca.ph[p].S = 1;
       ca.ph[p].in_phase = p - 1;
       ca.ph[p].in_N = p > 0 ? ca.ph[p - 1].N : 0;
+      ca.ph[p].in_S = p > 0 ? ca.ph[p - 1].S : 1;
       ca.ph[p].publish = p + 1 < ca.nphases ? 1 : 0;
     }
     LAUNCH(kind, launch_chain(cm, ca, G, s, pdl));
@@ -511,15 +521,15 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
           break;
         case IT_WO:
           ph_resid(d, m->layers[it.l].wo_p, d / kRowGroup, reader_gain(items[i + 1]), p);
-          cm.x[nph] = m->tm_o[bi];
+          cm.x[nph] = m->tm_o[cx];
           break;
         case IT_GU:
           ph_gu(it.l, ss_parts, p);
-          cm.x[nph] = m->tm_xa[bi];
+          cm.x[nph] = m->tm_xa[cx];
           break;
         case IT_DOWN:
           ph_resid(F, m->layers[it.l].wd_p, F / kRowGroup, reader_gain(items[i + 1]), p);
-          cm.x[nph] = m->tm_u[bi];
+          cm.x[nph] = m->tm_u[cx];
           break;
         default:
           ph_lm(ss_parts, p, cm.x[nph]);
@@ -622,6 +632,12 @@ bool build_tensor_maps(casspec_model* m) {
     ok = ok && encode_tmap_bf16(&m->tm_u[b], m->u, F, 2 * kMaxTree, F * 2, 64, BN);
     ok = ok && encode_tmap_bf16(&m->tm_xa[b], m->xa, d, 2 * kMaxTree, d * 2, 64, BN);
   }
+  {
+    const uint32_t rows = 2 * kMaxTree;
+    ok = ok && encode_tmap_bf16(&m->tm_o[4], m->o, d, rows, d * 2, 64, rows);
+    ok = ok && encode_tmap_bf16(&m->tm_u[4], m->u, F, rows, F * 2, 64, rows);
+    ok = ok && encode_tmap_bf16(&m->tm_xa[4], m->xa, d, rows, d * 2, 64, rows);
+  }
   return ok;
 }
 
@@ -646,14 +662,26 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   if (sms <= 0 || sms > kSmsBound) return CASSPEC_E_CUDA;
   {  // the projection chain's per-CTA slices must fit one MMA (and a residual slice the epilogue)
     const int G = chain_grid(sms), d = cfg->d_model, F = cfg->ffn;
-    if (chain_slice_rows(d, G, false) > 64 || chain_slice_rows(3 * d, G, false) > 256 ||
+    if (chain_slice_rows(3 * d, G, false) > 256 ||
         chain_slice_rows(F, G, true) > 256 || chain_slice_rows(roundup16(cfg->vocab), G, false) > 256 ||
         cdiv(F, 64) > kReadyPerPhase || cdiv(d, 64) > kReadyPerPhase)
+      return CASSPEC_E_SHAPE;
+  }
+  // The residual projections (d output rows) split K over CTA pairs when pairs of CTAs fit the GPU
+  // at once and a pair's rows fit its exchange buffer; otherwise each CTA runs all of K for its rows.
+  int resid_split = 1;
+  {
+    const int G = chain_grid(sms), d = cfg->d_model;
+    if (chain_slice_rows(d, G / 2, false) <= kPairMaxRows && cdiv(d, 64) >= 2 && cdiv(cfg->ffn, 64) >= 2 &&
+        chain_pairs_fit(G))
+      resid_split = 2;
+    else if (chain_slice_rows(d, G, false) > 64)
       return CASSPEC_E_SHAPE;
   }
   casspec_model* m = new (std::nothrow) casspec_model();
   if (m == nullptr) return CASSPEC_E_CAPACITY;
   m->cfg = *cfg;
+  m->resid_split = resid_split;
   m->lay = L;
   m->num_sms = sms;
   uint8_t* b = static_cast<uint8_t*>(dev_mem);

@@ -66,18 +66,20 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
     flags[1] = 0;
     fence_mbar_init();
   }
+  // The committed length P is written only between steps (compaction, set_prefix), by kernels that
+  // completed before this step's first kernel started, so it can be read before the dependency wait.
+  // The blocks of this split that lie wholly inside the committed prefix do not depend on the
+  // preceding kernels either: the producer loads the first of them into the ring before the wait,
+  // and asks L2 for the rest, while the previous kernel finishes.
+  const int Pp = *reinterpret_cast<const volatile int*>(a.dP);
+  const bool aligned = (smem_u32(sm) & 1023u) == 0;  // the swizzle addressing needs 1024-byte tiles
   if (tid == kAttnCompute) {
     tma_prefetch_desc(&tmKV);
-    // Before the dependency wait: pull this split's K/V blocks into L2 while the previous kernel
-    // finishes.  The committed prefix is written only by earlier steps, and an L2 prefetch is a
-    // coherent hint, so a P read here that a predecessor is about to change can only make the
-    // prefetch miss, never change a result.
-    const int Ph = *reinterpret_cast<const volatile int*>(a.dP);
-    if (Ph >= 0 && Ph <= a.ctx) {
-      const int nb = min((Ph + a.T + a.n + kAttnBlk - 1) / kAttnBlk, a.ctx / kAttnBlk);
+    if (Pp >= 0 && Pp <= a.ctx) {
+      const int nb = min((Pp + a.T + a.n + kAttnBlk - 1) / kAttnBlk, a.ctx / kAttnBlk);
       const int row_k = ((a.layer * 2 + 0) * a.n_heads + head) * a.ctx;
       const int row_v = ((a.layer * 2 + 1) * a.n_heads + head) * a.ctx;
-      for (int b = rank * nb / C; b < (rank + 1) * nb / C; ++b) {
+      for (int b = rank * nb / C + S; b < (rank + 1) * nb / C; ++b) {
 #pragma unroll
         for (int sub = 0; sub < HD / 64; ++sub) {
           tma_prefetch_l2_2d(&tmKV, sub * 64, row_k + b * kAttnBlk);
@@ -88,13 +90,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
   }
   __syncthreads();
   pdl_trigger();
-  pdl_wait();
+  if (warp != 4) pdl_wait();  // the producer waits after its prefix loads
 
-  const int P = __ldcg(a.dP);
+  const int P = warp == 4 ? Pp : __ldcg(a.dP);
   const int total = P + a.T + a.n;
   const int nblk = (total + kAttnBlk - 1) / kAttnBlk;
   const int b0 = rank * nblk / C, b1 = (rank + 1) * nblk / C;
-  const bool aligned = (smem_u32(sm) & 1023u) == 0;  // the swizzle addressing needs 1024-byte tiles
   if (!aligned && tid == 0) set_status(a.status, CASSPEC_E_CUDA);
 
   float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
@@ -116,7 +117,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
       uint32_t armed = 0, armed_parity = 0;
       const int row_k = ((a.layer * 2 + 0) * a.n_heads + head) * a.ctx;
       const int row_v = ((a.layer * 2 + 1) * a.n_heads + head) * a.ctx;
+      bool waited = false;
       for (int b = b0; b < b1; ++b) {
+        if (!waited && (b - b0 >= S || (b + 1) * kAttnBlk > P || P < 0 || P > a.ctx)) {
+          pdl_wait();  // from here on the blocks may hold this step's tree K/V
+          waited = true;
+          if (__ldcg(a.dP) != P) set_status(a.status, CASSPEC_E_STATE);  // P moved during a step
+        }
         if (!mbar_wait_bounded(&empty[stage], phase ^ 1, flags)) {
           flags[0] = 1;
           set_status(a.status, CASSPEC_E_TIMEOUT);
@@ -136,6 +143,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
           phase ^= 1;
         }
       }
+      if (!waited) pdl_wait();
       if (flags[0]) {  // abort: let the copies already issued land before the ring is reused
         for (int s = 0; s < S; ++s)
           if (armed & (1u << s)) mbar_wait_bounded(&full[s], (armed_parity >> s) & 1, nullptr);

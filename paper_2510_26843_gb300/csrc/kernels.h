@@ -104,6 +104,37 @@ __host__ __device__ inline int row_slice_owner(int g, int NG, int G) {
   return g < extra * (base + 1) ? g / (base + 1) : extra + (g - extra * (base + 1)) / (base > 0 ? base : 1);
 }
 
+// The part of a phase one CTA runs: rows [16 g0, 16 (g0 + ng)) of the output and the k-blocks
+// klo + (rot + j) % len, j = 0 .. len-1, of the input (S = 1: all of K; S = 2: CTA pair c / 2 shares
+// the rows, rank c % 2 takes one half of K).
+struct PhasePart {
+  int g0, ng, rank, klo, len, rot, slice;  // slice: index of the row slice (per-slice partials)
+};
+__host__ __device__ inline PhasePart phase_part(int c, int G, int NG, int kb, int S, int rot_groups) {
+  PhasePart q;
+  if (S == 2) {
+    const int Gc = G / 2, cl = c / 2;
+    const RowSlice s = row_slice(cl, NG, Gc);
+    q.g0 = s.g0;
+    q.ng = s.ng;
+    q.rank = c & 1;
+    q.klo = q.rank ? kb / 2 : 0;
+    q.len = q.rank ? kb - kb / 2 : kb / 2;
+    q.rot = q.len > 0 ? (cl * q.len) / Gc : 0;
+    q.slice = cl;
+  } else {
+    const RowSlice s = row_slice(c, NG, G);
+    q.g0 = s.g0;
+    q.ng = s.ng;
+    q.rank = 0;
+    q.klo = 0;
+    q.len = kb;
+    q.rot = rot_groups > 0 ? (row_slice(c, rot_groups, G).g0 * kRowGroup / 64) % kb : 0;
+    q.slice = c;
+  }
+  return q;
+}
+
 // How the rows of a projection's weights are packed (pack_rows_kernel).
 enum PackKind : int {
   PACK_PLAIN = 0,  // rows in order
@@ -126,10 +157,13 @@ struct ChainPhase {
   int in_phase;       // phase of this launch that produces the input, -1: an earlier kernel
   int in_N;           // output rows of that phase (the readiness targets)
   int publish;        // a later phase of this launch reads this phase's output
+  int in_S;           // split factor of that phase (its rows are counted in once per split)
+  int S;              // 1: the CTA's rows over all of K; 2 (EPI_RESID in a launch of CTA pairs): the
+                      // pair's rows, each CTA one half of K, the halves summed through shared memory
   const float* ss;    // partial sums of squares [ss_parts][64] of the normalised input (null: none)
   int ss_parts;
   float eps;
-  EpiParams ep;       // outputs; ss_out and the argmax partials are [G][64], indexed by CTA
+  EpiParams ep;       // outputs; ss_out and the argmax partials are [slices][64], indexed by slice
 };
 struct ChainArgs {
   int nphases;
@@ -139,9 +173,10 @@ struct ChainArgs {
   unsigned* done;      // [kMaxPhases + 1] CTAs finished per phase + exit counter, zero between launches
   int* status;
   int stall_phase;     // test hook: this phase's first readiness wait needs one row more than ever come (-1: off)
+  int pairs;           // 1: launched as clusters of two CTAs (phases with S = 2 allowed)
 };
 struct ChainMaps {
-  CUtensorMap x[kMaxPhases];  // split activations [128][K] bf16, 64 x bn boxes
+  CUtensorMap x[kMaxPhases];  // split activations [128][K] bf16: 64 x bn boxes (bn = 64: 64 x 128, both planes)
 };
 
 // ---- launchers (return cudaSuccess or the launch error) ----
@@ -166,9 +201,11 @@ int chain_grid(int num_sms);
 size_t chain_smem_bytes();
 int chain_slice_rows(int N, int G, bool glu);
 cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int grid, cudaStream_t stream, bool pdl);
+constexpr int kPairMaxRows = 64;  // rows of an S = 2 slice that the pair's exchange buffer holds
 size_t pack_rows_bytes(int N, int K, int kind);
-cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int rows, int K, int G, int kind, int d,
-                             int hd, int rot_groups, uint8_t* out, cudaStream_t s);
+cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int rows, int K, int G, int S, int kind,
+                             int d, int hd, int rot_groups, uint8_t* out, cudaStream_t s);
+int chain_pairs_fit(int grid);  // 1 if a launch of grid / 2 CTA pairs fits the GPU at once
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
                            cudaStream_t s, bool pdl);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
