@@ -55,6 +55,7 @@ for _n in (1, 2, 4, 8):
     WORKLOADS[f"draft7b-skip50-n{_n}"] = (32, 2048, _n, 8, None, 0.5, 0, False)
     WORKLOADS[f"draft7b-int8-n{_n}"] = (32, 2048, _n, 8, None, 0.0, 1, False)
     WORKLOADS[f"draft7b-skip50-int8-n{_n}"] = (32, 2048, _n, 8, None, 0.5, 1, False)
+    WORKLOADS[f"draft7b-w4a4-n{_n}"] = (32, 2048, _n, 8, None, 0.0, 2, False)
 FAMILY = {"verify13b": "13b", "cascade13b": "13b"}  # others: 7B shape
 CASCADE_SKIP = (0.4, 0.6)  # d1 (bf16) and d2 (W8A8) layer-skip fractions of the 13B cascade
 
@@ -68,12 +69,13 @@ def _shape(layers: int | None = None, family: str = "7b"):
 
 
 def algorithmic_bytes(shape, n: int, P: int, layers_on: int | None = None, quant: int = 0) -> dict:
-    """Bytes the step must move: every active weight once (int8 + fp32 row scales in W8A8 mode), the
-    prefix K/V of active layers, the tree K/V written once, fp32 logits written once (activations
-    are < 0.1% and left out)."""
+    """Bytes the step must move: every active weight once (int8, or 4-bit in W4A4 mode, + fp32 row
+    scales when quantised), the prefix K/V of active layers, the tree K/V written once, fp32 logits
+    written once (activations are < 0.1% and left out)."""
     L = shape.n_layers if layers_on is None else layers_on
     d, F, V = shape.d_model, shape.ffn, shape.vocab
-    w = L * (4 * d * d + 3 * d * F) * (1 if quant else 2) + (L * (5 * d + 2 * F) * 4 if quant else 0)
+    per_weight = {0: 2.0, 1: 1.0, 2: 0.5}[quant]
+    w = int(L * (4 * d * d + 3 * d * F) * per_weight) + (L * (5 * d + 2 * F) * 4 if quant else 0)
     lm = V * d * 2
     kv_read = L * 2 * P * d * 2
     kv_write = L * 2 * n * d * 2
@@ -97,7 +99,7 @@ def gateup_bytes(shape, n: int, quant: int = 0) -> int:
     """Wg, Wu read (+ row scales) + activations read + U written (bf16)."""
     d, F = shape.d_model, shape.ffn
     if quant:
-        return 2 * F * d + 2 * F * 4 + n * d + n * F * 2
+        return int(2 * F * d * (0.5 if quant == 2 else 1.0)) + 2 * F * 4 + n * d + n * F * 2
     return 2 * F * d * 2 + n * d * 2 + n * F * 2
 
 
@@ -210,7 +212,7 @@ class OracleSampler:
         self.mode = mode
         if mode:
             for name in ("wqkv", "wo", "wg", "wu", "wd"):
-                self.w.int8(name, 0)
+                self.w.intq(name, 0, 7 if mode == 2 else 127)
         self.t0 = None
 
     def _run(self, on: int) -> float:
@@ -265,7 +267,7 @@ def describe(name: str, wl) -> str:
                 f"(depth<={depth}): {int(CASCADE_SKIP[1] * 100)}%-skip W8A8 draft level by level, "
                 f"{int(CASCADE_SKIP[0] * 100)}%-skip bf16 re-check of all nodes, full verify + accept + compact")
     kind = "tree verify + accept + compact" if verify else "draft step (tree reset after)"
-    extra = (f", {int(skip * 100)}% layers skipped" if skip else "") + (", W8A8" if mode else ", bf16")
+    extra = (f", {int(skip * 100)}% layers skipped" if skip else "") + {0: ", bf16", 1: ", W8A8", 2: ", W4A4"}[mode]
     br = f", branching<={branch}" if branch else ""
     return (f"{name}: llama{fam}-shape {layers} layer(s), d{d}, n={n} nodes (depth<={depth}{br}), prefix {P}{extra}; "
             f"{kind}")
@@ -502,13 +504,13 @@ def run_gpu(args) -> None:
             T += b - a
         total += algorithmic_bytes(sh, n, P, on1, 0)["total"]
         ab["total"] = total
-    kern = ("gemm_i8_kernel (W8A8 gate/up + SwiGLU)" if mode else
+    kern = ((f"gemm_i8_kernel ({'W4A4' if mode == 2 else 'W8A8'} gate/up + SwiGLU)") if mode else
             "chain_kernel (Wo + residual, gate/up + SwiGLU, down + residual, next QKV or LM head)")
 
     out = {
         "metric": METRIC, "value": round(us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": False, "scaling": "weak",
-        "vs_baseline": None, "dtype": "int8" if mode else "bf16",
+        "vs_baseline": None, "dtype": {0: "bf16", 1: "int8", 2: "int4"}[mode],
         "data": "synthetic (seeded N(0,0.02) weights, N(0,1) prefix KV)",
         "config": config_block(args, args.workload, wl, graphs),
         "launch": {"cuda_graphs": graphs, "pdl": True},

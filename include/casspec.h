@@ -76,14 +76,16 @@ typedef struct casspec_kv casspec_kv;       /* opaque host handle */
  *   ATTN_NORM [d] fp32, FFN_NORM [d] fp32 (RMSNorm gains)
  *   WQKV [3d][d] bf16 (rows: Wq, then Wk, then Wv), WO [d][d], WG [F][d], WU [F][d], WD [d][F] bf16
  * The int8 copies (written by casspec_quantize_weights) are WQKV_Q .. WD_Q int8 with the same
- * shapes and WQKV_S .. WD_S fp32 per-output-row scales.
+ * shapes and WQKV_S .. WD_S fp32 per-output-row scales.  The int4 copies (W4A4, same call) are
+ * WQKV_Q4 .. WD_Q4 with rows of K / 2 bytes (column 2j in the low nibble of byte j, two's
+ * complement codes in [-7, 7]) and WQKV_S4 .. WD_S4 fp32 scales (amax / 7).
  * Step state (read-only views of the model's scratch, valid until the next step on the model; layer
  * ignored; for tests and for callers that want the hidden state):
  *   RESIDUAL [64][d] fp32: the residual stream after the step's last active layer (before the final
  *     RMSNorm), rows 0 .. n-1 valid;
  *   ACT_Q [64][K] int8 and ACT_S [64] fp32: codes and per-token scales of the latest quantised
- *     projection input of a W8A8 step (the down projection's input, K = ffn, when the last active
- *     layer ran its FFN block). */
+ *     projection input of a W8A8 or W4A4 step (the down projection's input, K = ffn, when the last
+ *     active layer ran its FFN block). */
 enum casspec_tensor_id {
   CASSPEC_T_EMBED = 0,
   CASSPEC_T_LM_HEAD = 1,
@@ -107,7 +109,17 @@ enum casspec_tensor_id {
   CASSPEC_T_WD_S = 19,
   CASSPEC_T_RESIDUAL = 20,
   CASSPEC_T_ACT_Q = 21,
-  CASSPEC_T_ACT_S = 22
+  CASSPEC_T_ACT_S = 22,
+  CASSPEC_T_WQKV_Q4 = 23,
+  CASSPEC_T_WO_Q4 = 24,
+  CASSPEC_T_WG_Q4 = 25,
+  CASSPEC_T_WU_Q4 = 26,
+  CASSPEC_T_WD_Q4 = 27,
+  CASSPEC_T_WQKV_S4 = 28,
+  CASSPEC_T_WO_S4 = 29,
+  CASSPEC_T_WG_S4 = 30,
+  CASSPEC_T_WU_S4 = 31,
+  CASSPEC_T_WD_S4 = 32
 };
 
 /* Option bits for casspec_set_options. */
@@ -204,7 +216,8 @@ CASSPEC_API int casspec_kv_length(casspec_kv* kv, int* P_out, int* T_out);
  *               slots (nested masks, as in a layer-sparsity cascade); otherwise E_STATE.
  *   quant_mode  0: bf16 weights, fp32 accumulation.  1: W8A8 GEMMs for WQKV, WO, WG/WU, WD with
  *               per-token dynamic int8 activations (activation-quantisation DSIA); attention, K/V
- *               and the LM head stay bf16.  Mode 1 needs casspec_quantize_weights first.
+ *               and the LM head stay bf16.  2: the same with 4-bit weights and activations (W4A4,
+ *               codes in [-7, 7]).  Modes 1 and 2 need casspec_quantize_weights first.
  *   logits_out  dev fp32 [n][vocab] or NULL.
  * The row argmax of the logits (ties to the lowest id) and the top-2 margin of every node are
  * always computed and kept in the model (casspec_argmax).  Invalid parent_idx values are reported
@@ -317,6 +330,10 @@ CASSPEC_API int casspec_rmsnorm(const float* x, const float* g, int n, int d, fl
 
 /* Per-row int8 quantisation of bf16 rows x [n][d] -> q [n][d], s [n] (same rule). */
 CASSPEC_API int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q_out, float* s_out, void* cuda_stream);
+/* The same with codes in [-7, 7] (the W4A4 draft's activations, App. C): inv = 7 / amax, scale amax / 7,
+ * q4_out (dev [n][d / 2] bytes) two codes per byte, column 2j in the low nibble of byte j.  d % 8 == 0. */
+CASSPEC_API int casspec_quantize_rows4(const uint16_t* x, int n, int d, uint8_t* q4_out, float* s_out,
+                                       void* cuda_stream);
 
 /* ---------------------------------------------------------------------------------------------
  * Dynamic Tree Cascade scheduling (DyTC): host code, no GPU work; thread-compatible (one scheduler

@@ -25,7 +25,8 @@ OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL = 1, 2, 4
 
 (T_EMBED, T_LM_HEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WG, T_WU, T_WD,
  T_WQKV_Q, T_WO_Q, T_WG_Q, T_WU_Q, T_WD_Q, T_WQKV_S, T_WO_S, T_WG_S, T_WU_S, T_WD_S,
- T_RESIDUAL, T_ACT_Q, T_ACT_S) = range(23)
+ T_RESIDUAL, T_ACT_Q, T_ACT_S,
+ T_WQKV_Q4, T_WO_Q4, T_WG_Q4, T_WU_Q4, T_WD_Q4, T_WQKV_S4, T_WO_S4, T_WG_S4, T_WU_S4, T_WD_S4) = range(33)
 
 EXPORTS = [
     "casspec_model_bytes", "casspec_create_model", "casspec_destroy_model", "casspec_set_stream",
@@ -34,7 +35,7 @@ EXPORTS = [
     "casspec_tree_step", "casspec_argmax", "casspec_accept_greedy", "casspec_kv_compact", "casspec_get_status",
     "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_linear_bf16_static", "casspec_linear_bf16_static_status",
     "casspec_rmsnorm",
-    "casspec_quantize_rows", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
+    "casspec_quantize_rows", "casspec_quantize_rows4", "casspec_profile", "casspec_profile_read", "casspec_launch_count",
     "casspec_ewif_sd", "casspec_ewif_hc", "casspec_ewif_vc", "casspec_dytc_objective", "casspec_dytc_create",
     "casspec_dytc_destroy", "casspec_dytc_get_params", "casspec_dytc_set_cost", "casspec_dytc_alpha", "casspec_dytc_cost", "casspec_dytc_best_config",
     "casspec_dytc_record", "casspec_dytc_end_step", "casspec_dytc_tree_reset", "casspec_dytc_tree_plan",
@@ -141,6 +142,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_linear_bf16_static_status": (_I, [_P, ctypes.POINTER(_I)]),
         "casspec_rmsnorm": (_I, [_P, _P, _I, _I, ctypes.c_float, _P, _P, _P, _P]),
         "casspec_quantize_rows": (_I, [_P, _I, _I, _P, _P, _P]),
+        "casspec_quantize_rows4": (_I, [_P, _I, _I, _P, _P, _P]),
         "casspec_profile": (_I, [_P, _I]),
         "casspec_profile_read": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(_I)]),
         "casspec_launch_count": (_I, [_P, ctypes.POINTER(ctypes.c_uint64)]),
@@ -323,6 +325,22 @@ def rmsnorm(x, g, n: int, d: int, eps: float, y=None, q=None, s=None, stream=Non
 
 def quantize_rows(x, n: int, d: int, q, s, stream=None) -> None:
     _check("casspec_quantize_rows", load_library().casspec_quantize_rows(_ptr(x), n, d, _ptr(q), _ptr(s), _stream(stream)))
+
+
+def quantize_rows4(x, n: int, d: int, q4, s, stream=None) -> None:
+    """casspec_quantize_rows4: codes in [-7, 7], two per byte (q4: [n][d / 2] uint8)."""
+    _check("casspec_quantize_rows4", load_library().casspec_quantize_rows4(_ptr(x), n, d, _ptr(q4), _ptr(s),
+                                                                            _stream(stream)))
+
+
+def unpack_int4(b: np.ndarray, K: int) -> np.ndarray:
+    """Codes of int4 rows ([rows][K / 2] bytes, column 2j in the low nibble of byte j) as int8 [rows][K]."""
+    b = np.asarray(b, dtype=np.uint8).reshape(-1, K // 2)
+    lo, hi = (b & 0x0F).astype(np.int16), (b >> 4).astype(np.int16)
+    out = np.empty((b.shape[0], K), dtype=np.int8)
+    out[:, 0::2] = np.where(lo > 7, lo - 16, lo)
+    out[:, 1::2] = np.where(hi > 7, hi - 16, hi)
+    return out
 
 
 def profile(m: int, enable: bool) -> None:

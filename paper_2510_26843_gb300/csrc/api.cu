@@ -25,6 +25,8 @@ struct LayerPtrs {
   uint16_t *wqkv, *wo, *wg, *wu, *wd;
   int8_t *qkv_q, *wo_q, *wg_q, *wu_q, *wd_q;
   float *qkv_s, *wo_s, *wg_s, *wu_s, *wd_s;
+  int8_t *qkv_q4, *wo_q4, *wg_q4, *wu_q4, *wd_q4;  // W4A4: two 4-bit codes per byte
+  float *qkv_s4, *wo_s4, *wg_s4, *wu_s4, *wd_s4;
   CUtensorMap tm_qkv, tm_o, tm_g, tm_u, tm_d;
   uint8_t *wqkv_p, *wo_p, *wgu_p, *wd_p;  // the projections packed per CTA for the chain (pack_rows_kernel)
 };
@@ -37,6 +39,7 @@ struct Layout {
   std::vector<size_t> qkv_q, wo_q, wg_q, wu_q, wd_q, qkv_s, wo_s, wg_s, wu_s, wd_s;
   std::vector<size_t> wqkv_p, wo_p, wgu_p, wd_p;
   size_t lm_p;
+  std::vector<size_t> qkv_q4, wo_q4, wg_q4, wu_q4, wd_q4, qkv_s4, wo_s4, wg_s4, wu_s4, wd_s4;
   size_t x, q, o, u, xa, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
   size_t gemm_part, gemm_cnt, chain_ready, chain_done, i8_part, i8_cnt, attn_part, attn_ml, attn_cnt, status;
   size_t scratch_begin;
@@ -101,6 +104,16 @@ Layout make_layout(const casspec_model_config& c) {
       L.wg_s.push_back(take(F * 4));
       L.wu_s.push_back(take(F * 4));
       L.wd_s.push_back(take(d * 4));
+      L.qkv_q4.push_back(take(3 * d * d / 2));
+      L.wo_q4.push_back(take(d * d / 2));
+      L.wg_q4.push_back(take(F * d / 2));
+      L.wu_q4.push_back(take(F * d / 2));
+      L.wd_q4.push_back(take(d * F / 2));
+      L.qkv_s4.push_back(take(3 * d * 4));
+      L.wo_s4.push_back(take(d * 4));
+      L.wg_s4.push_back(take(F * 4));
+      L.wu_s4.push_back(take(F * 4));
+      L.wd_s4.push_back(take(d * 4));
     }
   }
   L.scratch_begin = align_up(off, 256);
@@ -539,6 +552,9 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     }
     if ((rc = flush()) != CASSPEC_OK) return rc;
   } else {
+    // mode 1: W8A8 (codes in [-127, 127]); mode 2: W4A4 (codes in [-7, 7], weights two per byte)
+    const bool w4 = mode == 2;
+    const int qmax = w4 ? 7 : 127;
     auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
                      int epi, const EpiParams& e) -> cudaError_t {
       GemmI8Args g8 = {};
@@ -552,6 +568,7 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       g8.K = K;
       g8.tiles = tiles;
       g8.ksplit = gemm_i8_ksplit(tiles, K, m->num_sms);
+      g8.w4 = w4 ? 1 : 0;
       g8.partials = m->i8_part;
       g8.counters = m->i8_cnt;
       g8.status = m->status;
@@ -578,6 +595,10 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         continue;
       }
       LayerPtrs& Lp = m->layers[it.l];
+      const int8_t *q_qkv = w4 ? Lp.qkv_q4 : Lp.qkv_q, *q_wo = w4 ? Lp.wo_q4 : Lp.wo_q;
+      const int8_t *q_wg = w4 ? Lp.wg_q4 : Lp.wg_q, *q_wu = w4 ? Lp.wu_q4 : Lp.wu_q, *q_wd = w4 ? Lp.wd_q4 : Lp.wd_q;
+      const float *s_qkv = w4 ? Lp.qkv_s4 : Lp.qkv_s, *s_wo = w4 ? Lp.wo_s4 : Lp.wo_s;
+      const float *s_wg = w4 ? Lp.wg_s4 : Lp.wg_s, *s_wu = w4 ? Lp.wu_s4 : Lp.wu_s, *s_wd = w4 ? Lp.wd_s4 : Lp.wd_s;
       EpiParams ed = er;
       if ((it.kind == IT_WO || it.kind == IT_DOWN) && items[i + 1].kind == IT_LM) {
         ed.ss_out = m->ssp;  // the last residual projection leaves the LM head's RMSNorm inputs
@@ -585,26 +606,28 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         ed.g_next = m->final_norm;
       }
       if (it.kind == IT_QKV) {
-        LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
+        LAUNCH(CASSPEC_K_OTHER,
+               launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax));
         EpiParams e = base;
         e.N = 3 * d;
         e.q_out = m->q;
         e.kc = kv_layer_k(kv, it.l);
         e.vc = kv_layer_v(kv, it.l);
-        LAUNCH(CASSPEC_K_QKV, gemm8(Lp.qkv_q, Lp.qkv_s, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+        LAUNCH(CASSPEC_K_QKV, gemm8(q_qkv, s_qkv, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
       } else if (it.kind == IT_WO) {
         // W8A8 activations are the bf16 values: the hi plane of the split output
-        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl));
-        LAUNCH(CASSPEC_K_WO, gemm8(Lp.wo_q, Lp.wo_s, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl, qmax));
+        LAUNCH(CASSPEC_K_WO, gemm8(q_wo, s_wo, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
       } else if (it.kind == IT_GU) {
-        LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl));
+        LAUNCH(CASSPEC_K_OTHER,
+               launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax));
         EpiParams eg = base;
         eg.N = F;
         eg.u_out = m->u;
-        LAUNCH(CASSPEC_K_GATEUP, gemm8(Lp.wg_q, Lp.wg_s, Lp.wu_q, Lp.wu_s, F, d, cdiv(F, 64), EPI_GLU, eg));
+        LAUNCH(CASSPEC_K_GATEUP, gemm8(q_wg, s_wg, q_wu, s_wu, F, d, cdiv(F, 64), EPI_GLU, eg));
       } else {
-        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl));
-        LAUNCH(CASSPEC_K_DOWN, gemm8(Lp.wd_q, Lp.wd_s, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl, qmax));
+        LAUNCH(CASSPEC_K_DOWN, gemm8(q_wd, s_wd, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
       }
     }
   }
@@ -715,6 +738,16 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
       p.wg_s = reinterpret_cast<float*>(b + L.wg_s[l]);
       p.wu_s = reinterpret_cast<float*>(b + L.wu_s[l]);
       p.wd_s = reinterpret_cast<float*>(b + L.wd_s[l]);
+      p.qkv_q4 = reinterpret_cast<int8_t*>(b + L.qkv_q4[l]);
+      p.wo_q4 = reinterpret_cast<int8_t*>(b + L.wo_q4[l]);
+      p.wg_q4 = reinterpret_cast<int8_t*>(b + L.wg_q4[l]);
+      p.wu_q4 = reinterpret_cast<int8_t*>(b + L.wu_q4[l]);
+      p.wd_q4 = reinterpret_cast<int8_t*>(b + L.wd_q4[l]);
+      p.qkv_s4 = reinterpret_cast<float*>(b + L.qkv_s4[l]);
+      p.wo_s4 = reinterpret_cast<float*>(b + L.wo_s4[l]);
+      p.wg_s4 = reinterpret_cast<float*>(b + L.wg_s4[l]);
+      p.wu_s4 = reinterpret_cast<float*>(b + L.wu_s4[l]);
+      p.wd_s4 = reinterpret_cast<float*>(b + L.wd_s4[l]);
     }
   }
   m->x = reinterpret_cast<float*>(b + L.x);
@@ -801,7 +834,7 @@ int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size
   if (tensor <= CASSPEC_T_WD) m->pack_dirty = true;  // the caller may write through the pointer
   const auto& c = m->cfg;
   const size_t d = c.d_model, F = c.ffn, V = c.vocab;
-  const bool state = tensor >= CASSPEC_T_RESIDUAL;
+  const bool state = tensor >= CASSPEC_T_RESIDUAL && tensor <= CASSPEC_T_ACT_S;  // step state, not weights
   const bool per_layer = tensor >= CASSPEC_T_ATTN_NORM && !state;
   if (per_layer && (layer < 0 || layer >= c.n_layers)) return CASSPEC_E_INVAL;
   if (tensor >= CASSPEC_T_WQKV_Q && !state && !c.with_int8) return CASSPEC_E_INVAL;
@@ -832,6 +865,16 @@ int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size
     case CASSPEC_T_RESIDUAL: p = m->x; nb = (size_t)kMaxTree * d * 4; break;
     case CASSPEC_T_ACT_Q: p = m->xq; nb = (size_t)kMaxTree * std::max(d, F); break;
     case CASSPEC_T_ACT_S: p = m->xs; nb = (size_t)kMaxTree * 4; break;
+    case CASSPEC_T_WQKV_Q4: p = L->qkv_q4; nb = 3 * d * d / 2; break;
+    case CASSPEC_T_WO_Q4: p = L->wo_q4; nb = d * d / 2; break;
+    case CASSPEC_T_WG_Q4: p = L->wg_q4; nb = F * d / 2; break;
+    case CASSPEC_T_WU_Q4: p = L->wu_q4; nb = F * d / 2; break;
+    case CASSPEC_T_WD_Q4: p = L->wd_q4; nb = d * F / 2; break;
+    case CASSPEC_T_WQKV_S4: p = L->qkv_s4; nb = 3 * d * 4; break;
+    case CASSPEC_T_WO_S4: p = L->wo_s4; nb = d * 4; break;
+    case CASSPEC_T_WG_S4: p = L->wg_s4; nb = F * 4; break;
+    case CASSPEC_T_WU_S4: p = L->wu_s4; nb = F * 4; break;
+    case CASSPEC_T_WD_S4: p = L->wd_s4; nb = d * 4; break;
     default: return CASSPEC_E_INVAL;
   }
   *dev_ptr = p;
@@ -850,6 +893,12 @@ int casspec_quantize_weights(casspec_model* m) {
     CK(launch_quant_rows(p.wg, F, d, d, p.wg_q, d, p.wg_s, m->stream, false));
     CK(launch_quant_rows(p.wu, F, d, d, p.wu_q, d, p.wu_s, m->stream, false));
     CK(launch_quant_rows(p.wd, d, F, F, p.wd_q, F, p.wd_s, m->stream, false));
+    // the W4A4 copies: codes in [-7, 7], two per byte (row stride K / 2 bytes)
+    CK(launch_quant_rows(p.wqkv, 3 * d, d, d, p.qkv_q4, d / 2, p.qkv_s4, m->stream, false, 7, true));
+    CK(launch_quant_rows(p.wo, d, d, d, p.wo_q4, d / 2, p.wo_s4, m->stream, false, 7, true));
+    CK(launch_quant_rows(p.wg, F, d, d, p.wg_q4, d / 2, p.wg_s4, m->stream, false, 7, true));
+    CK(launch_quant_rows(p.wu, F, d, d, p.wu_q4, d / 2, p.wu_s4, m->stream, false, 7, true));
+    CK(launch_quant_rows(p.wd, d, F, F, p.wd_q4, F / 2, p.wd_s4, m->stream, false, 7, true));
   }
   return CASSPEC_OK;
 }
@@ -945,8 +994,8 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
                       const uint8_t* skip_mask, int quant_mode, float* logits_out) {
   if (m == nullptr || kv == nullptr || tokens == nullptr || parent_idx == nullptr || kv->m != m)
     return CASSPEC_E_INVAL;
-  if (quant_mode != 0 && quant_mode != 1) return CASSPEC_E_INVAL;
-  if (quant_mode == 1 && !m->cfg.with_int8) return CASSPEC_E_INVAL;
+  if (quant_mode < 0 || quant_mode > 2) return CASSPEC_E_INVAL;
+  if (quant_mode != 0 && !m->cfg.with_int8) return CASSPEC_E_INVAL;
   if (n < 1 || n > kMaxTree) return CASSPEC_E_SHAPE;
   if (kv->T + n > kMaxTree || kv->P_upper + kv->T + n > kv->ctx) return CASSPEC_E_CAPACITY;
   const int NL = m->cfg.n_layers;
@@ -1147,6 +1196,14 @@ int casspec_quantize_rows(const uint16_t* x, int n, int d, int8_t* q, float* s, 
   if (x == nullptr || q == nullptr || s == nullptr) return CASSPEC_E_INVAL;
   if (n < 1 || d < 1) return CASSPEC_E_SHAPE;
   CK(launch_quant_rows(x, n, d, d, q, d, s, static_cast<cudaStream_t>(stream), false));
+  return CASSPEC_OK;
+}
+
+int casspec_quantize_rows4(const uint16_t* x, int n, int d, uint8_t* q4, float* s, void* stream) {
+  if (x == nullptr || q4 == nullptr || s == nullptr) return CASSPEC_E_INVAL;
+  if (n < 1 || d < 8 || d % 8 != 0) return CASSPEC_E_SHAPE;
+  CK(launch_quant_rows(x, n, d, d, reinterpret_cast<int8_t*>(q4), d / 2, s, static_cast<cudaStream_t>(stream), false,
+                       7, true));
   return CASSPEC_OK;
 }
 

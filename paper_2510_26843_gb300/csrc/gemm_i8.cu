@@ -1,4 +1,4 @@
-// W8A8 projection for the activation-quantisation draft (App. C; W8A8 reading of QSpec-style DSIA).
+// W8A8 / W4A4 projection for the activation-quantisation drafts (App. C, QSpec-style DSIA).
 //
 // y[i][o] = (sum_k qx[i][k] * qw[o][k]) * sx[i] * sw[o], with the integer sum exact in int32
 // (|sum| <= K * 127^2 < 2^31 for K < 133,000).  tcgen05.mma has no integer kind on sm_103a, so the
@@ -11,6 +11,9 @@
 //     activation slice of the k-range is staged once in shared memory.  Both operands use the same
 //     permutation of the 128 columns of a block inside the fragments, which leaves the dot product
 //     unchanged: thread (group g, lane t) takes bytes [16t, 16t+16) and [64+16t, 64+16t+16);
+//   * W4A4: the weights are packed 4-bit codes (half the bytes again), loaded 8 bytes per fragment
+//     piece and widened to int8 in registers just before their MMA; the activations are int8 codes
+//     in [-7, 7], so the same s8 MMA gives the exact integer sum;
 //   * the CTA that finishes a tile last (atomic counter) sums the int32 partials, dequantises
 //     once, and runs the same fused epilogue as the bf16 projection.
 #include "common.cuh"
@@ -29,9 +32,30 @@ __device__ __forceinline__ uint4 ldg_nc16(const void* p) {
   return v;
 }
 
+__device__ __forceinline__ uint2 ldg_nc8(const void* p) {
+  uint2 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+  return v;
+}
+
+// 16 signed 4-bit codes (8 bytes, column 2j in the low nibble of byte j) -> 16 int8 in column order:
+// each nibble is sign-extended per byte as (v ^ 8) - 8, then low and high nibbles are interleaved.
+__device__ __forceinline__ uint4 unpack_s4x16(uint2 w) {
+  uint32_t out[4];
+  const uint32_t in[2] = {w.x, w.y};
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t lo = __vsub4((in[h] & 0x0F0F0F0Fu) ^ 0x08080808u, 0x08080808u);
+    const uint32_t hi = __vsub4(((in[h] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u, 0x08080808u);
+    out[2 * h] = __byte_perm(lo, hi, 0x5140);
+    out[2 * h + 1] = __byte_perm(lo, hi, 0x7362);
+  }
+  return make_uint4(out[0], out[1], out[2], out[3]);
+}
+
 constexpr int kI8MaxKb = 4;  // k-blocks of 128 per CTA (all of its weight loads in flight at once)
 
-template <int BN, int EPI>
+template <int BN, int EPI, bool W4>
 __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a) {
   extern __shared__ float stg[];  // the CTA's X slice, then the dequantised tile, then the epilogue staging
   __shared__ int s_last;
@@ -45,6 +69,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
   const int n = a.ep.n;
 
   // weight rows of this thread's fragments: tile rows lr and lr + 8
+  const size_t wld = W4 ? (size_t)a.K / 2 : (size_t)a.K;  // bytes per weight row
   const int8_t* wrow[2];
   bool wok[2];
 #pragma unroll
@@ -53,15 +78,17 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
     if (EPI == EPI_GLU) {
       const int ch = tile * 64 + (lr & 63);
       wok[h] = ch < a.N;
-      wrow[h] = (lr < 64 ? a.W : a.W2) + (size_t)(wok[h] ? ch : 0) * a.K;
+      wrow[h] = (lr < 64 ? a.W : a.W2) + (size_t)(wok[h] ? ch : 0) * wld;
     } else {
       const int o = tile * 128 + lr;
       wok[h] = o < a.N;
-      wrow[h] = a.W + (size_t)(wok[h] ? o : 0) * a.K;
+      wrow[h] = a.W + (size_t)(wok[h] ? o : 0) * wld;
     }
   }
-  // every weight load of the CTA's k-range first (the weights do not depend on the previous kernel)
-  uint4 A[kI8MaxKb][4];
+  // every weight load of the CTA's k-range first (the weights do not depend on the previous kernel);
+  // 4-bit codes stay packed in registers until their MMA
+  uint4 A[kI8MaxKb][W4 ? 1 : 4];
+  uint2 A4[kI8MaxKb][W4 ? 4 : 1];
 #pragma unroll
   for (int j = 0; j < kI8MaxKb; ++j) {
 #pragma unroll
@@ -69,7 +96,11 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         const int col = (kb0 + j) * 128 + c * 64 + 16 * t4;
-        A[j][2 * h + c] = (j < nkb && wok[h] && col < a.K) ? ldg_nc16(wrow[h] + col) : make_uint4(0, 0, 0, 0);
+        const bool ok = j < nkb && wok[h] && col < a.K;
+        if (W4)
+          A4[j][2 * h + c] = ok ? ldg_nc8(wrow[h] + col / 2) : make_uint2(0u, 0u);
+        else
+          A[j][2 * h + c] = ok ? ldg_nc16(wrow[h] + col) : make_uint4(0, 0, 0, 0);
       }
     }
   }
@@ -105,6 +136,9 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
 #pragma unroll
   for (int kbl = 0; kbl < kI8MaxKb; ++kbl) {
     if (kbl < nkb) {
+      uint4 Aw[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) Aw[e] = W4 ? unpack_s4x16(A4[kbl][e]) : A[kbl][W4 ? 0 : e];
 #pragma unroll
       for (int j = 0; j < BN / 8; ++j) {
         const int tok = 8 * j + g;
@@ -114,7 +148,7 @@ __global__ void __launch_bounds__(kI8Threads) gemm_i8_kernel(const GemmI8Args a)
           B[c] = *reinterpret_cast<const uint4*>(xs + tok * xrow + kbl * 128 + c * 64 + 16 * t4);
 #pragma unroll
         for (int s2 = 0; s2 < 4; ++s2) {
-          const uint4 lo = A[kbl][s2 >> 1], hi = A[kbl][2 + (s2 >> 1)], b = B[s2 >> 1];
+          const uint4 lo = Aw[s2 >> 1], hi = Aw[2 + (s2 >> 1)], b = B[s2 >> 1];
           const bool odd = s2 & 1;
           mma_s8_16832(acc[j], odd ? lo.z : lo.x, odd ? hi.z : hi.x, odd ? lo.w : lo.y, odd ? hi.w : hi.y,
                        odd ? b.z : b.x, odd ? b.w : b.y);
@@ -186,6 +220,7 @@ int gemm_i8_ksplit(int tiles, int K, int num_sms) {
 
 template <int BN, int EPI>
 static cudaError_t launch_t(const GemmI8Args& a, cudaStream_t s, bool pdl) {
+  if (a.w4 && a.K % 16 != 0) return cudaErrorInvalidValue;  // whole 8-byte groups of codes per fragment
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.tiles, a.ksplit);
   cfg.blockDim = dim3(kI8Threads);
@@ -196,7 +231,8 @@ static cudaError_t launch_t(const GemmI8Args& a, cudaStream_t s, bool pdl) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, gemm_i8_kernel<BN, EPI>, a);
+  return a.w4 ? cudaLaunchKernelEx(&cfg, gemm_i8_kernel<BN, EPI, true>, a)
+              : cudaLaunchKernelEx(&cfg, gemm_i8_kernel<BN, EPI, false>, a);
 }
 
 template <int BN>

@@ -57,7 +57,7 @@ struct GemmArgs {
 
 // int8 (W8A8) projection arguments
 struct GemmI8Args {
-  const int8_t* W;   // [N][K]
+  const int8_t* W;   // [N][K] int8, or with w4 [N][K / 2] bytes of two 4-bit codes (column 2j low nibble)
   const float* sw;   // [N]
   const int8_t* W2;  // EPI_GLU: up weights (gate in W)
   const float* sw2;
@@ -65,6 +65,7 @@ struct GemmI8Args {
   const float* sx;   // [64]
   int N, K, ksplit;  // ksplit CTAs share one 128-row tile along K
   int tiles;
+  int w4;            // weights are packed 4-bit codes (W4A4: activations are codes in [-7, 7] too)
   int* partials;     // [tiles][ksplit][64][128] int32
   unsigned* counters;
   int* status;
@@ -207,9 +208,9 @@ cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int r
                              int d, int hd, int rot_groups, uint8_t* out, cudaStream_t s);
 int chain_pairs_fit(int grid);  // 1 if a launch of grid / 2 CTA pairs fits the GPU at once
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
-                           cudaStream_t s, bool pdl);
+                           cudaStream_t s, bool pdl, int qmax = 127);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
-                              bool pdl);
+                              bool pdl, int qmax = 127, bool pack4 = false);
 cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,
                                  float* margin, cudaStream_t s, bool pdl);
 cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s);

@@ -110,9 +110,9 @@ __device__ __forceinline__ float block_max(float v, float* red) {
 // Per-row symmetric int8 quantisation rule (App. C activation-quantisation DSIA, W8A8 reading):
 // inv = 127 / amax (IEEE division), q = rint(x * inv) (IEEE multiply, ties to even), clamp +-127,
 // scale = amax / 127; amax = 0 gives q = 0, scale 0.
-__device__ __forceinline__ int8_t quant_one(float x, float inv) {
+__device__ __forceinline__ int8_t quant_one(float x, float inv, int qmax) {
   int q = __float2int_rn(__fmul_rn(x, inv));
-  q = q > 127 ? 127 : (q < -127 ? -127 : q);
+  q = q > qmax ? qmax : (q < -qmax ? -qmax : q);
   return (int8_t)q;
 }
 
@@ -164,7 +164,8 @@ constexpr int kRowVec = 8;  // float4 per thread: rows up to 16384 fp32 values
 
 __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g,
                                                               int d, float eps, uint16_t* __restrict__ y,
-                                                              int8_t* __restrict__ q, float* __restrict__ sq) {
+                                                              int8_t* __restrict__ q, float* __restrict__ sq,
+                                                              int qmax) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
@@ -210,35 +211,37 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __res
   }
   if (q == nullptr) return;
   amax = block_max(amax, red);
-  const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
+  const float inv = amax > 0.f ? __fdiv_rn((float)qmax, amax) : 0.f;
 #pragma unroll
   for (int k = 0; k < kRowVec; ++k) {
     const int c = threadIdx.x + k * kRowThreads;
     if (c < nv) {
       char4 o;
-      o.x = amax > 0.f ? quant_one(bf2f(b[k][0]), inv) : 0;
-      o.y = amax > 0.f ? quant_one(bf2f(b[k][1]), inv) : 0;
-      o.z = amax > 0.f ? quant_one(bf2f(b[k][2]), inv) : 0;
-      o.w = amax > 0.f ? quant_one(bf2f(b[k][3]), inv) : 0;
+      o.x = amax > 0.f ? quant_one(bf2f(b[k][0]), inv, qmax) : 0;
+      o.y = amax > 0.f ? quant_one(bf2f(b[k][1]), inv, qmax) : 0;
+      o.z = amax > 0.f ? quant_one(bf2f(b[k][2]), inv, qmax) : 0;
+      o.w = amax > 0.f ? quant_one(bf2f(b[k][3]), inv, qmax) : 0;
       reinterpret_cast<char4*>(q + (size_t)i * d)[c] = o;
     }
   }
-  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
+  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, (float)qmax) : 0.f;
 }
 
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
-                           cudaStream_t s, bool pdl) {
-  if (d % 4 != 0 || d > 4 * kRowVec * kRowThreads) return cudaErrorInvalidValue;
+                           cudaStream_t s, bool pdl, int qmax) {
+  if (d % 4 != 0 || d > 4 * kRowVec * kRowThreads || qmax < 1 || qmax > 127) return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, x, g, d, eps, y, q, sq);
+  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, x, g, d, eps, y, q, sq, qmax);
 }
 
-// Per-row int8 quantisation of bf16 rows (16-byte loads kept in registers; rows up to 16384).
+// Per-row symmetric quantisation of bf16 rows to codes in [-qmax, qmax] (16-byte loads kept in
+// registers; rows up to 16384).  pack4: two 4-bit codes per byte (column 2j in the low nibble of
+// byte j, 2j + 1 in the high one, two's complement), ldq then counted in bytes.
 constexpr int kQVec = 4;  // uint4 (8 bf16) per thread
 __global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t* __restrict__ x, int d, int ldx,
                                                                  int8_t* __restrict__ q, int ldq,
-                                                                 float* __restrict__ sq) {
+                                                                 float* __restrict__ sq, int qmax, int pack4) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
@@ -259,31 +262,37 @@ __global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t*
     for (int e = 0; e < 4; ++e) amax = fmaxf(amax, fmaxf(fabsf(bf2f(w[e] & 0xFFFF)), fabsf(bf2f(w[e] >> 16))));
   }
   amax = block_max(amax, red);
-  const float inv = amax > 0.f ? __fdiv_rn(127.f, amax) : 0.f;
+  const float inv = amax > 0.f ? __fdiv_rn((float)qmax, amax) : 0.f;
 #pragma unroll
   for (int k = 0; k < kQVec; ++k) {
     const int c = threadIdx.x + k * kRowThreads;
     if (c < nv) {
       const uint32_t w[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
-      uint32_t o[2] = {0u, 0u};
+      uint32_t o[2] = {0u, 0u}, p4 = 0u;
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
         const float v = bf2f(e & 1 ? (w[e >> 1] >> 16) : (w[e >> 1] & 0xFFFF));
-        const int8_t qq = amax > 0.f ? quant_one(v, inv) : (int8_t)0;
+        const int8_t qq = amax > 0.f ? quant_one(v, inv, qmax) : (int8_t)0;
         o[e >> 2] |= ((uint32_t)(uint8_t)qq) << (8 * (e & 3));
+        p4 |= ((uint32_t)qq & 0xFu) << (4 * e);
       }
-      reinterpret_cast<uint2*>(q + (size_t)i * ldq)[c] = make_uint2(o[0], o[1]);
+      if (pack4)
+        reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(q) + (size_t)i * ldq)[c] = p4;
+      else
+        reinterpret_cast<uint2*>(q + (size_t)i * ldq)[c] = make_uint2(o[0], o[1]);
     }
   }
-  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, 127.f) : 0.f;
+  if (threadIdx.x == 0) sq[i] = amax > 0.f ? __fdiv_rn(amax, (float)qmax) : 0.f;
 }
 
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
-                              bool pdl) {
-  if (d % 8 != 0 || ldx % 8 != 0 || ldq % 8 != 0 || d > 8 * kQVec * kRowThreads) return cudaErrorInvalidValue;
+                              bool pdl, int qmax, bool pack4) {
+  if (d % 8 != 0 || ldx % 8 != 0 || ldq % (pack4 ? 4 : 8) != 0 || d > 8 * kQVec * kRowThreads || qmax < 1 ||
+      qmax > 127 || (pack4 && qmax > 7))
+    return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq);
+  return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq, qmax, pack4 ? 1 : 0);
 }
 
 // ---------------------------------------------------------------------------------------------

@@ -123,3 +123,22 @@ def test_quantize_rows_bit_exact_including_golden_rows(cs):
     q_ref, s_ref = oracle.quantize_rows_f32(xb)
     assert np.array_equal(q.cpu().numpy(), q_ref)
     assert np.array_equal(s.cpu().numpy(), s_ref)
+
+
+def test_quantize_rows4_bit_exact(cs):
+    """W4A4 activation codes (App. C): the int4 rule on bf16 rows, bit-exact against the oracle's
+    fp32 rule with qmax 7, including rows with exact .5 ties and a zero row."""
+    width = 32
+    rng = np.random.default_rng(9)
+    x = (rng.standard_normal((48, width)) * rng.uniform(0.1, 20, (48, 1))).astype(np.float32)
+    x[0, :6] = [7, 3.5, -3.5, 0.5, -0.5, 2.5]  # amax 7: the codes are x itself, ties to even
+    x[1, :] = 0.0
+    bits = synth.bf16_bits_rne(x)
+    xb = synth.bf16_to_f32(bits)
+    q4 = torch.empty(x.shape[0], width // 2, dtype=torch.uint8, device="cuda")
+    s = torch.empty(x.shape[0], dtype=torch.float32, device="cuda")
+    cs.quantize_rows4(_bf16_dev(bits), x.shape[0], width, q4, s)
+    torch.cuda.synchronize()
+    q_ref, s_ref = oracle.quantize_rows_f32(xb, 7)
+    assert np.array_equal(cs.unpack_int4(q4.cpu().numpy(), width), q_ref)
+    assert np.array_equal(s.cpu().numpy(), s_ref)

@@ -97,6 +97,20 @@ def test_int8_weights_bit_exact(cs, dev_model, ow):
             assert np.array_equal(s, s_ref), (name, l)
 
 
+def test_int4_weights_bit_exact(cs, dev_model, ow):
+    """W4A4 weight codes and scales (casspec_quantize_weights) equal the oracle's int4 rule."""
+    d, F = SH.d_model, SH.ffn
+    for l in range(SH.n_layers):
+        for name, tq, ts, K in (("wqkv", cs.T_WQKV_Q4, cs.T_WQKV_S4, d), ("wo", cs.T_WO_Q4, cs.T_WO_S4, d),
+                                ("wg", cs.T_WG_Q4, cs.T_WG_S4, d), ("wu", cs.T_WU_Q4, cs.T_WU_S4, d),
+                                ("wd", cs.T_WD_Q4, cs.T_WD_S4, F)):
+            q_ref, s_ref = ow.intq(name, l, 7)
+            q = cs.unpack_int4(dev_model.slot(tq, l).cpu().numpy(), K)
+            s = dev_model.slot(ts, l).cpu().numpy().view(np.float32)
+            assert np.array_equal(q, q_ref), (name, l)
+            assert np.array_equal(s, s_ref), (name, l)
+
+
 def test_prefill_verify_accept_compact(cs, dev_model, ow, prefix):
     kv, okv = fresh_pair(cs, dev_model, ow, prefix)
     P0 = len(prefix)
@@ -239,6 +253,24 @@ def test_int8_mode_logits(cs, dev_model, ow, prefix):
     ref = oracle.tree_step(ow, okv, toks, parent, quant_mode=1)
     err = rel_err(got, ref)
     assert np.all(err < TOL_INT8), err
+    kv.close()
+
+
+def test_w4a4_mode_logits(cs, dev_model, ow, prefix):
+    """W4A4 draft logits.  A 4-bit code moves by a seventh of its row's range, so the logits follow
+    any bf16-sized perturbation strongly (0.14 of the range on this model); the bound is twice the
+    oracle's own movement when q and the new K/V are rounded to bf16, never below 5e-2.  The integer
+    parts are checked bit-exactly by test_int4_weights_bit_exact and test_quantize_rows4_bit_exact."""
+    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
+    _, okv2 = fresh_pair(cs, dev_model, ow, prefix)
+    parent = synth.tree(4, 8, 4)
+    toks = synth.tokens(4, 8, SH.vocab)
+    got = gpu_step(cs, dev_model, kv, toks, parent, mode=2)
+    assert cs.get_status(dev_model.h) == 0
+    ref = oracle.tree_step(ow, okv, toks, parent, quant_mode=2)
+    pert = oracle.tree_step(ow, okv2, toks, parent, quant_mode=2, attn_bf16=True)
+    err = rel_err(got, ref)
+    assert err.max() <= max(TOL_INT8, 2.0 * rel_err(pert, ref).max()), (err.max(), rel_err(pert, ref).max())
     kv.close()
 
 
