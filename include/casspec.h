@@ -78,7 +78,8 @@ typedef struct casspec_kv casspec_kv;       /* opaque host handle */
  * The int8 copies (written by casspec_quantize_weights) are WQKV_Q .. WD_Q int8 with the same
  * shapes and WQKV_S .. WD_S fp32 per-output-row scales.  The int4 copies (W4A4, same call) are
  * WQKV_Q4 .. WD_Q4 with rows of K / 2 bytes (column 2j in the low nibble of byte j, two's
- * complement codes in [-7, 7]) and WQKV_S4 .. WD_S4 fp32 scales (amax / 7).
+ * complement codes in [-7, 7]) and WQKV_S4 .. WD_S4 fp32 scales (amax / 7); WQKV_F8 .. WD_F8 hold
+ * the same codes as one FP8 e4m3 byte each (the tensor-core W4A4 path).
  * Step state (read-only views of the model's scratch, valid until the next step on the model; layer
  * ignored; for tests and for callers that want the hidden state):
  *   RESIDUAL [64][d] fp32: the residual stream after the step's last active layer (before the final
@@ -119,7 +120,12 @@ enum casspec_tensor_id {
   CASSPEC_T_WO_S4 = 29,
   CASSPEC_T_WG_S4 = 30,
   CASSPEC_T_WU_S4 = 31,
-  CASSPEC_T_WD_S4 = 32
+  CASSPEC_T_WD_S4 = 32,
+  CASSPEC_T_WQKV_F8 = 33,
+  CASSPEC_T_WO_F8 = 34,
+  CASSPEC_T_WG_F8 = 35,
+  CASSPEC_T_WU_F8 = 36,
+  CASSPEC_T_WD_F8 = 37
 };
 
 /* Option bits for casspec_set_options. */
@@ -131,6 +137,8 @@ enum casspec_tensor_id {
  * casspec_get_status, and the model stays usable once the bit is cleared.  Such steps run
  * eagerly (never captured into a graph). */
 #define CASSPEC_OPT_TEST_STALL 4u
+#define CASSPEC_OPT_W4_TC 8u /* quant_mode 2 on the tensor cores with e4m3 codes (default on); off: 4-bit
+                                codes through the integer mma.sync path */
 
 /* ---------------------------------------------------------------------------------------------
  * Model

@@ -21,12 +21,13 @@ TOPK_MAX = 8
 DYTC_MAX_CLASS = 4  # latency-model classes (one regression per step arithmetic)
 DYTC_WORK = 24 * MAX_TREE  # int32 entries of casspec_dytc_round's device scratch
 SKIP_ATTN, SKIP_FFN = 0x2, 0x4  # skip-mask flags on a non-zero byte: drop the attention / FFN block
-OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL = 1, 2, 4
+OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL, OPT_W4_TC = 1, 2, 4, 8
 
 (T_EMBED, T_LM_HEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WG, T_WU, T_WD,
  T_WQKV_Q, T_WO_Q, T_WG_Q, T_WU_Q, T_WD_Q, T_WQKV_S, T_WO_S, T_WG_S, T_WU_S, T_WD_S,
  T_RESIDUAL, T_ACT_Q, T_ACT_S,
- T_WQKV_Q4, T_WO_Q4, T_WG_Q4, T_WU_Q4, T_WD_Q4, T_WQKV_S4, T_WO_S4, T_WG_S4, T_WU_S4, T_WD_S4) = range(33)
+ T_WQKV_Q4, T_WO_Q4, T_WG_Q4, T_WU_Q4, T_WD_Q4, T_WQKV_S4, T_WO_S4, T_WG_S4, T_WU_S4, T_WD_S4,
+ T_WQKV_F8, T_WO_F8, T_WG_F8, T_WU_F8, T_WD_F8) = range(38)
 
 EXPORTS = [
     "casspec_model_bytes", "casspec_create_model", "casspec_destroy_model", "casspec_set_stream",
@@ -341,6 +342,16 @@ def unpack_int4(b: np.ndarray, K: int) -> np.ndarray:
     out[:, 0::2] = np.where(lo > 7, lo - 16, lo)
     out[:, 1::2] = np.where(hi > 7, hi - 16, hi)
     return out
+
+
+def decode_e4m3_codes(b: np.ndarray) -> np.ndarray:
+    """Integer codes in [-16, 16] from their FP8 e4m3 bytes (sign, 4 exponent bits with bias 7, 3
+    fraction bits); only exact integers are expected."""
+    b = np.asarray(b, dtype=np.uint8)
+    e = ((b >> 3) & 15).astype(np.int64)
+    f = (b & 7).astype(np.int64)
+    mag = np.where(e == 0, 0, ((8 + f) << np.maximum(e - 7, 0)) >> 3)
+    return np.where(b & 0x80, -mag, mag).astype(np.int8)
 
 
 def profile(m: int, enable: bool) -> None:

@@ -13,7 +13,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libcasspec.so")
 SOURCES = ["api.cu", "chain.cu", "gemm_tc.cu", "gemm_i8.cu", "attention.cu", "small_kernels.cu",
-           "linear_static.cu", "dytc.cpp", "pld.cu", "topk.cu"]
+           "linear_static.cu", "dytc.cpp", "pld.cu", "topk.cu", "gemm_f8.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-DCASSPEC_BUILD"]

@@ -27,6 +27,8 @@ struct LayerPtrs {
   float *qkv_s, *wo_s, *wg_s, *wu_s, *wd_s;
   int8_t *qkv_q4, *wo_q4, *wg_q4, *wu_q4, *wd_q4;  // W4A4: two 4-bit codes per byte
   float *qkv_s4, *wo_s4, *wg_s4, *wu_s4, *wd_s4;
+  uint8_t *qkv_f8, *wo_f8, *wg_f8, *wu_f8, *wd_f8;  // W4A4: the same codes as e4m3 bytes (tensor-core path)
+  CUtensorMap tm_qkv8, tm_o8, tm_g8, tm_u8, tm_d8;
   CUtensorMap tm_qkv, tm_o, tm_g, tm_u, tm_d;
   uint8_t *wqkv_p, *wo_p, *wgu_p, *wd_p;  // the projections packed per CTA for the chain (pack_rows_kernel)
 };
@@ -40,6 +42,7 @@ struct Layout {
   std::vector<size_t> wqkv_p, wo_p, wgu_p, wd_p;
   size_t lm_p;
   std::vector<size_t> qkv_q4, wo_q4, wg_q4, wu_q4, wd_q4, qkv_s4, wo_s4, wg_s4, wu_s4, wd_s4;
+  std::vector<size_t> qkv_f8, wo_f8, wg_f8, wu_f8, wd_f8;
   size_t x, q, o, u, xa, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
   size_t gemm_part, gemm_cnt, chain_ready, chain_done, i8_part, i8_cnt, attn_part, attn_ml, attn_cnt, status;
   size_t scratch_begin;
@@ -114,6 +117,11 @@ Layout make_layout(const casspec_model_config& c) {
       L.wg_s4.push_back(take(F * 4));
       L.wu_s4.push_back(take(F * 4));
       L.wd_s4.push_back(take(d * 4));
+      L.qkv_f8.push_back(take(3 * d * d));
+      L.wo_f8.push_back(take(d * d));
+      L.wg_f8.push_back(take(F * d));
+      L.wu_f8.push_back(take(F * d));
+      L.wd_f8.push_back(take(d * F));
     }
   }
   L.scratch_begin = align_up(off, 256);
@@ -183,7 +191,7 @@ struct casspec_model {
   uint8_t* base = nullptr;
   cudaStream_t stream = nullptr;
   cudaStream_t cap_stream = nullptr;
-  unsigned flags = CASSPEC_OPT_PDL;
+  unsigned flags = CASSPEC_OPT_PDL | CASSPEC_OPT_W4_TC;
   int num_sms = 0;
   uint16_t *embed, *lm_head;
   float* final_norm;
@@ -194,6 +202,7 @@ struct casspec_model {
   // their 64 x BN boxes, BN = 16, 32, 48, 64, and [4]: 64 x 128 boxes (both planes of all 64 tokens
   // in one load, used when n > 48)
   CUtensorMap tm_o[5], tm_u[5], tm_xa[5];
+  CUtensorMap tm_xq8_d[4], tm_xq8_f[4];    // e4m3 activation codes, rows of d or F bytes, 128 x BN boxes
   int8_t* xq;
   float* xs;
   unsigned *chain_ready, *chain_done;
@@ -555,6 +564,25 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     // mode 1: W8A8 (codes in [-127, 127]); mode 2: W4A4 (codes in [-7, 7], weights two per byte)
     const bool w4 = mode == 2;
     const int qmax = w4 ? 7 : 127;
+    // W4A4 on the tensor cores: e4m3 codes, exact fp32 accumulation (casspec gemm_f8); otherwise the
+    // 4-bit codes go through the s8 MMA of gemm_i8
+    const bool tc4 = w4 && (m->flags & CASSPEC_OPT_W4_TC) != 0;
+    const int afmt = tc4 ? 2 : 0;  // activation codes as e4m3 bytes for the tensor-core path
+    auto gemmf8 = [&](const CUtensorMap& tw, const CUtensorMap& tw2, const CUtensorMap& tx, const float* sw,
+                      const float* sw2, int N, int K, int tiles, int epi, const EpiParams& e) -> cudaError_t {
+      GemmF8Args g = {};
+      g.tiles = tiles;
+      g.kblocks = cdiv(K, 128);
+      g.N = N;
+      g.sw = sw;
+      g.sw2 = sw2;
+      g.sx = m->xs;
+      g.partials = m->gemm_part;
+      g.counters = m->gemm_cnt;
+      g.status = m->status;
+      g.ep = e;
+      return launch_gemm_f8(tw, tw2, tx, BN, epi, g, gemm_bf16_grid(tiles, g.kblocks, m->num_sms), s, pdl);
+    };
     auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
                      int epi, const EpiParams& e) -> cudaError_t {
       GemmI8Args g8 = {};
@@ -607,27 +635,42 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       }
       if (it.kind == IT_QKV) {
         LAUNCH(CASSPEC_K_OTHER,
-               launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax));
+               launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax, afmt));
         EpiParams e = base;
         e.N = 3 * d;
         e.q_out = m->q;
         e.kc = kv_layer_k(kv, it.l);
         e.vc = kv_layer_v(kv, it.l);
-        LAUNCH(CASSPEC_K_QKV, gemm8(q_qkv, s_qkv, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
+        if (tc4)
+          LAUNCH(CASSPEC_K_QKV, gemmf8(Lp.tm_qkv8, Lp.tm_qkv8, m->tm_xq8_d[bi], s_qkv, nullptr, 3 * d, d, 3 * d / 128,
+                                       EPI_QKV, e));
+        else
+          LAUNCH(CASSPEC_K_QKV, gemm8(q_qkv, s_qkv, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
       } else if (it.kind == IT_WO) {
         // W8A8 activations are the bf16 values: the hi plane of the split output
-        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl, qmax));
-        LAUNCH(CASSPEC_K_WO, gemm8(q_wo, s_wo, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl, qmax, afmt));
+        if (tc4)
+          LAUNCH(CASSPEC_K_WO, gemmf8(Lp.tm_o8, Lp.tm_o8, m->tm_xq8_d[bi], s_wo, nullptr, d, d, d / 128, EPI_RESID, ed));
+        else
+          LAUNCH(CASSPEC_K_WO, gemm8(q_wo, s_wo, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
       } else if (it.kind == IT_GU) {
         LAUNCH(CASSPEC_K_OTHER,
-               launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax));
+               launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax, afmt));
         EpiParams eg = base;
         eg.N = F;
         eg.u_out = m->u;
-        LAUNCH(CASSPEC_K_GATEUP, gemm8(q_wg, s_wg, q_wu, s_wu, F, d, cdiv(F, 64), EPI_GLU, eg));
+        if (tc4)
+          LAUNCH(CASSPEC_K_GATEUP, gemmf8(Lp.tm_g8, Lp.tm_u8, m->tm_xq8_d[bi], s_wg, s_wu, F, d, cdiv(F, 64), EPI_GLU,
+                                          eg));
+        else
+          LAUNCH(CASSPEC_K_GATEUP, gemm8(q_wg, s_wg, q_wu, s_wu, F, d, cdiv(F, 64), EPI_GLU, eg));
       } else {
-        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl, qmax));
-        LAUNCH(CASSPEC_K_DOWN, gemm8(q_wd, s_wd, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl, qmax, afmt));
+        if (tc4)
+          LAUNCH(CASSPEC_K_DOWN, gemmf8(Lp.tm_d8, Lp.tm_d8, m->tm_xq8_f[bi], s_wd, nullptr, d, F, d / 128, EPI_RESID,
+                                        ed));
+        else
+          LAUNCH(CASSPEC_K_DOWN, gemm8(q_wd, s_wd, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
       }
     }
   }
@@ -649,6 +692,21 @@ bool build_tensor_maps(casspec_model* m) {
     ok = ok && encode_tmap_bf16(&Lp.tm_d, Lp.wd, F, d, F * 2, 64, 128);
   }
   ok = ok && encode_tmap_bf16(&m->tm_lm, m->lm_head, d, V, d * 2, 64, 128);
+  if (c.with_int8) {
+    for (int l = 0; l < c.n_layers; ++l) {
+      LayerPtrs& Lp = m->layers[l];
+      ok = ok && encode_tmap_u8(&Lp.tm_qkv8, Lp.qkv_f8, d, 3 * d, d, 128, 128);
+      ok = ok && encode_tmap_u8(&Lp.tm_o8, Lp.wo_f8, d, d, d, 128, 128);
+      ok = ok && encode_tmap_u8(&Lp.tm_g8, Lp.wg_f8, d, F, d, 128, 64);
+      ok = ok && encode_tmap_u8(&Lp.tm_u8, Lp.wu_f8, d, F, d, 128, 64);
+      ok = ok && encode_tmap_u8(&Lp.tm_d8, Lp.wd_f8, F, d, F, 128, 128);
+    }
+    for (int b = 0; b < 4; ++b) {
+      const uint32_t BN = 16u * (uint32_t)(b + 1);
+      ok = ok && encode_tmap_u8(&m->tm_xq8_d[b], m->xq, d, kMaxTree, d, 128, BN);
+      ok = ok && encode_tmap_u8(&m->tm_xq8_f[b], m->xq, F, kMaxTree, F, 128, BN);
+    }
+  }
   for (int b = 0; b < 4; ++b) {
     const uint32_t BN = 16u * (uint32_t)(b + 1);
     ok = ok && encode_tmap_bf16(&m->tm_o[b], m->o, d, 2 * kMaxTree, d * 2, 64, BN);
@@ -748,6 +806,11 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
       p.wg_s4 = reinterpret_cast<float*>(b + L.wg_s4[l]);
       p.wu_s4 = reinterpret_cast<float*>(b + L.wu_s4[l]);
       p.wd_s4 = reinterpret_cast<float*>(b + L.wd_s4[l]);
+      p.qkv_f8 = b + L.qkv_f8[l];
+      p.wo_f8 = b + L.wo_f8[l];
+      p.wg_f8 = b + L.wg_f8[l];
+      p.wu_f8 = b + L.wu_f8[l];
+      p.wd_f8 = b + L.wd_f8[l];
     }
   }
   m->x = reinterpret_cast<float*>(b + L.x);
@@ -818,7 +881,8 @@ int casspec_set_stream(casspec_model* m, void* stream) {
 }
 
 int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
-  if (m == nullptr || (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS | CASSPEC_OPT_TEST_STALL)) != 0)
+  if (m == nullptr ||
+      (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS | CASSPEC_OPT_TEST_STALL | CASSPEC_OPT_W4_TC)) != 0)
     return CASSPEC_E_INVAL;
   if (old_flags) *old_flags = m->flags;
   if (flags != m->flags) {
@@ -875,6 +939,11 @@ int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size
     case CASSPEC_T_WG_S4: p = L->wg_s4; nb = F * 4; break;
     case CASSPEC_T_WU_S4: p = L->wu_s4; nb = F * 4; break;
     case CASSPEC_T_WD_S4: p = L->wd_s4; nb = d * 4; break;
+    case CASSPEC_T_WQKV_F8: p = L->qkv_f8; nb = 3 * d * d; break;
+    case CASSPEC_T_WO_F8: p = L->wo_f8; nb = d * d; break;
+    case CASSPEC_T_WG_F8: p = L->wg_f8; nb = F * d; break;
+    case CASSPEC_T_WU_F8: p = L->wu_f8; nb = F * d; break;
+    case CASSPEC_T_WD_F8: p = L->wd_f8; nb = d * F; break;
     default: return CASSPEC_E_INVAL;
   }
   *dev_ptr = p;
@@ -894,11 +963,17 @@ int casspec_quantize_weights(casspec_model* m) {
     CK(launch_quant_rows(p.wu, F, d, d, p.wu_q, d, p.wu_s, m->stream, false));
     CK(launch_quant_rows(p.wd, d, F, F, p.wd_q, F, p.wd_s, m->stream, false));
     // the W4A4 copies: codes in [-7, 7], two per byte (row stride K / 2 bytes)
-    CK(launch_quant_rows(p.wqkv, 3 * d, d, d, p.qkv_q4, d / 2, p.qkv_s4, m->stream, false, 7, true));
-    CK(launch_quant_rows(p.wo, d, d, d, p.wo_q4, d / 2, p.wo_s4, m->stream, false, 7, true));
-    CK(launch_quant_rows(p.wg, F, d, d, p.wg_q4, d / 2, p.wg_s4, m->stream, false, 7, true));
-    CK(launch_quant_rows(p.wu, F, d, d, p.wu_q4, d / 2, p.wu_s4, m->stream, false, 7, true));
-    CK(launch_quant_rows(p.wd, d, F, F, p.wd_q4, F / 2, p.wd_s4, m->stream, false, 7, true));
+    CK(launch_quant_rows(p.wqkv, 3 * d, d, d, p.qkv_q4, d / 2, p.qkv_s4, m->stream, false, 7, 1));
+    CK(launch_quant_rows(p.wo, d, d, d, p.wo_q4, d / 2, p.wo_s4, m->stream, false, 7, 1));
+    CK(launch_quant_rows(p.wg, F, d, d, p.wg_q4, d / 2, p.wg_s4, m->stream, false, 7, 1));
+    CK(launch_quant_rows(p.wu, F, d, d, p.wu_q4, d / 2, p.wu_s4, m->stream, false, 7, 1));
+    CK(launch_quant_rows(p.wd, d, F, F, p.wd_q4, F / 2, p.wd_s4, m->stream, false, 7, 1));
+    // ... and as e4m3 bytes for the tensor-core path (same codes, same scales)
+    CK(launch_quant_rows(p.wqkv, 3 * d, d, d, reinterpret_cast<int8_t*>(p.qkv_f8), d, p.qkv_s4, m->stream, false, 7, 2));
+    CK(launch_quant_rows(p.wo, d, d, d, reinterpret_cast<int8_t*>(p.wo_f8), d, p.wo_s4, m->stream, false, 7, 2));
+    CK(launch_quant_rows(p.wg, F, d, d, reinterpret_cast<int8_t*>(p.wg_f8), d, p.wg_s4, m->stream, false, 7, 2));
+    CK(launch_quant_rows(p.wu, F, d, d, reinterpret_cast<int8_t*>(p.wu_f8), d, p.wu_s4, m->stream, false, 7, 2));
+    CK(launch_quant_rows(p.wd, d, F, F, reinterpret_cast<int8_t*>(p.wd_f8), F, p.wd_s4, m->stream, false, 7, 2));
   }
   return CASSPEC_OK;
 }
@@ -1203,7 +1278,7 @@ int casspec_quantize_rows4(const uint16_t* x, int n, int d, uint8_t* q4, float* 
   if (x == nullptr || q4 == nullptr || s == nullptr) return CASSPEC_E_INVAL;
   if (n < 1 || d < 8 || d % 8 != 0) return CASSPEC_E_SHAPE;
   CK(launch_quant_rows(x, n, d, d, reinterpret_cast<int8_t*>(q4), d / 2, s, static_cast<cudaStream_t>(stream), false,
-                       7, true));
+                       7, 1));
   return CASSPEC_OK;
 }
 

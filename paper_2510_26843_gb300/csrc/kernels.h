@@ -72,6 +72,20 @@ struct GemmI8Args {
   EpiParams ep;
 };
 
+// exact W4A4 projection on the tensor cores (e4m3 codes in [-7, 7], fp32 accumulation is exact)
+struct GemmF8Args {
+  int tiles;     // 128-row output tiles (EPI_GLU: 64 gate + 64 up rows per tile)
+  int kblocks;   // ceil(K / 128)
+  int N;         // output channels (EPI_GLU: F)
+  const float* sw;   // [N] weight scales (EPI_GLU: gate)
+  const float* sw2;  // EPI_GLU: up weight scales
+  const float* sx;   // [64] activation scales
+  float* partials;     // stream-K partial tiles, (tiles + grid) slots of 64 x 128 fp32
+  unsigned* counters;  // [tiles], zero between launches
+  int* status;
+  EpiParams ep;
+};
+
 constexpr int kAttnMaxSplits = 16;
 struct AttnArgs {
   const uint16_t* q;    // [64][d] bf16 (rotated)
@@ -188,6 +202,11 @@ size_t gemm_partials_floats(int tiles, int grid);
 cudaError_t launch_gemm_bf16(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int BN, int epi,
                              const GemmArgs& args, int grid, cudaStream_t stream, bool pdl);
 
+bool encode_tmap_u8(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows, uint64_t row_stride_bytes,
+                    uint32_t box_inner, uint32_t box_rows);
+cudaError_t launch_gemm_f8(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int BN, int epi,
+                           const GemmF8Args& args, int grid, cudaStream_t stream, bool pdl);
+
 int gemm_i8_ksplit(int tiles, int K, int num_sms);
 cudaError_t launch_gemm_i8(const GemmI8Args& args, int BN, int epi, cudaStream_t stream, bool pdl);
 
@@ -207,10 +226,12 @@ size_t pack_rows_bytes(int N, int K, int kind);
 cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int rows, int K, int G, int S, int kind,
                              int d, int hd, int rot_groups, uint8_t* out, cudaStream_t s);
 int chain_pairs_fit(int grid);  // 1 if a launch of grid / 2 CTA pairs fits the GPU at once
+// Quantised outputs: fmt 0 int8 codes, 1 (quant_rows only) two 4-bit codes per byte, 2 e4m3 bytes of
+// codes in [-7, 7].
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
-                           cudaStream_t s, bool pdl, int qmax = 127);
+                           cudaStream_t s, bool pdl, int qmax = 127, int fmt = 0);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
-                              bool pdl, int qmax = 127, bool pack4 = false);
+                              bool pdl, int qmax = 127, int fmt = 0);
 cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,
                                  float* margin, cudaStream_t s, bool pdl);
 cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaStream_t s);

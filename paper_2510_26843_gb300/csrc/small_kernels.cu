@@ -110,6 +110,14 @@ __device__ __forceinline__ float block_max(float v, float* red) {
 // Per-row symmetric int8 quantisation rule (App. C activation-quantisation DSIA, W8A8 reading):
 // inv = 127 / amax (IEEE division), q = rint(x * inv) (IEEE multiply, ties to even), clamp +-127,
 // scale = amax / 127; amax = 0 gives q = 0, scale 0.
+// e4m3 byte of an integer code in [-7, 7] (exact: e4m3 holds every integer up to 16); byte a of the
+// constant is the code of +a
+__device__ __forceinline__ uint8_t e4m3_of_code(int q) {
+  const uint32_t a = (uint32_t)(q < 0 ? -q : q);
+  const uint8_t m = (uint8_t)((0x4E4C4A4844403800ull >> (8 * a)) & 0xFFu);
+  return q < 0 ? (uint8_t)(m | 0x80u) : m;
+}
+
 __device__ __forceinline__ int8_t quant_one(float x, float inv, int qmax) {
   int q = __float2int_rn(__fmul_rn(x, inv));
   q = q > qmax ? qmax : (q < -qmax ? -qmax : q);
@@ -165,7 +173,7 @@ constexpr int kRowVec = 8;  // float4 per thread: rows up to 16384 fp32 values
 __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g,
                                                               int d, float eps, uint16_t* __restrict__ y,
                                                               int8_t* __restrict__ q, float* __restrict__ sq,
-                                                              int qmax) {
+                                                              int qmax, int e4m3) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
@@ -221,6 +229,12 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __res
       o.y = amax > 0.f ? quant_one(bf2f(b[k][1]), inv, qmax) : 0;
       o.z = amax > 0.f ? quant_one(bf2f(b[k][2]), inv, qmax) : 0;
       o.w = amax > 0.f ? quant_one(bf2f(b[k][3]), inv, qmax) : 0;
+      if (e4m3) {
+        o.x = (int8_t)e4m3_of_code(o.x);
+        o.y = (int8_t)e4m3_of_code(o.y);
+        o.z = (int8_t)e4m3_of_code(o.z);
+        o.w = (int8_t)e4m3_of_code(o.w);
+      }
       reinterpret_cast<char4*>(q + (size_t)i * d)[c] = o;
     }
   }
@@ -228,20 +242,23 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* __res
 }
 
 cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float eps, uint16_t* y, int8_t* q, float* sq,
-                           cudaStream_t s, bool pdl, int qmax) {
-  if (d % 4 != 0 || d > 4 * kRowVec * kRowThreads || qmax < 1 || qmax > 127) return cudaErrorInvalidValue;
+                           cudaStream_t s, bool pdl, int qmax, int fmt) {
+  if (d % 4 != 0 || d > 4 * kRowVec * kRowThreads || qmax < 1 || qmax > 127 || (fmt != 0 && fmt != 2) ||
+      (fmt == 2 && qmax > 7))
+    return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, x, g, d, eps, y, q, sq, qmax);
+  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, x, g, d, eps, y, q, sq, qmax, fmt == 2 ? 1 : 0);
 }
 
 // Per-row symmetric quantisation of bf16 rows to codes in [-qmax, qmax] (16-byte loads kept in
-// registers; rows up to 16384).  pack4: two 4-bit codes per byte (column 2j in the low nibble of
-// byte j, 2j + 1 in the high one, two's complement), ldq then counted in bytes.
+// registers; rows up to 16384).  fmt 0: int8 codes; 1: two 4-bit codes per byte (column 2j in the
+// low nibble of byte j, 2j + 1 in the high one, two's complement), ldq then counted in bytes; 2: one
+// e4m3 byte per code (codes in [-7, 7]).
 constexpr int kQVec = 4;  // uint4 (8 bf16) per thread
 __global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t* __restrict__ x, int d, int ldx,
                                                                  int8_t* __restrict__ q, int ldq,
-                                                                 float* __restrict__ sq, int qmax, int pack4) {
+                                                                 float* __restrict__ sq, int qmax, int fmt) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
@@ -273,10 +290,10 @@ __global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t*
       for (int e = 0; e < 8; ++e) {
         const float v = bf2f(e & 1 ? (w[e >> 1] >> 16) : (w[e >> 1] & 0xFFFF));
         const int8_t qq = amax > 0.f ? quant_one(v, inv, qmax) : (int8_t)0;
-        o[e >> 2] |= ((uint32_t)(uint8_t)qq) << (8 * (e & 3));
+        o[e >> 2] |= ((uint32_t)(fmt == 2 ? e4m3_of_code(qq) : (uint8_t)qq)) << (8 * (e & 3));
         p4 |= ((uint32_t)qq & 0xFu) << (4 * e);
       }
-      if (pack4)
+      if (fmt == 1)
         reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(q) + (size_t)i * ldq)[c] = p4;
       else
         reinterpret_cast<uint2*>(q + (size_t)i * ldq)[c] = make_uint2(o[0], o[1]);
@@ -286,13 +303,13 @@ __global__ void __launch_bounds__(kRowThreads) quant_rows_kernel(const uint16_t*
 }
 
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
-                              bool pdl, int qmax, bool pack4) {
-  if (d % 8 != 0 || ldx % 8 != 0 || ldq % (pack4 ? 4 : 8) != 0 || d > 8 * kQVec * kRowThreads || qmax < 1 ||
-      qmax > 127 || (pack4 && qmax > 7))
+                              bool pdl, int qmax, int fmt) {
+  if (d % 8 != 0 || ldx % 8 != 0 || ldq % (fmt == 1 ? 4 : 8) != 0 || d > 8 * kQVec * kRowThreads || qmax < 1 ||
+      qmax > 127 || fmt < 0 || fmt > 2 || (fmt != 0 && qmax > 7))
     return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kRowThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq, qmax, pack4 ? 1 : 0);
+  return cudaLaunchKernelEx(&cfg, quant_rows_kernel, x, d, ldx, q, ldq, sq, qmax, fmt);
 }
 
 // ---------------------------------------------------------------------------------------------

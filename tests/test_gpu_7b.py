@@ -76,7 +76,7 @@ def test_single_layer_7b(cs):
     sh = synth.ModelShape(1, SH7.d_model, SH7.n_heads, SH7.head_dim, SH7.ffn, SH7.vocab)
     P, n = 1024, 32
     dm = DeviceModel(sh, SEED)
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC)
     kv = DeviceKV(dm, P + 64)
     kv.load_random_prefix(SEED, P)
     ow = oracle.Weights.from_seed(SEED, sh, keep_layers=1)
@@ -128,7 +128,7 @@ def dm7(cs):
     from paper_2510_26843_gb300.workload import DeviceModel
 
     dm = DeviceModel(SH7, SEED, with_int8=True)
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC)
     yield dm
     dm.close()
 

@@ -111,6 +111,17 @@ def test_int4_weights_bit_exact(cs, dev_model, ow):
             assert np.array_equal(s, s_ref), (name, l)
 
 
+def test_e4m3_weights_bit_exact(cs, dev_model, ow):
+    """The tensor-core W4A4 weights are the int4 codes as e4m3 bytes."""
+    d, F = SH.d_model, SH.ffn
+    for l in range(SH.n_layers):
+        for name, tq, K in (("wqkv", cs.T_WQKV_F8, d), ("wo", cs.T_WO_F8, d), ("wg", cs.T_WG_F8, d),
+                            ("wu", cs.T_WU_F8, d), ("wd", cs.T_WD_F8, F)):
+            q_ref, _ = ow.intq(name, l, 7)
+            q = cs.decode_e4m3_codes(dev_model.slot(tq, l).cpu().numpy()).reshape(q_ref.shape)
+            assert np.array_equal(q, q_ref), (name, l)
+
+
 def test_prefill_verify_accept_compact(cs, dev_model, ow, prefix):
     kv, okv = fresh_pair(cs, dev_model, ow, prefix)
     P0 = len(prefix)
@@ -272,6 +283,23 @@ def test_w4a4_mode_logits(cs, dev_model, ow, prefix):
     err = rel_err(got, ref)
     assert err.max() <= max(TOL_INT8, 2.0 * rel_err(pert, ref).max()), (err.max(), rel_err(pert, ref).max())
     kv.close()
+
+
+@pytest.mark.parametrize("n", [8, 33])
+def test_w4a4_tensor_core_path_equals_integer_path(cs, dev_model, ow, prefix, n):
+    """Both W4A4 paths take the same integer codes and scales, and both integer sums are exact (the
+    s8 MMA in int32, the e4m3 MMA in fp32 below 2^22), so the logits are bitwise equal."""
+    parent = synth.tree(40 + n, n, 8)
+    toks = synth.tokens(40 + n, n, SH.vocab)
+    out = []
+    for flags in (cs.OPT_PDL | cs.OPT_W4_TC, cs.OPT_PDL):
+        cs.set_options(dev_model.h, flags)
+        kv, _ = fresh_pair(cs, dev_model, ow, prefix)
+        out.append(gpu_step(cs, dev_model, kv, toks, parent, mode=2))
+        assert cs.get_status(dev_model.h) == 0
+        kv.close()
+    cs.set_options(dev_model.h, cs.OPT_PDL | cs.OPT_W4_TC)
+    np.testing.assert_array_equal(out[0], out[1])
 
 
 @pytest.mark.parametrize("n", [1, 16, 17, 33, 64])
