@@ -381,7 +381,8 @@ CASSPEC_API int casspec_latency_fit(const double* x, const double* y, int m, con
  * attention block runs (skip_mask as for casspec_tree_step, NULL = all on) its Wqkv and Wo, the prefix
  * K/V of P slots read and the n new K/V written; for every FFN block that runs its Wg, Wu and Wd; the
  * LM head read and the n rows of fp32 logits written.  Weights count 2 bytes in bf16 (quant_mode 0),
- * 1 byte plus 4 per output row in W8A8 (quant_mode 1).  Host only.  Returns -1 on bad arguments. */
+ * 1 byte plus 4 per output row in W8A8 (quant_mode 1), half a byte plus 4 per row in W4A4 (quant_mode
+ * 2, the 4-bit codes).  Host only.  Returns -1 on bad arguments. */
 CASSPEC_API double casspec_step_bytes(const casspec_model_config* cfg, const uint8_t* skip_mask, int quant_mode, int n,
                                       int P);
 

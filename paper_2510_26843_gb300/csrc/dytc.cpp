@@ -303,11 +303,11 @@ int casspec_dytc_tree_get(const casspec_dytc* s, int* n_out, int32_t* parent_out
 
 double casspec_step_bytes(const casspec_model_config* c, const uint8_t* skip_mask, int quant_mode, int n, int P) {
   if (c == nullptr || c->n_layers < 1 || c->d_model < 1 || c->ffn < 1 || c->vocab < 1 || n < 0 || P < 0 ||
-      quant_mode < 0 || quant_mode > 1)
+      quant_mode < 0 || quant_mode > 2)
     return -1.0;
   const double d = c->d_model, F = c->ffn, V = c->vocab;
-  const double wb = quant_mode == 1 ? 1.0 : 2.0;  // bytes per weight
-  const double sb = quant_mode == 1 ? 4.0 : 0.0;  // bytes per row scale
+  const double wb = quant_mode == 2 ? 0.5 : (quant_mode == 1 ? 1.0 : 2.0);  // bytes per weight
+  const double sb = quant_mode != 0 ? 4.0 : 0.0;                            // bytes per row scale
   double bytes = V * d * 2.0 + (double)n * V * 4.0;  // LM head read, fp32 logits written
   for (int l = 0; l < c->n_layers; ++l) {
     const uint8_t code = skip_mask ? skip_mask[l] : 1;

@@ -316,8 +316,9 @@ def test_step_bytes_match_the_bench_byte_model(cs):
     assert cs.step_bytes(cfg, no_attn, 0, 8, 2048) == head + L * 3 * d * F * 2  # no K/V either
     no_ffn = np.full(L, 1 | cs.SKIP_FFN, np.uint8)
     assert cs.step_bytes(cfg, no_ffn, 0, 8, 2048) == head + L * (4 * d * d * 2 + 2 * 2048 * d * 2 + 2 * 8 * d * 2)
+    assert cs.step_bytes(cfg, None, 2, 8, 2048) == bench.algorithmic_bytes(sh, 8, 2048, None, 2)["total"]
     with pytest.raises(cs.CasspecError):
-        cs.step_bytes(cfg, None, 2, 8, 2048)
+        cs.step_bytes(cfg, None, 3, 8, 2048)
 
 
 def test_costs_fitted_from_measured_steps(cs):
