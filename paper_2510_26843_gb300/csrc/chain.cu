@@ -40,12 +40,14 @@ constexpr int kChainThreads = 256;
 constexpr uint32_t kWStage = 32768;  // weight ring stage: whole k-blocks of the CTA's slice
 constexpr int kWStages = 4;
 constexpr uint32_t kXStage = 16384;  // one k-block of the split activation: 128 rows x 128 B
-constexpr int kXStages = 5;
+constexpr int kXStages = 4;
+constexpr int kRecvFloats = kPairMaxRows * 32;  // a pair partner's half-K partial of this CTA's 32 tokens
 constexpr int kStgFloats = 2048;     // epilogue hand-over buffer: 32 rows x 64 tokens fp32 (two of them)
 constexpr uint32_t kTmemCols = 512;  // one accumulator of up to 256 columns per MMA issuer
 
 __host__ __device__ constexpr size_t chain_smem() {
-  return 1024 + (size_t)kWStages * kWStage + (size_t)kXStages * kXStage + 2 * kStgFloats * 4 + 128 * 4 + 512;
+  return 1024 + (size_t)kWStages * kWStage + (size_t)kXStages * kXStage + 2 * kStgFloats * 4 + kRecvFloats * 4 +
+         128 * 4 + 512;
 }
 
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
@@ -86,7 +88,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint8_t* wring = smem;
   uint8_t* xring = wring + kWStages * kWStage;
   float* stg = reinterpret_cast<float*>(xring + kXStages * kXStage);  // [2][32][64]
-  float* rs = stg + 2 * kStgFloats;                                   // [64] RMSNorm factors
+  float* recv = stg + 2 * kStgFloats;                                 // [kPairMaxRows][32] from the partner
+  float* rs = recv + kRecvFloats;                                     // [64] RMSNorm factors
   float* rs2 = rs + 64;                                               // [64] second half of the sums
   uint64_t* wfull = reinterpret_cast<uint64_t*>(rs2 + 64);
   uint64_t* wempty = wfull + kWStages;
@@ -95,8 +98,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint64_t* tfull = xempty + kXStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;  // [2]: one per MMA issuer
-  uint64_t* pready = drain + 2;  // the partner CTA's half-K partial is in its staging area (S = 2)
-  uint64_t* pfree = pready + 1;  // the partner has finished reading this CTA's partial
+  uint64_t* pready = drain + 2;  // the partner CTA has written its half-K partial into `recv` (S = 2)
+  uint64_t* pfree = pready + 1;  // the partner has consumed what this CTA wrote into its `recv`
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pfree + 1);
   // [0] abort, [1] wait result, [2..5] accumulator-ready votes, [6] last CTA out
   volatile int* flags = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -403,9 +406,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
 
       // residual epilogue: this CTA's slice of the residual rows (written by this CTA's own earlier
       // phases, same slicing, or by an earlier kernel) is loaded while the MMAs run
-      float4 xo[16];
+      // Everything the epilogue reads from memory that does not depend on this phase's result is
+      // loaded while the MMAs run: the residual rows and the next norm's gains (S = 2), and the
+      // rotary coefficients of the first 16-row group (QKV).
+      float4 xo[4], gq[4], csn[4];
 #pragma unroll
-      for (int k = 0; k < 16; ++k) xo[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k = 0; k < 4; ++k) xo[k] = gq[k] = csn[k] = make_float4(0.f, 0.f, 0.f, 0.f);
       // S = 2: rank r finishes tokens 32 r .. 32 r + 31, four threads per token, R / 4 rows each
       const int t2 = 32 * s.rank + (et >> 2), cq = et & 3, wq = R / 4, c0q = cq * wq;
       if (S == 2) {
@@ -414,16 +420,28 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           for (int k = 0; k < 4; ++k)
             if (4 * k < wq) xo[k] = __ldcg(reinterpret_cast<const float4*>(ep.y + (size_t)t2 * ep.ldy + r0 + c0q) + k);
         }
-      } else if (epi == EPI_RESID && hi && t < n) {
+        if (ep.xa_out != nullptr) {
 #pragma unroll
-        for (int k = 0; k < 16; ++k)
-          if (4 * k < R) xo[k] = __ldcg(reinterpret_cast<const float4*>(ep.y + (size_t)t * ep.ldy + r0) + k);
+          for (int k = 0; k < 4; ++k)
+            if (4 * k < wq) gq[k] = __ldg(reinterpret_cast<const float4*>(ep.g_next + r0 + c0q) + k);
+        }
       }
       int pos_t = 0, P = 0;
       if (epi == EPI_QKV) {
         P = __ldcg(ep.dP);
         pos_t = t < n ? __ldcg(ep.pos + t) : 0;
       }
+      // rotary (cos, sin) of 16-row group `col` for this thread's token (zero for the v part)
+      auto rope_load = [&](int col, float4* dst) {
+        const int g = col / kRowGroup, gpp = ep.d / kRowGroup, part = g / gpp, gp = g - part * gpp;
+        const int gph = ep.hd / kRowGroup, head = gp / gph, a0 = (gp - head * gph) * 8;
+        if (part < 2) {
+          const float4* cs = reinterpret_cast<const float4*>(ep.rope + (size_t)pos_t * (ep.hd >> 1) + a0);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) dst[k] = __ldg(cs + k);
+        }
+      };
+      if (epi == EPI_QKV && hi) rope_load(r0, csn);
 
       // (2) the accumulator of this phase
       const bool got = mbar_wait_bounded(&tfull[buf], used[buf] & 1, flags);
@@ -450,7 +468,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         // pair's rows as partial(rank 0) + partial(rank 1), in that order on both.
         float* Pp = stg;
         const int nch = R / 16;  // <= kPairMaxRows / 16 = 4
-        float pv[4][16];         // both accumulators of the warp's lanes, read before the hand-over
+        float pv[4][16];         // both accumulators of the warp's lanes
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           if (c < nch) {
@@ -470,7 +488,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
               for (int i = 0; i < 16; ++i) Pp[(c * 16 + i) * 64 + t] = pv[c][i];
             }
         }
+        tc_fence_before();
         bar();
+        if (et == 0) mbar_arrive(&tempty[buf]);  // TMEM read: the next phase's MMAs may start
         if (hi) {
 #pragma unroll
           for (int c = 0; c < 4; ++c)
@@ -479,34 +499,51 @@ __global__ void __launch_bounds__(kChainThreads, 1)
               for (int i = 0; i < 16; ++i) Pp[(c * 16 + i) * 64 + t] += pv[c][i];
             }
         }
-        tc_fence_before();
-        bar();
+        // the partner's previous S = 2 phase has consumed what this CTA wrote into its `recv`
         if (et == 0) {
-          mbar_arrive(&tempty[buf]);  // TMEM read: the next phase's MMAs may start
-          mbar_arrive_remote(map_to_rank(smem_u32(pready), (uint32_t)(s.rank ^ 1)));
-          const bool okp = mbar_wait_cluster_bounded(pready, (uint32_t)(npair & 1), flags);
-          if (!okp) {
+          int okf = 1;
+          if (npair > 0 && !mbar_wait_cluster_bounded(pfree, (uint32_t)((npair - 1) & 1), flags)) {
+            okf = 0;
             flags[0] = 1;
             set_status(a.status, CASSPEC_E_TIMEOUT);
           }
-          flags[1] = okp ? 1 : 0;
+          flags[1] = okf;
         }
         bar();
-        const bool okp = flags[1] != 0;
-        if (okp) {
-          const uint32_t own = smem_u32(Pp), peer = map_to_rank(own, (uint32_t)(s.rank ^ 1));
-          const uint32_t p0 = s.rank == 0 ? own : peer, p1 = s.rank == 0 ? peer : own;
-          float v[16], v1[16];
-#pragma unroll
-          for (int c = 0; c < 16; ++c)  // every load issued before the first use
-            if (c < wq) {
-              const uint32_t off = (uint32_t)(((c0q + c) * 64 + t2) * 4);
-              v[c] = ld_dsmem_f32(p0 + off);
-              v1[c] = ld_dsmem_f32(p1 + off);
+        const int peer = s.rank ^ 1;
+        if (flags[1]) {
+          // push the partner's 32 tokens of this partial into its `recv` ([row][32], 16-byte stores)
+          const uint32_t rv = map_to_rank(smem_u32(recv), (uint32_t)peer);
+          for (int e = et; e < R * 8; e += 128) {
+            const int row = e >> 3, tq = (e & 7) * 4;
+            const float4 val = *reinterpret_cast<const float4*>(Pp + row * 64 + 32 * peer + tq);
+            st_dsmem_f4(rv + (uint32_t)((row * 32 + tq) * 4), val);
+          }
+        }
+        bar();
+        if (et == 0) {
+          int okp = flags[1];
+          if (okp) {
+            mbar_arrive_remote(map_to_rank(smem_u32(pready), (uint32_t)peer));
+            okp = mbar_wait_cluster_bounded(pready, (uint32_t)(npair & 1), flags) ? 1 : 0;
+            if (!okp) {
+              flags[0] = 1;
+              set_status(a.status, CASSPEC_E_TIMEOUT);
             }
+          }
+          flags[1] = okp;
+        }
+        bar();
+        if (flags[1]) {
+          // this CTA's 32 tokens: partial(rank 0) + partial(rank 1), the same order on both CTAs
+          const int tl = t2 - 32 * s.rank;  // token within this CTA's half
+          float v[16];
 #pragma unroll
           for (int c = 0; c < 16; ++c)
-            if (c < wq) v[c] += v1[c];
+            if (c < wq) {
+              const float own = Pp[(c0q + c) * 64 + t2], got = recv[(c0q + c) * 32 + tl];
+              v[c] = s.rank == 0 ? own + got : got + own;
+            }
           float ssq2 = 0.f;
           if (t2 < n) {
             float nv[16];
@@ -529,14 +566,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
 #pragma unroll
               for (int k = 0; k < 4; ++k) {
                 if (4 * k < wq) {
-                  const float4 g4 = __ldg(reinterpret_cast<const float4*>(ep.g_next + col) + k);
+                  const float4 g4 = gq[k];
                   const float g[4] = {nv[4 * k] * g4.x, nv[4 * k + 1] * g4.y, nv[4 * k + 2] * g4.z, nv[4 * k + 3] * g4.w};
                   uint16_t h[4];
                   float l[4];
 #pragma unroll
-                  for (int e = 0; e < 4; ++e) {
-                    h[e] = f2bf(g[e]);
-                    l[e] = g[e] - bf2f(h[e]);
+                  for (int e2 = 0; e2 < 4; ++e2) {
+                    h[e2] = f2bf(g[e2]);
+                    l[e2] = g[e2] - bf2f(h[e2]);
                   }
                   *reinterpret_cast<uint2*>(ep.xa_out + (size_t)t2 * ep.ldy + col + 4 * k) =
                       make_uint2((uint32_t)h[0] | ((uint32_t)h[1] << 16), (uint32_t)h[2] | ((uint32_t)h[3] << 16));
@@ -552,14 +589,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           if (cq == 0 && ep.ss_out != nullptr) ep.ss_out[(size_t)s.slice * 64 + t2] = t2 < n ? ssq2 : 0.f;
         }
         bar();
-        if (et == 0) {  // this CTA has read the partner's partial; wait until the partner has read ours
-          mbar_arrive_remote(map_to_rank(smem_u32(pfree), (uint32_t)(s.rank ^ 1)));
-          if (!mbar_wait_cluster_bounded(pfree, (uint32_t)(npair & 1), flags)) {
-            flags[0] = 1;
-            set_status(a.status, CASSPEC_E_TIMEOUT);
-          }
-        }
-        bar();
+        if (et == 0 && flags[1]) mbar_arrive_remote(map_to_rank(smem_u32(pfree), (uint32_t)peer));  // recv consumed
         ++npair;
       } else {
         // (3) 16 output rows (EPI_GLU: 16 channels, gate and up) at a time: the lo-plane warps hand
@@ -603,12 +633,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             if (t < n) {
               if (epi == EPI_RESID) {
                 float nv[16];
+                float4 ox[4];
+  #pragma unroll
+                for (int k = 0; k < 4; ++k) ox[k] = __ldcg(reinterpret_cast<const float4*>(ep.y + (size_t)t * ep.ldy + col) + k);
   #pragma unroll
                 for (int k = 0; k < 4; ++k) {
-                  float4 o4 = make_float4(0.f, 0.f, 0.f, 0.f);
-  #pragma unroll
-                  for (int kk = 0; kk < 16; ++kk)
-                    if (kk == 4 * c + k) o4 = xo[kk];  // register-resident old values (compile-time index)
+                  const float4 o4 = ox[k];
                   nv[4 * k + 0] = o4.x + v[4 * k + 0];
                   nv[4 * k + 1] = o4.y + v[4 * k + 1];
                   nv[4 * k + 2] = o4.z + v[4 * k + 2];
@@ -662,12 +692,15 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                 const int a0 = (gp - head * gph) * 8;
                 const int half = ep.hd >> 1;
                 float o[16];
+                float4 cur[4];
+  #pragma unroll
+                for (int k = 0; k < 4; ++k) cur[k] = csn[k];
+                if (c + 1 < nchunks) rope_load(col + 16, csn);  // the next group's, in flight meanwhile
                 if (part < 2) {
-                  const float4* cs = reinterpret_cast<const float4*>(ep.rope + (size_t)pos_t * half + a0);
                   float cv[8], sv[8];
   #pragma unroll
                   for (int k = 0; k < 4; ++k) {
-                    const float4 c4 = __ldg(cs + k);  // (cos, sin) of two frequencies
+                    const float4 c4 = cur[k];  // (cos, sin) of two frequencies
                     cv[2 * k] = c4.x;
                     sv[2 * k] = c4.y;
                     cv[2 * k + 1] = c4.z;

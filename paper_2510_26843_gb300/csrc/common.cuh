@@ -288,6 +288,10 @@ __device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
   asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr));
   return v;
 }
+__device__ __forceinline__ void st_dsmem_f4(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
 // Arrive on the mbarrier at cluster address `addr` (another CTA's, from map_to_rank), releasing this
 // thread's earlier writes (and those ordered before them) at cluster scope.
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t addr) {

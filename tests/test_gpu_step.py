@@ -453,7 +453,7 @@ def test_host_argument_errors(cs, dev_model):
     t = _i32([1] * 65)
     assert cs.tree_step(dev_model.h, kv.h, t, t, 0, None, 0, None, check=False) == cs.E_SHAPE
     assert cs.tree_step(dev_model.h, kv.h, t, t, 65, None, 0, None, check=False) == cs.E_SHAPE
-    assert cs.tree_step(dev_model.h, kv.h, t, t, 4, None, 2, None, check=False) == cs.E_INVAL
+    assert cs.tree_step(dev_model.h, kv.h, t, t, 4, None, 3, None, check=False) == cs.E_INVAL
     assert cs.tree_step(dev_model.h, kv.h, None, t, 4, None, 0, None, check=False) == cs.E_INVAL
     cs.kv_set_prefix(kv.h, 100)
     assert cs.tree_step(dev_model.h, kv.h, t, t, 64, None, 0, None, check=False) == cs.E_CAPACITY
