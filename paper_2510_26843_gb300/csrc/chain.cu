@@ -5,14 +5,16 @@
 // (+argmax) -- with one CTA per SM.
 //
 // Work split: every projection Y[token][row] = sum_k X[token][k] W[row][k] is divided among the CTAs
-// by OUTPUT ROWS only.  CTA c owns a contiguous slice of 16-row groups (row_slice) and runs the whole
-// K range for it, so no output element is shared between CTAs: there are no partial sums, no fix-up
-// round trips, and each output is reduced in one fixed order (results do not depend on timing).
+// by OUTPUT ROWS.  CTA c owns a contiguous slice of 16-row groups (row_slice) and runs the whole K
+// range for it.  The residual projections (Wo, Wdown: few rows per CTA) may instead give a slice to a
+// cluster pair of CTAs, each running one half of K (S = 2); the pair adds its two partials through
+// distributed shared memory as partial(rank 0) + partial(rank 1) on both CTAs.  Either way each output
+// is reduced in one fixed order, so results do not depend on timing.
 //
 // MMA shape: the tokens are on M.  A = the split activation of one 64-column k-block, the hi plane in
 // rows 0..63 and the lo plane in rows 64..127 (16 KB, 128-byte swizzle, TMA); B = the CTA's weight
 // rows of that k-block (N = slice rows <= 256); D in TMEM, lane = plane row, column = output row.
-// Two issuing threads split each k-block's four k-steps into two accumulators.  The epilogue adds the
+// Two issuing threads take alternate k-blocks, each into its own accumulator.  The epilogue adds the
 // accumulators, then the lo-plane lane to the hi-plane lane of each token, so 16 significant bits of
 // the activation reach the fp32 accumulation.
 //
@@ -49,6 +51,8 @@ __host__ __device__ constexpr size_t chain_smem() {
   return 1024 + (size_t)kWStages * kWStage + (size_t)kXStages * kXStage + 2 * kStgFloats * 4 + kRecvFloats * 4 +
          128 * 4 + 512;
 }
+static_assert(chain_smem() <= 232448, "the chain's shared memory exceeds the 227 KB a CTA may use");
+static_assert(kWStage % 1024 == 0 && kXStage % 1024 == 0, "ring stages keep the 1 KB alignment of the 128 B swizzle");
 
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
   unsigned v;
@@ -115,7 +119,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     }
     for (int s = 0; s < kXStages; ++s) {
       mbar_init(&xfull[s], 1);
-      mbar_init(&xempty[s], 2);
+      mbar_init(&xempty[s], 1);  // released by the issuer that consumed the k-block
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 2);
@@ -268,10 +272,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   } else if (warp == 1 || warp == 7) {
     if (lane == 0) {
       // ---------------- MMA issuers ----------------
-      // Two threads in two warps issue the MMAs of every k-block (k-steps 0, 1 and 2, 3), each into
-      // its own accumulator: one thread issues a tcgen05.mma only every ~80 cycles, so a single issuer
-      // would bound the small slices of the residual projections.  The epilogue adds the two.
+      // Two threads in two warps issue the MMAs, each into its own accumulator: the first takes the
+      // even k-blocks of a phase, the second the odd ones (a single k-block: the first alone), four
+      // k-steps per k-block.  A thread issues a tcgen05.mma only after its previous instructions, so
+      // the loop between MMAs is kept to a few integer adds: descriptors are offsets from per-ring
+      // bases, and one wait and one commit cover four MMAs.  The epilogue adds the accumulators.
       const int ib = warp == 1 ? 0 : 1;
+      const uint64_t xd0 = sw128_kmajor_desc(smem_u32(xring));
+      const uint64_t wd0 = sw128_kmajor_desc(smem_u32(wring));
       int ws = 0, xs = 0;
       uint32_t wph = 0, xph = 0;
       uint32_t used = 0;
@@ -292,6 +300,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ib * ncols);
+        uint32_t acc = 0;
         int j = 0;
         for (int j0 = 0; j0 < s.len && ok; j0 += kpb) {
           const int nk = min(kpb, s.len - j0);
@@ -299,22 +308,23 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             ok = false;
             break;
           }
+          const uint64_t wd = wd0 + (uint64_t)((uint32_t)ws * (kWStage >> 4));
           for (int jj = 0; jj < nk; ++jj, ++j) {
-            if (!mbar_wait_bounded(&xfull[xs], xph, flags)) {
-              ok = false;
-              break;
+            if ((j & 1) == ib) {
+              if (!mbar_wait_bounded(&xfull[xs], xph, flags)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint64_t ad = xd0 + (uint64_t)((uint32_t)xs * (kXStage >> 4));
+              const uint64_t bd = wd + (uint64_t)((uint32_t)jj * (chunk >> 4));
+              tc_mma_bf16(d_tmem, ad, bd, idesc, acc);  // k-step 0: 32 B further along K per step
+              tc_mma_bf16(d_tmem, ad + 2, bd + 2, idesc, 1u);
+              tc_mma_bf16(d_tmem, ad + 4, bd + 4, idesc, 1u);
+              tc_mma_bf16(d_tmem, ad + 6, bd + 6, idesc, 1u);
+              acc = 1u;
+              tc_commit(&xempty[xs]);
             }
-            tc_fence_after();
-            const uint32_t sa = smem_u32(xring + xs * kXStage);
-            const uint32_t sb = smem_u32(wring + ws * kWStage) + (uint32_t)jj * chunk;
-            // B = [hi; lo] planes stacked as M = 128 rows of the X stage; k-steps 2 ib, 2 ib + 1
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk) {
-              const uint32_t ko = (uint32_t)(2 * ib + kk) * 32u;
-              tc_mma_bf16(d_tmem, sw128_kmajor_desc(sa + ko), sw128_kmajor_desc(sb + ko), idesc,
-                          (j > 0 || kk > 0) ? 1u : 0u);
-            }
-            tc_commit(&xempty[xs]);
             if (++xs == kXStages) {
               xs = 0;
               xph ^= 1;
@@ -460,6 +470,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16);
       const uint32_t acc2 = (uint32_t)(R * mult);  // the second issuer's accumulator
+      const bool two = s.len > 1;                   // a single k-block leaves the second one unwritten
 
       if (S == 2) {
         // (3') the pair's residual projection: this CTA holds one half of K for the pair's rows.  Its
@@ -474,10 +485,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           if (c < nch) {
             float w2[16];
             tmem_ld_x16(tbase + (uint32_t)(c * 16), pv[c]);
-            tmem_ld_x16(tbase + acc2 + (uint32_t)(c * 16), w2);
+            if (two) tmem_ld_x16(tbase + acc2 + (uint32_t)(c * 16), w2);
             tmem_ld_wait();
+            if (two) {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) pv[c][i] += w2[i];
+              for (int i = 0; i < 16; ++i) pv[c][i] += w2[i];
+            }
           }
         }
         if (!hi) {
@@ -605,13 +618,15 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           // both lane groups read this chunk of both accumulators, then the lo-plane lanes hand over
           tmem_ld_x16(tbase + (uint32_t)(c * 16), v);
           if (mult == 2) tmem_ld_x16(tbase + (uint32_t)(R + c * 16), v + 16);
-          {
+          if (two) {
             float w2[32];
             tmem_ld_x16(tbase + acc2 + (uint32_t)(c * 16), w2);
             if (mult == 2) tmem_ld_x16(tbase + acc2 + (uint32_t)(R + c * 16), w2 + 16);
             tmem_ld_wait();
   #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] += w2[i];
+          } else {
+            tmem_ld_wait();
           }
           if (!hi) {
   #pragma unroll
@@ -899,7 +914,8 @@ cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int grid,
     const ChainPhase& ph = args.ph[p];
     if (ph.wp == nullptr || (reinterpret_cast<uintptr_t>(ph.wp) & 15) != 0 || ph.N % kRowGroup != 0 || ph.kb < 1)
       return cudaErrorInvalidValue;
-    if (chain_slice_rows(ph.N, grid, ph.epi == EPI_GLU) > 256) return cudaErrorInvalidValue;
+    // one k-block of the slice (rows x 128 B) fits a weight stage, and N <= 256
+    if (chain_slice_rows(ph.N, grid, ph.epi == EPI_GLU) > (int)min(256u, kWStage / 128u)) return cudaErrorInvalidValue;
     if (ph.S != 1 && (ph.S != 2 || !args.pairs || ph.epi != EPI_RESID || ph.kb < 2 ||
                       chain_slice_rows(ph.N, grid / 2, false) > kPairMaxRows))
       return cudaErrorInvalidValue;
