@@ -44,7 +44,7 @@ struct Layout {
   std::vector<size_t> qkv_q4, wo_q4, wg_q4, wu_q4, wd_q4, qkv_s4, wo_s4, wg_s4, wu_s4, wd_s4;
   std::vector<size_t> qkv_f8, wo_f8, wg_f8, wu_f8, wd_f8;
   size_t x, q, o, u, xa, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
-  size_t gemm_part, gemm_cnt, chain_ready, chain_done, i8_part, i8_cnt, attn_part, attn_ml, attn_cnt, status;
+  size_t gemm_part, gemm_cnt, chain_ready, chain_done, i8_part, i8_cnt, status;
   size_t scratch_begin;
   int max_tiles, lm_tiles;
 };
@@ -155,9 +155,6 @@ Layout make_layout(const casspec_model_config& c) {
     L.i8_part = take(slots * 64 * 128 * 4);
   }
   L.i8_cnt = take((size_t)L.max_tiles * 4);
-  L.attn_part = take((size_t)kAttnMaxSplits * c.n_heads * T * c.head_dim * 4);
-  L.attn_ml = take((size_t)kAttnMaxSplits * c.n_heads * T * 8);
-  L.attn_cnt = take((size_t)2 * c.n_heads * 4);
   L.status = take(256);
   L.total = align_up(off, 256);
   return L;
@@ -217,9 +214,6 @@ struct casspec_model {
   unsigned* gemm_cnt;
   int* i8_part;
   unsigned* i8_cnt;
-  float* attn_part;
-  float2* attn_ml;
-  unsigned* attn_cnt;
   int* status;
   std::map<GraphKey, std::pair<cudaGraphExec_t, int>> graphs;  // exec + kernels it contains
   std::mutex mu;
@@ -498,9 +492,6 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     at.n_heads = H;
     at.layer = l;
     at.splits = attn_splits(H, m->num_sms);
-    at.part_o = m->attn_part;
-    at.part_ml = m->attn_ml;
-    at.cnt = m->attn_cnt;
     at.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
     at.status = m->status;
     LAUNCH(CASSPEC_K_ATTN, launch_tree_attention(kv->tm_kv, at, hd, s, pdl));
@@ -836,9 +827,6 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   m->gemm_cnt = reinterpret_cast<unsigned*>(b + L.gemm_cnt);
   m->i8_part = reinterpret_cast<int*>(b + L.i8_part);
   m->i8_cnt = reinterpret_cast<unsigned*>(b + L.i8_cnt);
-  m->attn_part = reinterpret_cast<float*>(b + L.attn_part);
-  m->attn_ml = reinterpret_cast<float2*>(b + L.attn_ml);
-  m->attn_cnt = reinterpret_cast<unsigned*>(b + L.attn_cnt);
   m->status = reinterpret_cast<int*>(b + L.status);
 
   if (cudaMemset(b + L.scratch_begin, 0, L.total - L.scratch_begin) != cudaSuccess ||
@@ -1201,7 +1189,6 @@ int casspec_get_status(casspec_model* m, int* status_out) {
     CK(cudaMemset(m->i8_cnt, 0, (size_t)m->lay.max_tiles * 4));
     CK(cudaMemset(m->chain_ready, 0, (size_t)kMaxPhases * kReadyPerPhase * 4));
     CK(cudaMemset(m->chain_done, 0, 256));
-    CK(cudaMemset(m->attn_cnt, 0, (size_t)2 * m->cfg.n_heads * 4));
   }
   if (status_out) *status_out = st;
   return CASSPEC_OK;

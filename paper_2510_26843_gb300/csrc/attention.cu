@@ -1,125 +1,157 @@
-// Tree attention (Sec. 4.2: parallel verification / drafting of a token tree).
+// Tree attention (Sec. 4.2: parallel verification / drafting of a token tree) on the 5th-generation
+// tensor cores.
 //
 // Node i of the tree attends to every committed prefix slot [0, P) and to the tree slots of its
 // ancestors and itself (bit j of anc[i] <=> tree slot j, cache slot P + j).
-//   * S CTAs per head (split-KV, S * heads <= 2 per SM, so the whole grid is resident at once);
-//     split s handles the s-th contiguous share of the head's 64-slot KV blocks;
-//   * K/V blocks arrive by TMA (2-D tensor map over the whole cache, 128-byte swizzle, 64 slots x 64
-//     dims per box) in an S-stage mbarrier ring fed by a dedicated producer warp;
-//   * four compute warps, 16 query rows each, run QK^T and PV on tensor cores (mma.sync m16n8k16
-//     bf16 -> fp32) with ldmatrix addresses XOR-swizzled to match the TMA layout, the ancestor mask
-//     applied to the scores, and an online softmax whose row reductions are quad shuffles;
-//   * each split writes its partial (running max, sum, unnormalised output) to global scratch and
-//     counts itself in; once all S splits of the head have arrived, split s merges rows
-//     s, s + S, ... over the S partials in split order (fixed, so results do not depend on timing)
-//     and the last split out returns the head's counters to zero.
+//   * C CTAs per head (split-KV) form one thread-block cluster; heads * C <= 2 per SM, so the whole
+//     grid is resident at once.  Split s handles the s-th contiguous share of the head's 64-slot KV
+//     blocks;
+//   * K and V blocks arrive by TMA (2-D tensor map over the whole cache, 128-byte swizzle, 64 slots x
+//     64 dims per box) in two mbarrier rings (K: 3 stages, released once the block's scores are
+//     computed; V: 2 stages, released after P V), each fed by one producer thread, which loads the
+//     blocks that lie wholly in the committed prefix before waiting on the preceding kernel;
+//   * one thread issues tcgen05.mma: S = Q K^T per block (M = 64 query rows, N = 64 slots, both
+//     operands K-major) into one of two TMEM score buffers, and O += P V (N = head dim, V read
+//     MN-major straight from its cache layout) into a TMEM accumulator.  S of block i is issued
+//     before P V of block i - 1, so the scores of the next block are computed while the softmax
+//     warps work on the current one;
+//   * four softmax warps read S from TMEM (M = 64 puts query rows 16 q .. 16 q + 15 in lanes 0..15 of
+//     lane quarter q; the 16x256b load shape spreads each 16-row group over all 32 threads, two rows
+//     per quad), apply the ancestor mask, keep the online softmax state in registers against a
+//     reference max that moves only when a score exceeds it by 2^8 (then the O rows are rescaled in
+//     TMEM), and write P as bf16 into one of two 128-byte-swizzled tiles, the A operand of P V;
+//   * each split leaves its partial (running max, sum, unnormalised output) in its own shared memory;
+//     after a cluster barrier, split s merges rows s, s + C, ... over the C partials, read through
+//     distributed shared memory in split order (fixed, so results do not depend on timing).
 #include "common.cuh"
 #include "kernels.h"
 
 namespace casspec {
 
-constexpr int kAttnCompute = 128;                // 4 compute warps
-constexpr int kAttnThreads = kAttnCompute + 32;  // + producer warp
+constexpr int kAttnThreads = 192;  // warp 0 producers (lane 0: K, lane 1: V), warp 1 MMA, warps 2..5 softmax
 constexpr int kAttnBlk = 64;
-constexpr int kAttnStages = 3;
+constexpr int kAttnKStages = 3;
+constexpr int kAttnVStages = 2;
+constexpr uint32_t kAttnTmemCols = 256;  // two 64-column score buffers + the output (<= 128 columns)
+constexpr uint32_t kAttnO = 128;         // TMEM column of the output accumulator
+constexpr float kRescaleLog2 = 8.f;      // the reference max moves when a score exceeds it by 2^8
 
 template <int HD>
-__host__ __device__ constexpr uint32_t attn_tile_bytes() {
+__host__ __device__ constexpr uint32_t attn_tile_bytes() {  // a [64][HD] bf16 tile
   return (uint32_t)kAttnBlk * HD * 2;
 }
 template <int HD>
 __host__ __device__ constexpr size_t attn_smem_bytes() {
-  return (size_t)kAttnStages * 2 * attn_tile_bytes<HD>() + (size_t)64 * HD * 2 + 128;
+  // Q, the K and V rings, two P tiles, barriers (two CTAs per SM: <= 113 KB each)
+  return attn_tile_bytes<HD>() * (1 + kAttnKStages + kAttnVStages) + 2 * 8192 + 256;
 }
 
-// Address of 16-byte chunk `c` (0 .. HD/8-1) of row `r` in a [64][HD] bf16 tile stored as HD/64
+// Byte offset of 16-byte chunk `c` (0 .. HD/8-1) of row `r` in a [64][HD] bf16 tile stored as HD/64
 // sub-tiles of [64][128 B] with the 128-byte swizzle (TMA's layout; tile base 1024-byte aligned).
-__device__ __forceinline__ uint32_t swz(uint32_t tile, int r, int c) {
-  return tile + (uint32_t)(c >> 3) * 8192u + (uint32_t)r * 128u + ((uint32_t)((c & 7) ^ (r & 7)) << 4);
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+  return (uint32_t)(c >> 3) * 8192u + (uint32_t)r * 128u + ((uint32_t)((c & 7) ^ (r & 7)) << 4);
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {  // 2^x, ~2 ulp; 2^-inf = 0
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 template <int HD>
 __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid_constant__ CUtensorMap tmKV,
                                                                      const AttnArgs a) {
   constexpr uint32_t TILE = attn_tile_bytes<HD>();
-  constexpr uint32_t STAGE = 2 * TILE;
-  constexpr int S = kAttnStages;
+  constexpr int NK = kAttnKStages, NV = kAttnVStages;
   constexpr int NCH = HD / 8;  // 16-byte chunks per row
-  static_assert(64 * kAttnMaxSplits * 12 + 64 * 4 <= S * STAGE, "merge weights must fit in the K/V ring");
+  // the partial (O rows fp32 + (max, sum)) reuses the drained K/V rings
+  static_assert(64 * HD * 4 + 64 * 8 <= (NK + NV) * TILE, "the partial must fit in the K/V rings");
+  // The kernel has no static shared memory, so the dynamic block starts the CTA's shared window; the
+  // swizzled tiles need it 1 KB aligned (checked: results are flagged invalid otherwise).
   extern __shared__ __align__(1024) uint8_t sm[];
-  uint8_t* ring = sm;
-  uint8_t* qs = sm + S * STAGE;
-  uint64_t* full = reinterpret_cast<uint64_t*>(qs + 64 * HD * 2);
-  uint64_t* empty = full + S;
-  volatile int* flags = reinterpret_cast<volatile int*>(empty + S);  // [0] abort, [1] merge go-ahead
+  uint8_t* qs = sm;                // Q: [64][HD]
+  uint8_t* kring = qs + TILE;      // NK x K
+  uint8_t* vring = kring + NK * TILE;  // NV x V
+  uint8_t* ps = vring + NV * TILE;     // two P tiles [64][64]
+  uint64_t* k_full = reinterpret_cast<uint64_t*>(ps + 2 * 8192);
+  uint64_t* k_empty = k_full + NK;
+  uint64_t* v_full = k_empty + NK;
+  uint64_t* v_empty = v_full + NV;
+  uint64_t* s_full = v_empty + NV;  // [2]
+  uint64_t* s_free = s_full + 2;    // [2]
+  uint64_t* p_full = s_free + 2;    // [2]
+  uint64_t* pv_done = p_full + 2;   // [2]: P V of block j completes phase j / 2 of pv_done[j % 2]
+  uint64_t* q_full = pv_done + 2;
+  uint64_t* drain = q_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* flags = reinterpret_cast<volatile int*>(tmem_slot + 1);  // [0] abort
+  float* part_o = reinterpret_cast<float*>(kring);                        // [64][HD] after the blocks
+  float2* part_ml = reinterpret_cast<float2*>(kring + 64 * HD * 4);       // [64]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int C = a.splits;
   const int head = blockIdx.x / C;
-  const int rank = blockIdx.x % C;
+  const int rank = (int)cluster_ctarank();  // == blockIdx.x % C: the head's splits are one cluster
   if (tid == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 4);
+    for (int s = 0; s < NK; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
     }
+    for (int s = 0; s < NV; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], 4);  // one arrival per softmax warp
+    }
+    mbar_init(&p_full[0], 4);
+    mbar_init(&p_full[1], 4);
+    mbar_init(&pv_done[0], 1);
+    mbar_init(&pv_done[1], 1);
+    mbar_init(q_full, 4);
+    mbar_init(drain, 1);
     flags[0] = 0;
-    flags[1] = 0;
+    if ((smem_u32(sm) & 1023u) != 0) set_status(a.status, CASSPEC_E_CUDA);
     fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kAttnTmemCols);
+    tmem_relinquish();
   }
   // The committed length P is written only between steps (compaction, set_prefix), by kernels that
   // completed before this step's first kernel started, so it can be read before the dependency wait.
-  // The blocks of this split that lie wholly inside the committed prefix do not depend on the
-  // preceding kernels either: the producer loads the first of them into the ring before the wait,
-  // and asks L2 for the rest, while the previous kernel finishes.
   const int Pp = *reinterpret_cast<const volatile int*>(a.dP);
-  const bool aligned = (smem_u32(sm) & 1023u) == 0;  // the swizzle addressing needs 1024-byte tiles
-  if (tid == kAttnCompute) {
-    tma_prefetch_desc(&tmKV);
-    if (Pp >= 0 && Pp <= a.ctx) {
-      const int nb = min((Pp + a.T + a.n + kAttnBlk - 1) / kAttnBlk, a.ctx / kAttnBlk);
-      const int row_k = ((a.layer * 2 + 0) * a.n_heads + head) * a.ctx;
-      const int row_v = ((a.layer * 2 + 1) * a.n_heads + head) * a.ctx;
-      for (int b = rank * nb / C + S; b < (rank + 1) * nb / C; ++b) {
-#pragma unroll
-        for (int sub = 0; sub < HD / 64; ++sub) {
-          tma_prefetch_l2_2d(&tmKV, sub * 64, row_k + b * kAttnBlk);
-          tma_prefetch_l2_2d(&tmKV, sub * 64, row_v + b * kAttnBlk);
-        }
-      }
-    }
-  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
   pdl_trigger();
-  if (warp != 4) pdl_wait();  // the producer waits after its prefix loads
+  if (warp != 0) pdl_wait();  // the producers wait after their prefix loads
 
-  const int P = warp == 4 ? Pp : __ldcg(a.dP);
+  const int P = warp == 0 ? Pp : __ldcg(a.dP);
   const int total = P + a.T + a.n;
   const int nblk = (total + kAttnBlk - 1) / kAttnBlk;
   const int b0 = rank * nblk / C, b1 = (rank + 1) * nblk / C;
-  if (!aligned && tid == 0) set_status(a.status, CASSPEC_E_CUDA);
+  const int nb = b1 - b0;
 
-  float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
-  float oacc[HD / 8][4];
-#pragma unroll
-  for (int dt = 0; dt < HD / 8; ++dt) oacc[dt][0] = oacc[dt][1] = oacc[dt][2] = oacc[dt][3] = 0.f;
-  const int row0 = warp * 16;
-  const bool active = warp < 4 && row0 < a.n;
-  const int g = lane >> 2, t4 = lane & 3;
-  const int rA = row0 + g, rB = rA + 8;
-  auto cbar = [] { named_bar_sync(1, kAttnCompute); };
-
-  if (warp == 4) {
-    // ---------------- producer ----------------
-    if (lane == 0 && aligned) {
+  if (warp == 0) {
+    // ---------------- producers: lane 0 loads K blocks, lane 1 V blocks ----------------
+    if (lane < 2) {
+      if (lane == 0) tma_prefetch_desc(&tmKV);
+      const bool isk = lane == 0;
+      const int ns = isk ? NK : NV;
+      uint8_t* ring = isk ? kring : vring;
+      uint64_t* full = isk ? k_full : v_full;
+      uint64_t* empty = isk ? k_empty : v_empty;
       const uint64_t pol = policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
       uint32_t armed = 0, armed_parity = 0;
-      const int row_k = ((a.layer * 2 + 0) * a.n_heads + head) * a.ctx;
-      const int row_v = ((a.layer * 2 + 1) * a.n_heads + head) * a.ctx;
+      const int row0 = ((a.layer * 2 + (isk ? 0 : 1)) * a.n_heads + head) * a.ctx;
       bool waited = false;
       for (int b = b0; b < b1; ++b) {
-        if (!waited && (b - b0 >= S || (b + 1) * kAttnBlk > P || P < 0 || P > a.ctx)) {
+        if (!waited && (b - b0 >= ns || (b + 1) * kAttnBlk > P || P < 0 || P > a.ctx)) {
           pdl_wait();  // from here on the blocks may hold this step's tree K/V
           waited = true;
           if (__ldcg(a.dP) != P) set_status(a.status, CASSPEC_E_STATE);  // P moved during a step
@@ -129,272 +161,321 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
           set_status(a.status, CASSPEC_E_TIMEOUT);
           break;
         }
-        mbar_expect_tx(&full[stage], STAGE);
+        mbar_expect_tx(&full[stage], TILE);
         armed |= 1u << stage;
         armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
-        uint8_t* st = ring + stage * STAGE;
+        uint8_t* st = ring + stage * TILE;
 #pragma unroll
-        for (int sub = 0; sub < HD / 64; ++sub) {
-          tma_load_2d(st + sub * 8192, &tmKV, &full[stage], sub * 64, row_k + b * kAttnBlk, pol);
-          tma_load_2d(st + TILE + sub * 8192, &tmKV, &full[stage], sub * 64, row_v + b * kAttnBlk, pol);
-        }
-        if (++stage == S) {
+        for (int sub = 0; sub < HD / 64; ++sub)
+          tma_load_2d(st + sub * 8192, &tmKV, &full[stage], sub * 64, row0 + b * kAttnBlk, pol);
+        if (++stage == ns) {
           stage = 0;
           phase ^= 1;
         }
       }
       if (!waited) pdl_wait();
-      if (flags[0]) {  // abort: let the copies already issued land before the ring is reused
-        for (int s = 0; s < S; ++s)
+      if (flags[0]) {  // abort: let the copies already issued land before the shared memory is reused
+        for (int s = 0; s < ns; ++s)
           if (armed & (1u << s)) mbar_wait_bounded(&full[s], (armed_parity >> s) & 1, nullptr);
       }
     }
     __syncwarp();
-  } else if (aligned) {
-    // ---------------- compute warps ----------------
-    const uint32_t qbase = smem_u32(qs);
-    const unsigned long long ancA = rA < a.n ? __ldcg(a.anc + rA) : 0ull;
-    const unsigned long long ancB = rB < a.n ? __ldcg(a.anc + rB) : 0ull;
-    constexpr int QPT = 64 * NCH / kAttnCompute;  // 16-byte chunks of Q per thread
-    uint4 qv[QPT];  // every load in flight before the first shared-memory store
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16_f32(64, 64);
+      const uint32_t id_o = idesc_bf16_f32(64, HD) | kIdescBMnMajor;
+      const uint64_t qd = sw128_kmajor_desc(smem_u32(qs));
+      bool ok = nb == 0 || mbar_wait_bounded(q_full, 0, flags);
+      // P V of block j: A = P tile j & 1, 4 k-steps of 16 slots; B = V of its stage, MN-major
+      // (64-dim groups 8 KB apart, 8-slot groups 1 KB apart, 2 KB per k-step)
+      auto issue_pv = [&](int j) -> bool {
+        const int vs = j % NV;
+        const uint64_t pd = sw128_kmajor_desc(smem_u32(ps + (j & 1) * 8192));
+        if (!mbar_wait_bounded(&p_full[j & 1], (uint32_t)(j >> 1) & 1, flags)) return false;
+        if (!mbar_wait_bounded(&v_full[vs], (uint32_t)(j / NV) & 1, flags)) return false;
+        tc_fence_after();
+        const uint32_t vb = smem_u32(vring + vs * TILE);
 #pragma unroll
-    for (int k = 0; k < QPT; ++k) {
-      const int idx = tid + k * kAttnCompute, row = idx / NCH, c = idx % NCH;
-      qv[k] = row < a.n ? __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)row * a.d + head * HD + c * 8))
-                        : make_uint4(0, 0, 0, 0);
-    }
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_bf16(tmem + kAttnO, pd + (uint64_t)(2 * kk), sw128_mnmajor_desc(vb + 2048u * kk, 8192u, 1024u), id_o,
+                      (j > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&v_empty[vs]);
+        tc_commit(&pv_done[j & 1]);
+        return true;
+      };
+      if (ok) {
+        tc_fence_after();
+        for (int i = 0; i < nb && ok; ++i) {
+          const int sb = i & 1, ks = i % NK;
+          if (i >= 2 && !mbar_wait_bounded(&s_free[sb], (uint32_t)((i - 2) >> 1) & 1, flags)) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait_bounded(&k_full[ks], (uint32_t)(i / NK) & 1, flags)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t kd = sw128_kmajor_desc(smem_u32(kring + ks * TILE));
 #pragma unroll
-    for (int k = 0; k < QPT; ++k) {
-      const int idx = tid + k * kAttnCompute, row = idx / NCH, c = idx % NCH;
-      asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(swz(qbase, row, c)), "r"(qv[k].x), "r"(qv[k].y),
-                   "r"(qv[k].z), "r"(qv[k].w)
-                   : "memory");
-    }
-    cbar();
-    uint32_t qf[HD / 16][4];
-    if (active) {
-#pragma unroll
-      for (int kt = 0; kt < HD / 16; ++kt) {
-        const int mi = lane >> 3;
-        ldmatrix_x4_a(qf[kt][0], qf[kt][1], qf[kt][2], qf[kt][3],
-                      swz(qbase, row0 + (lane & 7) + 8 * (mi & 1), 2 * kt + (mi >> 1)));
+          for (int kk = 0; kk < HD / 16; ++kk) {
+            const uint64_t off = (uint64_t)((kk >> 2) * 512 + (kk & 3) * 2);  // 8 KB per 64 dims, 32 B per step
+            tc_mma_bf16(tmem + (uint32_t)(sb * 64), qd + off, kd + off, id_s, kk > 0 ? 1u : 0u);
+          }
+          tc_commit(&s_full[sb]);
+          tc_commit(&k_empty[ks]);  // the K block is consumed once its scores are complete
+          if (i >= 1 && !issue_pv(i - 1)) ok = false;
+        }
+        if (ok && nb > 0 && !issue_pv(nb - 1)) ok = false;
       }
-    }
-    int stage = 0;
-    uint32_t phase = 0;
-    for (int b = b0; b < b1; ++b) {
-      if (!mbar_wait_bounded(&full[stage], phase, flags)) {
+      if (!ok) {
         flags[0] = 1;
         set_status(a.status, CASSPEC_E_TIMEOUT);
+      }
+      tc_commit(drain);  // every MMA complete before TMEM is released
+      mbar_wait_bounded(drain, 0, nullptr);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- softmax warps 2..5 ----------------
+    // TMEM lane quarter qq holds query rows 16 qq .. 16 qq + 15 (M = 64).  Read with the 16x256b
+    // shape, thread t of the warp holds rows rA = 16 qq + t/4 and rB = rA + 8 at columns
+    // 8 j + 2 (t % 4) + {0, 1}: the four threads of a quad share a row pair, so row reductions are two
+    // quad shuffles.
+    const int qq = warp & 3;
+    const int g = lane >> 2, t4 = lane & 3;
+    const int rA = 16 * qq + g, rB = rA + 8;
+    const uint32_t tl = tmem + ((uint32_t)(qq * 32) << 16);
+    // Q of this head: rows >= n are zero
+    {
+      const int et = tid - 64;  // 0..127
+      constexpr int QPT = 64 * NCH / 128;
+      uint4 qv[QPT];
+#pragma unroll
+      for (int k = 0; k < QPT; ++k) {
+        const int idx = et + k * 128, r = idx / NCH, c = idx % NCH;
+        qv[k] = r < a.n ? __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)r * a.d + head * HD + c * 8))
+                        : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int k = 0; k < QPT; ++k) {
+        const int idx = et + k * 128, r = idx / NCH, c = idx % NCH;
+        *reinterpret_cast<uint4*>(qs + swz(r, c)) = qv[k];
+      }
+      fence_proxy_async_smem();  // generic-proxy writes -> the tensor cores' operand reads
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_full);
+    }
+    const unsigned long long ancA = rA < a.n ? __ldcg(a.anc + rA) : 0ull;
+    const unsigned long long ancB = rB < a.n ? __ldcg(a.anc + rB) : 0ull;
+    float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;  // lA, lB: this thread's columns only
+    bool ok = true;
+    for (int i = 0; i < nb; ++i) {
+      const int sb = i & 1;
+      if (!mbar_wait_bounded(&s_full[sb], (uint32_t)(i >> 1) & 1, flags)) {
+        ok = false;
         break;
       }
-      if (active) {
-        const uint32_t kb = smem_u32(ring + stage * STAGE), vb = kb + TILE;
-        float s[8][4];
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-#pragma unroll
-        for (int kt = 0; kt < HD / 16; ++kt) {
-#pragma unroll
-          for (int np = 0; np < 4; ++np) {
-            const int mi = lane >> 3;
-            uint32_t k0, k1, k2, k3;
-            ldmatrix_x4_a(k0, k1, k2, k3, swz(kb, 16 * np + 8 * (mi >> 1) + (lane & 7), 2 * kt + (mi & 1)));
-            mma_bf16_16816(s[2 * np], qf[kt][0], qf[kt][1], qf[kt][2], qf[kt][3], k0, k1);
-            mma_bf16_16816(s[2 * np + 1], qf[kt][0], qf[kt][1], qf[kt][2], qf[kt][3], k2, k3);
-          }
-        }
-        const int sbase = b * kAttnBlk;
-        float mxA = -INFINITY, mxB = -INFINITY;
-        if (sbase + kAttnBlk <= P) {  // a block of the committed prefix: visible to every node
-#pragma unroll
-          for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              s[nt][e] *= a.scale_log2;
-              s[nt][2 + e] *= a.scale_log2;
-              mxA = fmaxf(mxA, s[nt][e]);
-              mxB = fmaxf(mxB, s[nt][2 + e]);
-            }
-          }
-        } else {
-#pragma unroll
-          for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int slot = sbase + nt * 8 + 2 * t4 + e;
-              bool visA, visB;
-              if (slot < P) {
-                visA = visB = true;
-              } else if (slot < total) {
-                const int j = slot - P;
-                visA = (ancA >> j) & 1ull;
-                visB = (ancB >> j) & 1ull;
-              } else {
-                visA = visB = false;
-              }
-              s[nt][e] = visA ? s[nt][e] * a.scale_log2 : -INFINITY;
-              s[nt][2 + e] = visB ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
-              mxA = fmaxf(mxA, s[nt][e]);
-              mxB = fmaxf(mxB, s[nt][2 + e]);
-            }
-          }
-        }
-        mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 1));
-        mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 2));
-        mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 1));
-        mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 2));
-        const float nA = fmaxf(mA, mxA), nB = fmaxf(mB, mxB);
-        const float uA = (nA == -INFINITY) ? 0.f : nA, uB = (nB == -INFINITY) ? 0.f : nB;
-        const float cA = exp2f(mA - uA), cB = exp2f(mB - uB);
-        mA = nA;
-        mB = nB;
-        float sumA = 0.f, sumB = 0.f;
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-          s[nt][0] = exp2f(s[nt][0] - uA);
-          s[nt][1] = exp2f(s[nt][1] - uA);
-          s[nt][2] = exp2f(s[nt][2] - uB);
-          s[nt][3] = exp2f(s[nt][3] - uB);
-          sumA += s[nt][0] + s[nt][1];
-          sumB += s[nt][2] + s[nt][3];
-        }
-        lA = lA * cA + sumA;
-        lB = lB * cB + sumB;
-#pragma unroll
-        for (int dt = 0; dt < HD / 8; ++dt) {
-          oacc[dt][0] *= cA;
-          oacc[dt][1] *= cA;
-          oacc[dt][2] *= cB;
-          oacc[dt][3] *= cB;
-        }
-#pragma unroll
-        for (int kc = 0; kc < 4; ++kc) {
-          const uint32_t a0 = pack_bf16x2(s[2 * kc][0], s[2 * kc][1]);
-          const uint32_t a1 = pack_bf16x2(s[2 * kc][2], s[2 * kc][3]);
-          const uint32_t a2 = pack_bf16x2(s[2 * kc + 1][0], s[2 * kc + 1][1]);
-          const uint32_t a3 = pack_bf16x2(s[2 * kc + 1][2], s[2 * kc + 1][3]);
-#pragma unroll
-          for (int dp = 0; dp < HD / 16; ++dp) {
-            const int mi = lane >> 3;
-            uint32_t v0, v1, v2, v3;
-            ldmatrix_x4_trans_a(v0, v1, v2, v3, swz(vb, 16 * kc + (lane & 7) + 8 * (mi & 1), 2 * dp + (mi >> 1)));
-            mma_bf16_16816(oacc[2 * dp], a0, a1, a2, a3, v0, v1);
-            mma_bf16_16816(oacc[2 * dp + 1], a0, a1, a2, a3, v2, v3);
-          }
-        }
-      }
+      tc_fence_after();
+      float s[32];
+      tmem_ld_16x256b_x8(tl + (uint32_t)(sb * 64), s);
+      tmem_ld_wait();
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[stage]);
-      if (++stage == S) {
-        stage = 0;
-        phase ^= 1;
+      if (lane == 0) mbar_arrive(&s_free[sb]);  // the score buffer may take block i + 2
+      const int sbase = (b0 + i) * kAttnBlk;
+      float mxA = -INFINITY, mxB = -INFINITY;
+      if (sbase + kAttnBlk <= P) {  // a block of the committed prefix: visible to every node
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            s[4 * j + e] *= a.scale_log2;
+            s[4 * j + 2 + e] *= a.scale_log2;
+            mxA = fmaxf(mxA, s[4 * j + e]);
+            mxB = fmaxf(mxB, s[4 * j + 2 + e]);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int slot = sbase + 8 * j + 2 * t4 + e;
+            bool visA, visB;
+            if (slot < P) {
+              visA = visB = true;
+            } else if (slot < total) {
+              visA = (ancA >> (slot - P)) & 1ull;
+              visB = (ancB >> (slot - P)) & 1ull;
+            } else {
+              visA = visB = false;
+            }
+            s[4 * j + e] = visA ? s[4 * j + e] * a.scale_log2 : -INFINITY;
+            s[4 * j + 2 + e] = visB ? s[4 * j + 2 + e] * a.scale_log2 : -INFINITY;
+            mxA = fmaxf(mxA, s[4 * j + e]);
+            mxB = fmaxf(mxB, s[4 * j + 2 + e]);
+          }
+        }
       }
+      mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 1));
+      mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 2));
+      mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 1));
+      mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 2));
+      // Reference max per row: P = 2^(s - m) with m raised only when a score exceeds it by more than
+      // kRescaleLog2 (P <= 2^kRescaleLog2 otherwise).  Moving m rescales l and the O row by
+      // 2^(m_old - m_new), which needs the previous block's P V complete; most blocks skip that.
+      const bool upA = mxA > mA + kRescaleLog2, upB = mxB > mB + kRescaleLog2;
+      const float nA = upA ? mxA : mA, nB = upB ? mxB : mB;
+      const float uA = nA == -INFINITY ? 0.f : nA, uB = nB == -INFINITY ? 0.f : nB;
+      const float cA = upA ? fast_exp2(mA - uA) : 1.f, cB = upB ? fast_exp2(mB - uB) : 1.f;  // 0 from -inf
+      mA = nA;
+      mB = nB;
+      float sumA = 0.f, sumB = 0.f;
+      uint32_t pk[16];  // [2 j]: row A, [2 j + 1]: row B
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float a0 = fast_exp2(s[4 * j] - uA), a1 = fast_exp2(s[4 * j + 1] - uA);
+        const float b0v = fast_exp2(s[4 * j + 2] - uB), b1v = fast_exp2(s[4 * j + 3] - uB);
+        sumA += a0 + a1;
+        sumB += b0v + b1v;
+        pk[2 * j] = pack_bf16x2(a0, a1);
+        pk[2 * j + 1] = pack_bf16x2(b0v, b1v);
+      }
+      lA = lA * cA + sumA;
+      lB = lB * cB + sumB;
+      // The O rows of this warp move with m: P V of block i - 1 must have completed.  P tile i & 1
+      // was last read by P V of block i - 2.
+      const bool resc = i >= 1 && __any_sync(0xffffffffu, upA || upB);
+      if (resc || i >= 2) {
+        // (waits stay within one phase of each barrier: P V of block i + 1 or later needs this
+        // warp's P of block i first)
+        const int w = resc ? i - 1 : i - 2;
+        if (!mbar_wait_bounded(&pv_done[w & 1], (uint32_t)(w >> 1) & 1, flags)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+      }
+      if (resc) {
+#pragma unroll
+        for (int h = 0; h < HD / 64; ++h) {
+          float o[32];
+          tmem_ld_16x256b_x8(tl + kAttnO + (uint32_t)(64 * h), o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            o[4 * j] *= cA;
+            o[4 * j + 1] *= cA;
+            o[4 * j + 2] *= cB;
+            o[4 * j + 3] *= cB;
+          }
+          tmem_st_16x256b_x8(tl + kAttnO + (uint32_t)(64 * h), o);
+        }
+        tmem_st_wait();
+      }
+      {
+        uint8_t* pt = ps + sb * 8192;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          *reinterpret_cast<uint32_t*>(pt + (uint32_t)rA * 128u + ((uint32_t)(j ^ (rA & 7)) << 4) + 4u * t4) = pk[2 * j];
+          *reinterpret_cast<uint32_t*>(pt + (uint32_t)rB * 128u + ((uint32_t)(j ^ (rB & 7)) << 4) + 4u * t4) = pk[2 * j + 1];
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[sb]);
     }
-  }
-
-  // ---- this split's partial to global scratch, then count in ----
-  const int n = a.n;
-  const size_t pslot = (size_t)head * C + rank;
-  if (warp < 4) {
+    // this split's partial into its own shared memory (the rings are drained once the last P V
+    // completed): unnormalised O rows, (max, sum)
+    if (ok && nb > 0 && !mbar_wait_bounded(&pv_done[(nb - 1) & 1], (uint32_t)((nb - 1) >> 1) & 1, flags)) ok = false;
+    if (!ok) {
+      flags[0] = 1;
+      set_status(a.status, CASSPEC_E_TIMEOUT);
+    }
     lA += __shfl_xor_sync(0xffffffffu, lA, 1);
     lA += __shfl_xor_sync(0xffffffffu, lA, 2);
     lB += __shfl_xor_sync(0xffffffffu, lB, 1);
     lB += __shfl_xor_sync(0xffffffffu, lB, 2);
-    float* po = a.part_o + pslot * 64 * HD;
+    if (ok) tc_fence_after();
 #pragma unroll
-    for (int dt = 0; dt < HD / 8; ++dt) {
-      const int col = dt * 8 + 2 * t4;
-      if (rA < n) __stcg(reinterpret_cast<float2*>(po + rA * HD + col), make_float2(oacc[dt][0], oacc[dt][1]));
-      if (rB < n) __stcg(reinterpret_cast<float2*>(po + rB * HD + col), make_float2(oacc[dt][2], oacc[dt][3]));
+    for (int h = 0; h < HD / 64; ++h) {
+      float o[32];
+      if (ok && nb > 0) {
+        tmem_ld_16x256b_x8(tl + kAttnO + (uint32_t)(64 * h), o);
+        tmem_ld_wait();
+      } else {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) o[e] = 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int col = 64 * h + 8 * j + 2 * t4;
+        *reinterpret_cast<float2*>(part_o + rA * HD + col) = make_float2(o[4 * j], o[4 * j + 1]);
+        *reinterpret_cast<float2*>(part_o + rB * HD + col) = make_float2(o[4 * j + 2], o[4 * j + 3]);
+      }
     }
     if (t4 == 0) {
-      if (rA < n) __stcg(a.part_ml + pslot * 64 + rA, make_float2(mA, lA));
-      if (rB < n) __stcg(a.part_ml + pslot * 64 + rB, make_float2(mB, lB));
+      part_ml[rA] = make_float2(ok && nb > 0 ? mA : -INFINITY, lA);
+      part_ml[rB] = make_float2(ok && nb > 0 ? mB : -INFINITY, lB);
     }
   }
+  tc_fence_before();
   __syncthreads();
-  if (tid == 0) {
-    // every split of this head is resident (the grid fits the GPU at two CTAs per SM), so this
-    // wait ends as soon as the slowest split has written its partial
-    __threadfence();
-    atomicAdd(a.cnt + head, 1u);
-    const uint64_t t0 = globaltimer_ns();
-    int ok = 1;
-    while (ld_acquire_gpu(a.cnt + head) < (unsigned)C) {
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
-        ok = 0;
-        set_status(a.status, CASSPEC_E_TIMEOUT);
-        break;
-      }
-    }
-    flags[1] = ok;
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kAttnTmemCols);
   }
-  __syncthreads();
+  cluster_sync();  // every split's partial is in its shared memory
 
-  // ---- merge: this split finishes rows rank, rank + C, ... over all C partials, in split order ----
-  // (the K/V ring is drained: its shared memory holds the merge weights)
-  if (flags[1]) {
-    __threadfence();
-    constexpr int V4 = HD / 4;
-    const float* pob = a.part_o + (size_t)head * C * 64 * HD;
-    const float2* pml = a.part_ml + (size_t)head * C * 64;
-    const int nr = rank < n ? (n - rank + C - 1) / C : 0;  // rows of this split
-    float2* ml_s = reinterpret_cast<float2*>(ring);          // [nr][C] (max, sum)
-    float* w_s = reinterpret_cast<float*>(ring + 64 * kAttnMaxSplits * 8);  // [nr][C] weights
-    float* inv_s = w_s + 64 * kAttnMaxSplits;                                // [nr] 1 / sum
-    if (tid < nr * C) ml_s[tid] = __ldcg(pml + (tid % C) * 64 + rank + (tid / C) * C);
-    __syncthreads();
-    if (tid < nr) {
-      float M = -INFINITY;
-      for (int k = 0; k < C; ++k) M = fmaxf(M, ml_s[tid * C + k].x);
-      float L = 0.f;
-      for (int k = 0; k < C; ++k) {
-        const float2 ml = ml_s[tid * C + k];
-        const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);  // an empty split weighs 0
-        w_s[tid * C + k] = w;
-        L += ml.y * w;
-      }
-      inv_s[tid] = 1.f / L;
-    }
-    __syncthreads();
-    for (int idx = tid; idx < nr * V4; idx += kAttnThreads) {
-      const int j = idx / V4, c4 = (idx % V4) * 4, row = rank + j * C;
-      float4 ov[kAttnMaxSplits];  // every partial of this element in flight at once
+  // ---- merge: this split finishes rows rank, rank + C, ... over the C partials, in split order ----
+  // Each thread reads the (max, sum) and its four output columns of every partial at once (one
+  // round trip through distributed shared memory) and forms the weights itself.
+  const int n = a.n;
+  const int nr = rank < n ? (n - rank + C - 1) / C : 0;  // rows of this split
+  constexpr int V4 = HD / 4;
+  for (int idx = tid; idx < nr * V4; idx += kAttnThreads) {
+    const int j = idx / V4, c4 = (idx % V4) * 4, r = rank + j * C;
+    const uint32_t src = smem_u32(part_o + r * HD + c4), srm = smem_u32(part_ml + r);
+    float4 ov[kAttnMaxSplits];
+    float2 ml[kAttnMaxSplits];
 #pragma unroll
-      for (int k = 0; k < kAttnMaxSplits; ++k)
-        if (k < C) ov[k] = __ldcg(reinterpret_cast<const float4*>(pob + ((size_t)k * 64 + row) * HD + c4));
-      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int k = 0; k < kAttnMaxSplits; ++k) {
-        if (k < C) {
-          const float w = w_s[j * C + k];
-          o.x += ov[k].x * w;
-          o.y += ov[k].y * w;
-          o.z += ov[k].z * w;
-          o.w += ov[k].w * w;
-        }
+    for (int k = 0; k < kAttnMaxSplits; ++k)
+      if (k < C) {
+        ov[k] = ld_dsmem_f4(map_to_rank(src, (uint32_t)k));
+        ml[k] = ld_dsmem_f2(map_to_rank(srm, (uint32_t)k));
       }
-      const float inv = inv_s[j];
-      const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
-      const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
-      uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
-      hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
-      hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
-      lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
-      lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
-      *reinterpret_cast<uint2*>(a.o + (size_t)row * a.d + head * HD + c4) = hi;
-      *reinterpret_cast<uint2*>(a.o + (size_t)(64 + row) * a.d + head * HD + c4) = lo;
+    float M = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < kAttnMaxSplits; ++k)
+      if (k < C) M = fmaxf(M, ml[k].x);
+    float L = 0.f;
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < kAttnMaxSplits; ++k) {
+      if (k < C) {
+        const float w = ml[k].x == -INFINITY ? 0.f : exp2f(ml[k].x - M);  // an empty split weighs 0
+        L += ml[k].y * w;
+        o.x += ov[k].x * w;
+        o.y += ov[k].y * w;
+        o.z += ov[k].z * w;
+        o.w += ov[k].w * w;
+      }
     }
+    const float inv = 1.f / L;
+    const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
+    const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
+    uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
+    hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
+    hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
+    lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
+    lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
+    *reinterpret_cast<uint2*>(a.o + (size_t)r * a.d + head * HD + c4) = hi;
+    *reinterpret_cast<uint2*>(a.o + (size_t)(64 + r) * a.d + head * HD + c4) = lo;
   }
-  __syncthreads();
-  if (tid == 0) {  // the last split out (every split has stopped reading the arrival counter)
-    __threadfence();
-    if (atomicAdd(a.cnt + a.n_heads + head, 1u) == (unsigned)(C - 1)) {
-      a.cnt[head] = 0u;
-      a.cnt[a.n_heads + head] = 0u;
-    }
-  }
+  cluster_sync();  // no split leaves while another still reads its partial
 }
 
 int attn_splits(int n_heads, int num_sms) {
@@ -403,6 +484,8 @@ int attn_splits(int n_heads, int num_sms) {
   if (c < 1) c = 1;
   return c;
 }
+
+static_assert(attn_smem_bytes<128>() + 1024 <= 232448 / 2, "two attention CTAs per SM");
 
 template <int HD>
 static cudaError_t launch_hd(const CUtensorMap& tm, const AttnArgs& a, cudaStream_t stream, bool pdl) {
@@ -413,6 +496,8 @@ static cudaError_t launch_hd(const CUtensorMap& tm, const AttnArgs& a, cudaStrea
   cudaGetDevice(&dev);
   if (configured != dev) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    // the whole shared memory as carveout: two CTAs per SM
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
     configured = dev;
   }
@@ -421,16 +506,21 @@ static cudaError_t launch_hd(const CUtensorMap& tm, const AttnArgs& a, cudaStrea
   cfg.blockDim = dim3(kAttnThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)a.splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = pdl ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, kern, tm, a);
 }
 
 cudaError_t launch_tree_attention(const CUtensorMap& tm, const AttnArgs& a, int hd, cudaStream_t stream, bool pdl) {
-  if (a.splits < 1 || a.splits > kAttnMaxSplits) return cudaErrorInvalidValue;
+  if (a.splits < 1 || a.splits > kAttnMaxSplits || a.n < 1 || a.n > 64 || a.T < 0 || a.T + a.n > 64)
+    return cudaErrorInvalidValue;
   if (hd == 128) return launch_hd<128>(tm, a, stream, pdl);
   if (hd == 64) return launch_hd<64>(tm, a, stream, pdl);
   return cudaErrorInvalidValue;

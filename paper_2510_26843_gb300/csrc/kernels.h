@@ -86,7 +86,7 @@ struct GemmF8Args {
   EpiParams ep;
 };
 
-constexpr int kAttnMaxSplits = 16;
+constexpr int kAttnMaxSplits = 8;  // the splits of a head form one thread-block cluster (portable size)
 struct AttnArgs {
   const uint16_t* q;    // [64][d] bf16 (rotated)
   uint16_t* o;          // split attention output [128][d] bf16
@@ -94,11 +94,8 @@ struct AttnArgs {
   const int* dP;
   int T, n, ctx, d, n_heads;
   int layer;            // K/V rows of this layer in the cache tensor map: ((layer * 2 + kv) * H + h) * ctx + slot
-  int splits;           // CTAs per head (split-KV), <= kAttnMaxSplits; n_heads * splits <= 2 * SMs
+  int splits;           // CTAs per head (split-KV, one cluster), <= kAttnMaxSplits; n_heads * splits <= 2 * SMs
   float scale_log2;     // log2(e) / sqrt(hd)
-  float* part_o;        // [n_heads][splits][64][hd] fp32 unnormalised partial outputs
-  float2* part_ml;      // [n_heads][splits][64] (running max, sum) per row
-  unsigned* cnt;        // [2 * n_heads] arrival and exit counters per head, zero between launches
   int* status;
 };
 
