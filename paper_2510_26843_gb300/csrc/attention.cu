@@ -431,49 +431,63 @@ __global__ void __launch_bounds__(kAttnThreads, 2) tree_attn_kernel(const __grid
   cluster_sync();  // every split's partial is in its shared memory
 
   // ---- merge: this split finishes rows rank, rank + C, ... over the C partials, in split order ----
-  // Each thread reads the (max, sum) and its four output columns of every partial at once (one
-  // round trip through distributed shared memory) and forms the weights itself.
+  // A thread takes two (row, 4-column) items per batch and issues every load of both, the (max, sum)
+  // and the four output columns of all C partials, before using any: one round trip through
+  // distributed shared memory per batch.  The weights are formed per item.
   const int n = a.n;
   const int nr = rank < n ? (n - rank + C - 1) / C : 0;  // rows of this split
   constexpr int V4 = HD / 4;
-  for (int idx = tid; idx < nr * V4; idx += kAttnThreads) {
-    const int j = idx / V4, c4 = (idx % V4) * 4, r = rank + j * C;
-    const uint32_t src = smem_u32(part_o + r * HD + c4), srm = smem_u32(part_ml + r);
-    float4 ov[kAttnMaxSplits];
-    float2 ml[kAttnMaxSplits];
+  for (int base = 0; base < nr * V4; base += 2 * kAttnThreads) {  // 8 rows (C = 8): one batch
+    float4 ov[2][kAttnMaxSplits];
+    float2 ml[2][kAttnMaxSplits];
 #pragma unroll
-    for (int k = 0; k < kAttnMaxSplits; ++k)
-      if (k < C) {
-        ov[k] = ld_dsmem_f4(map_to_rank(src, (uint32_t)k));
-        ml[k] = ld_dsmem_f2(map_to_rank(srm, (uint32_t)k));
-      }
-    float M = -INFINITY;
+    for (int it = 0; it < 2; ++it) {
+      const int idx = base + tid + it * kAttnThreads;
+      if (idx < nr * V4) {
+        const int j = idx / V4, c4 = (idx % V4) * 4, r = rank + j * C;
+        const uint32_t src = smem_u32(part_o + r * HD + c4), srm = smem_u32(part_ml + r);
 #pragma unroll
-    for (int k = 0; k < kAttnMaxSplits; ++k)
-      if (k < C) M = fmaxf(M, ml[k].x);
-    float L = 0.f;
-    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int k = 0; k < kAttnMaxSplits; ++k) {
-      if (k < C) {
-        const float w = ml[k].x == -INFINITY ? 0.f : exp2f(ml[k].x - M);  // an empty split weighs 0
-        L += ml[k].y * w;
-        o.x += ov[k].x * w;
-        o.y += ov[k].y * w;
-        o.z += ov[k].z * w;
-        o.w += ov[k].w * w;
+        for (int k = 0; k < kAttnMaxSplits; ++k)
+          if (k < C) {
+            ov[it][k] = ld_dsmem_f4(map_to_rank(src, (uint32_t)k));
+            ml[it][k] = ld_dsmem_f2(map_to_rank(srm, (uint32_t)k));
+          }
       }
     }
-    const float inv = 1.f / L;
-    const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
-    const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
-    uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
-    hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
-    hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
-    lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
-    lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
-    *reinterpret_cast<uint2*>(a.o + (size_t)r * a.d + head * HD + c4) = hi;
-    *reinterpret_cast<uint2*>(a.o + (size_t)(64 + r) * a.d + head * HD + c4) = lo;
+#pragma unroll
+    for (int it = 0; it < 2; ++it) {
+      const int idx = base + tid + it * kAttnThreads;
+      if (idx < nr * V4) {
+        const int j = idx / V4, c4 = (idx % V4) * 4, r = rank + j * C;
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kAttnMaxSplits; ++k)
+          if (k < C) M = fmaxf(M, ml[it][k].x);
+        float L = 0.f;
+        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < kAttnMaxSplits; ++k) {
+          if (k < C) {
+            const float w = ml[it][k].x == -INFINITY ? 0.f : exp2f(ml[it][k].x - M);  // an empty split weighs 0
+            L += ml[it][k].y * w;
+            o.x += ov[it][k].x * w;
+            o.y += ov[it][k].y * w;
+            o.z += ov[it][k].z * w;
+            o.w += ov[it][k].w * w;
+          }
+        }
+        const float inv = 1.f / L;
+        const float r0 = o.x * inv, r1 = o.y * inv, r2 = o.z * inv, r3 = o.w * inv;
+        const uint16_t h0 = f2bf(r0), h1 = f2bf(r1), h2 = f2bf(r2), h3 = f2bf(r3);
+        uint2 hi, lo;  // split output: hi = bf16(o) in rows 0..63, lo = bf16(o - hi) in rows 64..127
+        hi.x = (uint32_t)h0 | ((uint32_t)h1 << 16);
+        hi.y = (uint32_t)h2 | ((uint32_t)h3 << 16);
+        lo.x = pack_bf16x2(r0 - bf2f(h0), r1 - bf2f(h1));
+        lo.y = pack_bf16x2(r2 - bf2f(h2), r3 - bf2f(h3));
+        *reinterpret_cast<uint2*>(a.o + (size_t)r * a.d + head * HD + c4) = hi;
+        *reinterpret_cast<uint2*>(a.o + (size_t)(64 + r) * a.d + head * HD + c4) = lo;
+      }
+    }
   }
   cluster_sync();  // no split leaves while another still reads its partial
 }
