@@ -547,16 +547,22 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           flags[1] = okp;
         }
         bar();
+        // this CTA's 32 tokens: partial(rank 0) + partial(rank 1), the same order on both CTAs
+        float v[16];
         if (flags[1]) {
-          // this CTA's 32 tokens: partial(rank 0) + partial(rank 1), the same order on both CTAs
           const int tl = t2 - 32 * s.rank;  // token within this CTA's half
-          float v[16];
 #pragma unroll
           for (int c = 0; c < 16; ++c)
             if (c < wq) {
               const float own = Pp[(c0q + c) * 64 + t2], got = recv[(c0q + c) * 32 + tl];
               v[c] = s.rank == 0 ? own + got : got + own;
             }
+        }
+        bar();
+        // `recv` is read: the partner may fill it for the next pair phase (released before this CTA's
+        // global stores below, which it does not depend on)
+        if (et == 0 && flags[1]) mbar_arrive_remote(map_to_rank(smem_u32(pfree), (uint32_t)peer));
+        if (flags[1]) {
           float ssq2 = 0.f;
           if (t2 < n) {
             float nv[16];
@@ -601,8 +607,6 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           ssq2 += __shfl_xor_sync(0xffffffffu, ssq2, 2);
           if (cq == 0 && ep.ss_out != nullptr) ep.ss_out[(size_t)s.slice * 64 + t2] = t2 < n ? ssq2 : 0.f;
         }
-        bar();
-        if (et == 0 && flags[1]) mbar_arrive_remote(map_to_rank(smem_u32(pfree), (uint32_t)peer));  // recv consumed
         ++npair;
       } else {
         // (3) 16 output rows (EPI_GLU: 16 channels, gate and up) at a time: the lo-plane warps hand
