@@ -39,12 +39,12 @@
 namespace casspec {
 
 constexpr int kChainThreads = 256;
-constexpr uint32_t kWStage = 32768;  // weight ring stage: whole k-blocks of the CTA's slice
+constexpr uint32_t kWStage = 28672;  // weight ring stage: whole k-blocks of the CTA's slice
 constexpr int kWStages = 4;
 constexpr uint32_t kXStage = 16384;  // one k-block of the split activation: 128 rows x 128 B
-constexpr int kXStages = 4;
+constexpr int kXStages = 5;
 constexpr int kRecvFloats = kPairMaxRows * 32;  // a pair partner's half-K partial of this CTA's 32 tokens
-constexpr int kStgFloats = 2048;     // epilogue hand-over buffer: 32 rows x 64 tokens fp32 (two of them)
+constexpr int kStgFloats = 2560;     // epilogue hand-over buffer: 32 rows x 64 tokens fp32 (two of them)
 constexpr uint32_t kTmemCols = 512;  // one accumulator of up to 256 columns per MMA issuer
 
 __host__ __device__ constexpr size_t chain_smem() {
@@ -419,20 +419,22 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       // Everything the epilogue reads from memory that does not depend on this phase's result is
       // loaded while the MMAs run: the residual rows and the next norm's gains (S = 2), and the
       // rotary coefficients of the first 16-row group (QKV).
-      float4 xo[4], gq[4], csn[4];
+      float4 xo[5], gq[5], csn[4];  // (S = 2: up to kPairMaxRows / 4 = 20 rows per thread)
 #pragma unroll
-      for (int k = 0; k < 4; ++k) xo[k] = gq[k] = csn[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k = 0; k < 5; ++k) xo[k] = gq[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) csn[k] = make_float4(0.f, 0.f, 0.f, 0.f);
       // S = 2: rank r finishes tokens 32 r .. 32 r + 31, four threads per token, R / 4 rows each
       const int t2 = 32 * s.rank + (et >> 2), cq = et & 3, wq = R / 4, c0q = cq * wq;
       if (S == 2) {
         if (t2 < n) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
+          for (int k = 0; k < 5; ++k)
             if (4 * k < wq) xo[k] = __ldcg(reinterpret_cast<const float4*>(ep.y + (size_t)t2 * ep.ldy + r0 + c0q) + k);
         }
         if (ep.xa_out != nullptr) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
+          for (int k = 0; k < 5; ++k)
             if (4 * k < wq) gq[k] = __ldg(reinterpret_cast<const float4*>(ep.g_next + r0 + c0q) + k);
         }
       }
@@ -478,40 +480,42 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         // partner reads it through distributed shared memory, and each CTA finishes 32 tokens of the
         // pair's rows as partial(rank 0) + partial(rank 1), in that order on both.
         float* Pp = stg;
-        const int nch = R / 16;  // <= kPairMaxRows / 16 = 4
-        float pv[4][16];         // both accumulators of the warp's lanes
+        const int nch = R / 16;  // <= kPairMaxRows / 16 = 5: read in passes of up to 4 chunks
+        for (int cb = 0; cb < nch; cb += 4) {
+          float pv[4][16];  // both accumulators of the warp's lanes
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          if (c < nch) {
-            float w2[16];
-            tmem_ld_x16(tbase + (uint32_t)(c * 16), pv[c]);
-            if (two) tmem_ld_x16(tbase + acc2 + (uint32_t)(c * 16), w2);
-            tmem_ld_wait();
-            if (two) {
+          for (int c = 0; c < 4; ++c) {
+            if (cb + c < nch) {
+              float w2[16];
+              tmem_ld_x16(tbase + (uint32_t)((cb + c) * 16), pv[c]);
+              if (two) tmem_ld_x16(tbase + acc2 + (uint32_t)((cb + c) * 16), w2);
+              tmem_ld_wait();
+              if (two) {
 #pragma unroll
-              for (int i = 0; i < 16; ++i) pv[c][i] += w2[i];
+                for (int i = 0; i < 16; ++i) pv[c][i] += w2[i];
+              }
             }
           }
-        }
-        if (!hi) {
+          if (!hi) {
 #pragma unroll
-          for (int c = 0; c < 4; ++c)
-            if (c < nch) {
+            for (int c = 0; c < 4; ++c)
+              if (cb + c < nch) {
 #pragma unroll
-              for (int i = 0; i < 16; ++i) Pp[(c * 16 + i) * 64 + t] = pv[c][i];
-            }
+                for (int i = 0; i < 16; ++i) Pp[((cb + c) * 16 + i) * 64 + t] = pv[c][i];
+              }
+          }
+          tc_fence_before();
+          bar();  // (the lo group's next pass writes other rows than the hi group adds here)
+          if (hi) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+              if (cb + c < nch) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) Pp[((cb + c) * 16 + i) * 64 + t] += pv[c][i];
+              }
+          }
         }
-        tc_fence_before();
-        bar();
         if (et == 0) mbar_arrive(&tempty[buf]);  // TMEM read: the next phase's MMAs may start
-        if (hi) {
-#pragma unroll
-          for (int c = 0; c < 4; ++c)
-            if (c < nch) {
-#pragma unroll
-              for (int i = 0; i < 16; ++i) Pp[(c * 16 + i) * 64 + t] += pv[c][i];
-            }
-        }
         // the partner's previous S = 2 phase has consumed what this CTA wrote into its `recv`
         if (et == 0) {
           int okf = 1;
@@ -548,11 +552,11 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         }
         bar();
         // this CTA's 32 tokens: partial(rank 0) + partial(rank 1), the same order on both CTAs
-        float v[16];
+        float v[20];
         if (flags[1]) {
           const int tl = t2 - 32 * s.rank;  // token within this CTA's half
 #pragma unroll
-          for (int c = 0; c < 16; ++c)
+          for (int c = 0; c < 20; ++c)
             if (c < wq) {
               const float own = Pp[(c0q + c) * 64 + t2], got = recv[(c0q + c) * 32 + tl];
               v[c] = s.rank == 0 ? own + got : got + own;
@@ -565,9 +569,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         if (flags[1]) {
           float ssq2 = 0.f;
           if (t2 < n) {
-            float nv[16];
+            float nv[20];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
+            for (int k = 0; k < 5; ++k) {
               nv[4 * k + 0] = xo[k].x + v[4 * k + 0];
               nv[4 * k + 1] = xo[k].y + v[4 * k + 1];
               nv[4 * k + 2] = xo[k].z + v[4 * k + 2];
@@ -576,14 +580,14 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             const int col = r0 + c0q;
             float4* dst = reinterpret_cast<float4*>(ep.y + (size_t)t2 * ep.ldy + col);
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
+            for (int k = 0; k < 5; ++k)
               if (4 * k < wq) dst[k] = make_float4(nv[4 * k], nv[4 * k + 1], nv[4 * k + 2], nv[4 * k + 3]);
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
+            for (int i = 0; i < 20; ++i)
               if (i < wq) ssq2 += nv[i] * nv[i];
             if (ep.xa_out != nullptr) {
 #pragma unroll
-              for (int k = 0; k < 4; ++k) {
+              for (int k = 0; k < 5; ++k) {
                 if (4 * k < wq) {
                   const float4 g4 = gq[k];
                   const float g[4] = {nv[4 * k] * g4.x, nv[4 * k + 1] * g4.y, nv[4 * k + 2] * g4.z, nv[4 * k + 3] * g4.w};
