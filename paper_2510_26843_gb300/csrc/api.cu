@@ -734,8 +734,8 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
   if (sms <= 0 || sms > kSmsBound) return CASSPEC_E_CUDA;
   {  // the projection chain's per-CTA slices must fit one MMA (and a residual slice the epilogue)
     const int G = chain_grid(sms), d = cfg->d_model, F = cfg->ffn;
-    if (chain_slice_rows(3 * d, G, false) > 256 ||
-        chain_slice_rows(F, G, true) > 256 || chain_slice_rows(roundup16(cfg->vocab), G, false) > 256 ||
+    if (chain_slice_rows(3 * d, G, false) > kChainMaxSliceRows || chain_slice_rows(F, G, true) > kChainMaxSliceRows ||
+        chain_slice_rows(roundup16(cfg->vocab), G, false) > kChainMaxSliceRows ||
         cdiv(F, 64) > kReadyPerPhase || cdiv(d, 64) > kReadyPerPhase)
       return CASSPEC_E_SHAPE;
   }

@@ -53,6 +53,7 @@ __host__ __device__ constexpr size_t chain_smem() {
 }
 static_assert(chain_smem() <= 232448, "the chain's shared memory exceeds the 227 KB a CTA may use");
 static_assert(kWStage % 1024 == 0 && kXStage % 1024 == 0, "ring stages keep the 1 KB alignment of the 128 B swizzle");
+static_assert(kChainMaxSliceRows * 128 <= (int)kWStage && kChainMaxSliceRows <= 256, "a slice's k-block fits a weight stage");
 
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
   unsigned v;
@@ -922,8 +923,7 @@ cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int grid,
     const ChainPhase& ph = args.ph[p];
     if (ph.wp == nullptr || (reinterpret_cast<uintptr_t>(ph.wp) & 15) != 0 || ph.N % kRowGroup != 0 || ph.kb < 1)
       return cudaErrorInvalidValue;
-    // one k-block of the slice (rows x 128 B) fits a weight stage, and N <= 256
-    if (chain_slice_rows(ph.N, grid, ph.epi == EPI_GLU) > (int)min(256u, kWStage / 128u)) return cudaErrorInvalidValue;
+    if (chain_slice_rows(ph.N, grid, ph.epi == EPI_GLU) > kChainMaxSliceRows) return cudaErrorInvalidValue;
     if (ph.S != 1 && (ph.S != 2 || !args.pairs || ph.epi != EPI_RESID || ph.kb < 2 ||
                       chain_slice_rows(ph.N, grid / 2, false) > kPairMaxRows))
       return cudaErrorInvalidValue;

@@ -218,6 +218,7 @@ int chain_grid(int num_sms);
 size_t chain_smem_bytes();
 int chain_slice_rows(int N, int G, bool glu);
 cudaError_t launch_chain(const ChainMaps& maps, const ChainArgs& args, int grid, cudaStream_t stream, bool pdl);
+constexpr int kChainMaxSliceRows = 224;  // output rows (GLU: 2 x channels) of a CTA's slice: one k-block per weight stage
 constexpr int kPairMaxRows = 80;  // rows of an S = 2 slice that the pair's exchange buffer holds
 size_t pack_rows_bytes(int N, int K, int kind);
 cudaError_t launch_pack_rows(const uint16_t* W, const uint16_t* W2, int N, int rows, int K, int G, int S, int kind,
