@@ -405,39 +405,76 @@ cudaError_t launch_row_argmax(const float* logits, int n, int V, int* am, cudaSt
 // ---------------------------------------------------------------------------------------------
 __global__ void accept_kernel(const int* __restrict__ am, const int* __restrict__ tokens,
                               const int* __restrict__ parent, int n, int* acc, int* status) {
-  __shared__ int s_par[kMaxTree], s_tok[kMaxTree], s_am[kMaxTree], s_depth[kMaxTree], s_match[kMaxTree];
-  const int tid = threadIdx.x;
-  if (tid < n) {
-    s_par[tid] = __ldcg(parent + tid);
-    s_tok[tid] = __ldcg(tokens + tid);
-    s_am[tid] = __ldcg(am + tid);
+  // Warp-parallel: thread c owns node c.  Pointer jumping (6 rounds for up to 64 nodes) gives every
+  // node its depth, whether every edge on its root path matches (child token == parent's argmax),
+  // and its ancestor set; a max-reduction picks the deepest matching node (lowest index on ties), and
+  // the nodes of its ancestor set write themselves into the path at their depth.
+  __shared__ int s_ptr[2][kMaxTree], s_depth[2][kMaxTree], s_match[2][kMaxTree], s_am[kMaxTree];
+  __shared__ unsigned long long s_anc[2][kMaxTree];
+  __shared__ int s_best, s_bad;
+  const int c = threadIdx.x;
+  const bool live = c < n;
+  int par = -1, tok = 0;
+  if (live) {
+    par = __ldcg(parent + c);
+    tok = __ldcg(tokens + c);
+    s_am[c] = __ldcg(am + c);
   }
+  if (c == 0) s_bad = 0;
   __syncthreads();
-  if (tid != 0) return;
-  bool ok = s_par[0] == -1;
-  for (int c = 1; c < n && ok; ++c) ok = s_par[c] >= 0 && s_par[c] < c;
-  if (!ok) {
-    set_status(status, CASSPEC_E_TREE);
-    acc[0] = 0;
+  if (live && (c == 0 ? par != -1 : (par < 0 || par >= c))) atomicOr(&s_bad, 1);
+  __syncthreads();
+  if (s_bad) {
+    if (c == 0) {
+      set_status(status, CASSPEC_E_TREE);
+      acc[0] = 0;
+    }
     return;
   }
-  s_depth[0] = 0;
-  s_match[0] = 1;
-  int best = 0;
-  for (int c = 1; c < n; ++c) {
-    const int p = s_par[c];
-    s_depth[c] = s_depth[p] + 1;
-    s_match[c] = s_match[p] && (s_tok[c] == s_am[p]);
-    if (s_match[c] && s_depth[c] > s_depth[best]) best = c;
+  int b = 0;
+  if (live) {
+    s_ptr[0][c] = par;
+    s_depth[0][c] = c == 0 ? 0 : 1;
+    s_match[0][c] = c == 0 ? 1 : (tok == s_am[par] ? 1 : 0);
+    s_anc[0][c] = 1ull << c;
   }
-  const int L = s_depth[best] + 1;
-  int node = best;
-  for (int k = L; k >= 1; --k) {
-    acc[k] = node;
-    node = s_par[node];
+  __syncthreads();
+  for (int r = 0; r < 6; ++r, b ^= 1) {  // 2^6 = 64 >= the deepest path
+    if (live) {
+      const int q = s_ptr[b][c];
+      if (q >= 0) {
+        s_ptr[b ^ 1][c] = s_ptr[b][q];
+        s_depth[b ^ 1][c] = s_depth[b][c] + s_depth[b][q];
+        s_match[b ^ 1][c] = s_match[b][c] & s_match[b][q];
+        s_anc[b ^ 1][c] = s_anc[b][c] | s_anc[b][q];
+      } else {
+        s_ptr[b ^ 1][c] = q;
+        s_depth[b ^ 1][c] = s_depth[b][c];
+        s_match[b ^ 1][c] = s_match[b][c];
+        s_anc[b ^ 1][c] = s_anc[b][c];
+      }
+    }
+    __syncthreads();
   }
-  acc[0] = L;
-  acc[L + 1] = s_am[best];
+  // deepest matching node, lowest index on ties: key = depth * 128 + (127 - c)
+  int key = (live && s_match[b][c]) ? s_depth[b][c] * 128 + (127 - c) : -1;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) key = max(key, __shfl_xor_sync(0xffffffffu, key, o));
+  if ((c & 31) == 0) s_ptr[b ^ 1][c >> 5] = key;  // (the other buffer is free now)
+  __syncthreads();
+  if (c == 0) {
+    int k = s_ptr[b ^ 1][0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) k = max(k, s_ptr[b ^ 1][w]);
+    s_best = 127 - (k & 127);
+  }
+  __syncthreads();
+  const int best = s_best;
+  const int L = s_depth[b][best] + 1;
+  if (live && ((s_anc[b][best] >> c) & 1ull)) acc[s_depth[b][c] + 1] = c;
+  if (c == 0) {
+    acc[0] = L;
+    acc[L + 1] = s_am[best];
+  }
 }
 
 cudaError_t launch_accept(const int* am, const int* tokens, const int* parent, int n, int* acc, int* status,
