@@ -54,8 +54,11 @@ typedef enum casspec_status {
 
 /* Model shape.  Requirements: d_model = n_heads * head_dim; head_dim in {64, 128};
  * d_model % 128 == 0, d_model <= 16384; ffn % 16 == 0, ffn <= 65536; vocab % 8 == 0,
- * vocab <= 131072; 1 <= n_layers <= 256.  The upper bounds keep every projection at most 1024
- * output tiles (one stream-K counter page per phase). */
+ * vocab <= 131072; 1 <= n_layers <= 256.  casspec_create_model further returns CASSPEC_E_SHAPE
+ * when the projection chain cannot hold the model on this GPU: a CTA's slice of any projection
+ * (rows / number of SMs, in 16-row groups; gate and up count twice) must stay within 224 rows, and a
+ * projection's input width within 256 blocks of 64 columns (d_model, ffn <= 16384).  On 152 SMs that
+ * is 3 * d_model, 2 * ffn and vocab <= 34048 (up to rounding to 16-row groups). */
 typedef struct casspec_model_config {
   int32_t n_layers;
   int32_t d_model;
