@@ -165,6 +165,22 @@ CASSPEC_API int casspec_set_stream(casspec_model* m, void* cuda_stream);
 /* Set option bits (CASSPEC_OPT_*); returns the previous bits in *old_flags if non-NULL. */
 CASSPEC_API int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags);
 
+/* Activation sparsity (App. C: the TEAL draft of the DSIA family), a model setting for bf16 steps.
+ * With 0 < s < 1, before each of Wqkv, Wo, Wgate/Wup and Wdown every token's floor(s * K) inputs of
+ * smallest magnitude (after RMSNorm) become 0; among equal magnitudes the lower index is kept.  The
+ * projections themselves stay dense, so a sparse step moves the same weight bytes as a dense one
+ * (this is the draft's arithmetic, not its speed).  s = 0, the default, is the dense step.  While
+ * s > 0, a step with quant_mode != 0 returns CASSPEC_E_INVAL.  Changing s drops captured graphs.
+ * Errors: CASSPEC_E_INVAL (null model, s outside [0, 1)). */
+CASSPEC_API int casspec_set_act_sparsity(casspec_model* m, float s);
+
+/* The sparsity rule of casspec_set_act_sparsity on a split activation x_split (dev, [128][ld] bf16:
+ * hi plane rows 0..63, lo plane rows 64..127, value = hi + lo in fp32): rows 0..n-1, columns
+ * 0..K-1, zeroed in both planes, in place, enqueued on `cuda_stream` (for tests and callers that
+ * apply the rule themselves).  Errors: CASSPEC_E_INVAL (null pointer, s outside [0, 1)),
+ * CASSPEC_E_SHAPE (n outside 1..64, K outside 1..16384, ld < K), CASSPEC_E_CUDA. */
+CASSPEC_API int casspec_sparsify_rows(uint16_t* x_split, int ld, int n, int K, float s, void* cuda_stream);
+
 /* Device address and size of weight tensor `tensor` (casspec_tensor_id) of `layer` (ignored for
  * the layer-independent tensors).  The caller writes weights there (e.g. cudaMemcpyAsync).
  * After writing the tensor maps stay valid: they are built once from these addresses.

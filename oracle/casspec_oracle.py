@@ -383,6 +383,8 @@ def tree_step(w: Weights, kv: KVCache, tokens: np.ndarray, parent: np.ndarray,
             x = _attention_block(x, w, kv, l, lin, pos, slots, all_anc, n, attn_bf16, trace)
         if ffn_on:
             xn2 = rmsnorm(x, w.gain("ffn_norm", l), sh.rms_eps)
+            if trace is not None:
+                trace.setdefault(l, {})["xn2"] = xn2
             g = _linear(xn2, w, "wg", l, lin)
             u = _linear(xn2, w, "wu", l, lin)
             hgu = silu(g) * u

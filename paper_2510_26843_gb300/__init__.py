@@ -31,7 +31,7 @@ OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL, OPT_W4_TC = 1, 2, 4, 8
 
 EXPORTS = [
     "casspec_model_bytes", "casspec_create_model", "casspec_destroy_model", "casspec_set_stream",
-    "casspec_set_options", "casspec_tensor", "casspec_quantize_weights", "casspec_kv_bytes", "casspec_kv_create",
+    "casspec_set_options", "casspec_set_act_sparsity", "casspec_sparsify_rows", "casspec_tensor", "casspec_quantize_weights", "casspec_kv_bytes", "casspec_kv_create",
     "casspec_kv_destroy", "casspec_kv_layer", "casspec_kv_set_prefix", "casspec_kv_reset_tree", "casspec_kv_length",
     "casspec_tree_step", "casspec_argmax", "casspec_accept_greedy", "casspec_kv_compact", "casspec_get_status",
     "casspec_status_string", "casspec_linear_workspace_bytes", "casspec_linear_bf16", "casspec_linear_bf16_static", "casspec_linear_bf16_static_status",
@@ -122,6 +122,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "casspec_destroy_model": (None, [_P]),
         "casspec_set_stream": (_I, [_P, _P]),
         "casspec_set_options": (_I, [_P, ctypes.c_uint, ctypes.POINTER(ctypes.c_uint)]),
+        "casspec_set_act_sparsity": (_I, [_P, ctypes.c_float]),
+        "casspec_sparsify_rows": (_I, [_P, _I, _I, _I, ctypes.c_float, _P]),
         "casspec_tensor": (_I, [_P, _I, _I, ctypes.POINTER(_P), ctypes.POINTER(_SZ)]),
         "casspec_quantize_weights": (_I, [_P]),
         "casspec_kv_bytes": (_SZ, [ctypes.POINTER(ModelConfig), _I]),
@@ -206,6 +208,17 @@ def set_options(m: int, flags: int) -> int:
     old = ctypes.c_uint()
     _check("casspec_set_options", load_library().casspec_set_options(m, flags, ctypes.byref(old)))
     return old.value
+
+
+def set_act_sparsity(m: int, s: float) -> None:
+    """casspec_set_act_sparsity: the activation sparsity s of the model's bf16 steps (0: dense)."""
+    _check("casspec_set_act_sparsity", load_library().casspec_set_act_sparsity(m, float(s)))
+
+
+def sparsify_rows(x_split, ld: int, n: int, K: int, s: float, stream=None) -> None:
+    """casspec_sparsify_rows: the sparsity rule on a split activation [128][ld] bf16, in place."""
+    _check("casspec_sparsify_rows", load_library().casspec_sparsify_rows(_ptr(x_split), ld, n, K, float(s),
+                                                                          _stream(stream)))
 
 
 def tensor(m: int, tensor_id: int, layer: int = 0) -> tuple[int, int]:

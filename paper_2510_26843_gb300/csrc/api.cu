@@ -205,6 +205,7 @@ struct casspec_model {
   unsigned *chain_ready, *chain_done;
   uint8_t* lm_p = nullptr;   // the LM head packed for the chain
   int resid_split = 1;       // 2: the chain runs as CTA pairs and the residual projections split K in two
+  float act_sparsity = 0.f;  // App. C activation sparsity of the bf16 steps (0: dense)
   bool pack_dirty = true;    // the row-major weights may have changed since the last packing
   int* pos;
   unsigned long long* anc;
@@ -526,6 +527,15 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         continue;
       }
       if (nph == kMaxPhases && (rc = flush()) != CASSPEC_OK) return rc;
+      // Activation sparsity (App. C): the projection's input loses its smallest-magnitude entries
+      // before the projection, so the projection starts its own launch after the sparsity kernel.
+      const float sp = m->act_sparsity;
+      if (sp > 0.f && it.kind != IT_LM) {
+        if ((rc = flush()) != CASSPEC_OK) return rc;
+        uint16_t* in = it.kind == IT_WO ? m->o : it.kind == IT_DOWN ? m->u : m->xa;
+        const int K = it.kind == IT_DOWN ? F : d;
+        LAUNCH(CASSPEC_K_OTHER, launch_sparsify(in, K, n, K, sp, s, pdl));
+      }
       const int ss_parts = i == 0 ? 1 : resid_parts;  // the embedding leaves one partial, a residual phase one per slice
       ChainPhase& p = ca.ph[nph];
       switch (it.kind) {
@@ -868,6 +878,23 @@ int casspec_set_stream(casspec_model* m, void* stream) {
   return CASSPEC_OK;
 }
 
+int casspec_set_act_sparsity(casspec_model* m, float s) {
+  if (m == nullptr || !(s >= 0.f && s < 1.f)) return CASSPEC_E_INVAL;
+  if (s != m->act_sparsity) {  // the step's launches differ: captured steps are rebuilt
+    for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second.first);
+    m->graphs.clear();
+  }
+  m->act_sparsity = s;
+  return CASSPEC_OK;
+}
+
+int casspec_sparsify_rows(uint16_t* x_split, int ld, int n, int K, float s, void* stream) {
+  if (x_split == nullptr || !(s >= 0.f && s < 1.f)) return CASSPEC_E_INVAL;
+  if (n < 1 || n > kMaxTree || K < 1 || K > 16384 || ld < K) return CASSPEC_E_SHAPE;
+  CK(launch_sparsify(x_split, ld, n, K, s, static_cast<cudaStream_t>(stream), false));
+  return CASSPEC_OK;
+}
+
 int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
   if (m == nullptr ||
       (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS | CASSPEC_OPT_TEST_STALL | CASSPEC_OPT_W4_TC)) != 0)
@@ -1059,6 +1086,7 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
     return CASSPEC_E_INVAL;
   if (quant_mode < 0 || quant_mode > 2) return CASSPEC_E_INVAL;
   if (quant_mode != 0 && !m->cfg.with_int8) return CASSPEC_E_INVAL;
+  if (quant_mode != 0 && m->act_sparsity > 0.f) return CASSPEC_E_INVAL;  // sparsity runs with bf16 steps only
   if (n < 1 || n > kMaxTree) return CASSPEC_E_SHAPE;
   if (kv->T + n > kMaxTree || kv->P_upper + kv->T + n > kv->ctx) return CASSPEC_E_CAPACITY;
   const int NL = m->cfg.n_layers;

@@ -313,6 +313,87 @@ cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* 
 }
 
 // ---------------------------------------------------------------------------------------------
+// Activation sparsity (App. C, TEAL's magnitude rule): in every token row t of a split activation
+// (hi plane row t, lo plane row 64 + t), the z = floor(s K) entries of smallest |hi + lo| become 0 in
+// both planes; among equal magnitudes the higher index goes first (the lower is kept).  One CTA per
+// row: a radix select over the magnitude's fp32 bits (4 passes of 8 bits) finds the z-th smallest
+// magnitude T and how many entries equal to T are to go; the entries below T and the highest-index
+// entries equal to T are zeroed.
+// ---------------------------------------------------------------------------------------------
+constexpr int kSpThreads = 256;
+__global__ void __launch_bounds__(kSpThreads) sparsify_kernel(uint16_t* __restrict__ x, int ld, int K, int z) {
+  extern __shared__ uint32_t sp_key[];  // [K] magnitude bits
+  __shared__ unsigned hist[256], part[kSpThreads];
+  __shared__ unsigned s_prefix, s_rem;
+  pdl_trigger();
+  pdl_wait();
+  const int t = blockIdx.x, tid = threadIdx.x;
+  uint16_t* hi = x + (size_t)t * ld;
+  uint16_t* lo = x + (size_t)(64 + t) * ld;
+  for (int c = tid; c < K; c += kSpThreads) sp_key[c] = __float_as_uint(fabsf(bf2f(hi[c]) + bf2f(lo[c])));
+  if (tid == 0) {
+    s_prefix = 0u;
+    s_rem = (unsigned)z;
+  }
+  unsigned mask = 0u;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int b = tid; b < 256; b += kSpThreads) hist[b] = 0u;
+    __syncthreads();
+    const unsigned prefix = s_prefix;
+    for (int c = tid; c < K; c += kSpThreads) {
+      const unsigned k = sp_key[c];
+      if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid == 0) {  // the bucket that holds the rem-th smallest candidate
+      unsigned rem = s_rem, b = 0u;
+      for (; b < 255u && hist[b] < rem; ++b) rem -= hist[b];
+      s_rem = rem;
+      s_prefix = prefix | (b << shift);
+    }
+    mask |= 255u << shift;
+    __syncthreads();
+  }
+  const unsigned T = s_prefix, rem = s_rem;  // z-th smallest magnitude; entries equal to it to zero
+  const int per = (K + kSpThreads - 1) / kSpThreads;
+  const int c0 = min(K, tid * per), c1 = min(K, c0 + per);
+  unsigned eq = 0u;
+  for (int c = c0; c < c1; ++c) eq += sp_key[c] == T ? 1u : 0u;
+  part[tid] = eq;
+  __syncthreads();
+  unsigned after = 0u;  // entries equal to T at higher indices than the one in hand
+  for (int k = tid + 1; k < kSpThreads; ++k) after += part[k];
+  for (int c = c1 - 1; c >= c0; --c) {
+    const unsigned k = sp_key[c];
+    bool drop = k < T;
+    if (k == T) drop = after++ < rem;
+    if (drop) {
+      hi[c] = 0;
+      lo[c] = 0;
+    }
+  }
+}
+
+cudaError_t launch_sparsify(uint16_t* x, int ld, int n, int K, float s, cudaStream_t st, bool pdl) {
+  if (n < 1 || n > 64 || K < 1 || ld < K || !(s >= 0.f && s < 1.f)) return cudaErrorInvalidValue;
+  const int z = (int)floor((double)s * K + 1e-9);
+  if (z <= 0) return cudaSuccess;
+  const size_t smem = (size_t)K * 4;
+  static int configured = -1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (configured != dev) {
+    const cudaError_t e = cudaFuncSetAttribute(sparsify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
+    if (e != cudaSuccess) return e;
+    configured = dev;
+  }
+  if (smem > 65536) return cudaErrorInvalidValue;
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kSpThreads), smem, st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, sparsify_kernel, x, ld, K, z);
+}
+
+// ---------------------------------------------------------------------------------------------
 // Argmax over the vocabulary: (max, lowest index of the max, second max) partials per LM-head
 // tile are merged; the merge is a total order (ties -> lower id), so lane order does not matter.
 // ---------------------------------------------------------------------------------------------
