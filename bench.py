@@ -401,7 +401,7 @@ def run_gpu(args) -> None:
     logits = torch.empty(n, sh.vocab, dtype=torch.float32, device="cuda")
     acc = torch.zeros(n + 2, dtype=torch.int32, device="cuda")
     graphs = not args.no_graphs
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC | (cs.OPT_GRAPHS if graphs else 0))
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC | (cs.OPT_GRAPHS if graphs else 0))
 
     def step():
         if cascade:
@@ -467,7 +467,7 @@ def run_gpu(args) -> None:
         assert 1 <= int(out_h[0]) <= n
 
     # ---- kernel-timing pass: eager launches bracketed by CUDA events on the launch stream ----
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC)
     cs.profile(dm.h, True)
     for _ in range(args.steps):
         if cascade:  # per-kernel figures of the round's verify step (the drafts mix kernel kinds)

@@ -142,6 +142,9 @@ enum casspec_tensor_id {
 #define CASSPEC_OPT_TEST_STALL 4u
 #define CASSPEC_OPT_W4_TC 8u /* quant_mode 2 on the tensor cores with e4m3 codes (default on); off: 4-bit
                                 codes through the integer mma.sync path */
+#define CASSPEC_OPT_W8_TC 16u /* quant_mode 1 on the tensor cores (default on): int8 codes widened to fp16
+                                 in shared memory, exact int32 sums (App. C's W8A8); off: the integer
+                                 mma.sync path.  Both give the same logits bit for bit. */
 
 /* ---------------------------------------------------------------------------------------------
  * Model

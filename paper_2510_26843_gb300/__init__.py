@@ -21,7 +21,7 @@ TOPK_MAX = 8
 DYTC_MAX_CLASS = 4  # latency-model classes (one regression per step arithmetic)
 DYTC_WORK = 24 * MAX_TREE  # int32 entries of casspec_dytc_round's device scratch
 SKIP_ATTN, SKIP_FFN = 0x2, 0x4  # skip-mask flags on a non-zero byte: drop the attention / FFN block
-OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL, OPT_W4_TC = 1, 2, 4, 8
+OPT_PDL, OPT_GRAPHS, OPT_TEST_STALL, OPT_W4_TC, OPT_W8_TC = 1, 2, 4, 8, 16
 
 (T_EMBED, T_LM_HEAD, T_FINAL_NORM, T_ATTN_NORM, T_FFN_NORM, T_WQKV, T_WO, T_WG, T_WU, T_WD,
  T_WQKV_Q, T_WO_Q, T_WG_Q, T_WU_Q, T_WD_Q, T_WQKV_S, T_WO_S, T_WG_S, T_WU_S, T_WD_S,

@@ -28,7 +28,11 @@ struct LayerPtrs {
   int8_t *qkv_q4, *wo_q4, *wg_q4, *wu_q4, *wd_q4;  // W4A4: two 4-bit codes per byte
   float *qkv_s4, *wo_s4, *wg_s4, *wu_s4, *wd_s4;
   uint8_t *qkv_f8, *wo_f8, *wg_f8, *wu_f8, *wd_f8;  // W4A4: the same codes as e4m3 bytes (tensor-core path)
+  // the tensor-core paths' weight codes as contiguous 16 KB tile images (launch_pack_tiles8): W8A8 int8
+  // codes (..._qp) and W4A4 e4m3 codes (..._fp); gate and up share one stream
+  uint8_t *qkv_qp, *wo_qp, *wgu_qp, *wd_qp, *qkv_fp, *wo_fp, *wgu_fp, *wd_fp;
   CUtensorMap tm_qkv8, tm_o8, tm_g8, tm_u8, tm_d8;
+  CUtensorMap tm_qkvq, tm_oq, tm_gq, tm_uq, tm_dq;  // W8A8 int8 codes as byte tiles (tensor-core path)
   CUtensorMap tm_qkv, tm_o, tm_g, tm_u, tm_d;
   uint8_t *wqkv_p, *wo_p, *wgu_p, *wd_p;  // the projections packed per CTA for the chain (pack_rows_kernel)
 };
@@ -43,6 +47,7 @@ struct Layout {
   size_t lm_p;
   std::vector<size_t> qkv_q4, wo_q4, wg_q4, wu_q4, wd_q4, qkv_s4, wo_s4, wg_s4, wu_s4, wd_s4;
   std::vector<size_t> qkv_f8, wo_f8, wg_f8, wu_f8, wd_f8;
+  std::vector<size_t> qkv_qp, wo_qp, wgu_qp, wd_qp, qkv_fp, wo_fp, wgu_fp, wd_fp;
   size_t x, q, o, u, xa, xq, xs, ssp, pos, anc, am_v1, am_i1, am_v2, am, margin, am2;
   size_t gemm_part, gemm_cnt, chain_ready, chain_done, i8_part, i8_cnt, status;
   size_t scratch_begin;
@@ -122,6 +127,12 @@ Layout make_layout(const casspec_model_config& c) {
       L.wg_f8.push_back(take(F * d));
       L.wu_f8.push_back(take(F * d));
       L.wd_f8.push_back(take(d * F));
+      for (int f = 0; f < 2; ++f) {
+        (f ? L.qkv_fp : L.qkv_qp).push_back(take(pack_tiles8_bytes((int)(3 * d), (int)d, 0)));
+        (f ? L.wo_fp : L.wo_qp).push_back(take(pack_tiles8_bytes((int)d, (int)d, 0)));
+        (f ? L.wgu_fp : L.wgu_qp).push_back(take(pack_tiles8_bytes((int)F, (int)d, 1)));
+        (f ? L.wd_fp : L.wd_qp).push_back(take(pack_tiles8_bytes((int)d, (int)F, 0)));
+      }
     }
   }
   L.scratch_begin = align_up(off, 256);
@@ -188,7 +199,7 @@ struct casspec_model {
   uint8_t* base = nullptr;
   cudaStream_t stream = nullptr;
   cudaStream_t cap_stream = nullptr;
-  unsigned flags = CASSPEC_OPT_PDL | CASSPEC_OPT_W4_TC;
+  unsigned flags = CASSPEC_OPT_PDL | CASSPEC_OPT_W4_TC | CASSPEC_OPT_W8_TC;
   int num_sms = 0;
   uint16_t *embed, *lm_head;
   float* final_norm;
@@ -199,7 +210,7 @@ struct casspec_model {
   // their 64 x BN boxes, BN = 16, 32, 48, 64, and [4]: 64 x 128 boxes (both planes of all 64 tokens
   // in one load, used when n > 48)
   CUtensorMap tm_o[5], tm_u[5], tm_xa[5];
-  CUtensorMap tm_xq8_d[4], tm_xq8_f[4];    // e4m3 activation codes, rows of d or F bytes, 128 x BN boxes
+  CUtensorMap tm_xq8_d[4], tm_xq8_f[4];    // activation codes (int8 or e4m3 bytes), rows of d or F, 128 x BN boxes
   int8_t* xq;
   float* xs;
   unsigned *chain_ready, *chain_done;
@@ -207,6 +218,7 @@ struct casspec_model {
   int resid_split = 1;       // 2: the chain runs as CTA pairs and the residual projections split K in two
   float act_sparsity = 0.f;  // App. C activation sparsity of the bf16 steps (0: dense)
   bool pack_dirty = true;    // the row-major weights may have changed since the last packing
+  bool pack8_dirty = true;   // the row-major W8A8 / W4A4 codes may have changed since their packing
   int* pos;
   unsigned long long* anc;
   float *am_v1, *am_v2, *margin;
@@ -313,6 +325,29 @@ int pack_weights(casspec_model* m, int& count) {
                       m->stream));
   ++count;
   m->pack_dirty = false;
+  return CASSPEC_OK;
+}
+
+// Refresh the tensor-core projections' tile images of the W8A8 int8 and W4A4 e4m3 codes.
+int pack_codes(casspec_model* m, int& count) {
+  const auto& c = m->cfg;
+  const int d = c.d_model, F = c.ffn;
+  for (int l = 0; l < c.n_layers; ++l) {
+    LayerPtrs& p = m->layers[l];
+    const uint8_t* q8[5] = {reinterpret_cast<uint8_t*>(p.qkv_q), reinterpret_cast<uint8_t*>(p.wo_q),
+                            reinterpret_cast<uint8_t*>(p.wg_q), reinterpret_cast<uint8_t*>(p.wu_q),
+                            reinterpret_cast<uint8_t*>(p.wd_q)};
+    const uint8_t* f8[5] = {p.qkv_f8, p.wo_f8, p.wg_f8, p.wu_f8, p.wd_f8};
+    for (int f = 0; f < 2; ++f) {
+      const uint8_t* const* w = f ? f8 : q8;
+      CK(launch_pack_tiles8(w[0], nullptr, 3 * d, d, 0, f ? p.qkv_fp : p.qkv_qp, m->stream));
+      CK(launch_pack_tiles8(w[1], nullptr, d, d, 0, f ? p.wo_fp : p.wo_qp, m->stream));
+      CK(launch_pack_tiles8(w[2], w[3], F, d, 1, f ? p.wgu_fp : p.wgu_qp, m->stream));
+      CK(launch_pack_tiles8(w[4], nullptr, d, F, 0, f ? p.wd_fp : p.wd_qp, m->stream));
+      count += 4;
+    }
+  }
+  m->pack8_dirty = false;
   return CASSPEC_OK;
 }
 
@@ -568,10 +603,16 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
     // W4A4 on the tensor cores: e4m3 codes, exact fp32 accumulation (casspec gemm_f8); otherwise the
     // 4-bit codes go through the s8 MMA of gemm_i8
     const bool tc4 = w4 && (m->flags & CASSPEC_OPT_W4_TC) != 0;
+    // W8A8 on the tensor cores: int8 codes widened to bf16 in shared memory (casspec gemm_s8tc), the
+    // same exact int32 sums as gemm_i8
+    const bool tc8 = !w4 && (m->flags & CASSPEC_OPT_W8_TC) != 0;
+    const bool tc = tc4 || tc8;
     const int afmt = tc4 ? 2 : 0;  // activation codes as e4m3 bytes for the tensor-core path
-    auto gemmf8 = [&](const CUtensorMap& tw, const CUtensorMap& tw2, const CUtensorMap& tx, const float* sw,
-                      const float* sw2, int N, int K, int tiles, int epi, const EpiParams& e) -> cudaError_t {
+    auto gemmf8 = [&](const CUtensorMap& tw, const CUtensorMap& tw2, const uint8_t* wpk, const CUtensorMap& tx,
+                      const float* sw, const float* sw2, int N, int K, int tiles, int epi,
+                      const EpiParams& e) -> cudaError_t {
       GemmF8Args g = {};
+      g.wpk = wpk;
       g.tiles = tiles;
       g.kblocks = cdiv(K, 128);
       g.N = N;
@@ -582,7 +623,9 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       g.counters = m->gemm_cnt;
       g.status = m->status;
       g.ep = e;
-      return launch_gemm_f8(tw, tw2, tx, BN, epi, g, gemm_bf16_grid(tiles, g.kblocks, m->num_sms), s, pdl);
+      const int grid = gemm_bf16_grid(tiles, g.kblocks, m->num_sms);
+      return tc8 ? launch_gemm_s8tc(tw, tw2, tx, BN, epi, g, grid, s, pdl)
+                 : launch_gemm_f8(tw, tw2, tx, BN, epi, g, grid, s, pdl);
     };
     auto gemm8 = [&](const int8_t* W, const float* sw, const int8_t* W2, const float* sw2, int N, int K, int tiles,
                      int epi, const EpiParams& e) -> cudaError_t {
@@ -634,6 +677,12 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         ed.xa_out = m->xa;
         ed.g_next = m->final_norm;
       }
+      // the tensor-core path's weight maps and tile images of this layer (W8A8 int8 / W4A4 e4m3 codes)
+      const CUtensorMap &t_qkv = tc8 ? Lp.tm_qkvq : Lp.tm_qkv8, &t_wo = tc8 ? Lp.tm_oq : Lp.tm_o8;
+      const CUtensorMap &t_wg = tc8 ? Lp.tm_gq : Lp.tm_g8, &t_wu = tc8 ? Lp.tm_uq : Lp.tm_u8;
+      const CUtensorMap& t_wd = tc8 ? Lp.tm_dq : Lp.tm_d8;
+      const uint8_t *p_qkv = tc8 ? Lp.qkv_qp : Lp.qkv_fp, *p_wo = tc8 ? Lp.wo_qp : Lp.wo_fp;
+      const uint8_t *p_wgu = tc8 ? Lp.wgu_qp : Lp.wgu_fp, *p_wd = tc8 ? Lp.wd_qp : Lp.wd_fp;
       if (it.kind == IT_QKV) {
         LAUNCH(CASSPEC_K_OTHER,
                launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax, afmt));
@@ -642,16 +691,16 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         e.q_out = m->q;
         e.kc = kv_layer_k(kv, it.l);
         e.vc = kv_layer_v(kv, it.l);
-        if (tc4)
-          LAUNCH(CASSPEC_K_QKV, gemmf8(Lp.tm_qkv8, Lp.tm_qkv8, m->tm_xq8_d[bi], s_qkv, nullptr, 3 * d, d, 3 * d / 128,
-                                       EPI_QKV, e));
+        if (tc)
+          LAUNCH(CASSPEC_K_QKV,
+                 gemmf8(t_qkv, t_qkv, p_qkv, m->tm_xq8_d[bi], s_qkv, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
         else
           LAUNCH(CASSPEC_K_QKV, gemm8(q_qkv, s_qkv, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
       } else if (it.kind == IT_WO) {
         // W8A8 activations are the bf16 values: the hi plane of the split output
         LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl, qmax, afmt));
-        if (tc4)
-          LAUNCH(CASSPEC_K_WO, gemmf8(Lp.tm_o8, Lp.tm_o8, m->tm_xq8_d[bi], s_wo, nullptr, d, d, d / 128, EPI_RESID, ed));
+        if (tc)
+          LAUNCH(CASSPEC_K_WO, gemmf8(t_wo, t_wo, p_wo, m->tm_xq8_d[bi], s_wo, nullptr, d, d, d / 128, EPI_RESID, ed));
         else
           LAUNCH(CASSPEC_K_WO, gemm8(q_wo, s_wo, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
       } else if (it.kind == IT_GU) {
@@ -660,16 +709,15 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         EpiParams eg = base;
         eg.N = F;
         eg.u_out = m->u;
-        if (tc4)
-          LAUNCH(CASSPEC_K_GATEUP, gemmf8(Lp.tm_g8, Lp.tm_u8, m->tm_xq8_d[bi], s_wg, s_wu, F, d, cdiv(F, 64), EPI_GLU,
-                                          eg));
+        if (tc)
+          LAUNCH(CASSPEC_K_GATEUP,
+                 gemmf8(t_wg, t_wu, p_wgu, m->tm_xq8_d[bi], s_wg, s_wu, F, d, cdiv(F, 64), EPI_GLU, eg));
         else
           LAUNCH(CASSPEC_K_GATEUP, gemm8(q_wg, s_wg, q_wu, s_wu, F, d, cdiv(F, 64), EPI_GLU, eg));
       } else {
         LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl, qmax, afmt));
-        if (tc4)
-          LAUNCH(CASSPEC_K_DOWN, gemmf8(Lp.tm_d8, Lp.tm_d8, m->tm_xq8_f[bi], s_wd, nullptr, d, F, d / 128, EPI_RESID,
-                                        ed));
+        if (tc)
+          LAUNCH(CASSPEC_K_DOWN, gemmf8(t_wd, t_wd, p_wd, m->tm_xq8_f[bi], s_wd, nullptr, d, F, d / 128, EPI_RESID, ed));
         else
           LAUNCH(CASSPEC_K_DOWN, gemm8(q_wd, s_wd, nullptr, nullptr, d, F, d / 128, EPI_RESID, ed));
       }
@@ -701,6 +749,11 @@ bool build_tensor_maps(casspec_model* m) {
       ok = ok && encode_tmap_u8(&Lp.tm_g8, Lp.wg_f8, d, F, d, 128, 64);
       ok = ok && encode_tmap_u8(&Lp.tm_u8, Lp.wu_f8, d, F, d, 128, 64);
       ok = ok && encode_tmap_u8(&Lp.tm_d8, Lp.wd_f8, F, d, F, 128, 128);
+      ok = ok && encode_tmap_u8(&Lp.tm_qkvq, Lp.qkv_q, d, 3 * d, d, 128, 128);
+      ok = ok && encode_tmap_u8(&Lp.tm_oq, Lp.wo_q, d, d, d, 128, 128);
+      ok = ok && encode_tmap_u8(&Lp.tm_gq, Lp.wg_q, d, F, d, 128, 64);
+      ok = ok && encode_tmap_u8(&Lp.tm_uq, Lp.wu_q, d, F, d, 128, 64);
+      ok = ok && encode_tmap_u8(&Lp.tm_dq, Lp.wd_q, F, d, F, 128, 128);
     }
     for (int b = 0; b < 4; ++b) {
       const uint32_t BN = 16u * (uint32_t)(b + 1);
@@ -812,6 +865,14 @@ int casspec_create_model(const casspec_model_config* cfg, void* dev_mem, size_t 
       p.wg_f8 = b + L.wg_f8[l];
       p.wu_f8 = b + L.wu_f8[l];
       p.wd_f8 = b + L.wd_f8[l];
+      p.qkv_qp = b + L.qkv_qp[l];
+      p.wo_qp = b + L.wo_qp[l];
+      p.wgu_qp = b + L.wgu_qp[l];
+      p.wd_qp = b + L.wd_qp[l];
+      p.qkv_fp = b + L.qkv_fp[l];
+      p.wo_fp = b + L.wo_fp[l];
+      p.wgu_fp = b + L.wgu_fp[l];
+      p.wd_fp = b + L.wd_fp[l];
     }
   }
   m->x = reinterpret_cast<float*>(b + L.x);
@@ -897,7 +958,8 @@ int casspec_sparsify_rows(uint16_t* x_split, int ld, int n, int K, float s, void
 
 int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
   if (m == nullptr ||
-      (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS | CASSPEC_OPT_TEST_STALL | CASSPEC_OPT_W4_TC)) != 0)
+      (flags & ~(CASSPEC_OPT_PDL | CASSPEC_OPT_GRAPHS | CASSPEC_OPT_TEST_STALL | CASSPEC_OPT_W4_TC |
+                 CASSPEC_OPT_W8_TC)) != 0)
     return CASSPEC_E_INVAL;
   if (old_flags) *old_flags = m->flags;
   if (flags != m->flags) {
@@ -911,6 +973,9 @@ int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags) {
 int casspec_tensor(casspec_model* m, int tensor, int layer, void** dev_ptr, size_t* bytes) {
   if (m == nullptr || dev_ptr == nullptr) return CASSPEC_E_INVAL;
   if (tensor <= CASSPEC_T_WD) m->pack_dirty = true;  // the caller may write through the pointer
+  if ((tensor >= CASSPEC_T_WQKV_Q && tensor <= CASSPEC_T_WD_Q) ||
+      (tensor >= CASSPEC_T_WQKV_F8 && tensor <= CASSPEC_T_WD_F8))
+    m->pack8_dirty = true;
   const auto& c = m->cfg;
   const size_t d = c.d_model, F = c.ffn, V = c.vocab;
   const bool state = tensor >= CASSPEC_T_RESIDUAL && tensor <= CASSPEC_T_ACT_S;  // step state, not weights
@@ -990,6 +1055,7 @@ int casspec_quantize_weights(casspec_model* m) {
     CK(launch_quant_rows(p.wu, F, d, d, reinterpret_cast<int8_t*>(p.wu_f8), d, p.wu_s4, m->stream, false, 7, 2));
     CK(launch_quant_rows(p.wd, d, F, F, reinterpret_cast<int8_t*>(p.wd_f8), F, p.wd_s4, m->stream, false, 7, 2));
   }
+  m->pack8_dirty = true;
   return CASSPEC_OK;
 }
 
@@ -1101,6 +1167,11 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
   if (m->pack_dirty) {  // outside any capture: a graph never holds the packing
     int count = 0;
     if ((rc = pack_weights(m, count)) != CASSPEC_OK) return rc;
+    m->launches += (uint64_t)count;
+  }
+  if (quant_mode != 0 && m->pack8_dirty) {
+    int count = 0;
+    if ((rc = pack_codes(m, count)) != CASSPEC_OK) return rc;
     m->launches += (uint64_t)count;
   }
   if ((m->flags & CASSPEC_OPT_GRAPHS) && !(m->flags & CASSPEC_OPT_TEST_STALL)) {

@@ -80,6 +80,8 @@ struct GemmF8Args {
   const float* sw;   // [N] weight scales (EPI_GLU: gate)
   const float* sw2;  // EPI_GLU: up weight scales
   const float* sx;   // [64] activation scales
+  const uint8_t* wpk;  // the weight codes packed as 16 KB tile images (launch_pack_tiles8), or null:
+                       // then read through the tensor maps
   float* partials;     // stream-K partial tiles, (tiles + grid) slots of 64 x 128 fp32
   unsigned* counters;  // [tiles], zero between launches
   int* status;
@@ -203,6 +205,15 @@ bool encode_tmap_u8(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t 
                     uint32_t box_inner, uint32_t box_rows);
 cudaError_t launch_gemm_f8(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int BN, int epi,
                            const GemmF8Args& args, int grid, cudaStream_t stream, bool pdl);
+// W8A8 on the tensor cores: int8 weight and activation codes (the 128-byte-swizzled byte tiles of
+// gemm_f8) widened to fp16 in shared memory; exact int32 sums, the same values as gemm_i8.
+// Weight codes ([N][K] bytes, K a multiple of 16; EPI_GLU: gate and up) as contiguous 16 KB images of
+// 128 x 128-code tiles with the 128-byte swizzle, in the order gemm_f8 / gemm_s8tc stream them.
+size_t pack_tiles8_bytes(int N, int K, int glu);
+cudaError_t launch_pack_tiles8(const uint8_t* src, const uint8_t* src2, int N, int K, int glu, uint8_t* dst,
+                               cudaStream_t stream);
+cudaError_t launch_gemm_s8tc(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int BN,
+                             int epi, const GemmF8Args& args, int grid, cudaStream_t stream, bool pdl);
 
 int gemm_i8_ksplit(int tiles, int K, int num_sms);
 cudaError_t launch_gemm_i8(const GemmI8Args& args, int BN, int epi, cudaStream_t stream, bool pdl);

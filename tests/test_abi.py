@@ -80,7 +80,8 @@ def test_binding_constants_match_the_header():
 
     h = _header_constants()
     pairs = {"MAX_TREE": "MAX_TREE", "TOPK_MAX": "TOPK_MAX", "DYTC_WORK": "DYTC_WORK", "DYTC_MAX_CLASS": "DYTC_MAX_CLASS", "SKIP_ATTN": "SKIP_ATTN",
-             "SKIP_FFN": "SKIP_FFN", "OPT_PDL": "OPT_PDL", "OPT_GRAPHS": "OPT_GRAPHS", "OPT_TEST_STALL": "OPT_TEST_STALL", "OK": "OK"}
+             "SKIP_FFN": "SKIP_FFN", "OPT_PDL": "OPT_PDL", "OPT_GRAPHS": "OPT_GRAPHS", "OPT_TEST_STALL": "OPT_TEST_STALL", "OPT_W4_TC": "OPT_W4_TC",
+             "OPT_W8_TC": "OPT_W8_TC", "OK": "OK"}
     for key in list(h):
         if key.startswith(("E_", "T_", "K_")):
             pairs[key] = key

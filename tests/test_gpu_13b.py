@@ -48,7 +48,7 @@ def dm13(cs):
     from paper_2510_26843_gb300.workload import DeviceModel
 
     dm = DeviceModel(SH13, SEED, with_int8=True)
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC | cs.OPT_W8_TC)
     yield dm
     dm.close()
 

@@ -76,7 +76,7 @@ def test_single_layer_7b(cs):
     sh = synth.ModelShape(1, SH7.d_model, SH7.n_heads, SH7.head_dim, SH7.ffn, SH7.vocab)
     P, n = 1024, 32
     dm = DeviceModel(sh, SEED)
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC | cs.OPT_W8_TC)
     kv = DeviceKV(dm, P + 64)
     kv.load_random_prefix(SEED, P)
     ow = oracle.Weights.from_seed(SEED, sh, keep_layers=1)
@@ -128,7 +128,7 @@ def dm7(cs):
     from paper_2510_26843_gb300.workload import DeviceModel
 
     dm = DeviceModel(SH7, SEED, with_int8=True)
-    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC | cs.OPT_W8_TC)
     yield dm
     dm.close()
 
@@ -197,6 +197,31 @@ def test_7b_draft_steps(cs, dm7, ow7, skip, mode, n):
     print(f"7B draft skip={skip} mode={mode} n={n}: per-row error / logit range {np.round(err, 4).tolist()}")
     assert np.all(err < (TOL_BF16 if mode == 0 else TOL_INT8_DEEP)), err.max()
     kv.close()
+
+
+@pytest.mark.parametrize("n", [1, 8, 64])
+def test_7b_w8a8_tensor_core_path_equals_integer_path(cs, dm7, n):
+    """The 32-layer W8A8 step on both paths: the same int8 codes and scales, exact int32 sums on both
+    (at K = 4096 and 11008 the tensor-core path adds 4 and up to 11 accumulators of <= 1024 columns,
+    each exact in fp32), so the logits are bitwise equal."""
+    from paper_2510_26843_gb300.workload import DeviceKV
+
+    P = 2048
+    parent = synth.tree(SEED + 11 + n, n, 8)
+    toks = synth.tokens(SEED + 11 + n, n, SH7.vocab)
+    base = cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC
+    out = []
+    for flags in (base | cs.OPT_W8_TC, base):
+        cs.set_options(dm7.h, flags)
+        kv = DeviceKV(dm7, P + 64)
+        kv.load_random_prefix(SEED, P)
+        got, _, _ = gpu_step(cs, dm7, kv, toks, parent, SH7.vocab, mode=1)
+        assert cs.get_status(dm7.h) == 0
+        kv.close()
+        out.append(got)
+    cs.set_options(dm7.h, base | cs.OPT_W8_TC)
+    assert np.all(np.isfinite(out[0]))
+    np.testing.assert_array_equal(out[0], out[1])
 
 
 def test_7b_int8_layerwise(cs, dm7, ow7):

@@ -298,7 +298,25 @@ def test_w4a4_tensor_core_path_equals_integer_path(cs, dev_model, ow, prefix, n)
         out.append(gpu_step(cs, dev_model, kv, toks, parent, mode=2))
         assert cs.get_status(dev_model.h) == 0
         kv.close()
-    cs.set_options(dev_model.h, cs.OPT_PDL | cs.OPT_W4_TC)
+    cs.set_options(dev_model.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC)
+    np.testing.assert_array_equal(out[0], out[1])
+
+
+@pytest.mark.parametrize("n", [1, 8, 33, 64])
+def test_w8a8_tensor_core_path_equals_integer_path(cs, dev_model, ow, prefix, n):
+    """Both W8A8 paths take the same int8 codes and scales, and both integer sums are exact (the s8
+    mma.sync in int32; the tensor-core path in fp32 accumulators of at most 1024 columns, each below
+    2^24, added in int32), so the logits are bitwise equal."""
+    parent = synth.tree(60 + n, n, 8)
+    toks = synth.tokens(60 + n, n, SH.vocab)
+    out = []
+    for flags in (cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC, cs.OPT_PDL | cs.OPT_W4_TC):
+        cs.set_options(dev_model.h, flags)
+        kv, _ = fresh_pair(cs, dev_model, ow, prefix)
+        out.append(gpu_step(cs, dev_model, kv, toks, parent, mode=1))
+        assert cs.get_status(dev_model.h) == 0
+        kv.close()
+    cs.set_options(dev_model.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC)
     np.testing.assert_array_equal(out[0], out[1])
 
 
