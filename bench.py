@@ -504,7 +504,10 @@ def run_gpu(args) -> None:
             T += b - a
         total += algorithmic_bytes(sh, n, P, on1, 0)["total"]
         ab["total"] = total
-    kern = ((f"gemm_i8_kernel ({'W4A4' if mode == 2 else 'W8A8'} gate/up + SwiGLU)") if mode else
+    # the quantised drafts' projections run on the tensor cores (gemm_f8_kernel: e4m3 codes for W4A4,
+    # int8 codes widened to fp16 for W8A8; the options set above keep both on)
+    kern = ((f"gemm_f8_kernel ({'W4A4 e4m3' if mode == 2 else 'W8A8 int8 widened to fp16'} gate/up + SwiGLU)")
+            if mode else
             "chain_kernel (Wo + residual, gate/up + SwiGLU, down + residual, next QKV or LM head)")
 
     out = {
@@ -564,7 +567,7 @@ def run_dytc(args) -> None:
     kv = DeviceKV(dm, P0 + 65 * rounds + 192)
     stream = torch.cuda.current_stream()
     cs.set_stream(dm.h, stream)
-    cs.set_options(dm.h, cs.OPT_PDL)
+    cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC)
     prompt = synth.prefix_tokens(SEED, P0, sh.vocab)
     logits = torch.empty(64, sh.vocab, dtype=torch.float32, device="cuda")
     for a in range(0, P0, 64):  # prefill in 64-token chains
