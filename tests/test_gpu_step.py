@@ -302,7 +302,7 @@ def test_w4a4_tensor_core_path_equals_integer_path(cs, dev_model, ow, prefix, n)
     np.testing.assert_array_equal(out[0], out[1])
 
 
-@pytest.mark.parametrize("n", [1, 8, 33, 64])
+@pytest.mark.parametrize("n", [1, 8, 24, 33, 64])  # token tiles BN = 16, 16, 32, 48, 64
 def test_w8a8_tensor_core_path_equals_integer_path(cs, dev_model, ow, prefix, n):
     """Both W8A8 paths take the same int8 codes and scales, and both integer sums are exact (the s8
     mma.sync in int32; the tensor-core path in fp32 accumulators of at most 1024 columns, each below
