@@ -286,10 +286,14 @@ QMAX = {1: 127, 2: 7}  # quant_mode -> largest code: W8A8, W4A4
 
 def _linear(x: np.ndarray, w: Weights, name: str, layer: int, lin: tuple) -> np.ndarray:
     """One projection of a draft: lin = (quant_mode, activation sparsity).  The sparsity rule
-    applies to the projection's input first; a quantised mode then quantises that input."""
+    applies to the projection's input first (in a quantised mode to its bf16 value, the value the
+    quantiser reads); a quantised mode then quantises that input."""
     mode, sparsity = lin
     if sparsity > 0.0:
-        x = sparsify_rows(x, sparsity)
+        # a quantised draft stores its activation in bf16 and quantises that value (reading of App. C
+        # above), so its magnitude selection is taken on the same bf16 value; a bf16 draft selects on
+        # the activation itself
+        x = sparsify_rows(round_bf16(x) if mode in QMAX else x, sparsity)
     if mode in QMAX:
         # The quantiser's integer decisions are taken on the activation as the draft stores it
         # (bf16) with the fp32 rule, i.e. in the kernel's precision.

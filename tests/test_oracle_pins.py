@@ -508,6 +508,31 @@ def test_w4a4_and_activation_sparsity_modes(tiny):
         oracle.tree_step(w, oracle.KVCache(SH.n_layers, SH.n_heads, SH.head_dim, 128), toks, parent, quant_mode=3)
 
 
+def test_quantised_sparsity_selects_on_the_bf16_activation(tiny):
+    """In a quantised draft the selection is taken on the bf16 activation the quantiser reads: two
+    inputs of different fp64 magnitude that round to the same bf16 value tie, and the lower index is
+    kept, where the bf16 draft keeps the larger fp64 one.  With one input kept, the W8A8 projection
+    is that input's code (127) times the weight column's codes, scaled."""
+    w, _, _ = tiny
+    from oracle import casspec_oracle
+
+    d = SH.d_model
+    x = np.zeros((1, d))
+    x[0, 5], x[0, 9] = 1.0 + 2.0 ** -12, 1.0 + 2.0 ** -11  # both round to 1.0 in bf16
+    keep_one = 1.0 - 1.0 / d
+    y16 = casspec_oracle._linear(x, w, "wo", 0, (0, keep_one))
+    np.testing.assert_array_equal(y16[0], x[0, 9] * w.f64("wo", 0)[:, 9])
+    y8 = casspec_oracle._linear(x, w, "wo", 0, (1, keep_one))
+    qw, sw = w.intq("wo", 0, 127)
+    kept = np.zeros((1, d))
+    kept[0, 5] = 1.0  # the selection under test: index 5, as bf16 (the quantiser's own scale rule)
+    qx, sx = oracle.quantize_rows_f32(kept, 127)
+    assert qx[0, 5] == 127 and np.count_nonzero(qx) == 1
+    want = (127.0 * qw[:, 5].astype(np.float64)) * float(sx[0]) * sw
+    np.testing.assert_allclose(y8[0], want, rtol=1e-15, atol=0)
+    assert not np.allclose(qw[:, 5], qw[:, 9])
+
+
 def test_attn_bf16_rounds_only_the_attention_operands(tiny):
     """attn_bf16 stores bf16 K/V and uses bf16 q: the cache entries it writes are bf16 values,
     everything else is the fp64 model, and the logits move by about the bf16 rounding."""
