@@ -168,13 +168,14 @@ CASSPEC_API int casspec_set_stream(casspec_model* m, void* cuda_stream);
 /* Set option bits (CASSPEC_OPT_*); returns the previous bits in *old_flags if non-NULL. */
 CASSPEC_API int casspec_set_options(casspec_model* m, unsigned flags, unsigned* old_flags);
 
-/* Activation sparsity (App. C: the TEAL draft of the DSIA family), a model setting for bf16 steps.
+/* Activation sparsity (App. C: the TEAL draft of the DSIA family), a model setting for every step.
  * With 0 < s < 1, before each of Wqkv, Wo, Wgate/Wup and Wdown every token's floor(s * K) inputs of
- * smallest magnitude (after RMSNorm) become 0; among equal magnitudes the lower index is kept.  The
+ * smallest magnitude (after RMSNorm) become 0; among equal magnitudes the lower index is kept.  A
+ * bf16 step selects on the split activation's value (hi + lo); a quantised step (App. C's mixed
+ * drafts, e.g. W4A4 with sparsity) selects on the bf16 activation it then quantises.  The
  * projections themselves stay dense, so a sparse step moves the same weight bytes as a dense one
- * (this is the draft's arithmetic, not its speed).  s = 0, the default, is the dense step.  While
- * s > 0, a step with quant_mode != 0 returns CASSPEC_E_INVAL.  Changing s drops captured graphs.
- * Errors: CASSPEC_E_INVAL (null model, s outside [0, 1)). */
+ * (this is the draft's arithmetic, not its speed).  s = 0, the default, is the dense step.  Changing
+ * s drops captured graphs.  Errors: CASSPEC_E_INVAL (null model, s outside [0, 1)). */
 CASSPEC_API int casspec_set_act_sparsity(casspec_model* m, float s);
 
 /* The sparsity rule of casspec_set_act_sparsity on a split activation x_split (dev, [128][ld] bf16:

@@ -683,9 +683,27 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
       const CUtensorMap& t_wd = tc8 ? Lp.tm_dq : Lp.tm_d8;
       const uint8_t *p_qkv = tc8 ? Lp.qkv_qp : Lp.qkv_fp, *p_wo = tc8 ? Lp.wo_qp : Lp.wo_fp;
       const uint8_t *p_wgu = tc8 ? Lp.wgu_qp : Lp.wgu_fp, *p_wd = tc8 ? Lp.wd_qp : Lp.wd_fp;
+      // the projection's quantised input: with activation sparsity (App. C's mixed draft) the bf16
+      // activation first loses its smallest-magnitude entries (selected on that bf16 value), then
+      // the same row quantiser runs on it
+      const float sp = m->act_sparsity;
+      auto norm_quant = [&](const float* gain) -> int {
+        if (sp > 0.f) {
+          LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, gain, n, d, c.rms_eps, m->xa, nullptr, nullptr, s, pdl, qmax, afmt));
+          LAUNCH(CASSPEC_K_OTHER, launch_sparsify(m->xa, d, n, d, sp, s, pdl, 1));
+          LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->xa, n, d, d, m->xq, d, m->xs, s, pdl, qmax, afmt));
+        } else {
+          LAUNCH(CASSPEC_K_OTHER, launch_rmsnorm(m->x, gain, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax, afmt));
+        }
+        return CASSPEC_OK;
+      };
+      auto quant = [&](uint16_t* in, int K) -> int {
+        if (sp > 0.f) LAUNCH(CASSPEC_K_OTHER, launch_sparsify(in, K, n, K, sp, s, pdl, 1));
+        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(in, n, K, K, m->xq, K, m->xs, s, pdl, qmax, afmt));
+        return CASSPEC_OK;
+      };
       if (it.kind == IT_QKV) {
-        LAUNCH(CASSPEC_K_OTHER,
-               launch_rmsnorm(m->x, Lp.attn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax, afmt));
+        if ((rc = norm_quant(Lp.attn_norm)) != CASSPEC_OK) return rc;
         EpiParams e = base;
         e.N = 3 * d;
         e.q_out = m->q;
@@ -698,14 +716,13 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
           LAUNCH(CASSPEC_K_QKV, gemm8(q_qkv, s_qkv, nullptr, nullptr, 3 * d, d, 3 * d / 128, EPI_QKV, e));
       } else if (it.kind == IT_WO) {
         // W8A8 activations are the bf16 values: the hi plane of the split output
-        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->o, n, d, d, m->xq, d, m->xs, s, pdl, qmax, afmt));
+        if ((rc = quant(m->o, d)) != CASSPEC_OK) return rc;
         if (tc)
           LAUNCH(CASSPEC_K_WO, gemmf8(t_wo, t_wo, p_wo, m->tm_xq8_d[bi], s_wo, nullptr, d, d, d / 128, EPI_RESID, ed));
         else
           LAUNCH(CASSPEC_K_WO, gemm8(q_wo, s_wo, nullptr, nullptr, d, d, d / 128, EPI_RESID, ed));
       } else if (it.kind == IT_GU) {
-        LAUNCH(CASSPEC_K_OTHER,
-               launch_rmsnorm(m->x, Lp.ffn_norm, n, d, c.rms_eps, nullptr, m->xq, m->xs, s, pdl, qmax, afmt));
+        if ((rc = norm_quant(Lp.ffn_norm)) != CASSPEC_OK) return rc;
         EpiParams eg = base;
         eg.N = F;
         eg.u_out = m->u;
@@ -715,7 +732,7 @@ int enqueue_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, const 
         else
           LAUNCH(CASSPEC_K_GATEUP, gemm8(q_wg, s_wg, q_wu, s_wu, F, d, cdiv(F, 64), EPI_GLU, eg));
       } else {
-        LAUNCH(CASSPEC_K_OTHER, launch_quant_rows(m->u, n, F, F, m->xq, F, m->xs, s, pdl, qmax, afmt));
+        if ((rc = quant(m->u, F)) != CASSPEC_OK) return rc;
         if (tc)
           LAUNCH(CASSPEC_K_DOWN, gemmf8(t_wd, t_wd, p_wd, m->tm_xq8_f[bi], s_wd, nullptr, d, F, d / 128, EPI_RESID, ed));
         else
@@ -1152,7 +1169,6 @@ int casspec_tree_step(casspec_model* m, casspec_kv* kv, const int32_t* tokens, c
     return CASSPEC_E_INVAL;
   if (quant_mode < 0 || quant_mode > 2) return CASSPEC_E_INVAL;
   if (quant_mode != 0 && !m->cfg.with_int8) return CASSPEC_E_INVAL;
-  if (quant_mode != 0 && m->act_sparsity > 0.f) return CASSPEC_E_INVAL;  // sparsity runs with bf16 steps only
   if (n < 1 || n > kMaxTree) return CASSPEC_E_SHAPE;
   if (kv->T + n > kMaxTree || kv->P_upper + kv->T + n > kv->ctx) return CASSPEC_E_CAPACITY;
   const int NL = m->cfg.n_layers;

@@ -241,7 +241,8 @@ cudaError_t launch_rmsnorm(const float* x, const float* g, int n, int d, float e
                            cudaStream_t s, bool pdl, int qmax = 127, int fmt = 0);
 // Activation sparsity of a split activation [128][ld] (hi rows 0..63, lo rows 64..127): in each of
 // the n token rows the floor(s K) smallest-magnitude entries of hi + lo become 0 (ties: lower index kept).
-cudaError_t launch_sparsify(uint16_t* x, int ld, int n, int K, float s, cudaStream_t st, bool pdl);
+// planes = 1: the magnitudes of the hi plane alone, and only the hi plane is written.
+cudaError_t launch_sparsify(uint16_t* x, int ld, int n, int K, float s, cudaStream_t st, bool pdl, int planes = 2);
 cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* q, int ldq, float* sq, cudaStream_t s,
                               bool pdl, int qmax = 127, int fmt = 0);
 cudaError_t launch_argmax_reduce(const float* v1, const int* i1, const float* v2, int tiles, int n, int* am,

@@ -315,13 +315,15 @@ cudaError_t launch_quant_rows(const uint16_t* x, int n, int d, int ldx, int8_t* 
 // ---------------------------------------------------------------------------------------------
 // Activation sparsity (App. C, TEAL's magnitude rule): in every token row t of a split activation
 // (hi plane row t, lo plane row 64 + t), the z = floor(s K) entries of smallest |hi + lo| become 0 in
-// both planes; among equal magnitudes the higher index goes first (the lower is kept).  One CTA per
+// both planes; among equal magnitudes the higher index goes first (the lower is kept).  With
+// planes = 1 only the hi plane is read and zeroed (the bf16 activation a quantised draft stores and
+// quantises; its lo plane is not used).  One CTA per
 // row: a radix select over the magnitude's fp32 bits (4 passes of 8 bits) finds the z-th smallest
 // magnitude T and how many entries equal to T are to go; the entries below T and the highest-index
 // entries equal to T are zeroed.
 // ---------------------------------------------------------------------------------------------
 constexpr int kSpThreads = 256;
-__global__ void __launch_bounds__(kSpThreads) sparsify_kernel(uint16_t* __restrict__ x, int ld, int K, int z) {
+__global__ void __launch_bounds__(kSpThreads) sparsify_kernel(uint16_t* __restrict__ x, int ld, int K, int z, int planes) {
   extern __shared__ uint32_t sp_key[];  // [K] magnitude bits
   __shared__ unsigned hist[256], part[kSpThreads];
   __shared__ unsigned s_prefix, s_rem;
@@ -330,7 +332,8 @@ __global__ void __launch_bounds__(kSpThreads) sparsify_kernel(uint16_t* __restri
   const int t = blockIdx.x, tid = threadIdx.x;
   uint16_t* hi = x + (size_t)t * ld;
   uint16_t* lo = x + (size_t)(64 + t) * ld;
-  for (int c = tid; c < K; c += kSpThreads) sp_key[c] = __float_as_uint(fabsf(bf2f(hi[c]) + bf2f(lo[c])));
+  for (int c = tid; c < K; c += kSpThreads)
+    sp_key[c] = __float_as_uint(fabsf(planes == 2 ? bf2f(hi[c]) + bf2f(lo[c]) : bf2f(hi[c])));
   if (tid == 0) {
     s_prefix = 0u;
     s_rem = (unsigned)z;
@@ -369,13 +372,14 @@ __global__ void __launch_bounds__(kSpThreads) sparsify_kernel(uint16_t* __restri
     if (k == T) drop = after++ < rem;
     if (drop) {
       hi[c] = 0;
-      lo[c] = 0;
+      if (planes == 2) lo[c] = 0;
     }
   }
 }
 
-cudaError_t launch_sparsify(uint16_t* x, int ld, int n, int K, float s, cudaStream_t st, bool pdl) {
-  if (n < 1 || n > 64 || K < 1 || ld < K || !(s >= 0.f && s < 1.f)) return cudaErrorInvalidValue;
+cudaError_t launch_sparsify(uint16_t* x, int ld, int n, int K, float s, cudaStream_t st, bool pdl, int planes) {
+  if (n < 1 || n > 64 || K < 1 || ld < K || !(s >= 0.f && s < 1.f) || (planes != 1 && planes != 2))
+    return cudaErrorInvalidValue;
   const int z = (int)floor((double)s * K + 1e-9);
   if (z <= 0) return cudaSuccess;
   const size_t smem = (size_t)K * 4;
@@ -390,7 +394,7 @@ cudaError_t launch_sparsify(uint16_t* x, int ld, int n, int K, float s, cudaStre
   if (smem > 65536) return cudaErrorInvalidValue;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n), dim3(kSpThreads), smem, st, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, sparsify_kernel, x, ld, K, z);
+  return cudaLaunchKernelEx(&cfg, sparsify_kernel, x, ld, K, z, planes);
 }
 
 // ---------------------------------------------------------------------------------------------

@@ -20,7 +20,14 @@
     median of up to 0.046);
   - s = 0.001 (z = floor(sK) = 0 for every K here): the sparsify launches run and zero nothing, and the
     logits equal the dense step's bit for bit; s = 0 again restores the dense step bit for bit;
-  - a quantised step is refused while s > 0.
+* Quantised steps with sparsity (App. C's mixed drafts, W8A8 and W4A4): the selection is taken on the
+  bf16 activation the quantiser then reads (the oracle's reading for quantised drafts):
+  - s = 0.001 (nothing zeroed): the sparse path (norm -> bf16 row -> selection -> row quantiser) gives
+    the fused norm-quantiser's codes, so the logits equal the dense quantised step's bit for bit;
+  - FFN-only layers at s = 0.99: within TOL_INT8 of the oracle (the dense quantised bound);
+  - the full model at s = 0.5 against the bf16-cache oracle: TOL_INT8_DEEP (W8A8) or TOL_W4 (W4A4,
+    whose attention-output codes follow the GPU's bf16 probabilities), with a median under half the
+    distance to the dense quantised step.
 """
 from __future__ import annotations
 
@@ -37,6 +44,7 @@ SH = synth.TINY
 SEED = 2468
 TOL_BF16 = 2e-2
 TOL_INT8_DEEP = 0.2  # as test_gpu_7b.TOL_INT8_DEEP
+TOL_W4 = 0.3  # as test_gpu_step.TOL_W4
 
 
 @pytest.fixture(scope="module")
@@ -159,11 +167,63 @@ def test_sparse_steps_match_oracle(cs):
             err = rel(got, ref)
             assert np.all(err < TOL_INT8_DEEP), (tseed, s, err.max())
             assert np.median(err) < 0.5 * np.median(rel(dense, ref)), (tseed, s, np.median(err))
-    rc, _ = run(0.5, toks, parent, mode=1)
-    assert rc == cs.E_INVAL
     _, dense0 = run(0.0, toks, parent)
     _, none0 = run(0.001, toks, parent)
     _, dense1 = run(0.0, toks, parent)
     assert np.array_equal(dense0, none0) and np.array_equal(dense0, dense1)
+    assert cs.get_status(dm.h) == 0
+    dm.close()
+
+
+def test_quantised_sparse_steps_match_oracle(cs):
+    from paper_2510_26843_gb300.workload import DeviceKV, DeviceModel
+
+    dm = DeviceModel(SH, SEED, with_int8=True)
+    ow = oracle.Weights.from_seed(SEED, SH, keep_layers=SH.n_layers)
+    TOL_INT8 = 5e-2
+
+    def run(s, toks, parent, mode, mask=None):
+        kv = DeviceKV(dm, 256)
+        kv.load_random_prefix(SEED, 96)
+        n = len(toks)
+        lg = torch.empty((n, SH.vocab), dtype=torch.float32, device="cuda")
+        cs.set_act_sparsity(dm.h, s)
+        t = torch.tensor(np.asarray(toks, dtype=np.int32), device="cuda")
+        p = torch.tensor(np.asarray(parent, dtype=np.int32), device="cuda")
+        rc = cs.tree_step(dm.h, kv.h, t, p, n, mask, mode, lg, check=False)
+        torch.cuda.synchronize()
+        kv.close()
+        assert rc == 0
+        return lg.cpu().numpy().astype(np.float64)
+
+    def oracle_cache():
+        okv = oracle.KVCache(SH.n_layers, SH.n_heads, SH.head_dim, 256)
+        for l in range(SH.n_layers):
+            k = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, SH, l, "k", 96)).astype(np.float64)
+            v = synth.bf16_to_f32(synth.prefix_kv_bf16(SEED, SH, l, "v", 96)).astype(np.float64)
+            okv.load_prefix(l, k, v)
+        return okv
+
+    def rel(a, ref):
+        return np.max(np.abs(a - ref) / np.ptp(ref, axis=1, keepdims=True), axis=1)
+
+    ffn_only = np.array([1 | cs.SKIP_ATTN, 1 | cs.SKIP_ATTN], np.uint8)
+    parent = synth.tree(6, 24, 6)
+    toks = synth.tokens(6, 24, SH.vocab)
+    for mode in (1, 2):
+        dense_q = run(0.0, toks, parent, mode)
+        np.testing.assert_array_equal(run(0.001, toks, parent, mode), dense_q)
+        got = run(0.99, toks, parent, mode, mask=ffn_only)
+        ref = oracle.tree_step(ow, oracle_cache(), toks, parent, skip_mask=ffn_only, quant_mode=mode,
+                               act_sparsity=0.99)
+        assert np.all(rel(got, ref) < TOL_INT8), (mode, rel(got, ref).max())
+        got = run(0.5, toks, parent, mode)
+        ref = oracle.tree_step(ow, oracle_cache(), toks, parent, quant_mode=mode, act_sparsity=0.5,
+                               attn_bf16=True)
+        dense = oracle.tree_step(ow, oracle_cache(), toks, parent, quant_mode=mode, attn_bf16=True)
+        err = rel(got, ref)
+        assert np.all(err < (TOL_INT8_DEEP if mode == 1 else TOL_W4)), (mode, err.max())
+        assert np.median(err) < 0.5 * np.median(rel(dense, ref)), (mode, np.median(err))
+    cs.set_act_sparsity(dm.h, 0.0)
     assert cs.get_status(dm.h) == 0
     dm.close()

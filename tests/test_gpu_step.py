@@ -22,6 +22,8 @@ pytestmark = pytest.mark.gpu
 SH = synth.TINY
 SEED = 1234
 TOL_BF16, TOL_INT8, MARGIN = 2e-2, 5e-2, 1e-3
+TOL_INT8_DEEP = 0.2  # as test_gpu_7b.TOL_INT8_DEEP
+TOL_W4 = 0.3  # full W4A4 steps (see test_w4a4_mode_logits)
 
 
 @pytest.fixture(scope="module")
@@ -268,20 +270,29 @@ def test_int8_mode_logits(cs, dev_model, ow, prefix):
 
 
 def test_w4a4_mode_logits(cs, dev_model, ow, prefix):
-    """W4A4 draft logits.  A 4-bit code moves by a seventh of its row's range, so the logits follow
-    any bf16-sized perturbation strongly (0.14 of the range on this model); the bound is twice the
-    oracle's own movement when q and the new K/V are rounded to bf16, never below 5e-2.  The integer
-    parts are checked bit-exactly by test_int4_weights_bit_exact and test_quantize_rows4_bit_exact."""
-    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
-    _, okv2 = fresh_pair(cs, dev_model, ow, prefix)
+    """W4A4 draft logits.  A 4-bit code moves by a seventh of its row's range, so any difference in the
+    values it quantises that crosses a rounding boundary moves the logits by a large step.  Without
+    attention (FFN-only layers, inputs the chain computes to fp32 accuracy) the step is held to the
+    dense quantised bound TOL_INT8.  With attention the GPU's probabilities enter P.V as bf16, which
+    the oracle's bf16-cache variant does not model, and the attention output's codes flip in most
+    rows: the full step is held to the fixed TOL_W4 (1.5 x the 0.2 the oracle's own fp64 and
+    bf16-cache variants differ by on these inputs), median row under TOL_W4 / 2.  The integer parts
+    are checked bit-exactly by test_int4_weights_bit_exact, test_quantize_rows4_bit_exact and the
+    equality of the two W4A4 paths."""
     parent = synth.tree(4, 8, 4)
     toks = synth.tokens(4, 8, SH.vocab)
+    ffn_only = np.array([1 | cs.SKIP_ATTN] * SH.n_layers, np.uint8)
+    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
+    got = gpu_step(cs, dev_model, kv, toks, parent, mask=ffn_only, mode=2)
+    ref = oracle.tree_step(ow, okv, toks, parent, skip_mask=ffn_only, quant_mode=2)
+    assert np.all(rel_err(got, ref) < TOL_INT8), rel_err(got, ref).max()
+    kv.close()
+    kv, okv = fresh_pair(cs, dev_model, ow, prefix)
     got = gpu_step(cs, dev_model, kv, toks, parent, mode=2)
     assert cs.get_status(dev_model.h) == 0
-    ref = oracle.tree_step(ow, okv, toks, parent, quant_mode=2)
-    pert = oracle.tree_step(ow, okv2, toks, parent, quant_mode=2, attn_bf16=True)
+    ref = oracle.tree_step(ow, okv, toks, parent, quant_mode=2, attn_bf16=True)
     err = rel_err(got, ref)
-    assert err.max() <= max(TOL_INT8, 2.0 * rel_err(pert, ref).max()), (err.max(), rel_err(pert, ref).max())
+    assert err.max() < TOL_W4 and np.median(err) < TOL_W4 / 2, (err.max(), np.median(err))
     kv.close()
 
 
