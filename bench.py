@@ -466,6 +466,30 @@ def run_gpu(args) -> None:
     if verify:
         assert 1 <= int(out_h[0]) <= n
 
+    # ---- per-step spread (each step between its own events) and the step without graphs ----
+    k = max(1, min(args.steps, 50))
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(k)]
+    barrier()
+    for a, b in evs:
+        a.record(stream)
+        step()
+        b.record(stream)
+    barrier()
+    per = sorted(a.elapsed_time(b) * 1e3 for a, b in evs)
+    step_stats = {"samples": k, "p50_us": round(per[len(per) // 2], 1),
+                  "p90_us": round(per[min(len(per) - 1, int(0.9 * len(per)))], 1)}
+    if graphs:
+        cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC)
+        for _ in range(3):
+            step()
+        barrier()
+        e0.record(stream)
+        for _ in range(k):
+            step()
+        e1.record(stream)
+        barrier()
+        step_stats["eager_us"] = round(e0.elapsed_time(e1) / k * 1e3, 1)
+
     # ---- kernel-timing pass: eager launches bracketed by CUDA events on the launch stream ----
     cs.set_options(dm.h, cs.OPT_PDL | cs.OPT_W4_TC | cs.OPT_W8_TC)
     cs.profile(dm.h, True)
@@ -527,6 +551,7 @@ def run_gpu(args) -> None:
                      "traffic": recorded_traffic() if (args.workload == "verify7b") else None,
                      "algorithmic_bytes_per_launch": gu_bytes},
         "kernels": per_kind,
+        "step_stats": step_stats,
         "e2e": {"value": round(e2e_us, 1), "unit": "us", "h2d_bytes_per_step": 2 * n * 4,
                 "d2h_bytes_per_step": int(out_d.numel() * out_d.element_size())},
         "gpu_launches": int(launches),
