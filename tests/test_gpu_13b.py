@@ -154,3 +154,27 @@ def test_13b_cascade_round(cs, dm13):
     if np.all(oracle.top2_margin(ref)[path] >= MARGIN):
         assert gpu_path == path and int(acc[L + 1]) == bonus
     kv.close()
+
+
+@pytest.mark.parametrize("n", [8, 64])
+def test_13b_w8a8_tensor_core_path_equals_integer_path(cs, dm13, n):
+    """The 40-layer 13B W8A8 step on both paths (K = 5120 and 13824: a gate/up output sums up to five
+    exact 1024-column accumulators): the same codes and scales, exact int32 sums on both, so the
+    logits are bitwise equal, at the 16- and 64-token tiles."""
+    from paper_2510_26843_gb300.workload import DeviceKV
+
+    parent = synth.tree(SEED + n, n, 8)
+    toks = synth.tokens(SEED + n, n, SH13.vocab)
+    base = cs.OPT_PDL | cs.OPT_GRAPHS | cs.OPT_W4_TC
+    out = []
+    for flags in (base | cs.OPT_W8_TC, base):
+        cs.set_options(dm13.h, flags)
+        kv = DeviceKV(dm13, P + 128)
+        kv.load_random_prefix(SEED, P)
+        got, _, _ = gpu_step(cs, dm13, kv, toks, parent, mode=1)
+        assert cs.get_status(dm13.h) == 0
+        kv.close()
+        out.append(got)
+    cs.set_options(dm13.h, base | cs.OPT_W8_TC)
+    assert np.all(np.isfinite(out[0]))
+    np.testing.assert_array_equal(out[0], out[1])
