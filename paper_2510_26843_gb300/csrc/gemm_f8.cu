@@ -30,6 +30,7 @@ namespace casspec {
 constexpr int kOpE4M3 = 0, kOpS8 = 1;
 constexpr uint32_t kF8ATile = 128 * 128;  // 128 rows x 128 codes
 constexpr int kS8Region = 8;              // k-blocks per fp32 accumulator in kOpS8 (1024 columns)
+constexpr int kF8MaxContrib = 8;          // stream-K contributors per tile whose partials are read together
 constexpr size_t kF8SmemMax = 232448;     // dynamic shared memory limit per CTA
 
 // kOpS8: converter warps (8 for the small token counts of drafts, 4 where the epilogue needs the
@@ -435,8 +436,7 @@ __global__ void __launch_bounds__(f8_threads(OP, BN), 1)
         finish = flags[1] != 0;
         if (finish) {
           __threadfence();
-          for (int cc = c_first; cc <= c_last; ++cc) {
-            if (cc == cta) continue;
+          auto add_partial = [&](int cc) {
             const float* pp = a.partials + (size_t)(t + cc) * (64 * 128);
 #pragma unroll
             for (int i = 0; i < BN; ++i)
@@ -447,6 +447,16 @@ __global__ void __launch_bounds__(f8_threads(OP, BN), 1)
                 else
                   v[i] += pv;
               }
+          };
+          if (BN <= 32 && c_last - c_first < kF8MaxContrib) {
+            // small token tiles: the loads of every contributor's partial are issued together, one
+            // memory round trip instead of one per contributor
+#pragma unroll
+            for (int k = 0; k < kF8MaxContrib; ++k)
+              if (k <= c_last - c_first && c_first + k != cta) add_partial(c_first + k);
+          } else {
+            for (int cc = c_first; cc <= c_last; ++cc)
+              if (cc != cta) add_partial(cc);
           }
           if (threadIdx.x == 64) a.counters[t] = 0u;
         }
