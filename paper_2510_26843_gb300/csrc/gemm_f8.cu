@@ -132,7 +132,9 @@ __device__ __forceinline__ void s8_widen_chunk(const uint8_t* raw, uint8_t* cv, 
   *reinterpret_cast<uint4*>(dst + (((j0 + 1) ^ sw) << 4)) = hi;
 }
 
-template <int BN, int EPI, int OP>
+// BATCH (kOpS8, BN <= 32, chosen for n >= 4): the stream-K fix-up reads every contributor's partial in
+// one batch; a separate instantiation, so the one-token drafts run the smaller code without it.
+template <int BN, int EPI, int OP, bool BATCH>
 __global__ void __launch_bounds__(f8_threads(OP, BN), 1)
     gemm_f8_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmW2,
                    const __grid_constant__ CUtensorMap tmX, const GemmF8Args a) {
@@ -448,9 +450,9 @@ __global__ void __launch_bounds__(f8_threads(OP, BN), 1)
                   v[i] += pv;
               }
           };
-          if (BN <= 32 && c_last - c_first < kF8MaxContrib) {
-            // small token tiles: the loads of every contributor's partial are issued together, one
-            // memory round trip instead of one per contributor
+          if (BATCH && c_last - c_first < kF8MaxContrib) {
+            // the loads of every contributor's partial are issued together: one memory round trip
+            // instead of one per contributor
 #pragma unroll
             for (int k = 0; k < kF8MaxContrib; ++k)
               if (k <= c_last - c_first && c_first + k != cta) add_partial(c_first + k);
@@ -557,10 +559,10 @@ bool encode_tmap_u8(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int EPI, int OP>
+template <int BN, int EPI, int OP, bool BATCH>
 static cudaError_t launch_f8_t(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX,
                                const GemmF8Args& args, int grid, cudaStream_t stream, bool pdl) {
-  auto kern = gemm_f8_kernel<BN, EPI, OP>;
+  auto kern = gemm_f8_kernel<BN, EPI, OP, BATCH>;
   constexpr size_t smem = f8_smem_bytes(OP, BN);
   static int configured = -1;
   int dev = 0;
@@ -583,16 +585,25 @@ static cudaError_t launch_f8_t(const CUtensorMap& tmW, const CUtensorMap& tmW2, 
   return cudaLaunchKernelEx(&cfg, kern, tmW, tmW2, tmX, args);
 }
 
+template <int BN, int OP, bool BATCH>
+static cudaError_t launch_f8_epi(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int epi,
+                                 const GemmF8Args& args, int grid, cudaStream_t s, bool pdl) {
+  switch (epi) {
+    case EPI_STORE: return launch_f8_t<BN, EPI_STORE, OP, BATCH>(tmW, tmW2, tmX, args, grid, s, pdl);
+    case EPI_RESID: return launch_f8_t<BN, EPI_RESID, OP, BATCH>(tmW, tmW2, tmX, args, grid, s, pdl);
+    case EPI_QKV: return launch_f8_t<BN, EPI_QKV, OP, BATCH>(tmW, tmW2, tmX, args, grid, s, pdl);
+    case EPI_GLU: return launch_f8_t<BN, EPI_GLU, OP, BATCH>(tmW, tmW2, tmX, args, grid, s, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
 template <int BN, int OP>
 static cudaError_t launch_f8_bn(const CUtensorMap& tmW, const CUtensorMap& tmW2, const CUtensorMap& tmX, int epi,
                                 const GemmF8Args& args, int grid, cudaStream_t s, bool pdl) {
-  switch (epi) {
-    case EPI_STORE: return launch_f8_t<BN, EPI_STORE, OP>(tmW, tmW2, tmX, args, grid, s, pdl);
-    case EPI_RESID: return launch_f8_t<BN, EPI_RESID, OP>(tmW, tmW2, tmX, args, grid, s, pdl);
-    case EPI_QKV: return launch_f8_t<BN, EPI_QKV, OP>(tmW, tmW2, tmX, args, grid, s, pdl);
-    case EPI_GLU: return launch_f8_t<BN, EPI_GLU, OP>(tmW, tmW2, tmX, args, grid, s, pdl);
+  if constexpr (OP == kOpS8 && BN <= 32) {
+    if (args.ep.n >= 4) return launch_f8_epi<BN, OP, true>(tmW, tmW2, tmX, epi, args, grid, s, pdl);
   }
-  return cudaErrorInvalidValue;
+  return launch_f8_epi<BN, OP, false>(tmW, tmW2, tmX, epi, args, grid, s, pdl);
 }
 
 template <int OP>
